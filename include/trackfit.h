@@ -1,0 +1,173 @@
+/*
+ * trackfit.h -- C-ABI of the GB300 (sm_103a) batched inference library for the
+ * bidirectional minGRU track-fit encoder of "Fast and Precise Learned
+ * Charged-Particle Trajectory Regression at the LHC".
+ *
+ * Problem statement (Sec. 3, first paragraph): the model maps the hit sequence
+ * of one track, ordered by measurement time, to the five perigee parameters
+ * (d0, z0, phi, theta, q/p) at the point of closest approach to the beam axis.
+ * This library runs that map for a batch of independent tracks (Sec. 4,
+ * "embarrassingly parallel across tracks").  The encoder computed is:
+ *
+ *   per hit   : u = min-max normalised features, e = [sin(pi s_k u_f), cos(pi s_k u_f)]
+ *               (Sec. 3.2, 16-scale Fourier featurisation), x0 = W_e2 SiLU(W_e1 e + b_e1) + b_e2
+ *   per layer : x_hat = RMSNorm(x) g ; [p_zf, n_f, p_zb, n_b, p_g] = W_in x_hat + b_in
+ *               forward and reverse scans h_t = h_{t-1} + z_t (n_t - h_{t-1}), z = sigma(p_z)
+ *               (Sec. 3.2, Eq. 2), masked to the track's hits, zero initial state
+ *               x' = x + (W_m [h_f; h_b] + b_m) * sigma(p_g)
+ *               x  = x' + W_2 SiLU(W_1 x' + b_1) + b_2        (padded hits set to 0)
+ *   per track : p = mean of x over the track's hits (or, pool = ENDPOINTS, the
+ *               forward state at the last hit and the reverse state at the first
+ *               hit, Sec. 3.2); q = W_h2 SiLU(W_h1 RMSNorm(p) g_h + b_h1) + b_h2,
+ *               35 = 5 parameters x 7 quantiles; output = the median quantile
+ *               (Sec. 3.2-3.3).
+ *
+ * Precision: TRACKFIT_FP32 computes everything in fp32.  TRACKFIT_BF16_PROJ rounds
+ * the operands of every per-hit matrix product (Fourier vector, embedding hidden,
+ * x_hat, [h_f; h_b], x', MLP hidden, and the weights of those products) to bf16
+ * and accumulates in fp32; gates, scan state, residual stream, pooling and the
+ * head stay fp32 (Sec. 3.5: reduced-precision projections, fp32 recurrence).
+ *
+ * Threading: a handle may be used from one host thread at a time and on one
+ * stream at a time (it owns a device workspace).  Different handles are
+ * independent.
+ */
+#ifndef TRACKFIT_H
+#define TRACKFIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TRACKFIT_ABI_VERSION 1
+#define TRACKFIT_MAX_FEATURES 5
+#define TRACKFIT_MAX_FOURIER 16
+
+typedef enum {
+  TRACKFIT_OK = 0,
+  TRACKFIT_ERR_INVALID_ARG = 1,  /* NULL pointer, n_tracks <= 0, misaligned pointer, bad sizes */
+  TRACKFIT_ERR_UNSUPPORTED = 2,  /* configuration outside what the kernels implement */
+  TRACKFIT_ERR_CUDA = 3,         /* a CUDA runtime call or kernel launch failed */
+  TRACKFIT_ERR_OOM = 4,          /* device allocation failed (create only) */
+  TRACKFIT_ERR_BAD_HITS = 5,     /* device-side: tracks with n_hits outside [1, max_hits] */
+  TRACKFIT_ERR_TIMEOUT = 6       /* device-side: a bounded wait inside a kernel expired */
+} trackfit_status;
+
+typedef enum { TRACKFIT_FP32 = 0, TRACKFIT_BF16_PROJ = 1 } trackfit_precision;
+typedef enum { TRACKFIT_POOL_MEAN = 0, TRACKFIT_POOL_ENDPOINTS = 1 } trackfit_pool;
+
+/* Encoder shape.  Supported: abi_version = 1, n_features = 5 (x, y, z [mm], r [mm],
+ * phi [rad]), n_fourier = 16, 1 <= max_hits <= 64, d_model in {16, 32, ..., 256}
+ * (multiple of 16), d_hidden = 3 * d_model / 2, 1 <= n_layers <= 16,
+ * head_hidden = 128, n_quantiles = 7 (odd).  feat_min/feat_max are fixed min-max
+ * constants (feat_max > feat_min); fourier_scale[k] = s_k, the feature argument
+ * is pi * s_k * u; rms_eps > 0. */
+typedef struct {
+  int32_t abi_version;
+  int32_t max_hits;
+  int32_t n_features;
+  int32_t n_fourier;
+  int32_t d_model;
+  int32_t d_hidden;
+  int32_t n_layers;
+  int32_t head_hidden;
+  int32_t n_quantiles;
+  int32_t precision;  /* trackfit_precision */
+  int32_t pool;       /* trackfit_pool */
+  float feat_min[TRACKFIT_MAX_FEATURES];
+  float feat_max[TRACKFIT_MAX_FEATURES];
+  float fourier_scale[TRACKFIT_MAX_FOURIER];
+  float rms_eps;
+} trackfit_config_t;
+
+typedef struct trackfit_ctx* trackfit_t;
+
+/* Number of fp32 values in the weight blob for cfg (0 if cfg is NULL or
+ * unsupported).  Blob order, every matrix in PyTorch [out][in] row-major order,
+ * with D = d_model, H = d_hidden, E = 2 * n_features * n_fourier,
+ * P = D (mean pooling) or 2H (endpoints), Hh = head_hidden, Q = 5 * n_quantiles:
+ *   W_e1[D][E] b_e1[D] W_e2[D][D] b_e2[D]
+ *   per layer: g[D] W_in[4H+D][D] b_in[4H+D] (row blocks z_f, n_f, z_b, n_b, gate)
+ *              W_m[D][2H] (columns: forward states, then reverse) b_m[D]
+ *              W_1[D][D] b_1[D] W_2[D][D] b_2[D]
+ *   g_h[P] W_h1[Hh][P] b_h1[Hh] W_h2[Q][Hh] b_h2[Q]   (Q rows parameter-major: [5][7]) */
+size_t trackfit_weight_count(const trackfit_config_t* cfg);
+
+/* Validate cfg, copy the host fp32 weights to the device (converted and repacked
+ * for the kernels) and allocate the handle's workspace.  Synchronous; launches no
+ * work on any user stream.  The caller keeps ownership of `weights` and may free
+ * it on return.  Errors: INVALID_ARG (NULL, n_weights != trackfit_weight_count),
+ * UNSUPPORTED (cfg outside the supported set), OOM, CUDA.  *out is set only on
+ * success. */
+int trackfit_create(const trackfit_config_t* cfg, const float* weights, size_t n_weights,
+                    trackfit_t* out);
+
+/* Run the encoder on n_tracks tracks, asynchronously on `stream` (a cudaStream_t;
+ * NULL = the legacy default stream).  No host synchronisation, no allocation.
+ *   hits       device, [n_tracks][max_hits][5] fp32, row-major, 16-byte aligned;
+ *              hit t of track b is valid for t < n_hits[b]; padded entries are
+ *              never read into the result (they may hold NaN).
+ *   n_hits     device, [n_tracks] int32.
+ *   out_params device, [n_tracks][5] fp32 (d0, z0, phi, theta, q/p), 16-byte aligned.
+ * The caller owns all three buffers.  Host-side checks (NULL, n_tracks <= 0,
+ * alignment) return INVALID_ARG and launch nothing; launch failures return CUDA.
+ * A track with n_hits outside [1, max_hits] gets a NaN row and is counted in the
+ * device error counter (trackfit_device_errors). */
+int trackfit_forward(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
+                     float* out_params, void* stream);
+
+/* As trackfit_forward, and optionally also writes (each pointer may be NULL):
+ *   out_quantiles device [n_tracks][5][7] fp32: all head outputs (Sec. 3.2-3.3);
+ *   out_pooled    device [n_tracks][P] fp32: the pooled vector before the head. */
+int trackfit_forward_ex(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
+                        float* out_params, float* out_quantiles, float* out_pooled, void* stream);
+
+/* End-to-end variant with HOST buffers: copies hits [n_tracks][max_hits][5] and
+ * n_hits [n_tracks] to the device, runs the encoder and copies out_params
+ * [n_tracks][5] back, all on `stream`, and returns after the stream has finished
+ * this work (synchronous).  Pinned (page-locked) host memory makes the copies
+ * asynchronous and faster; pageable memory works too.  The device staging
+ * buffers are owned by the handle and grow on demand (this call may allocate).
+ * Errors as trackfit_forward, plus OOM. */
+int trackfit_forward_host(trackfit_t h, const float* hits_host, const int32_t* n_hits_host,
+                          int64_t n_tracks, float* out_params_host, void* stream);
+
+/* Read and reset the device error counters: synchronises `stream`, returns the
+ * number of tracks with invalid n_hits since the last call in *n_bad, and
+ * returns TRACKFIT_ERR_TIMEOUT if a bounded device wait expired (else OK or
+ * BAD_HITS when *n_bad > 0). */
+int trackfit_device_errors(trackfit_t h, void* stream, int64_t* n_bad);
+
+/* Name of the kernel path the handle runs: "simt-fp32", "simt-bf16" or
+ * "tcgen05-bf16".  Static string, owned by the library. */
+const char* trackfit_path_name(trackfit_t h);
+
+/* Select the kernel path: 0 = automatic (tcgen05 for BF16_PROJ configs it
+ * supports, SIMT otherwise), 1 = force the SIMT path.  Returns UNSUPPORTED if the
+ * requested path cannot run this configuration. */
+int trackfit_set_path(trackfit_t h, int path);
+
+/* Free everything the handle owns.  Accepts NULL.  The caller must make sure no
+ * work using the handle is still running on any stream. */
+void trackfit_destroy(trackfit_t h);
+
+/* Static description of a status code. */
+const char* trackfit_strerror(int status);
+
+/* Test hook: masked bidirectional linear recurrence h_t = a_t h_{t-1} + b_t x_t
+ * (the spec form of Eq. 2 with a = 1 - z, b = z, x = n) on the device.
+ * a, b, x, h_fwd, h_bwd: device [n_tracks][T][C] fp32; n_hits device [n_tracks].
+ * Steps t >= n_hits[b] carry the state and output 0; the reverse scan starts at
+ * t = n_hits[b] - 1.  Asynchronous on `stream`. */
+int trackfit_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits,
+                        int64_t n_tracks, int32_t T, int32_t C, float* h_fwd, float* h_bwd,
+                        void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TRACKFIT_H */

@@ -1,0 +1,233 @@
+// Host side of the C-ABI (include/trackfit.h): validation, weight upload,
+// workspace, dispatch to the SIMT or tcgen05 kernel path, error counters.
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include "trackfit_internal.h"
+
+int tf_status_from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return TRACKFIT_OK;
+  if (e == cudaErrorMemoryAllocation) return TRACKFIT_ERR_OOM;
+  return TRACKFIT_ERR_CUDA;
+}
+
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Fill the shape summary and blob offsets; false if cfg is outside the supported set.
+static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
+  if (!c || c->abi_version != TRACKFIT_ABI_VERSION) return false;
+  if (c->n_features != TRACKFIT_MAX_FEATURES || c->n_fourier != TRACKFIT_MAX_FOURIER) return false;
+  if (c->max_hits < 1 || c->max_hits > TF_MAX_HITS) return false;
+  if (c->d_model < 16 || c->d_model > 256 || (c->d_model % 16) != 0) return false;
+  if (c->d_hidden != 3 * c->d_model / 2) return false;
+  if (c->n_layers < 1 || c->n_layers > TF_MAX_LAYERS) return false;
+  if (c->head_hidden != 128) return false;
+  if (c->n_quantiles < 1 || c->n_quantiles > 15 || (c->n_quantiles % 2) == 0) return false;
+  if (c->precision != TRACKFIT_FP32 && c->precision != TRACKFIT_BF16_PROJ) return false;
+  if (c->pool != TRACKFIT_POOL_MEAN && c->pool != TRACKFIT_POOL_ENDPOINTS) return false;
+  if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return false;
+  for (int f = 0; f < TRACKFIT_MAX_FEATURES; ++f)
+    if (!(c->feat_max[f] > c->feat_min[f]) || !std::isfinite(c->feat_max[f]) || !std::isfinite(c->feat_min[f]))
+      return false;
+  for (int k = 0; k < TRACKFIT_MAX_FOURIER; ++k)
+    if (!std::isfinite(c->fourier_scale[k])) return false;
+  s->T = c->max_hits;
+  s->F = c->n_features;
+  s->K = c->n_fourier;
+  s->E = 2 * s->F * s->K;
+  s->D = c->d_model;
+  s->H = c->d_hidden;
+  s->L = c->n_layers;
+  s->P = c->pool == TRACKFIT_POOL_MEAN ? s->D : 2 * s->H;
+  s->Hh = c->head_hidden;
+  s->NQ = c->n_quantiles;
+  s->Q = 5 * c->n_quantiles;
+  s->precision = c->precision;
+  s->pool = c->pool;
+  s->rms_eps = c->rms_eps;
+  for (int f = 0; f < s->F; ++f) {
+    s->feat_min[f] = c->feat_min[f];
+    s->feat_inv_range[f] = (float)(1.0 / ((double)c->feat_max[f] - (double)c->feat_min[f]));
+    s->feat_min_d[f] = c->feat_min[f];
+    s->feat_range_d[f] = (double)c->feat_max[f] - (double)c->feat_min[f];
+  }
+  for (int k = 0; k < s->K; ++k) s->scale[k] = c->fourier_scale[k];
+  const size_t D = s->D, H = s->H, E = s->E, P = s->P, Hh = s->Hh, Q = s->Q;
+  size_t p = 0;
+  o->emb_w1 = p; p += D * E;
+  o->emb_b1 = p; p += D;
+  o->emb_w2 = p; p += D * D;
+  o->emb_b2 = p; p += D;
+  for (int l = 0; l < s->L; ++l) {
+    tf_layer_off& y = o->layer[l];
+    y.g = p; p += D;
+    y.w_in = p; p += (4 * H + D) * D;
+    y.b_in = p; p += 4 * H + D;
+    y.w_m = p; p += D * 2 * H;
+    y.b_m = p; p += D;
+    y.w1 = p; p += D * D;
+    y.b1 = p; p += D;
+    y.w2 = p; p += D * D;
+    y.b2 = p; p += D;
+  }
+  o->head_g = p; p += P;
+  o->head_w1 = p; p += Hh * P;
+  o->head_b1 = p; p += Hh;
+  o->head_w2 = p; p += Q * Hh;
+  o->head_b2 = p; p += Q;
+  o->total = p;
+  return true;
+}
+
+extern "C" size_t trackfit_weight_count(const trackfit_config_t* cfg) {
+  tf_shape s;
+  tf_blob_off o;
+  if (!derive(cfg, &s, &o)) return 0;
+  return o.total;
+}
+
+extern "C" const char* trackfit_strerror(int status) {
+  switch (status) {
+    case TRACKFIT_OK: return "ok";
+    case TRACKFIT_ERR_INVALID_ARG: return "invalid argument";
+    case TRACKFIT_ERR_UNSUPPORTED: return "unsupported configuration";
+    case TRACKFIT_ERR_CUDA: return "CUDA error";
+    case TRACKFIT_ERR_OOM: return "out of device memory";
+    case TRACKFIT_ERR_BAD_HITS: return "tracks with hit counts outside [1, max_hits]";
+    case TRACKFIT_ERR_TIMEOUT: return "a bounded device wait expired";
+    default: return "unknown status";
+  }
+}
+
+extern "C" void trackfit_destroy(trackfit_t h) {
+  if (!h) return;
+  tf_tc_destroy(h);
+  cudaFree(h->d_w);
+  cudaFree(h->d_err);
+  cudaFree(h->ws);
+  cudaFree(h->st_hits);
+  cudaFree(h->st_n);
+  cudaFree(h->st_out);
+  delete h;
+}
+
+extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weights, size_t n_weights,
+                               trackfit_t* out) {
+  if (!cfg || !weights || !out) return TRACKFIT_ERR_INVALID_ARG;
+  tf_shape s;
+  tf_blob_off o;
+  if (cfg->abi_version != TRACKFIT_ABI_VERSION) return TRACKFIT_ERR_UNSUPPORTED;
+  if (!derive(cfg, &s, &o)) return TRACKFIT_ERR_UNSUPPORTED;
+  if (n_weights != o.total) return TRACKFIT_ERR_INVALID_ARG;
+  trackfit_ctx* h = new (std::nothrow) trackfit_ctx();
+  if (!h) return TRACKFIT_ERR_OOM;
+  h->cfg = *cfg;
+  h->s = s;
+  h->off = o;
+  h->path = TF_PATH_SIMT;
+  int st = tf_status_from_cuda(cudaMalloc(&h->d_w, o.total * sizeof(float)));
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(h->d_w, weights, o.total * sizeof(float), cudaMemcpyHostToDevice));
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMalloc(&h->d_err, 4 * sizeof(unsigned long long)));
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemset(h->d_err, 0, 4 * sizeof(unsigned long long)));
+  if (st == TRACKFIT_OK) st = tf_simt_workspace(h);
+  if (st == TRACKFIT_OK && s.precision == TRACKFIT_BF16_PROJ && tf_tc_supported(s)) {
+    st = tf_tc_create(h, weights);
+    if (st == TRACKFIT_OK) h->path = TF_PATH_TC;
+  }
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaDeviceSynchronize());
+  if (st != TRACKFIT_OK) {
+    trackfit_destroy(h);
+    return st;
+  }
+  *out = h;
+  return TRACKFIT_OK;
+}
+
+extern "C" const char* trackfit_path_name(trackfit_t h) {
+  if (!h) return "none";
+  if (h->path == TF_PATH_TC) return "tcgen05-bf16";
+  return h->s.precision == TRACKFIT_BF16_PROJ ? "simt-bf16" : "simt-fp32";
+}
+
+extern "C" int trackfit_set_path(trackfit_t h, int path) {
+  if (!h) return TRACKFIT_ERR_INVALID_ARG;
+  if (path == 1) {
+    h->path = TF_PATH_SIMT;
+    return TRACKFIT_OK;
+  }
+  if (path != 0) return TRACKFIT_ERR_INVALID_ARG;
+  h->path = (h->tc != nullptr) ? TF_PATH_TC : TF_PATH_SIMT;
+  return TRACKFIT_OK;
+}
+
+extern "C" int trackfit_forward_ex(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
+                                   float* out_params, float* out_q, float* out_pool, void* stream) {
+  if (!h || !hits || !n_hits || !out_params) return TRACKFIT_ERR_INVALID_ARG;
+  if (n_tracks <= 0) return TRACKFIT_ERR_INVALID_ARG;
+  if (!aligned16(hits) || !aligned16(out_params) || !aligned16(n_hits)) return TRACKFIT_ERR_INVALID_ARG;
+  if ((out_q && !aligned16(out_q)) || (out_pool && !aligned16(out_pool))) return TRACKFIT_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (h->path == TF_PATH_TC) return tf_tc_forward(h, hits, n_hits, n_tracks, out_params, out_q, out_pool, st);
+  return tf_simt_forward(h, hits, n_hits, n_tracks, out_params, out_q, out_pool, st);
+}
+
+extern "C" int trackfit_forward(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
+                                float* out_params, void* stream) {
+  return trackfit_forward_ex(h, hits, n_hits, n_tracks, out_params, nullptr, nullptr, stream);
+}
+
+extern "C" int trackfit_forward_host(trackfit_t h, const float* hits_host, const int32_t* n_hits_host,
+                                     int64_t n_tracks, float* out_host, void* stream) {
+  if (!h || !hits_host || !n_hits_host || !out_host || n_tracks <= 0) return TRACKFIT_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const size_t row = (size_t)h->s.T * 5;
+  if (n_tracks > h->st_cap) {
+    cudaStreamSynchronize(st);
+    cudaFree(h->st_hits);
+    cudaFree(h->st_n);
+    cudaFree(h->st_out);
+    h->st_hits = nullptr;
+    h->st_n = nullptr;
+    h->st_out = nullptr;
+    h->st_cap = 0;
+    int s1 = tf_status_from_cuda(cudaMalloc(&h->st_hits, n_tracks * row * sizeof(float)));
+    if (s1 == TRACKFIT_OK) s1 = tf_status_from_cuda(cudaMalloc(&h->st_n, ((n_tracks + 3) / 4) * 4 * sizeof(int32_t)));
+    if (s1 == TRACKFIT_OK) s1 = tf_status_from_cuda(cudaMalloc(&h->st_out, n_tracks * 5 * sizeof(float)));
+    if (s1 != TRACKFIT_OK) return s1;
+    h->st_cap = n_tracks;
+  }
+  cudaError_t e = cudaMemcpyAsync(h->st_hits, hits_host, n_tracks * row * sizeof(float), cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h->st_n, n_hits_host, n_tracks * sizeof(int32_t), cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  int r = trackfit_forward(h, h->st_hits, h->st_n, n_tracks, h->st_out, stream);
+  if (r != TRACKFIT_OK) return r;
+  e = cudaMemcpyAsync(out_host, h->st_out, n_tracks * 5 * sizeof(float), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  return tf_status_from_cuda(e);
+}
+
+extern "C" int trackfit_device_errors(trackfit_t h, void* stream, int64_t* n_bad) {
+  if (!h || !n_bad) return TRACKFIT_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  unsigned long long v[4] = {0, 0, 0, 0};
+  cudaError_t e = cudaMemcpyAsync(v, h->d_err, sizeof(v), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->d_err, 0, sizeof(v), st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  *n_bad = (int64_t)v[0];
+  if (v[1] != 0) return TRACKFIT_ERR_TIMEOUT;
+  return v[0] ? TRACKFIT_ERR_BAD_HITS : TRACKFIT_OK;
+}
+
+extern "C" int trackfit_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits,
+                                   int64_t n_tracks, int32_t T, int32_t C, float* h_fwd, float* h_bwd,
+                                   void* stream) {
+  if (!a || !b || !x || !n_hits || !h_fwd || !h_bwd) return TRACKFIT_ERR_INVALID_ARG;
+  if (n_tracks <= 0 || T < 1 || T > TF_MAX_HITS || C < 1) return TRACKFIT_ERR_INVALID_ARG;
+  return tf_simt_debug_scan(a, b, x, n_hits, n_tracks, T, C, h_fwd, h_bwd,
+                            reinterpret_cast<cudaStream_t>(stream));
+}

@@ -1,0 +1,348 @@
+// SIMT (CUDA-core) kernel path: the production path for TRACKFIT_FP32 configs
+// and a second, independent GPU implementation of the BF16_PROJ arithmetic.
+//
+// Layout: the batch is processed in chunks of whole tracks; inside a chunk every
+// per-hit tensor is row-major [tracks * max_hits][channels] in the handle's
+// workspace.  Padded rows are computed and then excluded by select (their
+// residual rows are forced to 0, the scans and pooling skip them).
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "trackfit_internal.h"
+
+namespace {
+
+enum { EPI_STORE = 0, EPI_SILU = 1, EPI_PROJ = 2, EPI_GATE_RES = 3, EPI_RES_MASK = 4, EPI_MASK = 5 };
+
+__device__ __forceinline__ float sigm(float x) { return 1.0f / (1.0f + expf(-x)); }
+__device__ __forceinline__ float silu(float x) { return x * sigm(x); }
+__device__ __forceinline__ float bf16r(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+__device__ __forceinline__ bool row_valid(int r, int T, const int32_t* n_hits) {
+  int b = r / T, t = r - b * T;
+  int n = n_hits[b];
+  return n >= 1 && n <= T && t < n;
+}
+
+struct GemmArgs {
+  const float* A; int lda;      // [R][lda], first K columns used
+  const float* W;               // [N][K] row-major (PyTorch [out][in])
+  const float* bias;            // [N]
+  float* C; int ldc;            // [R][ldc]
+  int R, N, K;
+  int bf16;                     // round both operands to bf16 on load
+  int epi;
+  const float* res; int ldr;    // residual input (GATE_RES, RES_MASK)
+  const float* gate; int ldg;   // sigmoid gate values (GATE_RES)
+  int H;                        // hidden width (PROJ: which columns are gates)
+  const int32_t* n_hits; int T; // padding mask (MASK, RES_MASK)
+};
+
+constexpr int BM = 64, BN = 64, BK = 16;
+
+// C = epilogue(A W^T + bias); 256 threads, 4x4 outputs per thread.
+__global__ void __launch_bounds__(256) gemm_kernel(GemmArgs g) {
+  __shared__ float As[BK][BM + 4];
+  __shared__ float Ws[BK][BN + 4];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int row0 = blockIdx.y * BM, col0 = blockIdx.x * BN;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < g.K; k0 += BK) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      int idx = tid + i * 256, m = idx >> 4, k = idx & 15;
+      int r = row0 + m, kk = k0 + k;
+      float a = (r < g.R && kk < g.K) ? g.A[(size_t)r * g.lda + kk] : 0.0f;
+      int n = col0 + m;
+      float w = (n < g.N && kk < g.K) ? g.W[(size_t)n * g.K + kk] : 0.0f;
+      if (g.bf16) { a = bf16r(a); w = bf16r(w); }
+      As[k][m] = a;
+      Ws[k][m] = w;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < BK; ++k) {
+      float a[4], w[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) { a[i] = As[k][ty * 4 + i]; w[i] = Ws[k][tx * 4 + i]; }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], w[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    int r = row0 + ty * 4 + i;
+    if (r >= g.R) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      int n = col0 + tx * 4 + j;
+      if (n >= g.N) continue;
+      float v = acc[i][j] + g.bias[n];
+      switch (g.epi) {
+        case EPI_SILU: v = silu(v); break;
+        case EPI_PROJ: {
+          bool is_gate = (n < g.H) || (n >= 2 * g.H && n < 3 * g.H) || (n >= 4 * g.H);
+          if (is_gate) v = sigm(v);
+        } break;
+        case EPI_GATE_RES: v = g.res[(size_t)r * g.ldr + n] + v * g.gate[(size_t)r * g.ldg + n]; break;
+        case EPI_RES_MASK:
+          v = row_valid(r, g.T, g.n_hits) ? g.res[(size_t)r * g.ldr + n] + v : 0.0f;
+          break;
+        case EPI_MASK: v = row_valid(r, g.T, g.n_hits) ? v : 0.0f; break;
+        default: break;
+      }
+      g.C[(size_t)r * g.ldc + n] = v;
+    }
+  }
+}
+
+// Fourier features (Sec. 3.2): one thread per (hit row, feature).  The argument
+// s_k * u is formed in fp64 and reduced modulo 2 before the fp32 sinpi/cospi, so
+// the fp32 result carries no argument error from the up-to-32x scale.
+__global__ void fourier_kernel(const float* __restrict__ hits, int64_t rows, float* __restrict__ e,
+                               tf_shape s) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= rows * s.F) return;
+  int64_t r = i / s.F;
+  int f = (int)(i - r * s.F);
+  double u = ((double)hits[r * s.F + f] - s.feat_min_d[f]) / s.feat_range_d[f];
+  float* o = e + r * s.E + f * 2 * s.K;
+  for (int k = 0; k < s.K; ++k) {
+    double a = u * (double)s.scale[k];
+    a -= 2.0 * rint(0.5 * a);
+    float af = (float)a;
+    o[k] = sinpif(af);
+    o[s.K + k] = cospif(af);
+  }
+}
+
+// x_hat = x / sqrt(mean(x^2) + eps) * g, one warp per row.
+__global__ void rmsnorm_kernel(const float* __restrict__ x, int64_t rows, int D, const float* __restrict__ gain,
+                               float eps, float* __restrict__ y) {
+  int64_t r = blockIdx.x * (int64_t)(blockDim.x / 32) + threadIdx.x / 32;
+  int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const float* xr = x + r * D;
+  float ss = 0.0f;
+  for (int c = lane; c < D; c += 32) ss = fmaf(xr[c], xr[c], ss);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  float inv = 1.0f / sqrtf(ss / (float)D + eps);
+  for (int c = lane; c < D; c += 32) y[r * D + c] = xr[c] * inv * gain[c];
+}
+
+// Bidirectional minGRU scans of one layer (Sec. 3.2, Eq. 2): one thread per
+// (track, channel); z already passed through the sigmoid by the projection.
+__global__ void mingru_scan_kernel(const float* __restrict__ pr, int ldp, const int32_t* __restrict__ n_hits,
+                                   int64_t B, int T, int H, float* __restrict__ y) {
+  int c = blockIdx.x * blockDim.x + threadIdx.x;
+  int64_t b = blockIdx.y;
+  if (c >= H || b >= B) return;
+  int n = n_hits[b];
+  if (n < 1 || n > T) n = 0;
+  const float* p = pr + b * T * (int64_t)ldp;
+  float* yo = y + b * T * (int64_t)(2 * H);
+  float h = 0.0f;
+  for (int t = 0; t < T; ++t) {
+    if (t < n) {
+      float z = p[t * ldp + c], cand = p[t * ldp + H + c];
+      h = fmaf(z, cand - h, h);
+      yo[t * 2 * H + c] = h;
+    } else {
+      yo[t * 2 * H + c] = 0.0f;
+    }
+  }
+  h = 0.0f;
+  for (int t = T - 1; t >= 0; --t) {
+    if (t < n) {
+      float z = p[t * ldp + 2 * H + c], cand = p[t * ldp + 3 * H + c];
+      h = fmaf(z, cand - h, h);
+      yo[t * 2 * H + H + c] = h;
+    } else {
+      yo[t * 2 * H + H + c] = 0.0f;
+    }
+  }
+}
+
+// Generic masked linear recurrence h_t = a_t h_{t-1} + b_t x_t, both directions.
+__global__ void linear_scan_kernel(const float* __restrict__ a, const float* __restrict__ bb,
+                                   const float* __restrict__ x, const int32_t* __restrict__ n_hits, int64_t B,
+                                   int T, int C, float* __restrict__ hf, float* __restrict__ hb) {
+  int c = blockIdx.x * blockDim.x + threadIdx.x;
+  int64_t b = blockIdx.y;
+  if (c >= C || b >= B) return;
+  int n = n_hits[b];
+  if (n < 0) n = 0;
+  if (n > T) n = T;
+  int64_t base = b * T * (int64_t)C + c;
+  float h = 0.0f;
+  for (int t = 0; t < T; ++t) {
+    int64_t i = base + (int64_t)t * C;
+    if (t < n) { h = fmaf(a[i], h, bb[i] * x[i]); hf[i] = h; } else { hf[i] = 0.0f; }
+  }
+  h = 0.0f;
+  for (int t = T - 1; t >= 0; --t) {
+    int64_t i = base + (int64_t)t * C;
+    if (t < n) { h = fmaf(a[i], h, bb[i] * x[i]); hb[i] = h; } else { hb[i] = 0.0f; }
+  }
+}
+
+// Pooling and head (Sec. 3.2-3.3): one 128-thread block per track.
+__global__ void __launch_bounds__(128) pool_head_kernel(const float* __restrict__ x, const float* __restrict__ y,
+                                                        const int32_t* __restrict__ n_hits, int64_t B, tf_shape s,
+                                                        const float* __restrict__ gh, const float* __restrict__ w1,
+                                                        const float* __restrict__ b1, const float* __restrict__ w2,
+                                                        const float* __restrict__ b2, float* __restrict__ out,
+                                                        float* __restrict__ out_q, float* __restrict__ out_pool,
+                                                        unsigned long long* err) {
+  __shared__ float pv[2 * 384];
+  __shared__ float hid[256];
+  __shared__ float red[4];
+  __shared__ float qv[5 * 15];
+  const int64_t b = blockIdx.x;
+  const int tid = threadIdx.x;
+  const int T = s.T, D = s.D, H = s.H, P = s.P;
+  int n = n_hits[b];
+  const bool bad = n < 1 || n > T;
+  if (bad) {
+    if (tid == 0) atomicAdd(err, 1ull);
+    n = 1;
+  }
+  if (s.pool == TRACKFIT_POOL_MEAN) {
+    for (int c = tid; c < D; c += blockDim.x) {
+      float acc = 0.0f;
+      for (int t = 0; t < n; ++t) acc += x[(b * T + t) * D + c];
+      pv[c] = acc / (float)n;
+    }
+  } else {
+    for (int c = tid; c < H; c += blockDim.x) {
+      pv[c] = y[(b * T + (n - 1)) * 2 * H + c];
+      pv[H + c] = y[(b * T) * 2 * H + H + c];
+    }
+  }
+  __syncthreads();
+  float ss = 0.0f;
+  for (int c = tid; c < P; c += blockDim.x) ss = fmaf(pv[c], pv[c], ss);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((tid & 31) == 0) red[tid >> 5] = ss;
+  __syncthreads();
+  float tot = 0.0f;
+  for (int i = 0; i < (int)(blockDim.x >> 5); ++i) tot += red[i];
+  const float inv = 1.0f / sqrtf(tot / (float)P + s.rms_eps);
+  if (out_pool)
+    for (int c = tid; c < P; c += blockDim.x) out_pool[b * P + c] = bad ? NAN : pv[c];
+  __syncthreads();
+  for (int c = tid; c < P; c += blockDim.x) pv[c] = pv[c] * inv * gh[c];
+  __syncthreads();
+  for (int j = tid; j < s.Hh; j += blockDim.x) {
+    float acc = b1[j];
+    const float* wr = w1 + (size_t)j * P;
+    for (int c = 0; c < P; ++c) acc = fmaf(wr[c], pv[c], acc);
+    hid[j] = silu(acc);
+  }
+  __syncthreads();
+  for (int o = tid; o < s.Q; o += blockDim.x) {
+    float acc = b2[o];
+    const float* wr = w2 + (size_t)o * s.Hh;
+    for (int j = 0; j < s.Hh; ++j) acc = fmaf(wr[j], hid[j], acc);
+    qv[o] = bad ? NAN : acc;
+    if (out_q) out_q[b * s.Q + o] = qv[o];
+  }
+  __syncthreads();
+  if (tid < 5) out[b * 5 + tid] = qv[tid * s.NQ + s.NQ / 2];
+}
+
+size_t ws_floats_per_track(const tf_shape& s) { return (size_t)s.T * (s.E + 14 * (size_t)s.D); }
+
+int launch_gemm(const GemmArgs& g, cudaStream_t st) {
+  dim3 grid((g.N + BN - 1) / BN, (g.R + BM - 1) / BM);
+  gemm_kernel<<<grid, 256, 0, st>>>(g);
+  return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
+}
+
+}  // namespace
+
+int tf_simt_workspace(trackfit_ctx* h) {
+  const size_t budget = (size_t)1 << 30;
+  size_t per = ws_floats_per_track(h->s) * sizeof(float);
+  int64_t n = (int64_t)(budget / per);
+  if (n < 1) n = 1;
+  if (n > 65535) n = 65535;                       // grid.y limit of the scan launch
+  if (n * h->s.T > 65535LL * 64) n = 65535LL * 64 / h->s.T;   // grid.y limit of the GEMM
+  h->ws_tracks = n;
+  h->ws_bytes = per * (size_t)n;
+  return tf_status_from_cuda(cudaMalloc(&h->ws, h->ws_bytes));
+}
+
+int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out,
+                    float* out_q, float* out_pool, cudaStream_t st) {
+  const tf_shape& s = h->s;
+  const float* W = h->d_w;
+  const tf_blob_off& o = h->off;
+  const int bf = s.precision == TRACKFIT_BF16_PROJ;
+  const int D = s.D, H = s.H, PD = 4 * s.H + s.D;
+  for (int64_t c0 = 0; c0 < B; c0 += h->ws_tracks) {
+    const int64_t nb = (B - c0 < h->ws_tracks) ? B - c0 : h->ws_tracks;
+    const int64_t R = nb * s.T;
+    float* EB = h->ws;
+    float* U = EB + R * s.E;
+    float* X = U + R * D;
+    float* XH = X + R * D;
+    float* PR = XH + R * D;
+    float* Y = PR + R * PD;
+    float* X1 = Y + R * 2 * H;
+    const float* hc = hits + c0 * s.T * 5;
+    const int32_t* nc = n_hits + c0;
+    int64_t nthreads = R * s.F;
+    fourier_kernel<<<(unsigned)((nthreads + 255) / 256), 256, 0, st>>>(hc, R, EB, s);
+    GemmArgs g{};
+    g.R = (int)R;
+    g.bf16 = bf;
+    g.n_hits = nc;
+    g.T = s.T;
+    g.H = H;
+    // embedding: U = SiLU(W_e1 e + b_e1); X = mask(W_e2 U + b_e2)
+    g.A = EB; g.lda = s.E; g.W = W + o.emb_w1; g.bias = W + o.emb_b1; g.C = U; g.ldc = D;
+    g.N = D; g.K = s.E; g.epi = EPI_SILU;
+    if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+    g.A = U; g.lda = D; g.W = W + o.emb_w2; g.bias = W + o.emb_b2; g.C = X; g.ldc = D;
+    g.N = D; g.K = D; g.epi = EPI_MASK;
+    if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+    for (int l = 0; l < s.L; ++l) {
+      const tf_layer_off& lo = o.layer[l];
+      rmsnorm_kernel<<<(unsigned)((R + 7) / 8), 256, 0, st>>>(X, R, D, W + lo.g, s.rms_eps, XH);
+      g.A = XH; g.lda = D; g.W = W + lo.w_in; g.bias = W + lo.b_in; g.C = PR; g.ldc = PD;
+      g.N = PD; g.K = D; g.epi = EPI_PROJ;
+      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+      dim3 sg((H + 127) / 128, (unsigned)nb);
+      mingru_scan_kernel<<<sg, 128, 0, st>>>(PR, PD, nc, nb, s.T, H, Y);
+      if (s.pool == TRACKFIT_POOL_ENDPOINTS && l == s.L - 1) break;
+      g.A = Y; g.lda = 2 * H; g.W = W + lo.w_m; g.bias = W + lo.b_m; g.C = X1; g.ldc = D;
+      g.N = D; g.K = 2 * H; g.epi = EPI_GATE_RES; g.res = X; g.ldr = D; g.gate = PR + 4 * H; g.ldg = PD;
+      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+      g.A = X1; g.lda = D; g.W = W + lo.w1; g.bias = W + lo.b1; g.C = U; g.ldc = D;
+      g.N = D; g.K = D; g.epi = EPI_SILU;
+      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+      g.A = U; g.lda = D; g.W = W + lo.w2; g.bias = W + lo.b2; g.C = X; g.ldc = D;
+      g.N = D; g.K = D; g.epi = EPI_RES_MASK; g.res = X1; g.ldr = D;
+      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+    }
+    pool_head_kernel<<<(unsigned)nb, 128, 0, st>>>(X, Y, nc, nb, s, W + o.head_g, W + o.head_w1, W + o.head_b1,
+                                                    W + o.head_w2, W + o.head_b2, out + c0 * 5,
+                                                    out_q ? out_q + c0 * s.Q : nullptr,
+                                                    out_pool ? out_pool + c0 * s.P : nullptr, h->d_err);
+    if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  }
+  return TRACKFIT_OK;
+}
+
+int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits, int64_t B, int T,
+                       int C, float* hf, float* hb, cudaStream_t st) {
+  dim3 grid((C + 127) / 128, (unsigned)B);
+  linear_scan_kernel<<<grid, 128, 0, st>>>(a, b, x, n_hits, B, T, C, hf, hb);
+  return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
+}

@@ -1,0 +1,71 @@
+// Internal declarations shared by the host API and the kernel translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "trackfit.h"
+
+#define TF_MAX_LAYERS 16
+#define TF_MAX_HITS 64
+
+// Offsets (in floats) of every tensor inside the fp32 weight blob.
+struct tf_layer_off {
+  size_t g, w_in, b_in, w_m, b_m, w1, b1, w2, b2;
+};
+struct tf_blob_off {
+  size_t emb_w1, emb_b1, emb_w2, emb_b2;
+  tf_layer_off layer[TF_MAX_LAYERS];
+  size_t head_g, head_w1, head_b1, head_w2, head_b2;
+  size_t total;
+};
+
+// Shape summary derived from the public config.
+struct tf_shape {
+  int T, F, K, E, D, H, L, P, Hh, NQ, Q, precision, pool;
+  float rms_eps;
+  float feat_min[TRACKFIT_MAX_FEATURES], feat_inv_range[TRACKFIT_MAX_FEATURES];
+  double feat_min_d[TRACKFIT_MAX_FEATURES], feat_range_d[TRACKFIT_MAX_FEATURES];
+  float scale[TRACKFIT_MAX_FOURIER];
+};
+
+struct tf_tc_state;  // tcgen05 path (tc_forward.cu)
+
+enum { TF_PATH_SIMT = 0, TF_PATH_TC = 1 };
+
+struct trackfit_ctx {
+  trackfit_config_t cfg;
+  tf_shape s;
+  tf_blob_off off;
+  int path;
+  float* d_w;                    // fp32 weight blob on the device
+  unsigned long long* d_err;     // [0] tracks with bad n_hits, [1] expired bounded waits
+  // SIMT workspace (one chunk of tracks at a time)
+  float* ws;
+  size_t ws_bytes;
+  int64_t ws_tracks;
+  // host-buffer staging
+  float* st_hits;
+  int32_t* st_n;
+  float* st_out;
+  int64_t st_cap;
+  tf_tc_state* tc;
+};
+
+// simt.cu
+int tf_simt_workspace(trackfit_ctx* h);
+int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,
+                    float* out, float* out_q, float* out_pool, cudaStream_t st);
+int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits,
+                       int64_t B, int T, int C, float* hf, float* hb, cudaStream_t st);
+
+// tc_forward.cu
+bool tf_tc_supported(const tf_shape& s);
+int tf_tc_create(trackfit_ctx* h, const float* host_w);
+void tf_tc_destroy(trackfit_ctx* h);
+int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,
+                  float* out, float* out_q, float* out_pool, cudaStream_t st);
+
+// api.cu
+int tf_status_from_cuda(cudaError_t e);

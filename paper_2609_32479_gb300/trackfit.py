@@ -1,0 +1,208 @@
+"""Thin ctypes binding of the C-ABI in include/trackfit.h.
+
+Argument marshalling only: every step of the encoder runs in the CUDA kernels of
+libtrackfit.so.  There is no CPU fallback; if the library is missing, load()
+raises.  Device buffers are torch CUDA tensors (torch supplies memory and
+streams), host buffers are numpy arrays."""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import numpy as np
+
+from . import workloads as W
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_lib", "libtrackfit.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_BAD_HITS, ERR_TIMEOUT = range(7)
+ABI_VERSION = 1
+
+# every function declared in include/trackfit.h
+EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trackfit_forward_ex",
+           "trackfit_forward_host", "trackfit_device_errors", "trackfit_path_name", "trackfit_set_path",
+           "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan")
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("abi_version", ctypes.c_int32), ("max_hits", ctypes.c_int32),
+                ("n_features", ctypes.c_int32), ("n_fourier", ctypes.c_int32),
+                ("d_model", ctypes.c_int32), ("d_hidden", ctypes.c_int32), ("n_layers", ctypes.c_int32),
+                ("head_hidden", ctypes.c_int32), ("n_quantiles", ctypes.c_int32),
+                ("precision", ctypes.c_int32), ("pool", ctypes.c_int32),
+                ("feat_min", ctypes.c_float * 5), ("feat_max", ctypes.c_float * 5),
+                ("fourier_scale", ctypes.c_float * 16), ("rms_eps", ctypes.c_float)]
+
+
+class TrackfitError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {strerror(status)} (status {status})")
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def load() -> ctypes.CDLL:
+    """Open libtrackfit.so (built by paper_2609_32479_gb300.build); raise if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; "
+                           f"g.build()'` (there is no CPU fallback)")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    lib.trackfit_weight_count.argtypes = [ctypes.POINTER(Config)]
+    lib.trackfit_weight_count.restype = ctypes.c_size_t
+    lib.trackfit_create.argtypes = [ctypes.POINTER(Config), vp, ctypes.c_size_t, ctypes.POINTER(vp)]
+    lib.trackfit_create.restype = ctypes.c_int
+    lib.trackfit_forward.argtypes = [vp, vp, vp, i64, vp, vp]
+    lib.trackfit_forward.restype = ctypes.c_int
+    lib.trackfit_forward_ex.argtypes = [vp, vp, vp, i64, vp, vp, vp, vp]
+    lib.trackfit_forward_ex.restype = ctypes.c_int
+    lib.trackfit_forward_host.argtypes = [vp, vp, vp, i64, vp, vp]
+    lib.trackfit_forward_host.restype = ctypes.c_int
+    lib.trackfit_device_errors.argtypes = [vp, vp, ctypes.POINTER(i64)]
+    lib.trackfit_device_errors.restype = ctypes.c_int
+    lib.trackfit_path_name.argtypes = [vp]
+    lib.trackfit_path_name.restype = ctypes.c_char_p
+    lib.trackfit_set_path.argtypes = [vp, ctypes.c_int]
+    lib.trackfit_set_path.restype = ctypes.c_int
+    lib.trackfit_destroy.argtypes = [vp]
+    lib.trackfit_destroy.restype = None
+    lib.trackfit_strerror.argtypes = [ctypes.c_int]
+    lib.trackfit_strerror.restype = ctypes.c_char_p
+    lib.trackfit_debug_scan.argtypes = [vp, vp, vp, vp, i64, i32, i32, vp, vp, vp]
+    lib.trackfit_debug_scan.restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def strerror(status: int) -> str:
+    return load().trackfit_strerror(int(status)).decode()
+
+
+def make_config(m: W.ModelConfig) -> Config:
+    c = Config()
+    c.abi_version = ABI_VERSION
+    c.max_hits, c.n_features, c.n_fourier = m.max_hits, m.n_features, m.n_fourier
+    c.d_model, c.d_hidden, c.n_layers = m.d_model, m.d_hidden, m.n_layers
+    c.head_hidden, c.n_quantiles = m.head_hidden, m.n_quantiles
+    c.precision, c.pool = m.precision, m.pool
+    for i in range(5):
+        c.feat_min[i], c.feat_max[i] = m.feat_min[i], m.feat_max[i]
+    for i in range(16):
+        c.fourier_scale[i] = m.fourier_scale[i]
+    c.rms_eps = m.rms_eps
+    return c
+
+
+def weight_count(m: W.ModelConfig) -> int:
+    c = make_config(m)
+    return int(load().trackfit_weight_count(ctypes.byref(c)))
+
+
+def _stream_handle(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+def _dev(t, dtype_name: str):
+    if t is None:
+        return None
+    if not (t.is_cuda and t.is_contiguous() and str(t.dtype) == dtype_name):
+        raise ValueError(f"expected a contiguous CUDA {dtype_name} tensor, got {t.dtype} on {t.device}")
+    return t.data_ptr()
+
+
+class Trackfit:
+    """A library handle: trackfit_create on construction, trackfit_destroy on close()."""
+
+    def __init__(self, model: W.ModelConfig, weights: np.ndarray):
+        self.lib = load()
+        self.model = model
+        self._cfg = make_config(model)
+        w = np.ascontiguousarray(weights, dtype=np.float32)
+        h = ctypes.c_void_p()
+        st = self.lib.trackfit_create(ctypes.byref(self._cfg), w.ctypes.data, w.size, ctypes.byref(h))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_create")
+        self._h = h
+
+    @property
+    def handle(self) -> int:
+        return self._h.value
+
+    @property
+    def path(self) -> str:
+        return self.lib.trackfit_path_name(self._h).decode()
+
+    def set_path(self, path: int) -> None:
+        st = self.lib.trackfit_set_path(self._h, int(path))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_set_path")
+
+    def forward(self, hits, n_hits, out, stream=None, quantiles=None, pooled=None) -> None:
+        """Device tensors: hits [B, T, 5] f32, n_hits [B] i32, out [B, 5] f32."""
+        B = int(n_hits.shape[0])
+        args = (self._h, _dev(hits, "torch.float32"), _dev(n_hits, "torch.int32"), B, _dev(out, "torch.float32"))
+        if quantiles is None and pooled is None:
+            st = self.lib.trackfit_forward(*args, _stream_handle(stream))
+        else:
+            st = self.lib.trackfit_forward_ex(*args, _dev(quantiles, "torch.float32"),
+                                              _dev(pooled, "torch.float32"), _stream_handle(stream))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_forward")
+
+    def forward_host(self, hits: np.ndarray, n_hits: np.ndarray, out: np.ndarray, stream=None) -> None:
+        """Host arrays (ideally pinned): copies in, runs, copies out, synchronises."""
+        for a, dt in ((hits, np.float32), (n_hits, np.int32), (out, np.float32)):
+            if a.dtype != dt or not a.flags["C_CONTIGUOUS"]:
+                raise ValueError("host buffers must be C-contiguous float32/int32/float32")
+        st = self.lib.trackfit_forward_host(self._h, hits.ctypes.data, n_hits.ctypes.data, int(n_hits.shape[0]),
+                                            out.ctypes.data, _stream_handle(stream))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_forward_host")
+
+    def forward_host_ptr(self, hits_ptr: int, n_ptr: int, B: int, out_ptr: int, stream=None) -> None:
+        st = self.lib.trackfit_forward_host(self._h, hits_ptr, n_ptr, int(B), out_ptr, _stream_handle(stream))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_forward_host")
+
+    def device_errors(self, stream=None):
+        """(status, n_bad): reads and resets the device error counters (synchronises)."""
+        n = ctypes.c_int64(0)
+        st = self.lib.trackfit_device_errors(self._h, _stream_handle(stream), ctypes.byref(n))
+        return st, int(n.value)
+
+    def close(self) -> None:
+        if getattr(self, "_h", None) is not None and self._h.value:
+            self.lib.trackfit_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *a):
+        self.close()
+
+
+def debug_scan(a, b, x, n_hits, h_fwd, h_bwd, stream=None) -> None:
+    """Device test hook for the masked linear recurrence (both directions)."""
+    B, T, C = a.shape
+    st = load().trackfit_debug_scan(_dev(a, "torch.float32"), _dev(b, "torch.float32"), _dev(x, "torch.float32"),
+                                    _dev(n_hits, "torch.int32"), B, T, C, _dev(h_fwd, "torch.float32"),
+                                    _dev(h_bwd, "torch.float32"), _stream_handle(stream))
+    if st != OK:
+        raise TrackfitError(st, "trackfit_debug_scan")

@@ -1,0 +1,220 @@
+"""GPU parity: the CUDA path through the C-ABI against the CPU oracle on the same
+seeded inputs, plus bit-exact checks of masking, indexing and determinism."""
+import dataclasses
+
+import numpy as np
+import pytest
+
+from oracle import trackfit_oracle as O
+from paper_2609_32479_gb300 import workloads as W
+from tests.helpers import BF16_TOL, FP32_TOL, parity_error
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="session")
+def T():
+    from paper_2609_32479_gb300 import trackfit
+    import os
+    if not os.path.exists(trackfit.LIB_PATH):
+        import __graft_entry__
+        __graft_entry__.build()
+    trackfit.load()
+    return trackfit
+
+
+def dev():
+    return torch.device("cuda:0")
+
+
+def tol_of(model):
+    return FP32_TOL if model.precision == W.PRECISION_FP32 else BF16_TOL
+
+
+def run(T, model, blob, hits, n_hits, path=0, extras=False):
+    with T.Trackfit(model, blob) as tf:
+        if path:
+            tf.set_path(path)
+        h = torch.from_numpy(np.ascontiguousarray(hits)).to(dev())
+        n = torch.from_numpy(np.ascontiguousarray(n_hits)).to(dev())
+        out = torch.full((n.shape[0], 5), -7.0, dtype=torch.float32, device=dev())
+        q = p = None
+        if extras:
+            q = torch.empty((n.shape[0], 5, model.n_quantiles), dtype=torch.float32, device=dev())
+            p = torch.empty((n.shape[0], model.pooled_dim), dtype=torch.float32, device=dev())
+        tf.forward(h, n, out, quantiles=q, pooled=p)
+        torch.cuda.synchronize()
+        st, nbad = tf.device_errors()
+        res = dict(out=out.cpu().numpy(), status=st, n_bad=nbad, path=tf.path)
+        if extras:
+            res.update(q=q.cpu().numpy(), pooled=p.cpu().numpy())
+        return res
+
+
+def oracle(model, blob, hits, n_hits, capture=None):
+    return O.forward(dataclasses.asdict(model), blob, hits, n_hits, capture=capture)
+
+
+CASES = [("tiny", None), ("small", None), ("medium", 1000), ("large", 300), ("sweep8", 515), ("sweep16", 300),
+         ("sweep32", 200), ("sweep64", 130)]
+
+
+@pytest.mark.parametrize("path", [0, 1], ids=["auto", "simt"])
+@pytest.mark.parametrize("name,n", CASES)
+def test_parity_against_oracle(T, name, n, path):
+    w = W.workload(name, n_tracks=n)
+    if path == 1 and w.model.precision == W.PRECISION_FP32:
+        pytest.skip("fp32 configs run the SIMT path under auto already")
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    r = run(T, w.model, blob, tb.hits, tb.n_hits, path=path)
+    ref = oracle(w.model, blob, tb.hits, tb.n_hits)
+    err = parity_error(r["out"], ref)
+    print(f"{name} [{r['path']}] parity error per parameter: {err}")
+    assert r["status"] == 0 and r["n_bad"] == 0
+    assert np.all(np.isfinite(r["out"]))
+    assert np.all(err <= tol_of(w.model)), err
+
+
+@pytest.mark.parametrize("name", ["medium", "large"])
+def test_full_size_sampled_parity(T, name):
+    """Full batch in the bench's launch configuration; the oracle recomputes a
+    sample of tracks covering every hit count."""
+    w = W.workload(name)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    r = run(T, w.model, blob, tb.hits, tb.n_hits)
+    rng = np.random.default_rng(3)
+    idx = []
+    for k in np.unique(tb.n_hits):
+        cand = np.nonzero(tb.n_hits == k)[0]
+        idx += list(rng.choice(cand, size=min(12, cand.size), replace=False))
+    idx += [0, w.n_tracks - 1]
+    idx = np.array(sorted(set(int(i) for i in idx)))
+    ref = oracle(w.model, blob, tb.hits[idx], tb.n_hits[idx])
+    err = parity_error(r["out"][idx], ref)
+    print(f"{name} full batch [{r['path']}], {idx.size} sampled tracks: {err}")
+    assert np.all(np.isfinite(r["out"]))
+    assert np.all(err <= tol_of(w.model)), err
+
+
+@pytest.mark.parametrize("name", ["tiny", "medium"])
+def test_endpoint_pooling_parity(T, name):
+    w = W.workload(name, n_tracks=300, pool=W.POOL_ENDPOINTS)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, 5)
+    r = run(T, w.model, blob, tb.hits, tb.n_hits)
+    err = parity_error(r["out"], oracle(w.model, blob, tb.hits, tb.n_hits))
+    assert np.all(err <= tol_of(w.model)), err
+
+
+@pytest.mark.parametrize("name", ["small", "medium"])
+def test_quantile_and_pooled_exports(T, name):
+    w = W.workload(name, n_tracks=200)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    r = run(T, w.model, blob, tb.hits, tb.n_hits, extras=True)
+    np.testing.assert_array_equal(r["out"], r["q"][:, :, w.model.n_quantiles // 2])
+    cap = {}
+    oracle(w.model, blob, tb.hits, tb.n_hits, capture=cap)
+    assert np.all(parity_error(r["pooled"], cap["pooled"]) <= tol_of(w.model))
+    assert np.all(parity_error(r["q"].reshape(200, -1), cap["quantiles"].reshape(200, -1)) <= tol_of(w.model))
+
+
+@pytest.mark.parametrize("name", ["small", "medium", "large"])
+def test_masking_and_indexing_bit_exact(T, name):
+    """NaN-filled pads, track permutation, batch split and repeated runs give
+    bit-identical outputs."""
+    w = W.workload(name, n_tracks=777)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    base = run(T, w.model, blob, tb.hits, tb.n_hits)["out"]
+    again = run(T, w.model, blob, tb.hits, tb.n_hits)["out"]
+    np.testing.assert_array_equal(base, again)
+    nanpad = tb.hits.copy()
+    Tm = w.model.max_hits
+    nanpad[np.arange(Tm)[None, :] >= tb.n_hits[:, None]] = np.nan
+    np.testing.assert_array_equal(run(T, w.model, blob, nanpad, tb.n_hits)["out"], base)
+    perm = np.random.default_rng(0).permutation(777)
+    np.testing.assert_array_equal(run(T, w.model, blob, tb.hits[perm], tb.n_hits[perm])["out"], base[perm])
+    parts = [run(T, w.model, blob, tb.hits[a:b], tb.n_hits[a:b])["out"] for a, b in ((0, 1), (1, 300), (300, 777))]
+    np.testing.assert_array_equal(np.concatenate(parts), base)
+
+
+@pytest.mark.parametrize("name", ["tiny", "medium"])
+def test_bad_hit_counts(T, name):
+    w = W.workload(name, n_tracks=64)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    base = run(T, w.model, blob, tb.hits, tb.n_hits)["out"]
+    n = tb.n_hits.copy()
+    n[3], n[10], n[63] = 0, w.model.max_hits + 1, -5
+    r = run(T, w.model, blob, tb.hits, n)
+    assert r["n_bad"] == 3 and r["status"] == 5
+    assert np.all(np.isnan(r["out"][[3, 10, 63]]))
+    keep = np.setdiff1d(np.arange(64), [3, 10, 63])
+    np.testing.assert_array_equal(r["out"][keep], base[keep])
+
+
+def test_host_buffer_entry_point_matches_device(T):
+    w = W.workload("medium", n_tracks=3000)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    base = run(T, w.model, blob, tb.hits, tb.n_hits)["out"]
+    with T.Trackfit(w.model, blob) as tf:
+        hits = torch.from_numpy(tb.hits).pin_memory()
+        n = torch.from_numpy(tb.n_hits).pin_memory()
+        out = torch.empty((3000, 5), dtype=torch.float32).pin_memory()
+        tf.forward_host_ptr(hits.data_ptr(), n.data_ptr(), 3000, out.data_ptr())
+        np.testing.assert_array_equal(out.numpy(), base)
+        o2 = np.zeros((3000, 5), np.float32)
+        tf.forward_host(tb.hits, tb.n_hits, o2)      # pageable memory works too
+        np.testing.assert_array_equal(o2, base)
+
+
+def test_abi_argument_errors_launch_nothing(T):
+    w = W.workload("tiny", n_tracks=8)
+    blob = W.gen_weights(w.model, 1)
+    with T.Trackfit(w.model, blob) as tf:
+        lib = tf.lib
+        hits = torch.zeros((8, w.model.max_hits, 5), device=dev())
+        n = torch.full((8,), 3, dtype=torch.int32, device=dev())
+        out = torch.full((8, 5), 1.5, device=dev())
+        s = torch.cuda.current_stream().cuda_stream
+        h = tf.handle
+        assert lib.trackfit_forward(h, hits.data_ptr(), n.data_ptr(), 0, out.data_ptr(), s) == T.ERR_INVALID_ARG
+        assert lib.trackfit_forward(h, hits.data_ptr(), n.data_ptr(), -3, out.data_ptr(), s) == T.ERR_INVALID_ARG
+        assert lib.trackfit_forward(h, None, n.data_ptr(), 8, out.data_ptr(), s) == T.ERR_INVALID_ARG
+        assert lib.trackfit_forward(h, hits.data_ptr() + 4, n.data_ptr(), 8, out.data_ptr(), s) == T.ERR_INVALID_ARG
+        assert lib.trackfit_forward(h, hits.data_ptr(), n.data_ptr(), 8, out.data_ptr() + 8, s) == T.ERR_INVALID_ARG
+        torch.cuda.synchronize()
+        assert torch.all(out == 1.5)
+
+
+def test_debug_scan_closed_forms(T):
+    rng = np.random.default_rng(11)
+    B, Tm, C = 37, 13, 70
+    n = rng.integers(0, Tm + 1, B).astype(np.int32)
+    a = rng.uniform(-1, 1, (B, Tm, C)).astype(np.float32)
+    b = rng.uniform(-1, 1, (B, Tm, C)).astype(np.float32)
+    x = rng.uniform(-2, 2, (B, Tm, C)).astype(np.float32)
+
+    def gpu(a, b, x):
+        ta, tb_, tx = (torch.from_numpy(v).to(dev()) for v in (a, b, x))
+        hf, hb = torch.empty_like(ta), torch.empty_like(ta)
+        T.debug_scan(ta, tb_, tx, torch.from_numpy(n).to(dev()), hf, hb)
+        torch.cuda.synchronize()
+        return hf.cpu().numpy(), hb.cpu().numpy()
+
+    valid = np.arange(Tm)[None, :] < n[:, None]
+    one = np.ones_like(a)
+    hf, hb = gpu(one, one, x)
+    np.testing.assert_allclose(hf, np.cumsum(np.where(valid[..., None], x, 0), axis=1) * valid[..., None],
+                               rtol=1e-5, atol=1e-5)
+    hf, hb = gpu(np.zeros_like(a), b, x)
+    np.testing.assert_array_equal(hf, np.where(valid[..., None], b * x, 0))
+    hf, hb = gpu(a, b, x)
+    np.testing.assert_allclose(hf, O.linear_scan(a, b, x, valid), rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(hb, O.linear_scan(a, b, x, valid, reverse=True), rtol=1e-5, atol=1e-6)
