@@ -166,6 +166,15 @@ int trackfit_debug_scan(const float* a, const float* b, const float* x, const in
                         int64_t n_tracks, int32_t T, int32_t C, float* h_fwd, float* h_bwd,
                         void* stream);
 
+/* Test hook for the tensor-core operand layouts: D = A * B on one 128 x 128
+ * tile through the same TMA, shared-memory descriptor and tensor-memory path as
+ * the fused kernel.  A device bf16 bits [128][K] row-major (K-major), Bkn device
+ * bf16 bits [K][128] row-major, D device fp32 [128][128]; K in {64, 128, 192,
+ * 256}; all 16-byte aligned.  h supplies the device error counter.
+ * Asynchronous on `stream`; requires an sm_100-family GPU. */
+int trackfit_debug_umma(trackfit_t h, const uint16_t* A, const uint16_t* Bkn, int32_t K, float* D,
+                        void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -231,3 +231,10 @@ extern "C" int trackfit_debug_scan(const float* a, const float* b, const float* 
   return tf_simt_debug_scan(a, b, x, n_hits, n_tracks, T, C, h_fwd, h_bwd,
                             reinterpret_cast<cudaStream_t>(stream));
 }
+
+extern "C" int trackfit_debug_umma(trackfit_t h, const uint16_t* A, const uint16_t* Bkn, int32_t K, float* D,
+                                   void* stream) {
+  if (!h || !A || !Bkn || !D) return TRACKFIT_ERR_INVALID_ARG;
+  if (!aligned16(A) || !aligned16(Bkn) || !aligned16(D)) return TRACKFIT_ERR_INVALID_ARG;
+  return tf_tc_probe(h, A, Bkn, K, D, reinterpret_cast<cudaStream_t>(stream));
+}

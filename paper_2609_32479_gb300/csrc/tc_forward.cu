@@ -1,9 +1,1126 @@
-// tcgen05 path placeholder (filled in by the fused kernel).
+// tcgen05 path: one persistent, warp-specialised kernel runs the whole encoder
+// forward (embedding, every minGRU layer, pooling, head) for BF16_PROJ configs.
+//
+// Orientation: every per-hit matrix product is computed transposed,
+//   D[channel][hit] = W[channel][k] * Act[k][hit],
+// with the weights as the M=128 operand (K-major, TMA-staged from L2/HBM with
+// 128-byte swizzle) and the activations of one tile of 128 packed hits as the
+// N=128 operand (MN-major, written by the epilogue warps straight into shared
+// memory).  The fp32 accumulator lives in tensor memory with lane = channel and
+// column = hit, so each epilogue thread owns one channel and walks the hits of
+// its tracks in order: the gated scans of Eq. 2 run in registers without any
+// cross-thread exchange.
+//
+// Tile: 128 hit columns = two 64-column slabs; each slab holds whole tracks
+// (packed greedily, unpadded).  Warp roles (320 threads):
+//   warp 0      TMA producer of weight blocks (one elected thread)
+//   warp 1      tcgen05.mma issuer (one elected thread), TMEM owner
+//   warps 2..9  epilogue: TMEM lane quadrant = warp % 4, column half = (warp-2)/4
+// TMEM (512 columns): R0,R1 = merge / MLP accumulators (d_model rows), R2,R3 =
+// z and n of one scan chunk, then the output-gate projection.
+// The fp32 residual stream of the tile lives in a per-CTA global scratch slab
+// (L2-resident), never in HBM-sized intermediates.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "sm100_ptx.cuh"
 #include "trackfit_internal.h"
 
-bool tf_tc_supported(const tf_shape&) { return false; }
-int tf_tc_create(trackfit_ctx*, const float*) { return TRACKFIT_ERR_UNSUPPORTED; }
-void tf_tc_destroy(trackfit_ctx*) {}
-int tf_tc_forward(trackfit_ctx*, const float*, const int32_t*, int64_t, float*, float*, float*, cudaStream_t) {
-  return TRACKFIT_ERR_UNSUPPORTED;
+using namespace sm100;
+
+namespace {
+
+constexpr int NT = 320;
+constexpr int NE = 256;
+constexpr int TILE = 128;
+constexpr int SLAB = 64;
+constexpr int MAX_TRK_SLAB = 16;
+constexpr int MAX_TRK_TILE = 2 * MAX_TRK_SLAB;
+constexpr int A_STAGE = 128 * 64 * 2;     // one 128-row x 64-k bf16 weight block
+constexpr int EB_BYTES = 160 * 256;       // Fourier operand: 160 k-rows x 128 hits bf16
+constexpr int MISC_BYTES = 8192;
+constexpr int MAX_STAGES = 8;
+constexpr int SEG = 1024;                 // tracks per packing segment
+constexpr int64_t MAXB = 4194304;         // tracks per launch chunk
+constexpr uint64_t WAIT_NS = 2000000000ull;
+constexpr uint64_t DRAIN_NS = 200000000ull;
+constexpr int B_SBO = 2048;               // k-group stride of the MN-major activation operand
+constexpr int B_LBO = 1024;               // 64-hit atom stride
+
+enum { MAP_E1 = 0, MAP_E2, MAP_IN, MAP_M, MAP_1, MAP_2, NMAPS };
+enum { BSEL_XB = 0, BSEL_HB = 1 };
+enum { F_FIRST = 1, F_LAST = 2, F_VALID = 4 };
+
+struct TcParams {
+  CUtensorMap tm[NMAPS];
+  const float* hits;
+  const int32_t* n_hits;
+  float* out;
+  float* out_q;
+  float* out_pool;
+  float* xs;
+  const int32_t* slab_start;
+  const int32_t* n_slabs;
+  const float* b_e1;
+  const float* b_e2;
+  const float* g;
+  const float* b_in;
+  const float* b_m;
+  const float* b_1;
+  const float* b_2;
+  const float* head_g;
+  const float* head_w1t;
+  const float* head_b1;
+  const float* head_w2;
+  const float* head_b2;
+  unsigned long long* err;
+  int T, D, H, L, NDC, ROWS_IN, NQ, Q, nst;
+  uint32_t idesc;
+  int off_xb, off_hb, off_a, off_misc;
+  float rms_eps;
+  float feat_min[5], feat_inv[5], scale[16];
+};
+
+struct Misc {
+  uint64_t full[MAX_STAGES], empty[MAX_STAGES];
+  uint64_t acc_bar, e_bar, drain_bar;
+  uint32_t tmem_base;
+  int abort_flag;
+  int n_slots;
+  int pad_;
+  int slot_track[MAX_TRK_TILE], slot_n[MAX_TRK_TILE], slot_bad[MAX_TRK_TILE];
+  uint8_t col_flags[TILE], col_slot[TILE], col_tpos[TILE], pad2_[128];
+  float part[4][TILE];
+  float rinv[TILE];
+  float hs[TILE][5];
+};
+static_assert(sizeof(Misc) <= MISC_BYTES, "misc region too small");
+
+__device__ __forceinline__ float sigm(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
+__device__ __forceinline__ float silu(float x) { return x * sigm(x); }
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);   // a -> low half (lower column)
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ uint16_t to_bf16(float a) {
+  __nv_bfloat16 v = __float2bfloat16_rn(a);
+  return *reinterpret_cast<uint16_t*>(&v);
+}
+
+// Byte offset, inside an MN-major 128-byte-swizzled operand with 128 columns, of
+// the 16-byte chunk that holds columns [8*n8, 8*n8+8) of k-row k.  Atoms are 8
+// k-rows x 64 columns (1 KB); the two column atoms of a k-group are adjacent.
+__device__ __forceinline__ uint32_t bchunk(int k, int n8) {
+  return (uint32_t)((k >> 3) * B_SBO + (n8 >> 3) * B_LBO + (k & 7) * 128 + (((n8 & 7) ^ (k & 7)) << 4));
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+__device__ __forceinline__ void st_shared_u16(uint32_t addr, uint16_t v) {
+  asm volatile("st.shared.u16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
+}
+
+// Write 32 consecutive columns [n0, n0+32) of k-row k (n0 % 32 == 0) as bf16.
+__device__ __forceinline__ void store_row32(uint32_t buf, int k, int n0, const float (&v)[32]) {
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    st_shared_v4(buf + bchunk(k, (n0 >> 3) + c), pack_bf16(v[8 * c + 0], v[8 * c + 1]),
+                 pack_bf16(v[8 * c + 2], v[8 * c + 3]), pack_bf16(v[8 * c + 4], v[8 * c + 5]),
+                 pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+  }
+}
+
+__device__ __forceinline__ void ebar_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+// Named-barrier vote over the 256 epilogue threads: true iff every thread passes true.
+__device__ __forceinline__ bool ebar_all(bool ok) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, 1, 256, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)ok)
+      : "memory");
+  return r != 0;
+}
+
+// After a butterfly reduce-scatter of v[32] (one value per column per lane),
+// lane L returns the sum over the 32 lanes of column L.
+__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) {
+    const bool upper = (lane & off) != 0;
+#pragma unroll
+    for (int i = 0; i < off; ++i) {
+      const float send = upper ? v[i] : v[i + off];
+      const float keep = upper ? v[i + off] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+    }
+  }
+  return v[0];
+}
+
+// The static sequence of 128x64 weight blocks of one tile, in the order the MMA
+// issuer consumes them.  f(map, row, col, nk, tmem_col, bsel, bk, acc, end):
+// nk MMAs of K=16 read the block, accumulate into TMEM columns tmem_col, with
+// the activation operand bsel starting at k-row bk; acc = accumulate onto the
+// existing accumulator; end = last block of a group (the epilogue runs next).
+template <class F>
+__device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
+  const int MT = p.D >> 7, KD = p.D >> 6;
+  for (int mt = 0; mt < MT; ++mt)
+    for (int kc = 0; kc < 3; ++kc)
+      f(MAP_E1, mt * 128, kc * 64, kc == 2 ? 2 : 4, mt * 128, BSEL_HB, kc * 64, kc > 0, mt == MT - 1 && kc == 2);
+  for (int mt = 0; mt < MT; ++mt)
+    for (int kc = 0; kc < KD; ++kc)
+      f(MAP_E2, mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, mt == MT - 1 && kc == KD - 1);
+  for (int l = 0; l < p.L; ++l) {
+    const int rb = l * p.ROWS_IN;
+    for (int dc = 0; dc <= p.NDC; ++dc) {
+      if (dc > 0) {  // merge of the previous scan chunk: M[D] += W_m[:, chunk] * h
+        for (int mt = 0; mt < MT; ++mt)
+          for (int kc = 0; kc < 2; ++kc)
+            f(MAP_M, l * p.D + mt * 128, (dc - 1) * 128 + kc * 64, 4, mt * 128, BSEL_HB, kc * 64,
+              dc > 1 || kc > 0, false);
+      }
+      if (dc < p.NDC) {  // z and n of scan chunk dc
+        for (int kc = 0; kc < KD; ++kc)
+          f(MAP_IN, rb + dc * 256, kc * 64, 4, 256, BSEL_XB, kc * 64, kc > 0, false);
+        for (int kc = 0; kc < KD; ++kc)
+          f(MAP_IN, rb + dc * 256 + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, kc == KD - 1);
+      }
+    }
+    for (int mt = 0; mt < MT; ++mt)  // output-gate projection
+      for (int kc = 0; kc < KD; ++kc)
+        f(MAP_IN, rb + p.NDC * 256 + mt * 128, kc * 64, 4, 256 + mt * 128, BSEL_XB, kc * 64, kc > 0,
+          mt == MT - 1 && kc == KD - 1);
+    for (int mt = 0; mt < MT; ++mt)
+      for (int kc = 0; kc < KD; ++kc)
+        f(MAP_1, l * p.D + mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, mt == MT - 1 && kc == KD - 1);
+    for (int mt = 0; mt < MT; ++mt)
+      for (int kc = 0; kc < KD; ++kc)
+        f(MAP_2, l * p.D + mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, mt == MT - 1 && kc == KD - 1);
+  }
+}
+
+__device__ __forceinline__ void set_abort(Misc* m, unsigned long long* err) {
+  if (atomicExch(&m->abort_flag, 1) == 0) atomicAdd(err + 1, 1ull);
+}
+
+// ------------------------------------------------------------------ epilogue
+struct ECtx {
+  const TcParams* p;
+  Misc* m;
+  uint32_t xb, hb, tq;
+  float* xs;
+  float* pooled;
+  float* hid;
+  int q, lane, half, c, col0, te, e, MT;
+};
+
+// silu(acc + bias) -> XB rows [mt*128 + c]
+__device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
+  for (int mt = 0; mt < x.MT; ++mt) {
+    const float b = bias[mt * 128 + x.c];
+#pragma unroll 1
+    for (int ch = 0; ch < 2; ++ch) {
+      float v[32];
+      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, v);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = silu(v[i] + b);
+      store_row32(x.xb, mt * 128 + x.c, x.col0 + 32 * ch, v);
+    }
+  }
+}
+
+// X = [xs +] acc + bias, zero on pad columns, stored to xs; then either the
+// RMS-normalised x_hat -> XB (next layer's projection operand) or mean pooling.
+__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bool add_xs, const float* gain,
+                                            bool pool) {
+  const TcParams& p = *x.p;
+  const int D = p.D;
+  float run[2] = {0.0f, 0.0f};
+#pragma unroll 1
+  for (int ch = 0; ch < 2; ++ch) {
+    float sq[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
+    for (int mt = 0; mt < x.MT; ++mt) {
+      const int ch_g = mt * 128 + x.c;
+      const float b = bias[ch_g];
+      float v[32];
+      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, v);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int col = x.col0 + 32 * ch + i;
+        float* xp = x.xs + (size_t)col * D + ch_g;
+        float val = v[i] + b;
+        if (add_xs) val += *xp;
+        const int fl = x.m->col_flags[col];
+        val = (fl & F_VALID) ? val : 0.0f;
+        *xp = val;
+        sq[i] = fmaf(val, val, sq[i]);
+        if (pool) {
+          if (fl & F_FIRST) run[mt] = 0.0f;
+          run[mt] += val;
+          if (fl & F_LAST) {
+            const int s = x.m->col_slot[col];
+            x.pooled[s * D + ch_g] = run[mt] / (float)x.m->slot_n[s];
+          }
+        }
+      }
+    }
+    if (!pool) {
+      const float s = reduce_scatter32(sq, x.lane);
+      x.m->part[x.q][x.col0 + 32 * ch + x.lane] = s;
+    }
+  }
+  if (pool) return;
+  ebar_sync();
+  if (x.te < TILE) {
+    const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
+    x.m->rinv[x.te] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
+  }
+  ebar_sync();
+  for (int mt = 0; mt < x.MT; ++mt) {
+    const int ch_g = mt * 128 + x.c;
+    const float g = gain[ch_g];
+#pragma unroll 1
+    for (int ch = 0; ch < 2; ++ch) {
+      float v[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int col = x.col0 + 32 * ch + i;
+        v[i] = x.xs[(size_t)col * D + ch_g] * g * x.m->rinv[col];
+      }
+      store_row32(x.xb, ch_g, x.col0 + 32 * ch, v);
+    }
+  }
+}
+
+// x' = X + (M + b_m) * sigma(p_g + b_g) -> xs and XB
+__device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
+  const TcParams& p = *x.p;
+  const int D = p.D;
+  for (int mt = 0; mt < x.MT; ++mt) {
+    const int ch_g = mt * 128 + x.c;
+    const float bm = p.b_m[l * D + ch_g];
+    const float bg = p.b_in[(size_t)l * p.ROWS_IN + p.NDC * 256 + ch_g];
+#pragma unroll 1
+    for (int ch = 0; ch < 2; ++ch) {
+      float mv[32], gv[32];
+      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, mv);
+      tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, gv);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int col = x.col0 + 32 * ch + i;
+        float* xp = x.xs + (size_t)col * D + ch_g;
+        const float x1 = *xp + (mv[i] + bm) * sigm(gv[i] + bg);
+        *xp = x1;
+        mv[i] = x1;
+      }
+      store_row32(x.xb, ch_g, x.col0 + 32 * ch, mv);
+    }
+  }
+}
+
+// Scan chunk dc (channel block dc/2, direction dc%2) of layer l -> HB.
+__device__ __forceinline__ void ep_scan(const ECtx& x, int l, int dc) {
+  const TcParams& p = *x.p;
+  const size_t rb = (size_t)l * p.ROWS_IN + dc * 256;
+  const float bz = p.b_in[rb + x.c], bn = p.b_in[rb + 128 + x.c];
+  const uint8_t* flags = x.m->col_flags;
+  float h = 0.0f;
+  if ((dc & 1) == 0) {
+#pragma unroll 1
+    for (int ch = 0; ch < 2; ++ch) {
+      float z[32], n[32];
+      tmem_ld32(x.tq + 256 + x.col0 + 32 * ch, z);
+      tmem_ld32(x.tq + 384 + x.col0 + 32 * ch, n);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int fl = flags[x.col0 + 32 * ch + i];
+        if (fl & F_FIRST) h = 0.0f;
+        if (fl & F_VALID) h = fmaf(sigm(z[i] + bz), (n[i] + bn) - h, h);
+        z[i] = (fl & F_VALID) ? h : 0.0f;
+      }
+      store_row32(x.hb, x.c, x.col0 + 32 * ch, z);
+    }
+  } else {
+#pragma unroll 1
+    for (int ch = 1; ch >= 0; --ch) {
+      float z[32], n[32];
+      tmem_ld32(x.tq + 256 + x.col0 + 32 * ch, z);
+      tmem_ld32(x.tq + 384 + x.col0 + 32 * ch, n);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 31; i >= 0; --i) {
+        const int fl = flags[x.col0 + 32 * ch + i];
+        if (fl & F_LAST) h = 0.0f;
+        if (fl & F_VALID) h = fmaf(sigm(z[i] + bz), (n[i] + bn) - h, h);
+        z[i] = (fl & F_VALID) ? h : 0.0f;
+      }
+      store_row32(x.hb, x.c, x.col0 + 32 * ch, z);
+    }
+  }
+}
+
+// Tile set-up: slot/column metadata, gather of the valid hits, Fourier operand.
+__device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
+  const TcParams& p = *x.p;
+  Misc* m = x.m;
+  if (x.te < TILE) m->col_flags[x.te] = 0;
+  ebar_sync();
+  if (x.e == 0) {
+    int ns = 0;
+    for (int hf = 0; hf < 2; ++hf) {
+      const int s = 2 * tile + hf;
+      if (s >= n_slabs) break;
+      const int b0 = p.slab_start[s];
+      const int cnt = p.slab_start[s + 1] - b0;
+      int n = 0, bad = 0;
+      if (x.lane < cnt) {
+        n = p.n_hits[b0 + x.lane];
+        bad = (n < 1 || n > p.T);
+        if (bad) n = 0;
+      }
+      int incl = n;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (x.lane >= o) incl += y;
+      }
+      if (x.lane < cnt) {
+        const int slot = ns + x.lane;
+        const int c0 = SLAB * hf + incl - n;
+        m->slot_track[slot] = b0 + x.lane;
+        m->slot_n[slot] = n;
+        m->slot_bad[slot] = bad;
+        for (int t = 0; t < n; ++t) {
+          const int col = c0 + t;
+          m->col_flags[col] = (uint8_t)(F_VALID | (t == 0 ? F_FIRST : 0) | (t == n - 1 ? F_LAST : 0));
+          m->col_slot[col] = (uint8_t)slot;
+          m->col_tpos[col] = (uint8_t)t;
+        }
+      }
+      ns += cnt;
+    }
+    if (x.lane == 0) m->n_slots = ns;
+  }
+  ebar_sync();
+  for (int idx = x.te; idx < TILE * 5; idx += NE) {
+    const int col = idx / 5, f = idx - col * 5;
+    float v = 0.0f;
+    if (m->col_flags[col] & F_VALID) {
+      const size_t trk = (size_t)m->slot_track[m->col_slot[col]];
+      v = p.hits[(trk * p.T + m->col_tpos[col]) * 5 + f];
+    }
+    m->hs[col][f] = v;
+  }
+  ebar_sync();
+  for (int idx = x.te; idx < TILE * 5; idx += NE) {
+    const int col = idx & (TILE - 1), f = idx >> 7;
+    const bool valid = (m->col_flags[col] & F_VALID) != 0;
+    const float u = (m->hs[col][f] - p.feat_min[f]) * p.feat_inv[f];
+    const uint32_t cb = x.hb + (uint32_t)((col & 7) * 2);
+#pragma unroll 4
+    for (int k = 0; k < 16; ++k) {
+      const float a = u * p.scale[k];
+      float sn = 0.0f, cs = 0.0f;
+      if (valid) {
+        sn = sinpif(a);
+        cs = cospif(a);
+      }
+      st_shared_u16(cb + bchunk(f * 32 + k, col >> 3), to_bf16(sn));
+      st_shared_u16(cb + bchunk(f * 32 + 16 + k, col >> 3), to_bf16(cs));
+    }
+  }
+}
+
+// Pooled vectors -> RMSNorm -> 2-layer head -> outputs (fp32 CUDA cores).
+__device__ __forceinline__ void ep_head(const ECtx& x) {
+  const TcParams& p = *x.p;
+  Misc* m = x.m;
+  const int D = p.D, ns = m->n_slots;
+  for (int s = x.e; s < ns; s += 8) {
+    const size_t trk = (size_t)m->slot_track[s];
+    const bool bad = m->slot_bad[s] != 0;
+    float ss = 0.0f;
+    for (int cc = x.lane; cc < D; cc += 32) {
+      const float v = x.pooled[s * D + cc];
+      ss = fmaf(v, v, ss);
+      if (p.out_pool) p.out_pool[trk * D + cc] = bad ? __int_as_float(0x7fc00000) : v;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    const float r = 1.0f / sqrtf(ss / (float)D + p.rms_eps);
+    for (int cc = x.lane; cc < D; cc += 32) x.pooled[s * D + cc] *= r * p.head_g[cc];
+  }
+  ebar_sync();
+  {
+    const int j = x.te & 127, sg = x.te >> 7;
+    float a[16];
+    const float b1 = p.head_b1[j];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) a[i] = b1;
+    const float* pv = x.pooled + (size_t)(sg * 16) * D;
+#pragma unroll 2
+    for (int cc = 0; cc < D; ++cc) {
+      const float w = p.head_w1t[cc * 128 + j];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) a[i] = fmaf(w, pv[i * D + cc], a[i]);
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (sg * 16 + i < ns) x.hid[(sg * 16 + i) * 128 + j] = silu(a[i]);
+  }
+  ebar_sync();
+  for (int idx = x.te; idx < ns * p.Q; idx += NE) {
+    const int s = idx / p.Q, o = idx - s * p.Q;
+    const float* w = p.head_w2 + (size_t)o * 128;
+    const float* hv = x.hid + s * 128;
+    float acc = p.head_b2[o];
+#pragma unroll 8
+    for (int j = 0; j < 128; ++j) acc = fmaf(w[j], hv[j], acc);
+    const size_t trk = (size_t)m->slot_track[s];
+    if (m->slot_bad[s]) acc = __int_as_float(0x7fc00000);
+    if (p.out_q) p.out_q[trk * p.Q + o] = acc;
+    const int qi = o % p.NQ;
+    if (qi == p.NQ / 2) p.out[trk * 5 + o / p.NQ] = acc;
+  }
+  for (int s = x.te; s < ns; s += NE)
+    if (m->slot_bad[s]) atomicAdd(p.err, 1ull);
+  ebar_sync();
+}
+
+__global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant__ TcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t xb = base + p.off_xb, hb = base + p.off_hb, ab = base + p.off_a;
+  Misc* m = reinterpret_cast<Misc*>(gbase + p.off_misc);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t full0 = smem_u32(&m->full[0]), empty0 = smem_u32(&m->empty[0]);
+  const uint32_t acc_bar = smem_u32(&m->acc_bar), e_bar = smem_u32(&m->e_bar);
+  const uint32_t drain_bar = smem_u32(&m->drain_bar);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.nst; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    mbar_init(acc_bar, 1);
+    mbar_init(e_bar, NE);
+    mbar_init(drain_bar, 1);
+    m->abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&m->tmem_base), 512);
+    tmem_relinquish();
+  }
+  if (warp == 0 && lane == 0)
+    for (int i = 0; i < NMAPS; ++i) prefetch_tmap(&p.tm[i]);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = m->tmem_base;
+  const int n_slabs = *p.n_slabs;
+  const int n_tiles = (n_slabs + 1) >> 1;
+  volatile int* abort = &m->abort_flag;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0;
+      bool ok = true;
+      int issued = 0;
+      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+        walk_tile(p, [&](int map, int row, int col, int, int, int, int, int, int) {
+          if (!ok) return;
+          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
+            set_abort(m, p.err);
+            ok = false;
+            return;
+          }
+          mbar_arrive_expect_tx(full0 + 8 * stage, A_STAGE);
+          tma_load_2d(ab + stage * A_STAGE, &p.tm[map], full0 + 8 * stage, col, row);
+          ++issued;
+          if (++stage == (uint32_t)p.nst) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        });
+      }
+      if (!ok) {
+        // let the copies already issued land before the CTA can exit
+        volatile int never = 0;
+        for (int k = 0; k < p.nst && k < issued; ++k) {
+          const int i = issued - 1 - k;
+          mbar_wait(full0 + 8 * (i % p.nst), (uint32_t)((i / p.nst) & 1), &never, DRAIN_NS);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0, e_phase = 0;
+      bool ok = true, need_e = true;
+      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+        walk_tile(p, [&](int, int, int, int nk, int tcol, int bsel, int bk, int acc, int end) {
+          if (!ok) return;
+          if (need_e) {
+            if (!mbar_wait(e_bar, e_phase, abort, WAIT_NS)) {
+              set_abort(m, p.err);
+              ok = false;
+              return;
+            }
+            e_phase ^= 1u;
+            need_e = false;
+            tc_fence_after();
+          }
+          if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
+            set_abort(m, p.err);
+            ok = false;
+            return;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = ab + stage * A_STAGE;
+          const uint32_t b_addr = bsel == BSEL_HB ? hb : xb;
+          for (int k = 0; k < nk; ++k) {
+            const uint64_t ad = sdesc_sw128(a_addr + 32 * k, 16, 1024);
+            const uint64_t bd = sdesc_sw128(b_addr + ((bk + 16 * k) >> 3) * B_SBO, B_LBO, B_SBO);
+            umma_f16(tmem + (uint32_t)tcol, ad, bd, p.idesc, (acc || k) ? 1u : 0u);
+          }
+          umma_commit(empty0 + 8 * stage);
+          if (end) {
+            umma_commit(acc_bar);
+            need_e = true;
+          }
+          if (++stage == (uint32_t)p.nst) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        });
+      }
+      // no MMA may still run when TMEM is released
+      umma_commit(drain_bar);
+      volatile int never = 0;
+      mbar_wait(drain_bar, 0, &never, DRAIN_NS);
+    }
+  } else {
+    ECtx x;
+    x.p = &p;
+    x.m = m;
+    x.xb = xb;
+    x.hb = hb;
+    x.e = warp - 2;
+    x.q = warp & 3;
+    x.half = x.e >> 2;
+    x.lane = lane;
+    x.c = 32 * x.q + lane;
+    x.col0 = SLAB * x.half;
+    x.te = threadIdx.x - 64;
+    x.MT = p.D >> 7;
+    x.tq = tmem + ((uint32_t)(32 * x.q) << 16);
+    x.xs = p.xs + (size_t)blockIdx.x * TILE * p.D;
+    x.pooled = reinterpret_cast<float*>(gbase + p.off_hb);
+    x.hid = reinterpret_cast<float*>(gbase + p.off_xb);
+    uint32_t acc_phase = 0;
+    auto signal = [&]() {
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(e_bar);
+    };
+    // The outcome of a wait is made uniform across the epilogue threads (they
+    // share named barriers); the wait itself ignores the abort flag so that a
+    // completed phase is seen by all of them.
+    volatile int no_abort = 0;
+    auto wait_acc = [&]() -> bool {
+      const bool mine = mbar_wait(acc_bar, acc_phase, &no_abort, WAIT_NS);
+      if (!ebar_all(mine)) {
+        set_abort(m, p.err);
+        return false;
+      }
+      acc_phase ^= 1u;
+      tc_fence_after();
+      return true;
+    };
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+      ep_setup(x, t, n_slabs);
+      signal();
+      if (!wait_acc()) break;
+      ep_silu(x, p.b_e1);
+      signal();
+      if (!wait_acc()) break;
+      ep_residual(x, p.b_e2, false, p.g, false);
+      signal();
+      bool ok = true;
+      for (int l = 0; l < p.L && ok; ++l) {
+        for (int dc = 0; dc < p.NDC; ++dc) {
+          if (!(ok = wait_acc())) break;
+          ep_scan(x, l, dc);
+          signal();
+        }
+        if (!ok || !(ok = wait_acc())) break;
+        ep_gate(x, l);
+        signal();
+        if (!(ok = wait_acc())) break;
+        ep_silu(x, p.b_1 + (size_t)l * p.D);
+        signal();
+        if (!(ok = wait_acc())) break;
+        const bool last = l == p.L - 1;
+        ep_residual(x, p.b_2 + (size_t)l * p.D, true, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
+        if (!last) signal();
+      }
+      if (!ok) break;
+      ebar_sync();
+      ep_head(x);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ------------------------------------------------------------------ packing
+// One warp per segment of SEG tracks packs whole tracks greedily into slabs of
+// at most 64 hits and MAX_TRK_SLAB tracks; every segment starts a new slab.
+__global__ void plan_segments(const int32_t* __restrict__ n_hits, int64_t B, int T, int32_t* __restrict__ seg_count,
+                              int32_t* __restrict__ seg_slabs) {
+  const int seg = blockIdx.x, lane = threadIdx.x;
+  const int64_t b0 = (int64_t)seg * SEG;
+  const int64_t b1 = (b0 + SEG < B) ? b0 + SEG : B;
+  int32_t* out = seg_slabs + (size_t)seg * (SEG + 1);
+  int cnt = 1, cur = 0, trk = 0;
+  if (lane == 0) out[0] = (int32_t)b0;
+  for (int64_t base = b0; base < b1; base += 32) {
+    int v = 0;
+    if (base + lane < b1) {
+      v = n_hits[base + lane];
+      if (v < 1 || v > T) v = 0;
+    }
+    const int lim = (int)((b1 - base) < 32 ? (b1 - base) : 32);
+    for (int i = 0; i < lim; ++i) {
+      const int ni = __shfl_sync(0xffffffffu, v, i);
+      if (trk == MAX_TRK_SLAB || cur + ni > SLAB) {
+        if (lane == 0) out[cnt] = (int32_t)(base + i);
+        ++cnt;
+        cur = 0;
+        trk = 0;
+      }
+      cur += ni;
+      ++trk;
+    }
+  }
+  if (lane == 0) seg_count[seg] = cnt;
+}
+
+// Exclusive scan of the per-segment slab counts (one block), total and sentinel.
+__global__ void plan_scan(const int32_t* __restrict__ seg_count, int nseg, int64_t B, int32_t* __restrict__ seg_off,
+                          int32_t* __restrict__ n_slabs, int32_t* __restrict__ slab_start) {
+  __shared__ int32_t part[1024];
+  const int tid = threadIdx.x;
+  const int per = (nseg + 1023) / 1024;
+  int32_t s = 0;
+  for (int i = 0; i < per; ++i) {
+    const int k = tid * per + i;
+    if (k < nseg) s += seg_count[k];
+  }
+  part[tid] = s;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {
+    const int32_t v = tid >= o ? part[tid - o] : 0;
+    __syncthreads();
+    part[tid] += v;
+    __syncthreads();
+  }
+  int32_t run = part[tid] - s;
+  for (int i = 0; i < per; ++i) {
+    const int k = tid * per + i;
+    if (k < nseg) {
+      seg_off[k] = run;
+      run += seg_count[k];
+    }
+  }
+  if (tid == 1023) {
+    n_slabs[0] = part[1023];
+    slab_start[part[1023]] = (int32_t)B;
+  }
+}
+
+__global__ void plan_scatter(const int32_t* __restrict__ seg_count, const int32_t* __restrict__ seg_off,
+                             const int32_t* __restrict__ seg_slabs, int32_t* __restrict__ slab_start) {
+  const int seg = blockIdx.x;
+  const int cnt = seg_count[seg], off = seg_off[seg];
+  for (int i = threadIdx.x; i < cnt; i += blockDim.x) slab_start[off + i] = seg_slabs[(size_t)seg * (SEG + 1) + i];
+}
+
+// ------------------------------------------------------------------ UMMA probe
+// D[128][128] = A[128][K] * B[K][128] through the same TMA / descriptor / TMEM
+// path as the fused kernel (test hook for the operand layouts).
+__global__ void __launch_bounds__(128, 1) umma_probe_kernel(const __grid_constant__ CUtensorMap tmA,
+                                                            const uint16_t* __restrict__ Bkn, int K,
+                                                            float* __restrict__ Dout, uint32_t idesc,
+                                                            unsigned long long* err) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t a_s = base;                 // K/64 blocks of 16 KB
+  const uint32_t b_s = base + (K / 64) * A_STAGE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(gbase + (K / 64) * A_STAGE + K * 256);
+  uint32_t* tbase = reinterpret_cast<uint32_t*>(bars + 2);
+  int* abortp = reinterpret_cast<int*>(bars + 3);
+  const uint32_t tma_bar = smem_u32(&bars[0]), mma_bar = smem_u32(&bars[1]);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(tma_bar, 1);
+    mbar_init(mma_bar, 1);
+    *abortp = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tbase), 128);
+    tmem_relinquish();
+  }
+  // B operand written by the threads, exactly as the epilogue does
+  for (int idx = threadIdx.x; idx < K * 16; idx += 128) {
+    const int k = idx >> 4, n8 = idx & 15;
+    const uint16_t* src = Bkn + (size_t)k * 128 + n8 * 8;
+    uint32_t w[4];
+    for (int i = 0; i < 4; ++i) w[i] = (uint32_t)src[2 * i] | ((uint32_t)src[2 * i + 1] << 16);
+    st_shared_v4(b_s + bchunk(k, n8), w[0], w[1], w[2], w[3]);
+  }
+  fence_proxy_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tbase;
+  volatile int* abort = abortp;
+  bool ok = true;
+  if (threadIdx.x == 0) {
+    mbar_arrive_expect_tx(tma_bar, (K / 64) * A_STAGE);
+    for (int kc = 0; kc < K / 64; ++kc) tma_load_2d(a_s + kc * A_STAGE, &tmA, tma_bar, kc * 64, 0);
+    ok = mbar_wait(tma_bar, 0, abort, WAIT_NS);
+    if (ok) {
+      tc_fence_after();
+      for (int kc = 0; kc < K / 64; ++kc)
+        for (int k = 0; k < 4; ++k) {
+          const uint64_t ad = sdesc_sw128(a_s + kc * A_STAGE + 32 * k, 16, 1024);
+          const uint64_t bd = sdesc_sw128(b_s + ((kc * 64 + 16 * k) >> 3) * B_SBO, B_LBO, B_SBO);
+          umma_f16(tmem, ad, bd, idesc, (kc || k) ? 1u : 0u);
+        }
+      umma_commit(mma_bar);
+    } else {
+      atomicAdd(err + 1, 1ull);
+      *abortp = 1;
+    }
+  }
+  __syncthreads();
+  if (!*abort) {
+    if (mbar_wait(mma_bar, 0, abort, WAIT_NS)) {
+      tc_fence_after();
+      const uint32_t tq = tmem + ((uint32_t)(32 * warp) << 16);
+      for (int ch = 0; ch < 4; ++ch) {
+        float v[32];
+        tmem_ld32(tq + 32 * ch, v);
+        tmem_ld_wait();
+        for (int i = 0; i < 32; ++i) Dout[(size_t)(32 * warp + lane) * 128 + 32 * ch + i] = v[i];
+      }
+    } else if (lane == 0) {
+      atomicAdd(err + 1, 1ull);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 128);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+uint16_t bf16_bits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7f800000u) == 0x7f800000u && (u & 0x007fffffu)) return 0x7fc0;
+  u += 0x7fffu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// bf16 matrix [rows][cols] row-major -> tensor map with 64 x 128 boxes, 128 B swizzle.
+bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, 128};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+struct tf_tc_state {
+  int nsm = 0, nst = 0, NDC = 0, ROWS_IN = 0, KM = 0;
+  size_t smem = 0;
+  int off_xb = 0, off_hb = 0, off_a = 0, off_misc = 0;
+  uint32_t idesc = 0;
+  void* dev = nullptr;  // one allocation for all weights
+  uint16_t *w_e1 = nullptr, *w_e2 = nullptr, *w_in = nullptr, *w_m = nullptr, *w_1 = nullptr, *w_2 = nullptr;
+  float *b_e1 = nullptr, *b_e2 = nullptr, *g = nullptr, *b_in = nullptr, *b_m = nullptr, *b_1 = nullptr,
+        *b_2 = nullptr, *hg = nullptr, *hw1t = nullptr, *hb1 = nullptr, *hw2 = nullptr, *hb2 = nullptr;
+  int32_t *seg_count = nullptr, *seg_off = nullptr, *seg_slabs = nullptr, *slab_start = nullptr, *n_slabs = nullptr;
+  float* xs = nullptr;
+  CUtensorMap tm[NMAPS];
+};
+
+bool tf_tc_supported(const tf_shape& s) {
+  return s.precision == TRACKFIT_BF16_PROJ && s.pool == TRACKFIT_POOL_MEAN && (s.D == 128 || s.D == 256) &&
+         s.T <= 64 && s.Hh == 128 && s.Q <= 75 && s.F == 5 && s.K == 16;
+}
+
+void tf_tc_destroy(trackfit_ctx* h) {
+  if (!h || !h->tc) return;
+  tf_tc_state* t = h->tc;
+  cudaFree(t->dev);
+  cudaFree(t->seg_count);
+  cudaFree(t->xs);
+  delete t;
+  h->tc = nullptr;
+}
+
+int tf_tc_create(trackfit_ctx* h, const float* W) {
+  const tf_shape& s = h->s;
+  const tf_blob_off& o = h->off;
+  tf_tc_state* t = new (std::nothrow) tf_tc_state();
+  if (!t) return TRACKFIT_ERR_OOM;
+  h->tc = t;
+  const int D = s.D, H = s.H, L = s.L, E = s.E;
+  const int nchunk = (H + 127) / 128;
+  t->NDC = 2 * nchunk;
+  t->ROWS_IN = t->NDC * 256 + D;
+  t->KM = t->NDC * 128;
+  t->idesc = idesc_f16(128, 128, 1u, false, true);
+  int dev = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&t->nsm, cudaDevAttrMultiProcessorCount, dev);
+  int smem_optin = 0;
+  cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  t->off_xb = 0;
+  t->off_hb = D * 256;
+  t->off_a = t->off_hb + EB_BYTES;
+  const int avail = smem_optin - 1024 - MISC_BYTES - t->off_a;
+  t->nst = avail / A_STAGE;
+  if (t->nst > MAX_STAGES) t->nst = MAX_STAGES;
+  if (t->nst < 2) return TRACKFIT_ERR_UNSUPPORTED;
+  t->off_misc = t->off_a + t->nst * A_STAGE;
+  t->smem = (size_t)t->off_misc + MISC_BYTES + 1024;
+  if ((size_t)(MAX_TRK_TILE * D * 4) > (size_t)EB_BYTES || MAX_TRK_TILE * 128 * 4 > D * 256)
+    return TRACKFIT_ERR_UNSUPPORTED;
+
+  // ---- repack weights (bf16 GEMM operands, fp32 biases/head)
+  const size_t n_e1 = (size_t)D * E, n_e2 = (size_t)D * D, n_in = (size_t)L * t->ROWS_IN * D,
+               n_m = (size_t)L * D * t->KM, n_11 = (size_t)L * D * D;
+  std::vector<uint16_t> we1(n_e1), we2(n_e2), win(n_in, 0), wm(n_m, 0), w1(n_11), w2(n_11);
+  std::vector<float> bin((size_t)L * t->ROWS_IN, 0.0f), gg((size_t)L * D), bm((size_t)L * D), b1((size_t)L * D),
+      b2((size_t)L * D), hw1t((size_t)s.P * 128);
+  for (size_t i = 0; i < n_e1; ++i) we1[i] = bf16_bits(W[o.emb_w1 + i]);
+  for (size_t i = 0; i < n_e2; ++i) we2[i] = bf16_bits(W[o.emb_w2 + i]);
+  for (int l = 0; l < L; ++l) {
+    const tf_layer_off& lo = o.layer[l];
+    const size_t rb = (size_t)l * t->ROWS_IN;
+    for (int dc = 0; dc < t->NDC; ++dc) {
+      const int j = dc >> 1, dir = dc & 1;
+      for (int c = 0; c < 128; ++c) {
+        const int ch = j * 128 + c;
+        if (ch >= H) continue;
+        const int src_z = (dir == 0 ? 0 : 2 * H) + ch, src_n = (dir == 0 ? H : 3 * H) + ch;
+        for (int k = 0; k < D; ++k) {
+          win[(rb + dc * 256 + c) * D + k] = bf16_bits(W[lo.w_in + (size_t)src_z * D + k]);
+          win[(rb + dc * 256 + 128 + c) * D + k] = bf16_bits(W[lo.w_in + (size_t)src_n * D + k]);
+        }
+        bin[rb + dc * 256 + c] = W[lo.b_in + src_z];
+        bin[rb + dc * 256 + 128 + c] = W[lo.b_in + src_n];
+        for (int r = 0; r < D; ++r)
+          wm[((size_t)l * D + r) * t->KM + dc * 128 + c] = bf16_bits(W[lo.w_m + (size_t)r * 2 * H + dir * H + ch]);
+      }
+    }
+    for (int c = 0; c < D; ++c) {
+      for (int k = 0; k < D; ++k)
+        win[(rb + t->NDC * 256 + c) * D + k] = bf16_bits(W[lo.w_in + (size_t)(4 * H + c) * D + k]);
+      bin[rb + t->NDC * 256 + c] = W[lo.b_in + 4 * H + c];
+    }
+    for (size_t i = 0; i < (size_t)D * D; ++i) {
+      w1[(size_t)l * D * D + i] = bf16_bits(W[lo.w1 + i]);
+      w2[(size_t)l * D * D + i] = bf16_bits(W[lo.w2 + i]);
+    }
+    for (int c = 0; c < D; ++c) {
+      gg[(size_t)l * D + c] = W[lo.g + c];
+      bm[(size_t)l * D + c] = W[lo.b_m + c];
+      b1[(size_t)l * D + c] = W[lo.b1 + c];
+      b2[(size_t)l * D + c] = W[lo.b2 + c];
+    }
+  }
+  for (int c = 0; c < s.P; ++c)
+    for (int j = 0; j < 128; ++j) hw1t[(size_t)c * 128 + j] = W[o.head_w1 + (size_t)j * s.P + c];
+
+  // ---- one device allocation for everything the kernel reads
+  struct Part {
+    const void* src;
+    size_t bytes;
+    void** dst;
+  };
+  std::vector<Part> parts = {
+      {we1.data(), n_e1 * 2, (void**)&t->w_e1},
+      {we2.data(), n_e2 * 2, (void**)&t->w_e2},
+      {win.data(), n_in * 2, (void**)&t->w_in},
+      {wm.data(), n_m * 2, (void**)&t->w_m},
+      {w1.data(), n_11 * 2, (void**)&t->w_1},
+      {w2.data(), n_11 * 2, (void**)&t->w_2},
+      {W + o.emb_b1, (size_t)D * 4, (void**)&t->b_e1},
+      {W + o.emb_b2, (size_t)D * 4, (void**)&t->b_e2},
+      {gg.data(), gg.size() * 4, (void**)&t->g},
+      {bin.data(), bin.size() * 4, (void**)&t->b_in},
+      {bm.data(), bm.size() * 4, (void**)&t->b_m},
+      {b1.data(), b1.size() * 4, (void**)&t->b_1},
+      {b2.data(), b2.size() * 4, (void**)&t->b_2},
+      {W + o.head_g, (size_t)s.P * 4, (void**)&t->hg},
+      {hw1t.data(), hw1t.size() * 4, (void**)&t->hw1t},
+      {W + o.head_b1, (size_t)128 * 4, (void**)&t->hb1},
+      {W + o.head_w2, (size_t)s.Q * 128 * 4, (void**)&t->hw2},
+      {W + o.head_b2, (size_t)s.Q * 4, (void**)&t->hb2},
+  };
+  size_t total = 0;
+  for (auto& pt : parts) total += (pt.bytes + 255) & ~(size_t)255;
+  if (cudaMalloc(&t->dev, total) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  size_t off = 0;
+  for (auto& pt : parts) {
+    *pt.dst = static_cast<char*>(t->dev) + off;
+    if (cudaMemcpy(*pt.dst, pt.src, pt.bytes, cudaMemcpyHostToDevice) != cudaSuccess) return TRACKFIT_ERR_CUDA;
+    off += (pt.bytes + 255) & ~(size_t)255;
+  }
+  // ---- packing buffers and the per-CTA residual scratch
+  const int nseg_max = (int)((MAXB + SEG - 1) / SEG);
+  const size_t plan_ints = (size_t)nseg_max * 2 + (size_t)nseg_max * (SEG + 1) + (size_t)MAXB + 2 + 64;
+  if (cudaMalloc(&t->seg_count, plan_ints * 4) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  t->seg_off = t->seg_count + nseg_max;
+  t->seg_slabs = t->seg_off + nseg_max;
+  t->slab_start = t->seg_slabs + (size_t)nseg_max * (SEG + 1);
+  t->n_slabs = t->slab_start + MAXB + 2;
+  if (cudaMalloc(&t->xs, (size_t)t->nsm * TILE * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  // ---- tensor maps
+  bool ok = make_map(&t->tm[MAP_E1], t->w_e1, D, E) && make_map(&t->tm[MAP_E2], t->w_e2, D, D) &&
+            make_map(&t->tm[MAP_IN], t->w_in, (uint64_t)L * t->ROWS_IN, D) &&
+            make_map(&t->tm[MAP_M], t->w_m, (uint64_t)L * D, t->KM) &&
+            make_map(&t->tm[MAP_1], t->w_1, (uint64_t)L * D, D) && make_map(&t->tm[MAP_2], t->w_2, (uint64_t)L * D, D);
+  if (!ok) return TRACKFIT_ERR_CUDA;
+  if (cudaFuncSetAttribute(tc_forward_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
+      cudaSuccess)
+    return TRACKFIT_ERR_CUDA;
+  return TRACKFIT_OK;
+}
+
+int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out, float* out_q,
+                  float* out_pool, cudaStream_t st) {
+  tf_tc_state* t = h->tc;
+  const tf_shape& s = h->s;
+  TcParams p;
+  std::memset(&p, 0, sizeof(p));
+  for (int i = 0; i < NMAPS; ++i) p.tm[i] = t->tm[i];
+  p.xs = t->xs;
+  p.slab_start = t->slab_start;
+  p.n_slabs = t->n_slabs;
+  p.b_e1 = t->b_e1;
+  p.b_e2 = t->b_e2;
+  p.g = t->g;
+  p.b_in = t->b_in;
+  p.b_m = t->b_m;
+  p.b_1 = t->b_1;
+  p.b_2 = t->b_2;
+  p.head_g = t->hg;
+  p.head_w1t = t->hw1t;
+  p.head_b1 = t->hb1;
+  p.head_w2 = t->hw2;
+  p.head_b2 = t->hb2;
+  p.err = h->d_err;
+  p.T = s.T;
+  p.D = s.D;
+  p.H = s.H;
+  p.L = s.L;
+  p.NDC = t->NDC;
+  p.ROWS_IN = t->ROWS_IN;
+  p.NQ = s.NQ;
+  p.Q = s.Q;
+  p.nst = t->nst;
+  p.idesc = t->idesc;
+  p.off_xb = t->off_xb;
+  p.off_hb = t->off_hb;
+  p.off_a = t->off_a;
+  p.off_misc = t->off_misc;
+  p.rms_eps = s.rms_eps;
+  for (int f = 0; f < 5; ++f) {
+    p.feat_min[f] = s.feat_min[f];
+    p.feat_inv[f] = s.feat_inv_range[f];
+  }
+  for (int k = 0; k < 16; ++k) p.scale[k] = s.scale[k];
+  for (int64_t c0 = 0; c0 < B; c0 += MAXB) {
+    const int64_t nb = (B - c0 < MAXB) ? B - c0 : MAXB;
+    const int nseg = (int)((nb + SEG - 1) / SEG);
+    plan_segments<<<nseg, 32, 0, st>>>(n_hits + c0, nb, s.T, t->seg_count, t->seg_slabs);
+    plan_scan<<<1, 1024, 0, st>>>(t->seg_count, nseg, nb, t->seg_off, t->n_slabs, t->slab_start);
+    plan_scatter<<<nseg, 128, 0, st>>>(t->seg_count, t->seg_off, t->seg_slabs, t->slab_start);
+    p.hits = hits + c0 * s.T * 5;
+    p.n_hits = n_hits + c0;
+    p.out = out + c0 * 5;
+    p.out_q = out_q ? out_q + c0 * s.Q : nullptr;
+    p.out_pool = out_pool ? out_pool + c0 * s.P : nullptr;
+    tc_forward_kernel<<<t->nsm, NT, t->smem, st>>>(p);
+    if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  }
+  return TRACKFIT_OK;
+}
+
+// UMMA layout probe: A device bf16 [128][K] (K-major), Bkn device bf16 [K][128],
+// D device fp32 [128][128]; K in {64, 128, 192, 256}.  Synchronous.
+int tf_tc_probe(trackfit_ctx* h, const uint16_t* A, const uint16_t* Bkn, int K, float* D, cudaStream_t st) {
+  if (K < 64 || K > 256 || (K % 64) != 0) return TRACKFIT_ERR_INVALID_ARG;
+  CUtensorMap m;
+  if (!make_map(&m, A, 128, (uint64_t)K)) return TRACKFIT_ERR_CUDA;
+  const size_t smem = (size_t)(K / 64) * A_STAGE + (size_t)K * 256 + 64 + 1024;
+  if (cudaFuncSetAttribute(umma_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return TRACKFIT_ERR_CUDA;
+  umma_probe_kernel<<<1, 128, smem, st>>>(m, Bkn, K, D, idesc_f16(128, 128, 1u, false, true), h->d_err);
+  if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  return TRACKFIT_OK;
 }

@@ -67,5 +67,7 @@ void tf_tc_destroy(trackfit_ctx* h);
 int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,
                   float* out, float* out_q, float* out_pool, cudaStream_t st);
 
+int tf_tc_probe(trackfit_ctx* h, const uint16_t* A, const uint16_t* Bkn, int K, float* D, cudaStream_t st);
+
 // api.cu
 int tf_status_from_cuda(cudaError_t e);

@@ -23,7 +23,7 @@ ABI_VERSION = 1
 # every function declared in include/trackfit.h
 EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trackfit_forward_ex",
            "trackfit_forward_host", "trackfit_device_errors", "trackfit_path_name", "trackfit_set_path",
-           "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan")
+           "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma")
 
 
 class Config(ctypes.Structure):
@@ -77,6 +77,8 @@ def load() -> ctypes.CDLL:
     lib.trackfit_strerror.restype = ctypes.c_char_p
     lib.trackfit_debug_scan.argtypes = [vp, vp, vp, vp, i64, i32, i32, vp, vp, vp]
     lib.trackfit_debug_scan.restype = ctypes.c_int
+    lib.trackfit_debug_umma.argtypes = [vp, vp, vp, i32, vp, vp]
+    lib.trackfit_debug_umma.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -206,3 +208,12 @@ def debug_scan(a, b, x, n_hits, h_fwd, h_bwd, stream=None) -> None:
                                     _dev(h_bwd, "torch.float32"), _stream_handle(stream))
     if st != OK:
         raise TrackfitError(st, "trackfit_debug_scan")
+
+
+def debug_umma(tf: "Trackfit", A, Bkn, D, stream=None) -> None:
+    """Device test hook: D[128][128] = A[128][K] * Bkn[K][128] (bf16 bits in int16 tensors)."""
+    K = int(A.shape[1])
+    st = load().trackfit_debug_umma(tf._h, _dev(A, "torch.int16"), _dev(Bkn, "torch.int16"), K,
+                                    _dev(D, "torch.float32"), _stream_handle(stream))
+    if st != OK:
+        raise TrackfitError(st, "trackfit_debug_umma")
