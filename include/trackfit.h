@@ -27,6 +27,7 @@
  * x_hat, [h_f; h_b], x', MLP hidden, and the weights of those products) to bf16
  * and accumulates in fp32; gates, scan state, residual stream, pooling and the
  * head stay fp32 (Sec. 3.5: reduced-precision projections, fp32 recurrence).
+ * TRACKFIT_FP16_PROJ is the same with fp16 operands, the format Sec. 3.5 names.
  *
  * Threading: a handle may be used from one host thread at a time and on one
  * stream at a time (it owns a device workspace).  Different handles are
@@ -56,7 +57,7 @@ typedef enum {
   TRACKFIT_ERR_TIMEOUT = 6       /* device-side: a bounded wait inside a kernel expired */
 } trackfit_status;
 
-typedef enum { TRACKFIT_FP32 = 0, TRACKFIT_BF16_PROJ = 1 } trackfit_precision;
+typedef enum { TRACKFIT_FP32 = 0, TRACKFIT_BF16_PROJ = 1, TRACKFIT_FP16_PROJ = 2 } trackfit_precision;
 typedef enum { TRACKFIT_POOL_MEAN = 0, TRACKFIT_POOL_ENDPOINTS = 1 } trackfit_pool;
 
 /* Encoder shape.  Supported: abi_version = 1, n_features = 5 (x, y, z [mm], r [mm],
@@ -141,14 +142,23 @@ int trackfit_forward_host(trackfit_t h, const float* hits_host, const int32_t* n
  * BAD_HITS when *n_bad > 0). */
 int trackfit_device_errors(trackfit_t h, void* stream, int64_t* n_bad);
 
-/* Name of the kernel path the handle runs: "simt-fp32", "simt-bf16" or
- * "tcgen05-bf16".  Static string, owned by the library. */
+/* Name of the kernel path the handle runs: "simt-fp32", "simt-bf16",
+ * "simt-fp16", "tcgen05-bf16" or "tcgen05-fp16".  Static string, owned by the
+ * library. */
 const char* trackfit_path_name(trackfit_t h);
 
-/* Select the kernel path: 0 = automatic (tcgen05 for BF16_PROJ configs it
- * supports, SIMT otherwise), 1 = force the SIMT path.  Returns UNSUPPORTED if the
+/* Select the kernel path: 0 = automatic (tcgen05 for the BF16_PROJ / FP16_PROJ
+ * configs it supports: mean pooling, d_model 128 or 256; SIMT otherwise), 1 = force the SIMT path.  Returns UNSUPPORTED if the
  * requested path cannot run this configuration. */
 int trackfit_set_path(trackfit_t h, int path);
+
+/* Timing hook: with enable = 1 every forward records CUDA events on its stream
+ * around the main compute kernel (the fused tcgen05 kernel, or the SIMT layer
+ * sequence); trackfit_profile_read synchronises on them, returns the summed
+ * kernel time in milliseconds and the number of timed launches since the last
+ * read, and resets both.  enable = 0 releases the events. */
+int trackfit_profile(trackfit_t h, int enable);
+int trackfit_profile_read(trackfit_t h, double* kernel_ms, int64_t* launches);
 
 /* Free everything the handle owns.  Accepts NULL.  The caller must make sure no
  * work using the handle is still running on any stream. */

@@ -11,13 +11,13 @@ it follows ("Fast and Precise Learned Charged-Particle Trajectory Regression at
 the LHC").  Where the paper is silent, the reading taken is stated in the
 function and collected in DESIGN.md.
 
-bf16 mode (configs with precision = 1): the paper runs the encoder GEMMs in
-reduced precision with fp32 recurrence state (Sec. 3.5).  The oracle then rounds
-exactly the operands of the per-hit GEMMs to bf16 (round to nearest even, from
-fp64): the Fourier vector, the embedding hidden activation, the pre-normed layer
-input, the concatenated scan states, the gated residual x', the MLP hidden
-activation, and the weights of those GEMMs.  Everything else (biases, gates, scan
-state, residual stream, pooling, head) stays fp64.
+Reduced-precision modes (precision = 1: bf16, precision = 2: fp16): the paper
+runs the encoder GEMMs in fp16 with fp32 recurrence state (Sec. 3.5).  The oracle
+then rounds exactly the operands of the per-hit GEMMs to that format (round to
+nearest even, from fp64): the Fourier vector, the embedding hidden activation,
+the pre-normed layer input, the concatenated scan states, the gated residual x',
+the MLP hidden activation, and the weights of those GEMMs.  Everything else
+(biases, gates, scan state, residual stream, pooling, head) stays fp64.
 
 Parity status: agreement with the paper's trained model is unpinned (no trained
 weights, data or printed activations exist); the functions here are pinned by
@@ -29,7 +29,7 @@ from typing import Dict, Optional
 
 import numpy as np
 
-__all__ = ["bf16_round", "sigmoid", "silu", "rmsnorm", "normalise", "fourier", "linear_scan",
+__all__ = ["bf16_round", "fp16_round", "sigmoid", "silu", "rmsnorm", "normalise", "fourier", "linear_scan",
            "mingru_layer_scans", "embed", "encoder_layer", "pool", "head", "forward", "split_blob"]
 
 
@@ -56,6 +56,13 @@ def bf16_round(x: np.ndarray) -> np.ndarray:
     out = np.where(np.isfinite(x), out, x)
     # values past the largest bf16 round to inf
     return out
+
+
+def fp16_round(x: np.ndarray) -> np.ndarray:
+    """Round fp64 values to the nearest IEEE binary16 value (ties to even); result
+    in fp64.  numpy converts float64 to float16 directly with that rounding."""
+    with np.errstate(over="ignore"):
+        return np.asarray(x, dtype=np.float64).astype(np.float16).astype(np.float64)
 
 
 def sigmoid(x):
@@ -137,14 +144,18 @@ def mingru_layer_scans(z_f, n_f, z_b, n_b, valid):
 # network blocks
 # ---------------------------------------------------------------------------
 
-def _op(x, bf16):
-    """Operand of a per-hit GEMM: bf16-rounded in bf16 mode, else unchanged."""
-    return bf16_round(x) if bf16 else x
+def _op(x, prec):
+    """Operand of a per-hit GEMM: rounded to bf16 (prec 1) or fp16 (prec 2), else unchanged."""
+    if prec == 1:
+        return bf16_round(x)
+    if prec == 2:
+        return fp16_round(x)
+    return x
 
 
-def _lin(x, w, b, bf16):
-    """y = x W^T + b with W in PyTorch [out][in] order; GEMM operands rounded in bf16 mode."""
-    return _op(x, bf16) @ _op(np.asarray(w, dtype=np.float64), bf16).T + b
+def _lin(x, w, b, prec):
+    """y = x W^T + b with W in PyTorch [out][in] order; GEMM operands rounded per prec."""
+    return _op(x, prec) @ _op(np.asarray(w, dtype=np.float64), prec).T + b
 
 
 def embed(e, W, bf16):
@@ -246,12 +257,12 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
     """Track parameters (d0, z0, phi, theta, q/p) for every track: [B, 5] fp64.
 
     cfg: dict with d_model, d_hidden, n_layers, n_features, n_fourier, head_hidden,
-    n_quantiles, precision (0 fp32, 1 bf16 operands), pool (0 mean, 1 endpoints),
+    n_quantiles, precision (0 fp32, 1 bf16 operands, 2 fp16 operands), pool (0 mean, 1 endpoints),
     feat_min, feat_max, fourier_scale, rms_eps.  hits: [B, T, 5]; n_hits: [B].
     Tracks whose hit count is outside [1, T] give a NaN row.  The output is the
     median quantile of the head directly (no seed decode)."""
     W = split_blob(cfg, blob)
-    bf16 = int(cfg["precision"]) == 1
+    bf16 = int(cfg["precision"])      # operand rounding: 0 none, 1 bf16, 2 fp16
     hits = np.asarray(hits)
     n_hits = np.asarray(n_hits).astype(np.int64)
     B, T, _ = hits.shape

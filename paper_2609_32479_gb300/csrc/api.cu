@@ -26,7 +26,8 @@ static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   if (c->n_layers < 1 || c->n_layers > TF_MAX_LAYERS) return false;
   if (c->head_hidden != 128) return false;
   if (c->n_quantiles < 1 || c->n_quantiles > 15 || (c->n_quantiles % 2) == 0) return false;
-  if (c->precision != TRACKFIT_FP32 && c->precision != TRACKFIT_BF16_PROJ) return false;
+  if (c->precision != TRACKFIT_FP32 && c->precision != TRACKFIT_BF16_PROJ && c->precision != TRACKFIT_FP16_PROJ)
+    return false;
   if (c->pool != TRACKFIT_POOL_MEAN && c->pool != TRACKFIT_POOL_ENDPOINTS) return false;
   if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return false;
   for (int f = 0; f < TRACKFIT_MAX_FEATURES; ++f)
@@ -102,8 +103,58 @@ extern "C" const char* trackfit_strerror(int status) {
   }
 }
 
+static void prof_collect(trackfit_ctx* h) {
+  for (int i = 0; i < h->prof_n; ++i) {
+    float ms = 0.0f;
+    cudaEventSynchronize(h->prof_ev[2 * i + 1]);
+    if (cudaEventElapsedTime(&ms, h->prof_ev[2 * i], h->prof_ev[2 * i + 1]) == cudaSuccess) h->prof_ms += ms;
+    ++h->prof_launches;
+  }
+  h->prof_n = 0;
+}
+
+void tf_prof_begin(trackfit_ctx* h, cudaStream_t st) {
+  if (!h->prof_on) return;
+  if (h->prof_n == 64) prof_collect(h);
+  cudaEventRecord(h->prof_ev[2 * h->prof_n], st);
+}
+
+void tf_prof_end(trackfit_ctx* h, cudaStream_t st) {
+  if (!h->prof_on) return;
+  cudaEventRecord(h->prof_ev[2 * h->prof_n + 1], st);
+  ++h->prof_n;
+}
+
+extern "C" int trackfit_profile(trackfit_t h, int enable) {
+  if (!h) return TRACKFIT_ERR_INVALID_ARG;
+  if (enable && !h->prof_on) {
+    for (int i = 0; i < 2 * 64; ++i)
+      if (cudaEventCreate(&h->prof_ev[i]) != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  }
+  if (!enable && h->prof_on) {
+    prof_collect(h);
+    for (int i = 0; i < 2 * 64; ++i) cudaEventDestroy(h->prof_ev[i]);
+  }
+  h->prof_on = enable ? 1 : 0;
+  h->prof_n = 0;
+  h->prof_ms = 0.0;
+  h->prof_launches = 0;
+  return TRACKFIT_OK;
+}
+
+extern "C" int trackfit_profile_read(trackfit_t h, double* kernel_ms, int64_t* launches) {
+  if (!h || !kernel_ms || !launches) return TRACKFIT_ERR_INVALID_ARG;
+  if (h->prof_on) prof_collect(h);
+  *kernel_ms = h->prof_ms;
+  *launches = h->prof_launches;
+  h->prof_ms = 0.0;
+  h->prof_launches = 0;
+  return TRACKFIT_OK;
+}
+
 extern "C" void trackfit_destroy(trackfit_t h) {
   if (!h) return;
+  if (h->prof_on) trackfit_profile(h, 0);
   tf_tc_destroy(h);
   cudaFree(h->d_w);
   cudaFree(h->d_err);
@@ -133,7 +184,7 @@ extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weight
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMalloc(&h->d_err, 4 * sizeof(unsigned long long)));
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemset(h->d_err, 0, 4 * sizeof(unsigned long long)));
   if (st == TRACKFIT_OK) st = tf_simt_workspace(h);
-  if (st == TRACKFIT_OK && s.precision == TRACKFIT_BF16_PROJ && tf_tc_supported(s)) {
+  if (st == TRACKFIT_OK && tf_tc_supported(s)) {
     st = tf_tc_create(h, weights);
     if (st == TRACKFIT_OK) h->path = TF_PATH_TC;
   }
@@ -148,8 +199,10 @@ extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weight
 
 extern "C" const char* trackfit_path_name(trackfit_t h) {
   if (!h) return "none";
-  if (h->path == TF_PATH_TC) return "tcgen05-bf16";
-  return h->s.precision == TRACKFIT_BF16_PROJ ? "simt-bf16" : "simt-fp32";
+  const bool tc = h->path == TF_PATH_TC;
+  if (h->s.precision == TRACKFIT_FP16_PROJ) return tc ? "tcgen05-fp16" : "simt-fp16";
+  if (h->s.precision == TRACKFIT_BF16_PROJ) return tc ? "tcgen05-bf16" : "simt-bf16";
+  return "simt-fp32";
 }
 
 extern "C" int trackfit_set_path(trackfit_t h, int path) {

@@ -6,6 +6,7 @@
 // workspace.  Padded rows are computed and then excluded by select (their
 // residual rows are forced to 0, the scans and pooling skip them).
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <math.h>
 
 #include "trackfit_internal.h"
@@ -17,6 +18,7 @@ enum { EPI_STORE = 0, EPI_SILU = 1, EPI_PROJ = 2, EPI_GATE_RES = 3, EPI_RES_MASK
 __device__ __forceinline__ float sigm(float x) { return 1.0f / (1.0f + expf(-x)); }
 __device__ __forceinline__ float silu(float x) { return x * sigm(x); }
 __device__ __forceinline__ float bf16r(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+__device__ __forceinline__ float fp16r(float x) { return __half2float(__float2half_rn(x)); }
 
 __device__ __forceinline__ bool row_valid(int r, int T, const int32_t* n_hits) {
   int b = r / T, t = r - b * T;
@@ -30,7 +32,7 @@ struct GemmArgs {
   const float* bias;            // [N]
   float* C; int ldc;            // [R][ldc]
   int R, N, K;
-  int bf16;                     // round both operands to bf16 on load
+  int rnd;                      // round both operands on load: 0 none, 1 bf16, 2 fp16
   int epi;
   const float* res; int ldr;    // residual input (GATE_RES, RES_MASK)
   const float* gate; int ldg;   // sigmoid gate values (GATE_RES)
@@ -55,7 +57,8 @@ __global__ void __launch_bounds__(256) gemm_kernel(GemmArgs g) {
       float a = (r < g.R && kk < g.K) ? g.A[(size_t)r * g.lda + kk] : 0.0f;
       int n = col0 + m;
       float w = (n < g.N && kk < g.K) ? g.W[(size_t)n * g.K + kk] : 0.0f;
-      if (g.bf16) { a = bf16r(a); w = bf16r(w); }
+      if (g.rnd == 1) { a = bf16r(a); w = bf16r(w); }
+      if (g.rnd == 2) { a = fp16r(a); w = fp16r(w); }
       As[k][m] = a;
       Ws[k][m] = w;
     }
@@ -283,7 +286,7 @@ int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, i
   const tf_shape& s = h->s;
   const float* W = h->d_w;
   const tf_blob_off& o = h->off;
-  const int bf = s.precision == TRACKFIT_BF16_PROJ;
+  const int rnd = s.precision;   // TRACKFIT_FP32 = 0, BF16_PROJ = 1, FP16_PROJ = 2
   const int D = s.D, H = s.H, PD = 4 * s.H + s.D;
   for (int64_t c0 = 0; c0 < B; c0 += h->ws_tracks) {
     const int64_t nb = (B - c0 < h->ws_tracks) ? B - c0 : h->ws_tracks;
@@ -297,11 +300,12 @@ int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, i
     float* X1 = Y + R * 2 * H;
     const float* hc = hits + c0 * s.T * 5;
     const int32_t* nc = n_hits + c0;
+    tf_prof_begin(h, st);
     int64_t nthreads = R * s.F;
     fourier_kernel<<<(unsigned)((nthreads + 255) / 256), 256, 0, st>>>(hc, R, EB, s);
     GemmArgs g{};
     g.R = (int)R;
-    g.bf16 = bf;
+    g.rnd = rnd;
     g.n_hits = nc;
     g.T = s.T;
     g.H = H;
@@ -335,6 +339,7 @@ int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, i
                                                     W + o.head_w2, W + o.head_b2, out + c0 * 5,
                                                     out_q ? out_q + c0 * s.Q : nullptr,
                                                     out_pool ? out_pool + c0 * s.P : nullptr, h->d_err);
+    tf_prof_end(h, st);
     if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
   }
   return TRACKFIT_OK;

@@ -84,8 +84,9 @@ struct TcParams {
   int T, D, H, L, NDC, ROWS_IN, NQ, Q, nst;
   uint32_t idesc;
   int off_xb, off_hb, off_a, off_misc;
+  int fp16;
   float rms_eps;
-  float feat_min[5], feat_inv[5], scale[16];
+  float feat_min[5], feat_inv_hi[5], feat_inv_lo[5], scale[16];
 };
 
 struct Misc {
@@ -106,13 +107,26 @@ static_assert(sizeof(Misc) <= MISC_BYTES, "misc region too small");
 __device__ __forceinline__ float sigm(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
 __device__ __forceinline__ float silu(float x) { return x * sigm(x); }
 
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);   // a -> low half (lower column)
-  return *reinterpret_cast<uint32_t*>(&v);
+// Operand conversion (round to nearest even): bf16, or fp16 when FP16 is set.
+template <bool FP16>
+__device__ __forceinline__ uint32_t pack2(float a, float b) {   // a -> low half (lower column)
+  if constexpr (FP16) {
+    __half2 v = __floats2half2_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&v);
+  } else {
+    __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&v);
+  }
 }
-__device__ __forceinline__ uint16_t to_bf16(float a) {
-  __nv_bfloat16 v = __float2bfloat16_rn(a);
-  return *reinterpret_cast<uint16_t*>(&v);
+template <bool FP16>
+__device__ __forceinline__ uint16_t to16(float a) {
+  if constexpr (FP16) {
+    __half v = __float2half_rn(a);
+    return *reinterpret_cast<uint16_t*>(&v);
+  } else {
+    __nv_bfloat16 v = __float2bfloat16_rn(a);
+    return *reinterpret_cast<uint16_t*>(&v);
+  }
 }
 
 // Byte offset, inside an MN-major 128-byte-swizzled operand with 128 columns, of
@@ -129,13 +143,14 @@ __device__ __forceinline__ void st_shared_u16(uint32_t addr, uint16_t v) {
   asm volatile("st.shared.u16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
 }
 
-// Write 32 consecutive columns [n0, n0+32) of k-row k (n0 % 32 == 0) as bf16.
+// Write 32 consecutive columns [n0, n0+32) of k-row k (n0 % 32 == 0) as 16-bit operands.
+template <bool FP16>
 __device__ __forceinline__ void store_row32(uint32_t buf, int k, int n0, const float (&v)[32]) {
 #pragma unroll
   for (int c = 0; c < 4; ++c) {
-    st_shared_v4(buf + bchunk(k, (n0 >> 3) + c), pack_bf16(v[8 * c + 0], v[8 * c + 1]),
-                 pack_bf16(v[8 * c + 2], v[8 * c + 3]), pack_bf16(v[8 * c + 4], v[8 * c + 5]),
-                 pack_bf16(v[8 * c + 6], v[8 * c + 7]));
+    st_shared_v4(buf + bchunk(k, (n0 >> 3) + c), pack2<FP16>(v[8 * c + 0], v[8 * c + 1]),
+                 pack2<FP16>(v[8 * c + 2], v[8 * c + 3]), pack2<FP16>(v[8 * c + 4], v[8 * c + 5]),
+                 pack2<FP16>(v[8 * c + 6], v[8 * c + 7]));
   }
 }
 
@@ -227,6 +242,7 @@ struct ECtx {
 };
 
 // silu(acc + bias) -> XB rows [mt*128 + c]
+template <bool FP16>
 __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
   for (int mt = 0; mt < x.MT; ++mt) {
     const float b = bias[mt * 128 + x.c];
@@ -237,13 +253,14 @@ __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = silu(v[i] + b);
-      store_row32(x.xb, mt * 128 + x.c, x.col0 + 32 * ch, v);
+      store_row32<FP16>(x.xb, mt * 128 + x.c, x.col0 + 32 * ch, v);
     }
   }
 }
 
 // X = [xs +] acc + bias, zero on pad columns, stored to xs; then either the
 // RMS-normalised x_hat -> XB (next layer's projection operand) or mean pooling.
+template <bool FP16>
 __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bool add_xs, const float* gain,
                                             bool pool) {
   const TcParams& p = *x.p;
@@ -303,12 +320,13 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
         const int col = x.col0 + 32 * ch + i;
         v[i] = x.xs[(size_t)col * D + ch_g] * g * x.m->rinv[col];
       }
-      store_row32(x.xb, ch_g, x.col0 + 32 * ch, v);
+      store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, v);
     }
   }
 }
 
 // x' = X + (M + b_m) * sigma(p_g + b_g) -> xs and XB
+template <bool FP16>
 __device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
   const TcParams& p = *x.p;
   const int D = p.D;
@@ -330,12 +348,13 @@ __device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
         *xp = x1;
         mv[i] = x1;
       }
-      store_row32(x.xb, ch_g, x.col0 + 32 * ch, mv);
+      store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, mv);
     }
   }
 }
 
 // Scan chunk dc (channel block dc/2, direction dc%2) of layer l -> HB.
+template <bool FP16>
 __device__ __forceinline__ void ep_scan(const ECtx& x, int l, int dc) {
   const TcParams& p = *x.p;
   const size_t rb = (size_t)l * p.ROWS_IN + dc * 256;
@@ -356,7 +375,7 @@ __device__ __forceinline__ void ep_scan(const ECtx& x, int l, int dc) {
         if (fl & F_VALID) h = fmaf(sigm(z[i] + bz), (n[i] + bn) - h, h);
         z[i] = (fl & F_VALID) ? h : 0.0f;
       }
-      store_row32(x.hb, x.c, x.col0 + 32 * ch, z);
+      store_row32<FP16>(x.hb, x.c, x.col0 + 32 * ch, z);
     }
   } else {
 #pragma unroll 1
@@ -372,12 +391,13 @@ __device__ __forceinline__ void ep_scan(const ECtx& x, int l, int dc) {
         if (fl & F_VALID) h = fmaf(sigm(z[i] + bz), (n[i] + bn) - h, h);
         z[i] = (fl & F_VALID) ? h : 0.0f;
       }
-      store_row32(x.hb, x.c, x.col0 + 32 * ch, z);
+      store_row32<FP16>(x.hb, x.c, x.col0 + 32 * ch, z);
     }
   }
 }
 
 // Tile set-up: slot/column metadata, gather of the valid hits, Fourier operand.
+template <bool FP16>
 __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
   const TcParams& p = *x.p;
   Misc* m = x.m;
@@ -430,21 +450,32 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
     m->hs[col][f] = v;
   }
   ebar_sync();
+  // u = (v - min) / (max - min) and the argument s_k * u as unevaluated sums of
+  // two floats (error-free TwoSum / TwoProduct with fma), reduced modulo 2
+  // exactly, so sin(pi s_k u) carries only the final fp32 rounding.
   for (int idx = x.te; idx < TILE * 5; idx += NE) {
     const int col = idx & (TILE - 1), f = idx >> 7;
     const bool valid = (m->col_flags[col] & F_VALID) != 0;
-    const float u = (m->hs[col][f] - p.feat_min[f]) * p.feat_inv[f];
+    const float v = m->hs[col][f], mn = -p.feat_min[f];
+    const float dh = v + mn;
+    const float bv = dh - v;
+    const float dl = (v - (dh - bv)) + (mn - bv);
+    const float uh = dh * p.feat_inv_hi[f];
+    const float ul = fmaf(dh, p.feat_inv_hi[f], -uh) + fmaf(dh, p.feat_inv_lo[f], dl * p.feat_inv_hi[f]);
     const uint32_t cb = x.hb + (uint32_t)((col & 7) * 2);
 #pragma unroll 4
     for (int k = 0; k < 16; ++k) {
-      const float a = u * p.scale[k];
+      const float sk = p.scale[k];
+      const float xh = uh * sk;
+      const float xl = fmaf(uh, sk, -xh) + ul * sk;
+      const float r = (xh - 2.0f * rintf(0.5f * xh)) + xl;
       float sn = 0.0f, cs = 0.0f;
       if (valid) {
-        sn = sinpif(a);
-        cs = cospif(a);
+        sn = sinpif(r);
+        cs = cospif(r);
       }
-      st_shared_u16(cb + bchunk(f * 32 + k, col >> 3), to_bf16(sn));
-      st_shared_u16(cb + bchunk(f * 32 + 16 + k, col >> 3), to_bf16(cs));
+      st_shared_u16(cb + bchunk(f * 32 + k, col >> 3), to16<FP16>(sn));
+      st_shared_u16(cb + bchunk(f * 32 + 16 + k, col >> 3), to16<FP16>(cs));
     }
   }
 }
@@ -505,6 +536,7 @@ __device__ __forceinline__ void ep_head(const ECtx& x) {
   ebar_sync();
 }
 
+template <bool FP16>
 __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -658,30 +690,30 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       return true;
     };
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
-      ep_setup(x, t, n_slabs);
+      ep_setup<FP16>(x, t, n_slabs);
       signal();
       if (!wait_acc()) break;
-      ep_silu(x, p.b_e1);
+      ep_silu<FP16>(x, p.b_e1);
       signal();
       if (!wait_acc()) break;
-      ep_residual(x, p.b_e2, false, p.g, false);
+      ep_residual<FP16>(x, p.b_e2, false, p.g, false);
       signal();
       bool ok = true;
       for (int l = 0; l < p.L && ok; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
           if (!(ok = wait_acc())) break;
-          ep_scan(x, l, dc);
+          ep_scan<FP16>(x, l, dc);
           signal();
         }
         if (!ok || !(ok = wait_acc())) break;
-        ep_gate(x, l);
+        ep_gate<FP16>(x, l);
         signal();
         if (!(ok = wait_acc())) break;
-        ep_silu(x, p.b_1 + (size_t)l * p.D);
+        ep_silu<FP16>(x, p.b_1 + (size_t)l * p.D);
         signal();
         if (!(ok = wait_acc())) break;
         const bool last = l == p.L - 1;
-        ep_residual(x, p.b_2 + (size_t)l * p.D, true, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
+        ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, true, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
         if (!last) signal();
       }
       if (!ok) break;
@@ -855,6 +887,10 @@ __global__ void __launch_bounds__(128, 1) umma_probe_kernel(const __grid_constan
 }
 
 // ------------------------------------------------------------------ host side
+uint16_t fp16_bits(float f) {
+  const __half v = __float2half_rn(f);
+  return *reinterpret_cast<const uint16_t*>(&v);
+}
 uint16_t bf16_bits(float f) {
   uint32_t u;
   std::memcpy(&u, &f, 4);
@@ -877,14 +913,14 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 // bf16 matrix [rows][cols] row-major -> tensor map with 64 x 128 boxes, 128 B swizzle.
-bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols) {
+bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, bool fp16 = false) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
   cuuint32_t box[2] = {64, 128};
   cuuint32_t es[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
+  return fn(m, fp16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -906,7 +942,7 @@ struct tf_tc_state {
 };
 
 bool tf_tc_supported(const tf_shape& s) {
-  return s.precision == TRACKFIT_BF16_PROJ && s.pool == TRACKFIT_POOL_MEAN && (s.D == 128 || s.D == 256) &&
+  return (s.precision == TRACKFIT_BF16_PROJ || s.precision == TRACKFIT_FP16_PROJ) && s.pool == TRACKFIT_POOL_MEAN && (s.D == 128 || s.D == 256) &&
          s.T <= 64 && s.Hh == 128 && s.Q <= 75 && s.F == 5 && s.K == 16;
 }
 
@@ -931,7 +967,8 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   t->NDC = 2 * nchunk;
   t->ROWS_IN = t->NDC * 256 + D;
   t->KM = t->NDC * 128;
-  t->idesc = idesc_f16(128, 128, 1u, false, true);
+  const bool fp16 = s.precision == TRACKFIT_FP16_PROJ;
+  t->idesc = idesc_f16(128, 128, fp16 ? 0u : 1u, false, true);
   int dev = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&t->nsm, cudaDevAttrMultiProcessorCount, dev);
@@ -955,8 +992,9 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   std::vector<uint16_t> we1(n_e1), we2(n_e2), win(n_in, 0), wm(n_m, 0), w1(n_11), w2(n_11);
   std::vector<float> bin((size_t)L * t->ROWS_IN, 0.0f), gg((size_t)L * D), bm((size_t)L * D), b1((size_t)L * D),
       b2((size_t)L * D), hw1t((size_t)s.P * 128);
-  for (size_t i = 0; i < n_e1; ++i) we1[i] = bf16_bits(W[o.emb_w1 + i]);
-  for (size_t i = 0; i < n_e2; ++i) we2[i] = bf16_bits(W[o.emb_w2 + i]);
+  uint16_t (*cv)(float) = fp16 ? fp16_bits : bf16_bits;
+  for (size_t i = 0; i < n_e1; ++i) we1[i] = cv(W[o.emb_w1 + i]);
+  for (size_t i = 0; i < n_e2; ++i) we2[i] = cv(W[o.emb_w2 + i]);
   for (int l = 0; l < L; ++l) {
     const tf_layer_off& lo = o.layer[l];
     const size_t rb = (size_t)l * t->ROWS_IN;
@@ -967,23 +1005,23 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
         if (ch >= H) continue;
         const int src_z = (dir == 0 ? 0 : 2 * H) + ch, src_n = (dir == 0 ? H : 3 * H) + ch;
         for (int k = 0; k < D; ++k) {
-          win[(rb + dc * 256 + c) * D + k] = bf16_bits(W[lo.w_in + (size_t)src_z * D + k]);
-          win[(rb + dc * 256 + 128 + c) * D + k] = bf16_bits(W[lo.w_in + (size_t)src_n * D + k]);
+          win[(rb + dc * 256 + c) * D + k] = cv(W[lo.w_in + (size_t)src_z * D + k]);
+          win[(rb + dc * 256 + 128 + c) * D + k] = cv(W[lo.w_in + (size_t)src_n * D + k]);
         }
         bin[rb + dc * 256 + c] = W[lo.b_in + src_z];
         bin[rb + dc * 256 + 128 + c] = W[lo.b_in + src_n];
         for (int r = 0; r < D; ++r)
-          wm[((size_t)l * D + r) * t->KM + dc * 128 + c] = bf16_bits(W[lo.w_m + (size_t)r * 2 * H + dir * H + ch]);
+          wm[((size_t)l * D + r) * t->KM + dc * 128 + c] = cv(W[lo.w_m + (size_t)r * 2 * H + dir * H + ch]);
       }
     }
     for (int c = 0; c < D; ++c) {
       for (int k = 0; k < D; ++k)
-        win[(rb + t->NDC * 256 + c) * D + k] = bf16_bits(W[lo.w_in + (size_t)(4 * H + c) * D + k]);
+        win[(rb + t->NDC * 256 + c) * D + k] = cv(W[lo.w_in + (size_t)(4 * H + c) * D + k]);
       bin[rb + t->NDC * 256 + c] = W[lo.b_in + 4 * H + c];
     }
     for (size_t i = 0; i < (size_t)D * D; ++i) {
-      w1[(size_t)l * D * D + i] = bf16_bits(W[lo.w1 + i]);
-      w2[(size_t)l * D * D + i] = bf16_bits(W[lo.w2 + i]);
+      w1[(size_t)l * D * D + i] = cv(W[lo.w1 + i]);
+      w2[(size_t)l * D * D + i] = cv(W[lo.w2 + i]);
     }
     for (int c = 0; c < D; ++c) {
       gg[(size_t)l * D + c] = W[lo.g + c];
@@ -1040,13 +1078,16 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   t->n_slabs = t->slab_start + MAXB + 2;
   if (cudaMalloc(&t->xs, (size_t)t->nsm * TILE * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
   // ---- tensor maps
-  bool ok = make_map(&t->tm[MAP_E1], t->w_e1, D, E) && make_map(&t->tm[MAP_E2], t->w_e2, D, D) &&
-            make_map(&t->tm[MAP_IN], t->w_in, (uint64_t)L * t->ROWS_IN, D) &&
-            make_map(&t->tm[MAP_M], t->w_m, (uint64_t)L * D, t->KM) &&
-            make_map(&t->tm[MAP_1], t->w_1, (uint64_t)L * D, D) && make_map(&t->tm[MAP_2], t->w_2, (uint64_t)L * D, D);
+  bool ok = make_map(&t->tm[MAP_E1], t->w_e1, D, E, fp16) && make_map(&t->tm[MAP_E2], t->w_e2, D, D, fp16) &&
+            make_map(&t->tm[MAP_IN], t->w_in, (uint64_t)L * t->ROWS_IN, D, fp16) &&
+            make_map(&t->tm[MAP_M], t->w_m, (uint64_t)L * D, t->KM, fp16) &&
+            make_map(&t->tm[MAP_1], t->w_1, (uint64_t)L * D, D, fp16) &&
+            make_map(&t->tm[MAP_2], t->w_2, (uint64_t)L * D, D, fp16);
   if (!ok) return TRACKFIT_ERR_CUDA;
-  if (cudaFuncSetAttribute(tc_forward_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
-      cudaSuccess)
+  if (cudaFuncSetAttribute(tc_forward_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(tc_forward_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
+          cudaSuccess)
     return TRACKFIT_ERR_CUDA;
   return TRACKFIT_OK;
 }
@@ -1089,9 +1130,12 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   p.off_a = t->off_a;
   p.off_misc = t->off_misc;
   p.rms_eps = s.rms_eps;
+  p.fp16 = s.precision == TRACKFIT_FP16_PROJ;
   for (int f = 0; f < 5; ++f) {
+    const double inv = 1.0 / s.feat_range_d[f];
     p.feat_min[f] = s.feat_min[f];
-    p.feat_inv[f] = s.feat_inv_range[f];
+    p.feat_inv_hi[f] = (float)inv;
+    p.feat_inv_lo[f] = (float)(inv - (double)p.feat_inv_hi[f]);
   }
   for (int k = 0; k < 16; ++k) p.scale[k] = s.scale[k];
   for (int64_t c0 = 0; c0 < B; c0 += MAXB) {
@@ -1105,7 +1149,12 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
     p.out = out + c0 * 5;
     p.out_q = out_q ? out_q + c0 * s.Q : nullptr;
     p.out_pool = out_pool ? out_pool + c0 * s.P : nullptr;
-    tc_forward_kernel<<<t->nsm, NT, t->smem, st>>>(p);
+    tf_prof_begin(h, st);
+    if (p.fp16)
+      tc_forward_kernel<true><<<t->nsm, NT, t->smem, st>>>(p);
+    else
+      tc_forward_kernel<false><<<t->nsm, NT, t->smem, st>>>(p);
+    tf_prof_end(h, st);
     if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
   }
   return TRACKFIT_OK;

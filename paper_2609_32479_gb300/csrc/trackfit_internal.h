@@ -51,7 +51,17 @@ struct trackfit_ctx {
   float* st_out;
   int64_t st_cap;
   tf_tc_state* tc;
+  // optional timing of the main compute kernel (trackfit_profile)
+  int prof_on;
+  int prof_n;
+  cudaEvent_t prof_ev[2 * 64];
+  double prof_ms;
+  int64_t prof_launches;
 };
+
+// Record the start / end of the main kernel of one forward when profiling is on.
+void tf_prof_begin(trackfit_ctx* h, cudaStream_t st);
+void tf_prof_end(trackfit_ctx* h, cudaStream_t st);
 
 // simt.cu
 int tf_simt_workspace(trackfit_ctx* h);

@@ -23,7 +23,8 @@ ABI_VERSION = 1
 # every function declared in include/trackfit.h
 EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trackfit_forward_ex",
            "trackfit_forward_host", "trackfit_device_errors", "trackfit_path_name", "trackfit_set_path",
-           "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma")
+           "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma",
+           "trackfit_profile", "trackfit_profile_read")
 
 
 class Config(ctypes.Structure):
@@ -79,6 +80,10 @@ def load() -> ctypes.CDLL:
     lib.trackfit_debug_scan.restype = ctypes.c_int
     lib.trackfit_debug_umma.argtypes = [vp, vp, vp, i32, vp, vp]
     lib.trackfit_debug_umma.restype = ctypes.c_int
+    lib.trackfit_profile.argtypes = [vp, ctypes.c_int]
+    lib.trackfit_profile.restype = ctypes.c_int
+    lib.trackfit_profile_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64)]
+    lib.trackfit_profile_read.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -181,6 +186,19 @@ class Trackfit:
         n = ctypes.c_int64(0)
         st = self.lib.trackfit_device_errors(self._h, _stream_handle(stream), ctypes.byref(n))
         return st, int(n.value)
+
+    def profile(self, enable: bool) -> None:
+        st = self.lib.trackfit_profile(self._h, 1 if enable else 0)
+        if st != OK:
+            raise TrackfitError(st, "trackfit_profile")
+
+    def profile_read(self):
+        """(summed main-kernel milliseconds, timed launches) since the last read."""
+        ms, n = ctypes.c_double(0.0), ctypes.c_int64(0)
+        st = self.lib.trackfit_profile_read(self._h, ctypes.byref(ms), ctypes.byref(n))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_profile_read")
+        return ms.value, n.value
 
     def close(self) -> None:
         if getattr(self, "_h", None) is not None and self._h.value:

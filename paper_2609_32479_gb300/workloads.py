@@ -42,6 +42,7 @@ import numpy as np
 
 PRECISION_FP32 = 0
 PRECISION_BF16 = 1
+PRECISION_FP16 = 2
 POOL_MEAN = 0
 POOL_ENDPOINTS = 1
 
@@ -346,13 +347,33 @@ def _positions(kin, A, K, rng, w: Workload, smear: bool):
     return x, y, z
 
 
+GEN_CHUNK = 65536
+
+
 def gen_tracks(w: Workload, n_tracks: Optional[int] = None, seed: Optional[int] = None,
                smear: bool = True, pad_value: float = 0.0) -> TrackBatch:
     """Seeded synthetic helix tracks for workload w: hits [B, T, 5] fp32 in
-    (x, y, z, r, phi), n_hits [B] int32, pads filled with pad_value."""
+    (x, y, z, r, phi), n_hits [B] int32, pads filled with pad_value.
+
+    Tracks are drawn in chunks of GEN_CHUNK; chunk c uses the stream
+    PCG64(SeedSequence([seed, c])), so a batch is the same on every machine and
+    its memory use stays bounded."""
     B = w.n_tracks if n_tracks is None else int(n_tracks)
+    s0 = w.track_seed if seed is None else seed
+    parts = []
+    for c, b0 in enumerate(range(0, B, GEN_CHUNK)):
+        rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([s0, c])))
+        parts.append(_gen_chunk(w, min(GEN_CHUNK, B - b0), rng, smear, pad_value))
+    if len(parts) == 1:
+        return parts[0]
+    return TrackBatch(hits=np.concatenate([p.hits for p in parts]),
+                      n_hits=np.concatenate([p.n_hits for p in parts]),
+                      truth=np.concatenate([p.truth for p in parts]),
+                      kin={k: np.concatenate([p.kin[k] for p in parts]) for k in parts[0].kin})
+
+
+def _gen_chunk(w: Workload, B: int, rng, smear: bool, pad_value: float) -> TrackBatch:
     T = w.model.max_hits
-    rng = np.random.Generator(np.random.PCG64(w.track_seed if seed is None else seed))
     max_keep = MAX_TRACK_HITS if w.layout == "barrel_endcap" else T
 
     kin_all: Dict[str, List[np.ndarray]] = {}

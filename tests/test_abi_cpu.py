@@ -43,7 +43,7 @@ def test_weight_count_matches_layout(lib, name):
 
 @pytest.mark.parametrize("bad", [dict(d_model=24), dict(d_hidden=100), dict(max_hits=65), dict(max_hits=0),
                                  dict(n_layers=0), dict(n_layers=17), dict(head_hidden=64), dict(n_quantiles=6),
-                                 dict(precision=2), dict(pool=3), dict(n_fourier=8), dict(rms_eps=0.0),
+                                 dict(precision=3), dict(pool=3), dict(n_fourier=8), dict(rms_eps=0.0),
                                  dict(d_model=272, d_hidden=408)])
 def test_unsupported_configs_rejected_on_host(lib, bad):
     m = W.workload("tiny").model.with_(**bad)

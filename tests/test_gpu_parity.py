@@ -55,6 +55,7 @@ def oracle(model, blob, hits, n_hits, capture=None):
 
 CASES = [("tiny", None), ("small", None), ("medium", 1000), ("large", 300), ("sweep8", 515), ("sweep16", 300),
          ("sweep32", 200), ("sweep64", 130)]
+FP16_CASES = [("medium", 1000), ("large", 300), ("sweep8", 515), ("sweep64", 130)]
 
 
 @pytest.mark.parametrize("path", [0, 1], ids=["auto", "simt"])
@@ -71,6 +72,20 @@ def test_parity_against_oracle(T, name, n, path):
     print(f"{name} [{r['path']}] parity: {msg}; per parameter max {parity_error(r['out'], ref)}")
     assert r["status"] == 0 and r["n_bad"] == 0
     assert np.all(np.isfinite(r["out"]))
+    assert ok, msg
+
+
+@pytest.mark.parametrize("path", [0, 1], ids=["auto", "simt"])
+@pytest.mark.parametrize("name,n", FP16_CASES)
+def test_fp16_parity_against_oracle(T, name, n, path):
+    """fp16 operands (the format of Sec. 3.5) hold the 2e-3 bar on every track."""
+    w = W.workload(name, n_tracks=n, precision=W.PRECISION_FP16)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    r = run(T, w.model, blob, tb.hits, tb.n_hits, path=path)
+    ok, msg = parity_ok(r["out"], oracle(w.model, blob, tb.hits, tb.n_hits), w.model.precision)
+    print(f"{name} [{r['path']}] fp16 parity: {msg}")
+    assert r["path"].endswith("fp16")
     assert ok, msg
 
 
@@ -96,9 +111,9 @@ def test_full_size_sampled_parity(T, name):
     assert ok, msg
 
 
-@pytest.mark.parametrize("name", ["tiny", "medium"])
-def test_endpoint_pooling_parity(T, name):
-    w = W.workload(name, n_tracks=300, pool=W.POOL_ENDPOINTS)
+@pytest.mark.parametrize("name,prec", [("tiny", W.PRECISION_FP32), ("medium", W.PRECISION_FP16)])
+def test_endpoint_pooling_parity(T, name, prec):
+    w = W.workload(name, n_tracks=300, pool=W.POOL_ENDPOINTS, precision=prec)
     tb = W.gen_tracks(w)
     blob = W.gen_weights(w.model, 5)
     r = run(T, w.model, blob, tb.hits, tb.n_hits)

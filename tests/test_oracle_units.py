@@ -34,6 +34,14 @@ def test_bf16_round_matches_torch_on_fp32_values():
     np.testing.assert_array_equal(got, want)
 
 
+def test_fp16_round_matches_torch_on_fp32_values():
+    x = np.concatenate([rng.standard_normal(20000).astype(np.float32),
+                        (rng.standard_normal(2000) * 1e-6).astype(np.float32),     # fp16 subnormals
+                        np.array([0.0, 65504.0, 65520.0, 1e6, -1e6, 1.0 + 2.0 ** -11], np.float32)])
+    want = torch.from_numpy(x).to(torch.float16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.fp16_round(x.astype(np.float64)), want)
+
+
 def test_bf16_round_specials():
     v = np.array([np.inf, -np.inf, np.nan])
     got = O.bf16_round(v)
