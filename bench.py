@@ -1,0 +1,352 @@
+"""Throughput benchmark of the track-fit encoder on GB300.
+
+One step = one forward of the whole hot path (Fourier embedding, every minGRU
+layer, pooling, head) over the full synthetic batch of the workload (default:
+large, 1,048,576 tracks, d_model 256, 8 layers, bf16 operands).  Inputs are
+resident in HBM when the timed region starts; the hit batch (503 MB) is larger
+than L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload large] [--impl ours|reference]
+
+N > 1 runs under torch.distributed.run, one rank per GPU; every rank processes
+its own full batch (replicas, weak scaling; the path has no exchange step).
+--impl reference times the CPU oracle on bounded samples of the same workload
+(rank 0 only).  Prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import dataclasses
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_32479_gb300 import workloads as W  # noqa: E402
+
+METRIC = "tracks/sec at 1 GB300 (device-timed) and % of HBM/tensor roofline vs CPU oracle"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KERNEL_SRC = os.path.join(ROOT, "paper_2609_32479_gb300", "csrc", "tc_forward.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "tc_forward_large.traffic.json")
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as fh:
+            d = json.load(fh)
+        return d, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+def flops_per_hit(m: W.ModelConfig) -> int:
+    """Algorithmic multiply-add work per valid hit: embedding 2(E D + D^2) plus, per
+    layer, 2 D (4H + D) + 2 (2H) D + 2 (2 D^2) (= 24 D^2 at H = 1.5 D)."""
+    D, H, E = m.d_model, m.d_hidden, m.embed_dim
+    per_layer = 2 * D * (4 * H + D) + 2 * 2 * H * D + 4 * D * D
+    return 2 * (E * D + D * D) + m.n_layers * per_layer
+
+
+def flops_per_track_head(m: W.ModelConfig) -> int:
+    return 2 * (m.pooled_dim * m.head_hidden + m.head_hidden * m.n_out)
+
+
+def bytes_per_track(m: W.ModelConfig) -> int:
+    """Compulsory HBM traffic of one track: padded hits in, hit count in, 5 outputs out."""
+    return m.max_hits * 5 * 4 + 4 + 5 * 4
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.flush()
+        self.f.seek(0)
+        rows = [r.split(",") for r in self.f.read().strip().splitlines() if r.strip()]
+        os.unlink(self.f.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+                for n, v in zip(names, r[5:9]):
+                    if v.strip().lower() == "active":
+                        reasons.add(n)
+            except (ValueError, IndexError):
+                continue
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def stratified_sample(n_hits: np.ndarray, n: int, seed: int = 7) -> np.ndarray:
+    """n track indices covering every hit count present in proportion."""
+    rng = np.random.default_rng(seed)
+    idx = rng.choice(n_hits.size, size=min(n, n_hits.size), replace=False)
+    extra = [int(np.nonzero(n_hits == k)[0][0]) for k in np.unique(n_hits)]
+    return np.unique(np.concatenate([idx, extra]))
+
+
+def run_oracle_sample(w: W.Workload, blob, tb, budget_s: float):
+    """Time the CPU oracle (as it stands) on a bounded sample: returns
+    (tracks/s, sample indices, outputs, seconds)."""
+    from oracle import trackfit_oracle as O
+    cfg = dataclasses.asdict(w.model)
+    cal = stratified_sample(tb.n_hits, 64, seed=1)[:64]
+    t0 = time.perf_counter()
+    O.forward(cfg, blob, tb.hits[cal], tb.n_hits[cal])
+    per = (time.perf_counter() - t0) / len(cal)
+    n = int(max(16, min(4096, budget_s / max(per, 1e-6))))
+    idx = stratified_sample(tb.n_hits, n)
+    t0 = time.perf_counter()
+    out = np.concatenate([O.forward(cfg, blob, tb.hits[idx[i:i + 128]], tb.n_hits[idx[i:i + 128]])
+                          for i in range(0, idx.size, 128)])
+    dt = time.perf_counter() - t0
+    return idx.size / dt, idx, out, dt
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def config_block(w: W.Workload, tb) -> dict:
+    m = w.model
+    hist = W.length_histogram(tb.n_hits)
+    return {"workload": w.name, "n_tracks": w.n_tracks, "max_hits": m.max_hits, "d_model": m.d_model,
+            "d_hidden": m.d_hidden, "n_layers": m.n_layers, "pool": "mean" if m.pool == 0 else "endpoints",
+            "precision": {0: "fp32", 1: "bf16", 2: "fp16"}[m.precision],
+            "mean_hits": float(tb.n_hits.mean()), "hit_histogram": hist,
+            "l2": "inputs larger than L2 (hits %.0f MB > 129 MB); no flush" % (tb.hits.nbytes / 1e6),
+            "parallelism": "replicas"}
+
+
+def reference_main(args, w: W.Workload):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    budget = max(2.0, min(15.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        run_oracle_sample(w, blob, tb, min(budget, 3.0))
+    vals, tot_t, tot_n = [], 0.0, 0
+    for _ in range(args.steps):
+        v, idx, _, dt = run_oracle_sample(w, blob, tb, budget)
+        vals.append(v)
+        tot_t += dt
+        tot_n += idx.size
+    value = tot_n / tot_t
+    cores = host_cores()
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tracks/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": config_block(w, tb),
+            "cpu_baseline": {"value": value, "unit": "tracks/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{tot_n // args.steps} stratified tracks of {w.name} per step (numpy fp64)"},
+            "e2e": {"value": value, "unit": "tracks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def traffic_for_kernel():
+    """dram bytes per launch from the committed ncu summary, if it was taken on the
+    current kernel source (else null)."""
+    try:
+        with open(TRAFFIC_FILE) as fh:
+            d = json.load(fh)
+        with open(KERNEL_SRC, "rb") as fh:
+            h = hashlib.sha256(fh.read()).hexdigest()
+        if d.get("kernel_sha256") != h:
+            return None
+        return float(d["dram_bytes_per_launch_full"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="large")
+    ap.add_argument("--n-tracks", type=int, default=None)
+    ap.add_argument("--precision", choices=["config", "bf16", "fp16"], default="config")
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    kw = {}
+    if args.precision != "config":
+        kw["precision"] = W.PRECISION_BF16 if args.precision == "bf16" else W.PRECISION_FP16
+    w = W.workload(args.workload, n_tracks=args.n_tracks, **kw)
+    if args.impl == "reference":
+        return reference_main(args, w)
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    from paper_2609_32479_gb300 import trackfit as TF
+
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    m = w.model
+    B = w.n_tracks
+    tf = TF.Trackfit(m, blob)
+    hits = torch.from_numpy(tb.hits).to(dev)
+    n_hits = torch.from_numpy(tb.n_hits).to(dev)
+    out = torch.empty((B, 5), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(max(args.warmup, 0)):
+        tf.forward(hits, n_hits, out, stream)
+    torch.cuda.synchronize(dev)
+    st, nbad = tf.device_errors(stream)
+    if st not in (TF.OK, TF.ERR_BAD_HITS):
+        raise RuntimeError(f"device error status {st} during warm-up")
+
+    tf.profile(True)
+    tf.profile_read()
+    clocks = ClockSampler() if rank == 0 else None
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ev[0].record(stream)
+    for k in range(args.steps):
+        tf.forward(hits, n_hits, out, stream)
+        ev[k + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    if dist is not None:
+        dist.barrier()
+    clk = clocks.stop() if clocks else None
+    step_ms = [ev[k].elapsed_time(ev[k + 1]) for k in range(args.steps)]
+    total_ms = ev[0].elapsed_time(ev[args.steps])
+    kern_ms, kern_n = tf.profile_read()
+    tf.profile(False)
+    st, nbad = tf.device_errors(stream)
+    if dist is not None:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    n_ranks = world
+    value = n_ranks * B * args.steps / (total_ms * 1e-3)
+
+    # ---- end to end through the C-ABI with host buffers (pinned), copies inside
+    gpu_out = out.cpu().numpy()
+    e2e_value, same = None, None
+    if args.e2e_steps > 0:
+        hits_h = torch.from_numpy(tb.hits).pin_memory()
+        n_h = torch.from_numpy(tb.n_hits).pin_memory()
+        out_h = torch.empty((B, 5), dtype=torch.float32).pin_memory()
+        tf.forward_host_ptr(hits_h.data_ptr(), n_h.data_ptr(), B, out_h.data_ptr(), stream)
+        if dist is not None:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            tf.forward_host_ptr(hits_h.data_ptr(), n_h.data_ptr(), B, out_h.data_ptr(), stream)
+        e2e_s = time.perf_counter() - t0
+        if dist is not None:
+            t = torch.tensor([e2e_s], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        e2e_value = n_ranks * B * args.e2e_steps / e2e_s
+        same = bool(np.array_equal(out_h.numpy(), gpu_out))
+
+    if rank != 0:
+        tf.close()
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+
+    peaks, peak_kind = load_peaks()
+    valid_hits = int(tb.n_hits.clip(0, m.max_hits).sum())
+    flops = valid_hits * flops_per_hit(m) + B * flops_per_track_head(m)
+    kern_avg_s = (kern_ms / max(kern_n, 1)) * 1e-3
+    dtype_tf = {1: "bf16_tflops", 2: "bf16_tflops"}.get(m.precision, "bf16_tflops")
+    peak = float(peaks.get(dtype_tf, FALLBACK_PEAKS["bf16_tflops"]))
+    peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    achieved = flops / kern_avg_s / 1e12 if kern_n else None
+    traffic = traffic_for_kernel()
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                "peak_kind": f"{peak_kind} bf16 dense burst (fp16 runs at the bf16 rate)",
+                "frac_of_sustained": (achieved / peak_sus) if achieved else None,
+                "kernel": "tc_forward_kernel" if tf.path.startswith("tcgen05") else "simt layer sequence",
+                "kernel_ms_avg": kern_avg_s * 1e3, "flops_per_launch": flops,
+                "algorithmic_bytes_per_launch": B * bytes_per_track(m),
+                "hbm_frac_of_time": (B * bytes_per_track(m) / (peaks.get("hbm_gbs", 6800.0) * 1e9)) / kern_avg_s
+                if kern_n else None}
+    line = {"metric": METRIC, "value": value, "unit": "tracks/s", "n_gpus": n_ranks, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+            "ms_per_step_min": float(min(step_ms)), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": {0: "f32", 1: "bf16", 2: "f16"}[m.precision],
+            "data": "synthetic helix tracks + random-init weights (seeded)", "config": config_block(w, tb),
+            "path": tf.path, "roofline": roofline, "clocks": clk,
+            "e2e": {"value": e2e_value, "unit": "tracks/s", "h2d_bytes_per_step": int(tb.hits.nbytes + tb.n_hits.nbytes),
+                    "d2h_bytes_per_step": int(B * 5 * 4), "matches_device_result": same},
+            "gpu_launches": int(4 * math.ceil(B / 4194304) * args.steps) if tf.path.startswith("tcgen05") else None,
+            "device_errors": {"status": st, "bad_tracks": nbad}}
+    if not args.no_cpu_baseline and world == 1:
+        v, idx, ref, dt = run_oracle_sample(w, blob, tb, args.cpu_budget)
+        from tests.helpers import normalised_errors
+        e = normalised_errors(gpu_out[idx], ref)
+        line["cpu_baseline"] = {"value": v, "unit": "tracks/s", "cores": host_cores(), "kind": "oracle",
+                                "sample": f"{idx.size} stratified tracks of {w.name} (numpy fp64, {dt:.1f} s)"}
+        line["parity_on_sample"] = {"tracks": int(idx.size), "p90": float(np.percentile(e, 90)),
+                                    "max": float(e.max())}
+    tf.close()
+    print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

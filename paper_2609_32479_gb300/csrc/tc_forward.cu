@@ -258,43 +258,51 @@ __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
   }
 }
 
-// X = [xs +] acc + bias, zero on pad columns, stored to xs; then either the
-// RMS-normalised x_hat -> XB (next layer's projection operand) or mean pooling.
+// X = acc + bias [+ x'], zero on pad columns.  x' (the gated residual of this
+// layer) sits in TMEM columns 256.. where the gate epilogue left it.  X goes to
+// the per-CTA scratch (read back once, by the next layer's gate epilogue), then
+// either the RMS-normalised x_hat -> XB (recomputing X from TMEM) or mean pooling.
 template <bool FP16>
-__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bool add_xs, const float* gain,
+__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bool add_x1, const float* gain,
                                             bool pool) {
   const TcParams& p = *x.p;
   const int D = p.D;
+  const uint8_t* flags = x.m->col_flags;
   float run[2] = {0.0f, 0.0f};
 #pragma unroll 1
   for (int ch = 0; ch < 2; ++ch) {
     float sq[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
+#pragma unroll 1
     for (int mt = 0; mt < x.MT; ++mt) {
       const int ch_g = mt * 128 + x.c;
       const float b = bias[ch_g];
-      float v[32];
+      float v[32], r[32];
       tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, v);
+      if (add_x1) tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, r);
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
         const int col = x.col0 + 32 * ch + i;
-        float* xp = x.xs + (size_t)col * D + ch_g;
         float val = v[i] + b;
-        if (add_xs) val += *xp;
-        const int fl = x.m->col_flags[col];
+        if (add_x1) val += r[i];
+        const int fl = flags[col];
         val = (fl & F_VALID) ? val : 0.0f;
-        *xp = val;
+        v[i] = val;
         sq[i] = fmaf(val, val, sq[i]);
         if (pool) {
-          if (fl & F_FIRST) run[mt] = 0.0f;
-          run[mt] += val;
+          run[mt] = (fl & F_FIRST) ? val : run[mt] + val;
           if (fl & F_LAST) {
             const int s = x.m->col_slot[col];
             x.pooled[s * D + ch_g] = run[mt] / (float)x.m->slot_n[s];
           }
         }
+      }
+      if (!pool) {
+        float* xp = x.xs + (size_t)(x.col0 + 32 * ch) * D + ch_g;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) xp[(size_t)i * D] = v[i];
       }
     }
     if (!pool) {
@@ -309,48 +317,57 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
     x.m->rinv[x.te] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
   }
   ebar_sync();
+#pragma unroll 1
   for (int mt = 0; mt < x.MT; ++mt) {
     const int ch_g = mt * 128 + x.c;
+    const float b = bias[ch_g];
     const float g = gain[ch_g];
 #pragma unroll 1
     for (int ch = 0; ch < 2; ++ch) {
-      float v[32];
+      float v[32], r[32];
+      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, v);
+      if (add_x1) tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, r);
+      tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
         const int col = x.col0 + 32 * ch + i;
-        v[i] = x.xs[(size_t)col * D + ch_g] * g * x.m->rinv[col];
+        float val = v[i] + b;
+        if (add_x1) val += r[i];
+        val = (flags[col] & F_VALID) ? val : 0.0f;
+        v[i] = val * g * x.m->rinv[col];
       }
       store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, v);
     }
   }
 }
 
-// x' = X + (M + b_m) * sigma(p_g + b_g) -> xs and XB
+// x' = X + (M + b_m) * sigma(p_g + b_g) -> TMEM columns 256.. (in place of the gate
+// projection) and XB.  X is read back from the scratch with one batch of loads.
 template <bool FP16>
 __device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
   const TcParams& p = *x.p;
   const int D = p.D;
+#pragma unroll 1
   for (int mt = 0; mt < x.MT; ++mt) {
     const int ch_g = mt * 128 + x.c;
     const float bm = p.b_m[l * D + ch_g];
     const float bg = p.b_in[(size_t)l * p.ROWS_IN + p.NDC * 256 + ch_g];
 #pragma unroll 1
     for (int ch = 0; ch < 2; ++ch) {
-      float mv[32], gv[32];
+      float xv[32], mv[32], gv[32];
+      const float* xp = x.xs + (size_t)(x.col0 + 32 * ch) * D + ch_g;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) xv[i] = xp[(size_t)i * D];
       tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, mv);
       tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, gv);
       tmem_ld_wait();
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int col = x.col0 + 32 * ch + i;
-        float* xp = x.xs + (size_t)col * D + ch_g;
-        const float x1 = *xp + (mv[i] + bm) * sigm(gv[i] + bg);
-        *xp = x1;
-        mv[i] = x1;
-      }
+      for (int i = 0; i < 32; ++i) mv[i] = xv[i] + (mv[i] + bm) * sigm(gv[i] + bg);
+      tmem_st32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, mv);
       store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, mv);
     }
   }
+  tmem_st_wait();
 }
 
 // Scan chunk dc (channel block dc/2, direction dc%2) of layer l -> HB.
@@ -371,8 +388,10 @@ __device__ __forceinline__ void ep_scan(const ECtx& x, int l, int dc) {
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
         const int fl = flags[x.col0 + 32 * ch + i];
-        if (fl & F_FIRST) h = 0.0f;
-        if (fl & F_VALID) h = fmaf(sigm(z[i] + bz), (n[i] + bn) - h, h);
+        const float zz = sigm(z[i] + bz), nn = n[i] + bn;
+        h = (fl & F_FIRST) ? 0.0f : h;
+        const float hn = fmaf(zz, nn - h, h);
+        h = (fl & F_VALID) ? hn : h;
         z[i] = (fl & F_VALID) ? h : 0.0f;
       }
       store_row32<FP16>(x.hb, x.c, x.col0 + 32 * ch, z);
@@ -387,8 +406,10 @@ __device__ __forceinline__ void ep_scan(const ECtx& x, int l, int dc) {
 #pragma unroll
       for (int i = 31; i >= 0; --i) {
         const int fl = flags[x.col0 + 32 * ch + i];
-        if (fl & F_LAST) h = 0.0f;
-        if (fl & F_VALID) h = fmaf(sigm(z[i] + bz), (n[i] + bn) - h, h);
+        const float zz = sigm(z[i] + bz), nn = n[i] + bn;
+        h = (fl & F_LAST) ? 0.0f : h;
+        const float hn = fmaf(zz, nn - h, h);
+        h = (fl & F_VALID) ? hn : h;
         z[i] = (fl & F_VALID) ? h : 0.0f;
       }
       store_row32<FP16>(x.hb, x.c, x.col0 + 32 * ch, z);
@@ -507,11 +528,15 @@ __device__ __forceinline__ void ep_head(const ECtx& x) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) a[i] = b1;
     const float* pv = x.pooled + (size_t)(sg * 16) * D;
-#pragma unroll 2
-    for (int cc = 0; cc < D; ++cc) {
-      const float w = p.head_w1t[cc * 128 + j];
+#pragma unroll 1
+    for (int c0 = 0; c0 < D; c0 += 16) {
+      float w[16];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) a[i] = fmaf(w, pv[i * D + cc], a[i]);
+      for (int u = 0; u < 16; ++u) w[u] = p.head_w1t[(c0 + u) * 128 + j];
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+#pragma unroll
+        for (int i = 0; i < 16; ++i) a[i] = fmaf(w[u], pv[i * D + c0 + u], a[i]);
     }
 #pragma unroll
     for (int i = 0; i < 16; ++i)
@@ -523,8 +548,14 @@ __device__ __forceinline__ void ep_head(const ECtx& x) {
     const float* w = p.head_w2 + (size_t)o * 128;
     const float* hv = x.hid + s * 128;
     float acc = p.head_b2[o];
-#pragma unroll 8
-    for (int j = 0; j < 128; ++j) acc = fmaf(w[j], hv[j], acc);
+#pragma unroll 1
+    for (int j0 = 0; j0 < 128; j0 += 16) {
+      float wv[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) wv[u] = w[j0 + u];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) acc = fmaf(wv[u], hv[j0 + u], acc);
+    }
     const size_t trk = (size_t)m->slot_track[s];
     if (m->slot_bad[s]) acc = __int_as_float(0x7fc00000);
     if (p.out_q) p.out_q[trk * p.Q + o] = acc;
@@ -696,7 +727,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       ep_silu<FP16>(x, p.b_e1);
       signal();
       if (!wait_acc()) break;
-      ep_residual<FP16>(x, p.b_e2, false, p.g, false);
+      ep_residual<FP16>(x, p.b_e2, false, p.g, false);   // embedding output X0
       signal();
       bool ok = true;
       for (int l = 0; l < p.L && ok; ++l) {
