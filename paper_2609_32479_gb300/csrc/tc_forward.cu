@@ -268,7 +268,7 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
   const TcParams& p = *x.p;
   const int D = p.D;
   const uint8_t* flags = x.m->col_flags;
-  float run[2] = {0.0f, 0.0f};
+  float run0 = 0.0f, run1 = 0.0f;
 #pragma unroll 1
   for (int ch = 0; ch < 2; ++ch) {
     float sq[32];
@@ -276,6 +276,7 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
     for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
 #pragma unroll 1
     for (int mt = 0; mt < x.MT; ++mt) {
+      float run = mt ? run1 : run0;
       const int ch_g = mt * 128 + x.c;
       const float b = bias[ch_g];
       float v[32], r[32];
@@ -292,13 +293,14 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
         v[i] = val;
         sq[i] = fmaf(val, val, sq[i]);
         if (pool) {
-          run[mt] = (fl & F_FIRST) ? val : run[mt] + val;
+          run = (fl & F_FIRST) ? val : run + val;
           if (fl & F_LAST) {
             const int s = x.m->col_slot[col];
-            x.pooled[s * D + ch_g] = run[mt] / (float)x.m->slot_n[s];
+            x.pooled[s * D + ch_g] = run / (float)x.m->slot_n[s];
           }
         }
       }
+      if (mt) run1 = run; else run0 = run;
       if (!pool) {
         float* xp = x.xs + (size_t)(x.col0 + 32 * ch) * D + ch_g;
 #pragma unroll
@@ -372,10 +374,7 @@ __device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
 
 // Scan chunk dc (channel block dc/2, direction dc%2) of layer l -> HB.
 template <bool FP16>
-__device__ __forceinline__ void ep_scan(const ECtx& x, int l, int dc) {
-  const TcParams& p = *x.p;
-  const size_t rb = (size_t)l * p.ROWS_IN + dc * 256;
-  const float bz = p.b_in[rb + x.c], bn = p.b_in[rb + 128 + x.c];
+__device__ __forceinline__ void ep_scan(const ECtx& x, int dc, float bz, float bn) {
   const uint8_t* flags = x.m->col_flags;
   float h = 0.0f;
   if ((dc & 1) == 0) {
@@ -732,8 +731,11 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       bool ok = true;
       for (int l = 0; l < p.L && ok; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
+          // biases are loaded before the wait so their latency hides behind it
+          const size_t rb = (size_t)l * p.ROWS_IN + dc * 256;
+          const float bz = p.b_in[rb + x.c], bn = p.b_in[rb + 128 + x.c];
           if (!(ok = wait_acc())) break;
-          ep_scan<FP16>(x, l, dc);
+          ep_scan<FP16>(x, dc, bz, bn);
           signal();
         }
         if (!ok || !(ok = wait_acc())) break;
