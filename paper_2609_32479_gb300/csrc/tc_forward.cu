@@ -238,6 +238,7 @@ struct ECtx {
   float* xs;
   float* pooled;
   float* hid;
+  float* w2s;   // staged W_h2 [Q][128]
   int q, lane, half, c, col0, te, e, MT;
 };
 
@@ -501,10 +502,15 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
 }
 
 // Pooled vectors -> RMSNorm -> 2-layer head -> outputs (fp32 CUDA cores).
+// pooled: [32][D] in the HB region; the XB region holds the hidden layer
+// [32][128] and a copy of W_h2 [Q][128] staged with coalesced loads.
 __device__ __forceinline__ void ep_head(const ECtx& x) {
   const TcParams& p = *x.p;
   Misc* m = x.m;
   const int D = p.D, ns = m->n_slots;
+  float* w2s = x.w2s;
+  for (int i = x.te; i < p.Q * 32; i += NE)   // stage W_h2 as float4s
+    reinterpret_cast<float4*>(w2s)[i] = reinterpret_cast<const float4*>(p.head_w2)[i];
   for (int s = x.e; s < ns; s += 8) {
     const size_t trk = (size_t)m->slot_track[s];
     const bool bad = m->slot_bad[s] != 0;
@@ -521,39 +527,57 @@ __device__ __forceinline__ void ep_head(const ECtx& x) {
   }
   ebar_sync();
   {
+    // thread: hidden unit j, slots sg, sg + 2, ... (only the tile's slots)
     const int j = x.te & 127, sg = x.te >> 7;
+    const int nmine = (ns - sg + 1) >> 1;
     float a[16];
     const float b1 = p.head_b1[j];
 #pragma unroll
     for (int i = 0; i < 16; ++i) a[i] = b1;
-    const float* pv = x.pooled + (size_t)(sg * 16) * D;
+    float w[8], wn[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) w[u] = p.head_w1t[u * 128 + j];
 #pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 16) {
-      float w[16];
+    for (int c0 = 0; c0 < D; c0 += 8) {
+      if (c0 + 8 < D) {
 #pragma unroll
-      for (int u = 0; u < 16; ++u) w[u] = p.head_w1t[(c0 + u) * 128 + j];
+        for (int u = 0; u < 8; ++u) wn[u] = p.head_w1t[(c0 + 8 + u) * 128 + j];
+      }
 #pragma unroll
-      for (int u = 0; u < 16; ++u)
+      for (int i = 0; i < 16; ++i) {
+        if (i < nmine) {
+          const float4* pv = reinterpret_cast<const float4*>(x.pooled + (size_t)(sg + 2 * i) * D + c0);
+          const float4 p0 = pv[0], p1 = pv[1];
+          a[i] = fmaf(w[0], p0.x, a[i]);
+          a[i] = fmaf(w[1], p0.y, a[i]);
+          a[i] = fmaf(w[2], p0.z, a[i]);
+          a[i] = fmaf(w[3], p0.w, a[i]);
+          a[i] = fmaf(w[4], p1.x, a[i]);
+          a[i] = fmaf(w[5], p1.y, a[i]);
+          a[i] = fmaf(w[6], p1.z, a[i]);
+          a[i] = fmaf(w[7], p1.w, a[i]);
+        }
+      }
 #pragma unroll
-        for (int i = 0; i < 16; ++i) a[i] = fmaf(w[u], pv[i * D + c0 + u], a[i]);
+      for (int u = 0; u < 8; ++u) w[u] = wn[u];
     }
 #pragma unroll
     for (int i = 0; i < 16; ++i)
-      if (sg * 16 + i < ns) x.hid[(sg * 16 + i) * 128 + j] = silu(a[i]);
+      if (i < nmine) x.hid[(sg + 2 * i) * 128 + j] = silu(a[i]);
   }
   ebar_sync();
   for (int idx = x.te; idx < ns * p.Q; idx += NE) {
     const int s = idx / p.Q, o = idx - s * p.Q;
-    const float* w = p.head_w2 + (size_t)o * 128;
-    const float* hv = x.hid + s * 128;
+    const float4* w = reinterpret_cast<const float4*>(w2s + o * 128);
+    const float4* hv = reinterpret_cast<const float4*>(x.hid + s * 128);
     float acc = p.head_b2[o];
-#pragma unroll 1
-    for (int j0 = 0; j0 < 128; j0 += 16) {
-      float wv[16];
-#pragma unroll
-      for (int u = 0; u < 16; ++u) wv[u] = w[j0 + u];
-#pragma unroll
-      for (int u = 0; u < 16; ++u) acc = fmaf(wv[u], hv[j0 + u], acc);
+#pragma unroll 8
+    for (int j4 = 0; j4 < 32; ++j4) {
+      const float4 a4 = w[j4], h4 = hv[j4];
+      acc = fmaf(a4.x, h4.x, acc);
+      acc = fmaf(a4.y, h4.y, acc);
+      acc = fmaf(a4.z, h4.z, acc);
+      acc = fmaf(a4.w, h4.w, acc);
     }
     const size_t trk = (size_t)m->slot_track[s];
     if (m->slot_bad[s]) acc = __int_as_float(0x7fc00000);
@@ -639,6 +663,8 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     if (lane == 0) {
       uint32_t stage = 0, phase = 0, e_phase = 0;
       bool ok = true, need_e = true;
+      const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
+      const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
         walk_tile(p, [&](int, int, int, int nk, int tcol, int bsel, int bk, int acc, int end) {
           if (!ok) return;
@@ -658,12 +684,17 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
             return;
           }
           tc_fence_after();
-          const uint32_t a_addr = ab + stage * A_STAGE;
-          const uint32_t b_addr = bsel == BSEL_HB ? hb : xb;
-          for (int k = 0; k < nk; ++k) {
-            const uint64_t ad = sdesc_sw128(a_addr + 32 * k, 16, 1024);
-            const uint64_t bd = sdesc_sw128(b_addr + ((bk + 16 * k) >> 3) * B_SBO, B_LBO, B_SBO);
-            umma_f16(tmem + (uint32_t)tcol, ad, bd, p.idesc, (acc || k) ? 1u : 0u);
+          // descriptors advance by plain adds: 32 B per K=16 step inside a
+          // 128-byte swizzled weight row, two 8-row groups (2 x 2 KB) per step
+          // of the activation operand
+          const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE) >> 4);
+          const uint64_t bd = (bsel == BSEL_HB ? b_desc_hb : b_desc_xb) + (uint64_t)(((bk >> 3) * B_SBO) >> 4);
+          const uint32_t d = tmem + (uint32_t)tcol;
+          umma_f16(d, ad, bd, p.idesc, acc ? 1u : 0u);
+          umma_f16(d, ad + 2, bd + (2 * B_SBO >> 4), p.idesc, 1u);
+          if (nk == 4) {
+            umma_f16(d, ad + 4, bd + (4 * B_SBO >> 4), p.idesc, 1u);
+            umma_f16(d, ad + 6, bd + (6 * B_SBO >> 4), p.idesc, 1u);
           }
           umma_commit(empty0 + 8 * stage);
           if (end) {
@@ -699,6 +730,10 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     x.xs = p.xs + (size_t)blockIdx.x * TILE * p.D;
     x.pooled = reinterpret_cast<float*>(gbase + p.off_hb);
     x.hid = reinterpret_cast<float*>(gbase + p.off_xb);
+    // W_h2 goes after the hidden layer in XB when it fits (d_model 256), else after
+    // the pooled vectors in the HB region (d_model 128)
+    x.w2s = (p.D * 256 >= (MAX_TRK_TILE + p.Q) * 128 * 4) ? x.hid + MAX_TRK_TILE * 128
+                                                           : x.pooled + MAX_TRK_TILE * p.D;
     uint32_t acc_phase = 0;
     auto signal = [&]() {
       fence_proxy_async_smem();
@@ -1016,7 +1051,9 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   if (t->nst < 2) return TRACKFIT_ERR_UNSUPPORTED;
   t->off_misc = t->off_a + t->nst * A_STAGE;
   t->smem = (size_t)t->off_misc + MISC_BYTES + 1024;
-  if ((size_t)(MAX_TRK_TILE * D * 4) > (size_t)EB_BYTES || MAX_TRK_TILE * 128 * 4 > D * 256)
+  const bool w2_in_xb = D * 256 >= (MAX_TRK_TILE + s.Q) * 128 * 4;
+  if (MAX_TRK_TILE * 128 * 4 > D * 256 ||
+      (size_t)(MAX_TRK_TILE * D + (w2_in_xb ? 0 : s.Q * 128)) * 4 > (size_t)EB_BYTES)
     return TRACKFIT_ERR_UNSUPPORTED;
 
   // ---- repack weights (bf16 GEMM operands, fp32 biases/head)
