@@ -609,7 +609,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       mbar_init(empty0 + 8 * s, 1);
     }
     mbar_init(acc_bar, 1);
-    mbar_init(e_bar, NE);
+    mbar_init(e_bar, 1);
     mbar_init(drain_bar, 1);
     m->abort_flag = 0;
     fence_mbar_init();
@@ -735,17 +735,22 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     x.w2s = (p.D * 256 >= (MAX_TRK_TILE + p.Q) * 128 * 4) ? x.hid + MAX_TRK_TILE * 128
                                                            : x.pooled + MAX_TRK_TILE * p.D;
     uint32_t acc_phase = 0;
+    // Every thread makes its shared-memory operand writes visible to the async
+    // proxy and orders its TMEM reads, the named barrier collects them, then a
+    // single arrival hands the phase to the MMA issuer.
     auto signal = [&]() {
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(e_bar);
+      ebar_sync();
+      if (x.te == 0) mbar_arrive(e_bar);
     };
-    // The outcome of a wait is made uniform across the epilogue threads (they
-    // share named barriers); the wait itself ignores the abort flag so that a
-    // completed phase is seen by all of them.
-    volatile int no_abort = 0;
+    // One elected epilogue thread polls the barrier; the others wait in the
+    // hardware named barrier (no shared-memory polling traffic competing with
+    // the tensor core's operand reads).  The vote makes the outcome uniform; the
+    // barrier also orders the shared-memory view for all participants.
     auto wait_acc = [&]() -> bool {
-      const bool mine = mbar_wait(acc_bar, acc_phase, &no_abort, WAIT_NS);
+      bool mine = true;
+      if (x.te == 0) mine = mbar_wait(acc_bar, acc_phase, abort, WAIT_NS);
       if (!ebar_all(mine)) {
         set_abort(m, p.err);
         return false;
