@@ -43,7 +43,8 @@ constexpr int TILE = 128;
 constexpr int SLAB = 64;
 constexpr int MAX_TRK_SLAB = 16;
 constexpr int MAX_TRK_TILE = 2 * MAX_TRK_SLAB;
-constexpr int A_STAGE = 128 * 64 * 2;     // one 128-row x 64-k bf16 weight block
+constexpr int A_BLOCK = 128 * 64 * 2;     // one 128-row x 64-k 16-bit weight block
+constexpr int A_STAGE = 2 * A_BLOCK;      // a pipeline stage holds two consecutive blocks
 constexpr int EB_BYTES = 160 * 256;       // Fourier operand: 160 k-rows x 128 hits bf16
 constexpr int MISC_BYTES = 8192;
 constexpr int MAX_STAGES = 8;
@@ -373,12 +374,14 @@ __device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
   tmem_st_wait();
 }
 
-// Scan chunk dc (channel block dc/2, direction dc%2) of layer l -> HB.
+// Scan chunk dc of one layer -> HB.  The chunk holds 64 channels of both
+// directions: TMEM lanes 0-63 (quadrants 0, 1) run the forward recurrence over
+// the hits in time order, lanes 64-127 (quadrants 2, 3) the reverse one.
 template <bool FP16>
 __device__ __forceinline__ void ep_scan(const ECtx& x, int dc, float bz, float bn) {
   const uint8_t* flags = x.m->col_flags;
   float h = 0.0f;
-  if ((dc & 1) == 0) {
+  if (x.q < 2) {   // lanes 0-63 of the chunk: forward direction
 #pragma unroll 1
     for (int ch = 0; ch < 2; ++ch) {
       float z[32], n[32];
@@ -628,33 +631,50 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   const int n_tiles = (n_slabs + 1) >> 1;
   volatile int* abort = &m->abort_flag;
 
+  // Blocks are consumed in walk order; a stage holds two consecutive blocks
+  // (one full-barrier wait and one release per 8 MMAs).  Both roles count the
+  // blocks of this CTA so the last stage may hold a single block.
+  int total_blocks = 0;
+  if (warp < 2 && lane == 0) {
+    int my_tiles = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
+    int per_tile = 0;
+    walk_tile(p, [&](int, int, int, int, int, int, int, int, int) { ++per_tile; });
+    total_blocks = per_tile * my_tiles;
+  }
   if (warp == 0) {
     if (lane == 0) {
       uint32_t stage = 0, phase = 0;
       bool ok = true;
-      int issued = 0;
+      int issued = 0, half = 0;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
         walk_tile(p, [&](int map, int row, int col, int, int, int, int, int, int) {
           if (!ok) return;
-          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
-            set_abort(m, p.err);
-            ok = false;
-            return;
+          if (half == 0) {
+            if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
+              set_abort(m, p.err);
+              ok = false;
+              return;
+            }
+            mbar_arrive_expect_tx(full0 + 8 * stage, issued + 1 < total_blocks ? A_STAGE : A_BLOCK);
           }
-          mbar_arrive_expect_tx(full0 + 8 * stage, A_STAGE);
-          tma_load_2d(ab + stage * A_STAGE, &p.tm[map], full0 + 8 * stage, col, row);
+          tma_load_2d(ab + stage * A_STAGE + half * A_BLOCK, &p.tm[map], full0 + 8 * stage, col, row);
           ++issued;
-          if (++stage == (uint32_t)p.nst) {
-            stage = 0;
-            phase ^= 1u;
+          if (++half == 2) {
+            half = 0;
+            if (++stage == (uint32_t)p.nst) {
+              stage = 0;
+              phase ^= 1u;
+            }
           }
         });
       }
       if (!ok) {
         // let the copies already issued land before the CTA can exit
         volatile int never = 0;
-        for (int k = 0; k < p.nst && k < issued; ++k) {
-          const int i = issued - 1 - k;
+        const int stages_used = (issued + 1) / 2;
+        for (int k = 0; k < p.nst && k < stages_used; ++k) {
+          const int i = stages_used - 1 - k;
           mbar_wait(full0 + 8 * (i % p.nst), (uint32_t)((i / p.nst) & 1), &never, DRAIN_NS);
         }
       }
@@ -665,6 +685,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       bool ok = true, need_e = true;
       const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
       const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
+      int half = 0, consumed = 0;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
         walk_tile(p, [&](int, int, int, int nk, int tcol, int bsel, int bk, int acc, int end) {
           if (!ok) return;
@@ -678,16 +699,18 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
             need_e = false;
             tc_fence_after();
           }
-          if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
-            set_abort(m, p.err);
-            ok = false;
-            return;
+          if (half == 0) {
+            if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
+              set_abort(m, p.err);
+              ok = false;
+              return;
+            }
+            tc_fence_after();
           }
-          tc_fence_after();
           // descriptors advance by plain adds: 32 B per K=16 step inside a
           // 128-byte swizzled weight row, two 8-row groups (2 x 2 KB) per step
           // of the activation operand
-          const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE) >> 4);
+          const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE + half * A_BLOCK) >> 4);
           const uint64_t bd = (bsel == BSEL_HB ? b_desc_hb : b_desc_xb) + (uint64_t)(((bk >> 3) * B_SBO) >> 4);
           const uint32_t d = tmem + (uint32_t)tcol;
           umma_f16(d, ad, bd, p.idesc, acc ? 1u : 0u);
@@ -696,14 +719,18 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
             umma_f16(d, ad + 4, bd + (4 * B_SBO >> 4), p.idesc, 1u);
             umma_f16(d, ad + 6, bd + (6 * B_SBO >> 4), p.idesc, 1u);
           }
-          umma_commit(empty0 + 8 * stage);
           if (end) {
             umma_commit(acc_bar);
             need_e = true;
           }
-          if (++stage == (uint32_t)p.nst) {
-            stage = 0;
-            phase ^= 1u;
+          ++consumed;
+          if (++half == 2 || consumed == total_blocks) {
+            umma_commit(empty0 + 8 * stage);
+            half = 0;
+            if (++stage == (uint32_t)p.nst) {
+              stage = 0;
+              phase ^= 1u;
+            }
           }
         });
       }
@@ -887,8 +914,8 @@ __global__ void __launch_bounds__(128, 1) umma_probe_kernel(const __grid_constan
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
   const uint32_t a_s = base;                 // K/64 blocks of 16 KB
-  const uint32_t b_s = base + (K / 64) * A_STAGE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(gbase + (K / 64) * A_STAGE + K * 256);
+  const uint32_t b_s = base + (K / 64) * A_BLOCK;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(gbase + (K / 64) * A_BLOCK + K * 256);
   uint32_t* tbase = reinterpret_cast<uint32_t*>(bars + 2);
   int* abortp = reinterpret_cast<int*>(bars + 3);
   const uint32_t tma_bar = smem_u32(&bars[0]), mma_bar = smem_u32(&bars[1]);
@@ -919,14 +946,14 @@ __global__ void __launch_bounds__(128, 1) umma_probe_kernel(const __grid_constan
   volatile int* abort = abortp;
   bool ok = true;
   if (threadIdx.x == 0) {
-    mbar_arrive_expect_tx(tma_bar, (K / 64) * A_STAGE);
-    for (int kc = 0; kc < K / 64; ++kc) tma_load_2d(a_s + kc * A_STAGE, &tmA, tma_bar, kc * 64, 0);
+    mbar_arrive_expect_tx(tma_bar, (K / 64) * A_BLOCK);
+    for (int kc = 0; kc < K / 64; ++kc) tma_load_2d(a_s + kc * A_BLOCK, &tmA, tma_bar, kc * 64, 0);
     ok = mbar_wait(tma_bar, 0, abort, WAIT_NS);
     if (ok) {
       tc_fence_after();
       for (int kc = 0; kc < K / 64; ++kc)
         for (int k = 0; k < 4; ++k) {
-          const uint64_t ad = sdesc_sw128(a_s + kc * A_STAGE + 32 * k, 16, 1024);
+          const uint64_t ad = sdesc_sw128(a_s + kc * A_BLOCK + 32 * k, 16, 1024);
           const uint64_t bd = sdesc_sw128(b_s + ((kc * 64 + 16 * k) >> 3) * B_SBO, B_LBO, B_SBO);
           umma_f16(tmem, ad, bd, idesc, (kc || k) ? 1u : 0u);
         }
@@ -1016,7 +1043,7 @@ struct tf_tc_state {
 
 bool tf_tc_supported(const tf_shape& s) {
   return (s.precision == TRACKFIT_BF16_PROJ || s.precision == TRACKFIT_FP16_PROJ) && s.pool == TRACKFIT_POOL_MEAN && (s.D == 128 || s.D == 256) &&
-         s.T <= 64 && s.Hh == 128 && s.Q <= 75 && s.F == 5 && s.K == 16;
+         s.H % 64 == 0 && s.T <= 64 && s.Hh == 128 && s.Q <= 75 && s.F == 5 && s.K == 16;
 }
 
 void tf_tc_destroy(trackfit_ctx* h) {
@@ -1036,8 +1063,7 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   if (!t) return TRACKFIT_ERR_OOM;
   h->tc = t;
   const int D = s.D, H = s.H, L = s.L, E = s.E;
-  const int nchunk = (H + 127) / 128;
-  t->NDC = 2 * nchunk;
+  t->NDC = H / 64;
   t->ROWS_IN = t->NDC * 256 + D;
   t->KM = t->NDC * 128;
   const bool fp16 = s.precision == TRACKFIT_FP16_PROJ;
@@ -1073,11 +1099,11 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   for (int l = 0; l < L; ++l) {
     const tf_layer_off& lo = o.layer[l];
     const size_t rb = (size_t)l * t->ROWS_IN;
+    // scan chunk dc = 64 channels of both directions: rows 0-63 forward,
+    // rows 64-127 reverse (z block, then n block); the merge columns follow
     for (int dc = 0; dc < t->NDC; ++dc) {
-      const int j = dc >> 1, dir = dc & 1;
       for (int c = 0; c < 128; ++c) {
-        const int ch = j * 128 + c;
-        if (ch >= H) continue;
+        const int dir = c >> 6, ch = dc * 64 + (c & 63);
         const int src_z = (dir == 0 ? 0 : 2 * H) + ch, src_n = (dir == 0 ? H : 3 * H) + ch;
         for (int k = 0; k < D; ++k) {
           win[(rb + dc * 256 + c) * D + k] = cv(W[lo.w_in + (size_t)src_z * D + k]);
@@ -1241,7 +1267,7 @@ int tf_tc_probe(trackfit_ctx* h, const uint16_t* A, const uint16_t* Bkn, int K, 
   if (K < 64 || K > 256 || (K % 64) != 0) return TRACKFIT_ERR_INVALID_ARG;
   CUtensorMap m;
   if (!make_map(&m, A, 128, (uint64_t)K)) return TRACKFIT_ERR_CUDA;
-  const size_t smem = (size_t)(K / 64) * A_STAGE + (size_t)K * 256 + 64 + 1024;
+  const size_t smem = (size_t)(K / 64) * A_BLOCK + (size_t)K * 256 + 64 + 1024;
   if (cudaFuncSetAttribute(umma_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
     return TRACKFIT_ERR_CUDA;
   umma_probe_kernel<<<1, 128, smem, st>>>(m, Bkn, K, D, idesc_f16(128, 128, 1u, false, true), h->d_err);
