@@ -43,8 +43,8 @@ constexpr int TILE = 128;
 constexpr int SLAB = 64;
 constexpr int MAX_TRK_SLAB = 16;
 constexpr int MAX_TRK_TILE = 2 * MAX_TRK_SLAB;
-constexpr int A_BLOCK = 128 * 64 * 2;     // one 128-row x 64-k 16-bit weight block
-constexpr int A_STAGE = 2 * A_BLOCK;      // a pipeline stage holds two consecutive blocks
+constexpr int A_BLOCK = 128 * 64 * 2;     // one 128-row x 64-k 16-bit weight block = one pipeline stage
+constexpr int MAX_SCHED = 4096;           // schedule entries per tile
 constexpr int EB_BYTES = 160 * 256;       // Fourier operand: 160 k-rows x 128 hits bf16
 constexpr int MISC_BYTES = 8192;
 constexpr int MAX_STAGES = 8;
@@ -69,6 +69,9 @@ struct TcParams {
   float* xs;
   const int32_t* slab_start;
   const int32_t* n_slabs;
+  const uint32_t* sched_p;   // per block: map | col/64 << 4 | row << 8
+  const uint32_t* sched_m;   // per block: b offset | bsel << 13 | tcol/128 << 14 | nk4 << 16 | acc << 17 | end << 18
+  int n_sched;
   const float* b_e1;
   const float* b_e2;
   const float* g;
@@ -631,108 +634,88 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   const int n_tiles = (n_slabs + 1) >> 1;
   volatile int* abort = &m->abort_flag;
 
-  // Blocks are consumed in walk order; a stage holds two consecutive blocks
-  // (one full-barrier wait and one release per 8 MMAs).  Both roles count the
-  // blocks of this CTA so the last stage may hold a single block.
-  int total_blocks = 0;
-  if (warp < 2 && lane == 0) {
-    int my_tiles = 0;
-    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
-    int per_tile = 0;
-    walk_tile(p, [&](int, int, int, int, int, int, int, int, int) { ++per_tile; });
-    total_blocks = per_tile * my_tiles;
-  }
   if (warp == 0) {
     if (lane == 0) {
+      // TMA producer: one 16 KB weight block per stage, in schedule order
       uint32_t stage = 0, phase = 0;
       bool ok = true;
-      int issued = 0, half = 0;
+      int issued = 0;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-        walk_tile(p, [&](int map, int row, int col, int, int, int, int, int, int) {
-          if (!ok) return;
-          if (half == 0) {
-            if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
-              set_abort(m, p.err);
-              ok = false;
-              return;
-            }
-            mbar_arrive_expect_tx(full0 + 8 * stage, issued + 1 < total_blocks ? A_STAGE : A_BLOCK);
+        for (int i = 0; i < p.n_sched; ++i) {
+          const uint32_t e = __ldg(p.sched_p + i);
+          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
+            set_abort(m, p.err);
+            ok = false;
+            break;
           }
-          tma_load_2d(ab + stage * A_STAGE + half * A_BLOCK, &p.tm[map], full0 + 8 * stage, col, row);
+          mbar_arrive_expect_tx(full0 + 8 * stage, A_BLOCK);
+          tma_load_2d(ab + stage * A_BLOCK, &p.tm[e & 15u], full0 + 8 * stage, (int)((e >> 4) & 15u) * 64,
+                      (int)(e >> 8));
           ++issued;
-          if (++half == 2) {
-            half = 0;
-            if (++stage == (uint32_t)p.nst) {
-              stage = 0;
-              phase ^= 1u;
-            }
+          if (++stage == (uint32_t)p.nst) {
+            stage = 0;
+            phase ^= 1u;
           }
-        });
+        }
       }
       if (!ok) {
         // let the copies already issued land before the CTA can exit
         volatile int never = 0;
-        const int stages_used = (issued + 1) / 2;
-        for (int k = 0; k < p.nst && k < stages_used; ++k) {
-          const int i = stages_used - 1 - k;
+        for (int k = 0; k < p.nst && k < issued; ++k) {
+          const int i = issued - 1 - k;
           mbar_wait(full0 + 8 * (i % p.nst), (uint32_t)((i / p.nst) & 1), &never, DRAIN_NS);
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
+      // MMA issuer: per block one full-barrier wait, 2 or 4 MMAs with
+      // descriptors advanced by adds, one release; a group end commits the
+      // accumulator to the epilogue and waits for its next hand-over.
       uint32_t stage = 0, phase = 0, e_phase = 0;
       bool ok = true, need_e = true;
       const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
       const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
-      int half = 0, consumed = 0;
+      constexpr uint32_t BSTEP = (2 * B_SBO) >> 4;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-        walk_tile(p, [&](int, int, int, int nk, int tcol, int bsel, int bk, int acc, int end) {
-          if (!ok) return;
+        for (int i = 0; i < p.n_sched; ++i) {
+          const uint32_t e = __ldg(p.sched_m + i);
           if (need_e) {
             if (!mbar_wait(e_bar, e_phase, abort, WAIT_NS)) {
               set_abort(m, p.err);
               ok = false;
-              return;
+              break;
             }
             e_phase ^= 1u;
             need_e = false;
             tc_fence_after();
           }
-          if (half == 0) {
-            if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
-              set_abort(m, p.err);
-              ok = false;
-              return;
-            }
-            tc_fence_after();
+          if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
+            set_abort(m, p.err);
+            ok = false;
+            break;
           }
-          // descriptors advance by plain adds: 32 B per K=16 step inside a
-          // 128-byte swizzled weight row, two 8-row groups (2 x 2 KB) per step
-          // of the activation operand
-          const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE + half * A_BLOCK) >> 4);
-          const uint64_t bd = (bsel == BSEL_HB ? b_desc_hb : b_desc_xb) + (uint64_t)(((bk >> 3) * B_SBO) >> 4);
-          const uint32_t d = tmem + (uint32_t)tcol;
-          umma_f16(d, ad, bd, p.idesc, acc ? 1u : 0u);
-          umma_f16(d, ad + 2, bd + (2 * B_SBO >> 4), p.idesc, 1u);
-          if (nk == 4) {
-            umma_f16(d, ad + 4, bd + (4 * B_SBO >> 4), p.idesc, 1u);
-            umma_f16(d, ad + 6, bd + (6 * B_SBO >> 4), p.idesc, 1u);
+          tc_fence_after();
+          const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BLOCK >> 4));
+          const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
+          const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
+          const uint32_t idesc = p.idesc;
+          umma_f16(d, ad, bd, idesc, (e >> 17) & 1u);
+          umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
+          if (e & (1u << 16)) {
+            umma_f16(d, ad + 4, bd + 2 * BSTEP, idesc, 1u);
+            umma_f16(d, ad + 6, bd + 3 * BSTEP, idesc, 1u);
           }
-          if (end) {
+          umma_commit(empty0 + 8 * stage);
+          if (e & (1u << 18)) {
             umma_commit(acc_bar);
             need_e = true;
           }
-          ++consumed;
-          if (++half == 2 || consumed == total_blocks) {
-            umma_commit(empty0 + 8 * stage);
-            half = 0;
-            if (++stage == (uint32_t)p.nst) {
-              stage = 0;
-              phase ^= 1u;
-            }
+          if (++stage == (uint32_t)p.nst) {
+            stage = 0;
+            phase ^= 1u;
           }
-        });
+        }
       }
       // no MMA may still run when TMEM is released
       umma_commit(drain_bar);
@@ -827,6 +810,22 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
+}
+
+// ------------------------------------------------------------------ schedule
+// One thread expands walk_tile into the compact per-block entries read by the
+// producer and the MMA issuer (identical for every tile).
+__global__ void build_schedule(const __grid_constant__ TcParams p, uint32_t* sp, uint32_t* sm, int* count) {
+  int n = 0;
+  walk_tile(p, [&](int map, int row, int col, int nk, int tcol, int bsel, int bk, int acc, int end) {
+    if (n < MAX_SCHED) {
+      sp[n] = (uint32_t)map | ((uint32_t)(col >> 6) << 4) | ((uint32_t)row << 8);
+      sm[n] = (uint32_t)(((bk >> 3) * B_SBO) >> 4) | ((uint32_t)bsel << 13) | ((uint32_t)(tcol >> 7) << 14) |
+              ((uint32_t)(nk == 4) << 16) | ((uint32_t)acc << 17) | ((uint32_t)end << 18);
+    }
+    ++n;
+  });
+  *count = n;
 }
 
 // ------------------------------------------------------------------ packing
@@ -1037,6 +1036,8 @@ struct tf_tc_state {
   float *b_e1 = nullptr, *b_e2 = nullptr, *g = nullptr, *b_in = nullptr, *b_m = nullptr, *b_1 = nullptr,
         *b_2 = nullptr, *hg = nullptr, *hw1t = nullptr, *hb1 = nullptr, *hw2 = nullptr, *hb2 = nullptr;
   int32_t *seg_count = nullptr, *seg_off = nullptr, *seg_slabs = nullptr, *slab_start = nullptr, *n_slabs = nullptr;
+  uint32_t* sched = nullptr;   // [2][MAX_SCHED]: producer entries, then MMA entries
+  int n_sched = 0;
   float* xs = nullptr;
   CUtensorMap tm[NMAPS];
 };
@@ -1052,6 +1053,7 @@ void tf_tc_destroy(trackfit_ctx* h) {
   cudaFree(t->dev);
   cudaFree(t->seg_count);
   cudaFree(t->xs);
+  cudaFree(t->sched);
   delete t;
   h->tc = nullptr;
 }
@@ -1077,10 +1079,10 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   t->off_hb = D * 256;
   t->off_a = t->off_hb + EB_BYTES;
   const int avail = smem_optin - 1024 - MISC_BYTES - t->off_a;
-  t->nst = avail / A_STAGE;
+  t->nst = avail / A_BLOCK;
   if (t->nst > MAX_STAGES) t->nst = MAX_STAGES;
   if (t->nst < 2) return TRACKFIT_ERR_UNSUPPORTED;
-  t->off_misc = t->off_a + t->nst * A_STAGE;
+  t->off_misc = t->off_a + t->nst * A_BLOCK;
   t->smem = (size_t)t->off_misc + MISC_BYTES + 1024;
   const bool w2_in_xb = D * 256 >= (MAX_TRK_TILE + s.Q) * 128 * 4;
   if (MAX_TRK_TILE * 128 * 4 > D * 256 ||
@@ -1185,6 +1187,21 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
             make_map(&t->tm[MAP_1], t->w_1, (uint64_t)L * D, D, fp16) &&
             make_map(&t->tm[MAP_2], t->w_2, (uint64_t)L * D, D, fp16);
   if (!ok) return TRACKFIT_ERR_CUDA;
+  // ---- the per-tile block schedule, expanded once on the device
+  {
+    TcParams q;
+    std::memset(&q, 0, sizeof(q));
+    q.D = D;
+    q.L = L;
+    q.NDC = t->NDC;
+    q.ROWS_IN = t->ROWS_IN;
+    int* d_count = nullptr;
+    if (cudaMalloc(&t->sched, 2 * MAX_SCHED * sizeof(uint32_t) + 16) != cudaSuccess) return TRACKFIT_ERR_OOM;
+    d_count = reinterpret_cast<int*>(t->sched + 2 * MAX_SCHED);
+    build_schedule<<<1, 1>>>(q, t->sched, t->sched + MAX_SCHED, d_count);
+    if (cudaMemcpy(&t->n_sched, d_count, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return TRACKFIT_ERR_CUDA;
+    if (t->n_sched < 1 || t->n_sched > MAX_SCHED) return TRACKFIT_ERR_UNSUPPORTED;
+  }
   if (cudaFuncSetAttribute(tc_forward_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
           cudaSuccess ||
       cudaFuncSetAttribute(tc_forward_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
@@ -1203,6 +1220,9 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   p.xs = t->xs;
   p.slab_start = t->slab_start;
   p.n_slabs = t->n_slabs;
+  p.sched_p = t->sched;
+  p.sched_m = t->sched + MAX_SCHED;
+  p.n_sched = t->n_sched;
   p.b_e1 = t->b_e1;
   p.b_e2 = t->b_e2;
   p.g = t->g;
