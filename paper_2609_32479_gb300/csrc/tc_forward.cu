@@ -37,7 +37,7 @@ using namespace sm100;
 
 namespace {
 
-constexpr int NT = 320;
+constexpr int NT = 352;                   // warp 0 TMA, warps 1 and 10 MMA issuers, warps 2..9 epilogue
 constexpr int NE = 256;
 constexpr int TILE = 128;
 constexpr int SLAB = 64;
@@ -614,9 +614,9 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
-    mbar_init(acc_bar, 1);
+    mbar_init(acc_bar, 2);    // one commit from each MMA issuer
     mbar_init(e_bar, 1);
-    mbar_init(drain_bar, 1);
+    mbar_init(drain_bar, 2);
     m->abort_flag = 0;
     fence_mbar_init();
   }
@@ -626,6 +626,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   }
   if (warp == 0 && lane == 0)
     for (int i = 0; i < NMAPS; ++i) prefetch_tmap(&p.tm[i]);
+  static_assert(NT == 352, "warp roles assume 11 warps");
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -667,19 +668,24 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         }
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == 1 || warp == 10) {
     if (lane == 0) {
-      // MMA issuer: per block one full-barrier wait, 2 or 4 MMAs with
-      // descriptors advanced by adds, one release; a group end commits the
-      // accumulator to the epilogue and waits for its next hand-over.
+      // Two MMA issuers: warp 1 drives the accumulators in TMEM regions R0/R2,
+      // warp 10 those in R1/R3, so one issues while the other waits on a stage
+      // or commits.  Both walk the whole schedule (stage and phase counters
+      // stay in step), issue only their own blocks, and both commit to the
+      // accumulator barrier at every group end.
+      const uint32_t mine = warp == 1 ? 0u : 1u;
       uint32_t stage = 0, phase = 0, e_phase = 0;
       bool ok = true, need_e = true;
       const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
       const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
       constexpr uint32_t BSTEP = (2 * B_SBO) >> 4;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+        uint32_t e_next = __ldg(p.sched_m);
         for (int i = 0; i < p.n_sched; ++i) {
-          const uint32_t e = __ldg(p.sched_m + i);
+          const uint32_t e = e_next;
+          if (i + 1 < p.n_sched) e_next = __ldg(p.sched_m + i + 1);
           if (need_e) {
             if (!mbar_wait(e_bar, e_phase, abort, WAIT_NS)) {
               set_abort(m, p.err);
@@ -690,23 +696,25 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
             need_e = false;
             tc_fence_after();
           }
-          if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
-            set_abort(m, p.err);
-            ok = false;
-            break;
+          if (((e >> 14) & 1u) == mine) {
+            if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
+              set_abort(m, p.err);
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BLOCK >> 4));
+            const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
+            const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
+            const uint32_t idesc = p.idesc;
+            umma_f16(d, ad, bd, idesc, (e >> 17) & 1u);
+            umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
+            if (e & (1u << 16)) {
+              umma_f16(d, ad + 4, bd + 2 * BSTEP, idesc, 1u);
+              umma_f16(d, ad + 6, bd + 3 * BSTEP, idesc, 1u);
+            }
+            umma_commit(empty0 + 8 * stage);
           }
-          tc_fence_after();
-          const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BLOCK >> 4));
-          const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
-          const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
-          const uint32_t idesc = p.idesc;
-          umma_f16(d, ad, bd, idesc, (e >> 17) & 1u);
-          umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
-          if (e & (1u << 16)) {
-            umma_f16(d, ad + 4, bd + 2 * BSTEP, idesc, 1u);
-            umma_f16(d, ad + 6, bd + 3 * BSTEP, idesc, 1u);
-          }
-          umma_commit(empty0 + 8 * stage);
           if (e & (1u << 18)) {
             umma_commit(acc_bar);
             need_e = true;
