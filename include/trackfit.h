@@ -185,6 +185,28 @@ int trackfit_debug_scan(const float* a, const float* b, const float* x, const in
 int trackfit_debug_umma(trackfit_t h, const uint16_t* A, const uint16_t* Bkn, int32_t K, float* D,
                         void* stream);
 
+/* Forward pass that allocates no device memory, for callers that cannot call
+ * cudaMalloc (code whose device memory is owned by an outer framework or pool,
+ * or that must not let an allocation synchronise the device).  The paper has no
+ * counterpart: it is a deployment variant of the CUDA-core (SIMT) path.
+ *   cfg        host, as for trackfit_create (any supported precision / pooling).
+ *   weights    device, the fp32 blob of trackfit_weight_count(cfg) values in the
+ *              layout documented there, 16-byte aligned (used as given, no repack).
+ *   hits, n_hits, n_tracks, out_params: as for trackfit_forward.
+ * All workspace comes from one file-scope device array of 32 MiB that every GPU
+ * loading this library keeps until the process exits; the batch is processed in
+ * chunks of whole tracks that fit in it.  A configuration whose workspace for a
+ * single track exceeds 32 MiB returns TRACKFIT_ERR_UNSUPPORTED.  The first call
+ * on a device looks up the array's device address (cudaGetSymbolAddress) with
+ * that device current; make that first call before any stream capture.  Every
+ * call shares the array: calls that overlap on the GPU (different streams or
+ * devices' contexts sharing it concurrently) race and must be serialised by the
+ * caller.  Tracks with n_hits outside [1, max_hits] get NaN rows (no counter is
+ * read back).  Asynchronous on `stream`; makes no cudaMalloc / cudaFree call.
+ * Errors: INVALID_ARG (NULL, n_tracks <= 0, misalignment), UNSUPPORTED, CUDA. */
+int trackfit_forward_noalloc(const trackfit_config_t* cfg, const float* weights, const float* hits,
+                             const int32_t* n_hits, int64_t n_tracks, float* out_params, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

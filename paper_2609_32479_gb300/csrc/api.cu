@@ -291,3 +291,6 @@ extern "C" int trackfit_debug_umma(trackfit_t h, const uint16_t* A, const uint16
   if (!aligned16(A) || !aligned16(Bkn) || !aligned16(D)) return TRACKFIT_ERR_INVALID_ARG;
   return tf_tc_probe(h, A, Bkn, K, D, reinterpret_cast<cudaStream_t>(stream));
 }
+
+// Validation and blob offsets for callers outside this file (no-allocation entry point).
+bool tf_derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) { return derive(c, s, o); }

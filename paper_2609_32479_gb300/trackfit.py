@@ -24,7 +24,7 @@ ABI_VERSION = 1
 EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trackfit_forward_ex",
            "trackfit_forward_host", "trackfit_device_errors", "trackfit_path_name", "trackfit_set_path",
            "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma",
-           "trackfit_profile", "trackfit_profile_read")
+           "trackfit_profile", "trackfit_profile_read", "trackfit_forward_noalloc")
 
 
 class Config(ctypes.Structure):
@@ -84,6 +84,8 @@ def load() -> ctypes.CDLL:
     lib.trackfit_profile.restype = ctypes.c_int
     lib.trackfit_profile_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(i64)]
     lib.trackfit_profile_read.restype = ctypes.c_int
+    lib.trackfit_forward_noalloc.argtypes = [ctypes.POINTER(Config), vp, vp, vp, i64, vp, vp]
+    lib.trackfit_forward_noalloc.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -235,3 +237,14 @@ def debug_umma(tf: "Trackfit", A, Bkn, D, stream=None) -> None:
                                     _dev(D, "torch.float32"), _stream_handle(stream))
     if st != OK:
         raise TrackfitError(st, "trackfit_debug_umma")
+
+
+def forward_noalloc(model: W.ModelConfig, weights, hits, n_hits, out, stream=None) -> None:
+    """No-allocation forward: device fp32 weight blob, hits, n_hits and out as
+    torch CUDA tensors; the library's static device scratch supplies the workspace."""
+    cfg = make_config(model)
+    st = load().trackfit_forward_noalloc(ctypes.byref(cfg), _dev(weights, "torch.float32"),
+                                         _dev(hits, "torch.float32"), _dev(n_hits, "torch.int32"),
+                                         int(n_hits.shape[0]), _dev(out, "torch.float32"), _stream_handle(stream))
+    if st != OK:
+        raise TrackfitError(st, "trackfit_forward_noalloc")
