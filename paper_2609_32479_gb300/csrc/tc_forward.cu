@@ -37,13 +37,14 @@ using namespace sm100;
 
 namespace {
 
-constexpr int NT = 352;                   // warp 0 TMA, warps 1 and 10 MMA issuers, warps 2..9 epilogue
+constexpr int NT = 320;                   // warp 0 TMA, warp 1 MMA issuer, warps 2..9 epilogue
 constexpr int NE = 256;
 constexpr int TILE = 128;
 constexpr int SLAB = 64;
 constexpr int MAX_TRK_SLAB = 16;
 constexpr int MAX_TRK_TILE = 2 * MAX_TRK_SLAB;
-constexpr int A_BLOCK = 128 * 64 * 2;     // one 128-row x 64-k 16-bit weight block = one pipeline stage
+constexpr int A_BLOCK = 128 * 64 * 2;     // one 128-row x 64-k 16-bit weight block
+constexpr int A_STAGE = 2 * A_BLOCK;      // a pipeline stage holds two consecutive blocks
 constexpr int MAX_SCHED = 4096;           // schedule entries per tile
 constexpr int EB_BYTES = 160 * 256;       // Fourier operand: 160 k-rows x 128 hits bf16
 constexpr int MISC_BYTES = 8192;
@@ -614,9 +615,9 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
-    mbar_init(acc_bar, 2);    // one commit from each MMA issuer
+    mbar_init(acc_bar, 1);
     mbar_init(e_bar, 1);
-    mbar_init(drain_bar, 2);
+    mbar_init(drain_bar, 1);
     m->abort_flag = 0;
     fence_mbar_init();
   }
@@ -626,7 +627,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   }
   if (warp == 0 && lane == 0)
     for (int i = 0; i < NMAPS; ++i) prefetch_tmap(&p.tm[i]);
-  static_assert(NT == 352, "warp roles assume 11 warps");
+  static_assert(NT == 320, "warp roles assume 10 warps");
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -637,47 +638,59 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
 
   if (warp == 0) {
     if (lane == 0) {
-      // TMA producer: one 16 KB weight block per stage, in schedule order
+      // TMA producer: two consecutive 16 KB weight blocks per stage, in
+      // schedule order (the CTA's block sequence runs on across tiles; a final
+      // odd block occupies a stage alone)
       uint32_t stage = 0, phase = 0;
       bool ok = true;
-      int issued = 0;
+      int issued = 0, half = 0;
+      int my_tiles = 0;
+      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
+      const int total = my_tiles * p.n_sched;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
         for (int i = 0; i < p.n_sched; ++i) {
           const uint32_t e = __ldg(p.sched_p + i);
-          if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
-            set_abort(m, p.err);
-            ok = false;
-            break;
+          if (half == 0) {
+            if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
+              set_abort(m, p.err);
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(full0 + 8 * stage, issued + 1 < total ? A_STAGE : A_BLOCK);
           }
-          mbar_arrive_expect_tx(full0 + 8 * stage, A_BLOCK);
-          tma_load_2d(ab + stage * A_BLOCK, &p.tm[e & 15u], full0 + 8 * stage, (int)((e >> 4) & 15u) * 64,
-                      (int)(e >> 8));
+          tma_load_2d(ab + stage * A_STAGE + half * A_BLOCK, &p.tm[e & 15u], full0 + 8 * stage,
+                      (int)((e >> 4) & 15u) * 64, (int)(e >> 8));
           ++issued;
-          if (++stage == (uint32_t)p.nst) {
-            stage = 0;
-            phase ^= 1u;
+          if (++half == 2) {
+            half = 0;
+            if (++stage == (uint32_t)p.nst) {
+              stage = 0;
+              phase ^= 1u;
+            }
           }
         }
       }
       if (!ok) {
         // let the copies already issued land before the CTA can exit
         volatile int never = 0;
-        for (int k = 0; k < p.nst && k < issued; ++k) {
-          const int i = issued - 1 - k;
+        const int used = (issued + 1) / 2;
+        for (int k = 0; k < p.nst && k < used; ++k) {
+          const int i = used - 1 - k;
           mbar_wait(full0 + 8 * (i % p.nst), (uint32_t)((i / p.nst) & 1), &never, DRAIN_NS);
         }
       }
     }
-  } else if (warp == 1 || warp == 10) {
+  } else if (warp == 1) {
     if (lane == 0) {
-      // Two MMA issuers: warp 1 drives the accumulators in TMEM regions R0/R2,
-      // warp 10 those in R1/R3, so one issues while the other waits on a stage
-      // or commits.  Both walk the whole schedule (stage and phase counters
-      // stay in step), issue only their own blocks, and both commit to the
-      // accumulator barrier at every group end.
-      const uint32_t mine = warp == 1 ? 0u : 1u;
+      // MMA issuer: per stage (two blocks) one full-barrier wait and one
+      // release; per block 2 or 4 MMAs with descriptors advanced by adds; a
+      // group end commits the accumulator to the epilogue and waits for its
+      // next hand-over.
       uint32_t stage = 0, phase = 0, e_phase = 0;
       bool ok = true, need_e = true;
+      int half = 0, consumed = 0, my_tiles = 0;
+      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
+      const int total = my_tiles * p.n_sched;
       const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
       const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
       constexpr uint32_t BSTEP = (2 * B_SBO) >> 4;
@@ -696,32 +709,36 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
             need_e = false;
             tc_fence_after();
           }
-          if (((e >> 14) & 1u) == mine) {
+          if (half == 0) {
             if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
               set_abort(m, p.err);
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint64_t ad = a_desc0 + (uint64_t)(stage * (A_BLOCK >> 4));
-            const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
-            const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
-            const uint32_t idesc = p.idesc;
-            umma_f16(d, ad, bd, idesc, (e >> 17) & 1u);
-            umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
-            if (e & (1u << 16)) {
-              umma_f16(d, ad + 4, bd + 2 * BSTEP, idesc, 1u);
-              umma_f16(d, ad + 6, bd + 3 * BSTEP, idesc, 1u);
-            }
-            umma_commit(empty0 + 8 * stage);
+          }
+          const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE + half * A_BLOCK) >> 4);
+          const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
+          const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
+          const uint32_t idesc = p.idesc;
+          umma_f16(d, ad, bd, idesc, (e >> 17) & 1u);
+          umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
+          if (e & (1u << 16)) {
+            umma_f16(d, ad + 4, bd + 2 * BSTEP, idesc, 1u);
+            umma_f16(d, ad + 6, bd + 3 * BSTEP, idesc, 1u);
           }
           if (e & (1u << 18)) {
             umma_commit(acc_bar);
             need_e = true;
           }
-          if (++stage == (uint32_t)p.nst) {
-            stage = 0;
-            phase ^= 1u;
+          ++consumed;
+          if (++half == 2 || consumed == total) {
+            umma_commit(empty0 + 8 * stage);
+            half = 0;
+            if (++stage == (uint32_t)p.nst) {
+              stage = 0;
+              phase ^= 1u;
+            }
           }
         }
       }
@@ -1087,10 +1104,10 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   t->off_hb = D * 256;
   t->off_a = t->off_hb + EB_BYTES;
   const int avail = smem_optin - 1024 - MISC_BYTES - t->off_a;
-  t->nst = avail / A_BLOCK;
+  t->nst = avail / A_STAGE;
   if (t->nst > MAX_STAGES) t->nst = MAX_STAGES;
   if (t->nst < 2) return TRACKFIT_ERR_UNSUPPORTED;
-  t->off_misc = t->off_a + t->nst * A_BLOCK;
+  t->off_misc = t->off_a + t->nst * A_STAGE;
   t->smem = (size_t)t->off_misc + MISC_BYTES + 1024;
   const bool w2_in_xb = D * 256 >= (MAX_TRK_TILE + s.Q) * 128 * 4;
   if (MAX_TRK_TILE * 128 * 4 > D * 256 ||
