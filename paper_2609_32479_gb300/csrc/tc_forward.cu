@@ -45,9 +45,10 @@ constexpr int MAX_TRK_SLAB = 16;
 constexpr int MAX_TRK_TILE = 2 * MAX_TRK_SLAB;
 constexpr int A_BLOCK = 128 * 64 * 2;     // one 128-row x 64-k 16-bit weight block
 constexpr int A_STAGE = 2 * A_BLOCK;      // a pipeline stage holds two consecutive blocks
-constexpr int MAX_SCHED = 4096;           // schedule entries per tile
+constexpr int MAX_SCHED = 2048;           // schedule entries per tile
 constexpr int EB_BYTES = 160 * 256;       // Fourier operand: 160 k-rows x 128 hits bf16
 constexpr int MISC_BYTES = 8192;
+constexpr int SCHED_BYTES = 2 * MAX_SCHED * 4;   // both schedule tables, copied to shared memory
 constexpr int MAX_STAGES = 8;
 constexpr int SEG = 1024;                 // tracks per packing segment
 constexpr int64_t MAXB = 4194304;         // tracks per launch chunk
@@ -621,6 +622,11 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     m->abort_flag = 0;
     fence_mbar_init();
   }
+  uint32_t* sched_s = reinterpret_cast<uint32_t*>(gbase + p.off_misc + MISC_BYTES);   // [2][MAX_SCHED]
+  for (int i = threadIdx.x; i < p.n_sched; i += blockDim.x) {
+    sched_s[i] = p.sched_p[i];
+    sched_s[MAX_SCHED + i] = p.sched_m[i];
+  }
   if (warp == 1) {
     tmem_alloc(smem_u32(&m->tmem_base), 512);
     tmem_relinquish();
@@ -649,7 +655,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       const int total = my_tiles * p.n_sched;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
         for (int i = 0; i < p.n_sched; ++i) {
-          const uint32_t e = __ldg(p.sched_p + i);
+          const uint32_t e = sched_s[i];
           if (half == 0) {
             if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
               set_abort(m, p.err);
@@ -695,12 +701,13 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
       constexpr uint32_t BSTEP = (2 * B_SBO) >> 4;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-        uint32_t e_next = __ldg(p.sched_m);
+        const uint32_t* sm_tab = sched_s + MAX_SCHED;
+        uint32_t e_next = sm_tab[0];
         for (int i = 0; i < p.n_sched; ++i) {
           const uint32_t e = e_next;
-          if (i + 1 < p.n_sched) e_next = __ldg(p.sched_m + i + 1);
+          if (i + 1 < p.n_sched) e_next = sm_tab[i + 1];
           if (need_e) {
-            if (!mbar_wait(e_bar, e_phase, abort, WAIT_NS)) {
+            if (!mbar_wait_spin(e_bar, e_phase, abort, WAIT_NS)) {
               set_abort(m, p.err);
               ok = false;
               break;
@@ -785,7 +792,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     // barrier also orders the shared-memory view for all participants.
     auto wait_acc = [&]() -> bool {
       bool mine = true;
-      if (x.te == 0) mine = mbar_wait(acc_bar, acc_phase, abort, WAIT_NS);
+      if (x.te == 0) mine = mbar_wait_spin(acc_bar, acc_phase, abort, WAIT_NS);
       if (!ebar_all(mine)) {
         set_abort(m, p.err);
         return false;
@@ -1103,12 +1110,12 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   t->off_xb = 0;
   t->off_hb = D * 256;
   t->off_a = t->off_hb + EB_BYTES;
-  const int avail = smem_optin - 1024 - MISC_BYTES - t->off_a;
+  const int avail = smem_optin - 1024 - MISC_BYTES - SCHED_BYTES - t->off_a;
   t->nst = avail / A_STAGE;
   if (t->nst > MAX_STAGES) t->nst = MAX_STAGES;
   if (t->nst < 2) return TRACKFIT_ERR_UNSUPPORTED;
   t->off_misc = t->off_a + t->nst * A_STAGE;
-  t->smem = (size_t)t->off_misc + MISC_BYTES + 1024;
+  t->smem = (size_t)t->off_misc + MISC_BYTES + SCHED_BYTES + 1024;
   const bool w2_in_xb = D * 256 >= (MAX_TRK_TILE + s.Q) * 128 * 4;
   if (MAX_TRK_TILE * 128 * 4 > D * 256 ||
       (size_t)(MAX_TRK_TILE * D + (w2_in_xb ? 0 : s.Q * 128)) * 4 > (size_t)EB_BYTES)
