@@ -13,8 +13,8 @@
 //
 // Tile: 128 hit columns = two 64-column slabs; each slab holds whole tracks
 // (packed greedily, unpadded).  Warp roles (320 threads):
-//   warp 0      TMA producer of weight blocks (one elected thread)
-//   warp 1      tcgen05.mma issuer (one elected thread), TMEM owner
+//   warp 0      TMA producer of weight blocks (warp-wide loop, one elected lane issues)
+//   warp 1      tcgen05.mma issuer (warp-wide loop, one elected lane issues), TMEM owner
 //   warps 2..9  epilogue: TMEM lane quadrant = warp % 4, column half = (warp-2)/4
 // TMEM (512 columns): R0,R1 = merge / MLP accumulators (d_model rows), R2,R3 =
 // z and n of one scan chunk, then the output-gate projection.
@@ -59,6 +59,14 @@ constexpr int B_LBO = 1024;               // 64-hit atom stride
 
 enum { MAP_E1 = 0, MAP_E2, MAP_IN, MAP_M, MAP_1, MAP_2, NMAPS };
 enum { BSEL_XB = 0, BSEL_HB = 1 };
+// Hand-overs around a schedule block: before its first MMA the issuer waits for
+// the epilogue's next arrival on e_bar (W_E) or eh_bar (W_H); after its last MMA
+// it commits to acc_bar (C_ACC) or hb_bar (C_HB).
+enum { W_NONE = 0, W_E = 1, W_H = 2 };
+enum { C_NONE = 0, C_ACC = 1, C_HB = 2 };
+// bits of an MMA schedule entry
+constexpr uint32_t S_NK4 = 1u << 16, S_ACC = 1u << 17, S_C_ACC = 1u << 18, S_C_HB = 1u << 19, S_W_E = 1u << 20,
+                   S_W_H = 1u << 21;
 enum { F_FIRST = 1, F_LAST = 2, F_VALID = 4 };
 
 struct TcParams {
@@ -72,7 +80,7 @@ struct TcParams {
   const int32_t* slab_start;
   const int32_t* n_slabs;
   const uint32_t* sched_p;   // per block: map | col/64 << 4 | row << 8
-  const uint32_t* sched_m;   // per block: b offset | bsel << 13 | tcol/128 << 14 | nk4 << 16 | acc << 17 | end << 18
+  const uint32_t* sched_m;   // per block: b offset | bsel << 13 | tcol/128 << 14 | S_* flags
   int n_sched;
   const float* b_e1;
   const float* b_e2;
@@ -97,7 +105,7 @@ struct TcParams {
 
 struct Misc {
   uint64_t full[MAX_STAGES], empty[MAX_STAGES];
-  uint64_t acc_bar, e_bar, drain_bar;
+  uint64_t acc_bar, e_bar, hb_bar, eh_bar, drain_bar;
   uint32_t tmem_base;
   int abort_flag;
   int n_slots;
@@ -190,45 +198,59 @@ __device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
 }
 
 // The static sequence of 128x64 weight blocks of one tile, in the order the MMA
-// issuer consumes them.  f(map, row, col, nk, tmem_col, bsel, bk, acc, end):
+// issuer consumes them.  f(map, row, col, nk, tmem_col, bsel, bk, acc, wait, commit):
 // nk MMAs of K=16 read the block, accumulate into TMEM columns tmem_col, with
 // the activation operand bsel starting at k-row bk; acc = accumulate onto the
-// existing accumulator; end = last block of a group (the epilogue runs next).
+// existing accumulator; wait / commit = hand-overs (W_*, C_*).
+//
+// Within a layer the scan chunks are software-pipelined: as soon as the
+// epilogue has copied the z/n accumulators of chunk k into registers, the
+// issuer computes z/n of chunk k+1 into the same TMEM columns, and the merge
+// product of chunk k follows once its states h(k) are in shared memory.
 template <class F>
 __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
   const int MT = p.D >> 7, KD = p.D >> 6;
   for (int mt = 0; mt < MT; ++mt)
     for (int kc = 0; kc < 3; ++kc)
-      f(MAP_E1, mt * 128, kc * 64, kc == 2 ? 2 : 4, mt * 128, BSEL_HB, kc * 64, kc > 0, mt == MT - 1 && kc == 2);
-  for (int mt = 0; mt < MT; ++mt)
-    for (int kc = 0; kc < KD; ++kc)
-      f(MAP_E2, mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, mt == MT - 1 && kc == KD - 1);
+      f(MAP_E1, mt * 128, kc * 64, kc == 2 ? 2 : 4, mt * 128, BSEL_HB, kc * 64, kc > 0,
+        (mt == 0 && kc == 0) ? W_E : W_NONE, (mt == MT - 1 && kc == 2) ? C_ACC : C_NONE);
+  // a dense D x D product from XB into accumulator columns 0.. (MT tiles of 128 rows)
+  auto dense = [&](int map, int r0) {
+    for (int mt = 0; mt < MT; ++mt)
+      for (int kc = 0; kc < KD; ++kc)
+        f(map, r0 + mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, (mt == 0 && kc == 0) ? W_E : W_NONE,
+          (mt == MT - 1 && kc == KD - 1) ? C_ACC : C_NONE);
+  };
+  dense(MAP_E2, 0);
   for (int l = 0; l < p.L; ++l) {
     const int rb = l * p.ROWS_IN;
-    for (int dc = 0; dc <= p.NDC; ++dc) {
-      if (dc > 0) {  // merge of the previous scan chunk: M[D] += W_m[:, chunk] * h
+    auto zn = [&](int k) {   // z and n of scan chunk k -> TMEM columns 256.. and 384..
+      for (int kc = 0; kc < KD; ++kc)
+        f(MAP_IN, rb + k * 256, kc * 64, 4, 256, BSEL_XB, kc * 64, kc > 0, kc == 0 ? W_E : W_NONE, C_NONE);
+      for (int kc = 0; kc < KD; ++kc)
+        f(MAP_IN, rb + k * 256 + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, W_NONE,
+          kc == KD - 1 ? C_ACC : C_NONE);
+    };
+    zn(0);
+    for (int k = 0; k < p.NDC; ++k) {
+      if (k + 1 < p.NDC) {
+        zn(k + 1);
+      } else {   // output-gate projection into the z/n columns once the last chunk is out
         for (int mt = 0; mt < MT; ++mt)
-          for (int kc = 0; kc < 2; ++kc)
-            f(MAP_M, l * p.D + mt * 128, (dc - 1) * 128 + kc * 64, 4, mt * 128, BSEL_HB, kc * 64,
-              dc > 1 || kc > 0, false);
+          for (int kc = 0; kc < KD; ++kc)
+            f(MAP_IN, rb + p.NDC * 256 + mt * 128, kc * 64, 4, 256 + mt * 128, BSEL_XB, kc * 64, kc > 0,
+              (mt == 0 && kc == 0) ? W_E : W_NONE, C_NONE);
       }
-      if (dc < p.NDC) {  // z and n of scan chunk dc
-        for (int kc = 0; kc < KD; ++kc)
-          f(MAP_IN, rb + dc * 256, kc * 64, 4, 256, BSEL_XB, kc * 64, kc > 0, false);
-        for (int kc = 0; kc < KD; ++kc)
-          f(MAP_IN, rb + dc * 256 + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, kc == KD - 1);
-      }
+      // merge of chunk k: M[D] += W_m[:, chunk] * h(k); the last one also
+      // completes the gate product for the epilogue
+      for (int mt = 0; mt < MT; ++mt)
+        for (int kc = 0; kc < 2; ++kc)
+          f(MAP_M, l * p.D + mt * 128, k * 128 + kc * 64, 4, mt * 128, BSEL_HB, kc * 64, k > 0 || kc > 0,
+            (mt == 0 && kc == 0) ? W_H : W_NONE,
+            (mt == MT - 1 && kc == 1) ? (k + 1 < p.NDC ? C_HB : C_ACC) : C_NONE);
     }
-    for (int mt = 0; mt < MT; ++mt)  // output-gate projection
-      for (int kc = 0; kc < KD; ++kc)
-        f(MAP_IN, rb + p.NDC * 256 + mt * 128, kc * 64, 4, 256 + mt * 128, BSEL_XB, kc * 64, kc > 0,
-          mt == MT - 1 && kc == KD - 1);
-    for (int mt = 0; mt < MT; ++mt)
-      for (int kc = 0; kc < KD; ++kc)
-        f(MAP_1, l * p.D + mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, mt == MT - 1 && kc == KD - 1);
-    for (int mt = 0; mt < MT; ++mt)
-      for (int kc = 0; kc < KD; ++kc)
-        f(MAP_2, l * p.D + mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, mt == MT - 1 && kc == KD - 1);
+    dense(MAP_1, l * p.D);
+    dense(MAP_2, l * p.D);
   }
 }
 
@@ -379,50 +401,51 @@ __device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
   tmem_st_wait();
 }
 
-// Scan chunk dc of one layer -> HB.  The chunk holds 64 channels of both
-// directions: TMEM lanes 0-63 (quadrants 0, 1) run the forward recurrence over
-// the hits in time order, lanes 64-127 (quadrants 2, 3) the reverse one.
-template <bool FP16>
-__device__ __forceinline__ void ep_scan(const ECtx& x, int dc, float bz, float bn) {
-  const uint8_t* flags = x.m->col_flags;
+// Scan chunk of one layer.  The chunk holds 64 channels of both directions:
+// TMEM lanes 0-63 (quadrants 0, 1) run the forward recurrence over the hits in
+// time order, lanes 64-127 (quadrants 2, 3) the reverse one.  The z/n
+// accumulators are first copied to registers (scan_load) so the issuer can
+// reuse their TMEM columns for the next chunk while the recurrence runs
+// (scan_run); the states then go to HB (scan_store).
+__device__ __forceinline__ void scan_load(const ECtx& x, float (&z)[2][32], float (&n)[2][32]) {
+  tmem_ld32(x.tq + 256 + x.col0, z[0]);
+  tmem_ld32(x.tq + 256 + x.col0 + 32, z[1]);
+  tmem_ld32(x.tq + 384 + x.col0, n[0]);
+  tmem_ld32(x.tq + 384 + x.col0 + 32, n[1]);
+  tmem_ld_wait();
+}
+// Eq. 2 per channel over the packed hits of this thread's 64 columns; the states
+// (zero at padding) replace z.
+__device__ __forceinline__ void scan_run(const ECtx& x, float (&z)[2][32], const float (&n)[2][32], float bz,
+                                         float bn) {
+  const uint8_t* flags = x.m->col_flags + x.col0;
   float h = 0.0f;
-  if (x.q < 2) {   // lanes 0-63 of the chunk: forward direction
-#pragma unroll 1
-    for (int ch = 0; ch < 2; ++ch) {
-      float z[32], n[32];
-      tmem_ld32(x.tq + 256 + x.col0 + 32 * ch, z);
-      tmem_ld32(x.tq + 384 + x.col0 + 32 * ch, n);
-      tmem_ld_wait();
+  if (x.q < 2) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int fl = flags[x.col0 + 32 * ch + i];
-        const float zz = sigm(z[i] + bz), nn = n[i] + bn;
-        h = (fl & F_FIRST) ? 0.0f : h;
-        const float hn = fmaf(zz, nn - h, h);
-        h = (fl & F_VALID) ? hn : h;
-        z[i] = (fl & F_VALID) ? h : 0.0f;
-      }
-      store_row32<FP16>(x.hb, x.c, x.col0 + 32 * ch, z);
+    for (int j = 0; j < 64; ++j) {
+      const int fl = flags[j];
+      const float zz = sigm(z[j >> 5][j & 31] + bz), nn = n[j >> 5][j & 31] + bn;
+      h = (fl & F_FIRST) ? 0.0f : h;
+      const float hn = fmaf(zz, nn - h, h);
+      h = (fl & F_VALID) ? hn : h;
+      z[j >> 5][j & 31] = (fl & F_VALID) ? h : 0.0f;
     }
   } else {
-#pragma unroll 1
-    for (int ch = 1; ch >= 0; --ch) {
-      float z[32], n[32];
-      tmem_ld32(x.tq + 256 + x.col0 + 32 * ch, z);
-      tmem_ld32(x.tq + 384 + x.col0 + 32 * ch, n);
-      tmem_ld_wait();
 #pragma unroll
-      for (int i = 31; i >= 0; --i) {
-        const int fl = flags[x.col0 + 32 * ch + i];
-        const float zz = sigm(z[i] + bz), nn = n[i] + bn;
-        h = (fl & F_LAST) ? 0.0f : h;
-        const float hn = fmaf(zz, nn - h, h);
-        h = (fl & F_VALID) ? hn : h;
-        z[i] = (fl & F_VALID) ? h : 0.0f;
-      }
-      store_row32<FP16>(x.hb, x.c, x.col0 + 32 * ch, z);
+    for (int j = 63; j >= 0; --j) {
+      const int fl = flags[j];
+      const float zz = sigm(z[j >> 5][j & 31] + bz), nn = n[j >> 5][j & 31] + bn;
+      h = (fl & F_LAST) ? 0.0f : h;
+      const float hn = fmaf(zz, nn - h, h);
+      h = (fl & F_VALID) ? hn : h;
+      z[j >> 5][j & 31] = (fl & F_VALID) ? h : 0.0f;
     }
   }
+}
+template <bool FP16>
+__device__ __forceinline__ void scan_store(const ECtx& x, const float (&hv)[2][32]) {
+  store_row32<FP16>(x.hb, x.c, x.col0, hv[0]);
+  store_row32<FP16>(x.hb, x.c, x.col0 + 32, hv[1]);
 }
 
 // Tile set-up: slot/column metadata, gather of the valid hits, Fourier operand.
@@ -609,6 +632,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t full0 = smem_u32(&m->full[0]), empty0 = smem_u32(&m->empty[0]);
   const uint32_t acc_bar = smem_u32(&m->acc_bar), e_bar = smem_u32(&m->e_bar);
+  const uint32_t hb_bar = smem_u32(&m->hb_bar), eh_bar = smem_u32(&m->eh_bar);
   const uint32_t drain_bar = smem_u32(&m->drain_bar);
 
   if (threadIdx.x == 0) {
@@ -618,6 +642,8 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     }
     mbar_init(acc_bar, 1);
     mbar_init(e_bar, 1);
+    mbar_init(hb_bar, 1);
+    mbar_init(eh_bar, 1);
     mbar_init(drain_bar, 1);
     m->abort_flag = 0;
     fence_mbar_init();
@@ -643,117 +669,122 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   volatile int* abort = &m->abort_flag;
 
   if (warp == 0) {
-    if (lane == 0) {
-      // TMA producer: two consecutive 16 KB weight blocks per stage, in
-      // schedule order (the CTA's block sequence runs on across tiles; a final
-      // odd block occupies a stage alone)
-      uint32_t stage = 0, phase = 0;
-      bool ok = true;
-      int issued = 0, half = 0;
-      int my_tiles = 0;
-      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
-      const int total = my_tiles * p.n_sched;
-      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-        for (int i = 0; i < p.n_sched; ++i) {
-          const uint32_t e = sched_s[i];
-          if (half == 0) {
-            if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS)) {
-              set_abort(m, p.err);
-              ok = false;
-              break;
-            }
-            mbar_arrive_expect_tx(full0 + 8 * stage, issued + 1 < total ? A_STAGE : A_BLOCK);
+    // TMA producer: two consecutive 16 KB weight blocks per stage, in schedule
+    // order (the CTA's block sequence runs on across tiles; a final odd block
+    // occupies a stage alone).  The whole warp walks the schedule and waits; one
+    // elected lane issues (a loop run by a lone lane issues far slower).
+    uint32_t stage = 0, phase = 0;
+    bool ok = true;
+    int issued = 0, half = 0;
+    int my_tiles = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
+    const int total = my_tiles * p.n_sched;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      for (int i = 0; i < p.n_sched; ++i) {
+        const uint32_t e = sched_s[i];
+        if (half == 0) {
+          const bool got = mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS);
+          if (!__all_sync(0xffffffffu, got)) {
+            if (lane == 0) set_abort(m, p.err);
+            ok = false;
+            break;
           }
+        }
+        if (elect_one()) {
+          if (half == 0) mbar_arrive_expect_tx(full0 + 8 * stage, issued + 1 < total ? A_STAGE : A_BLOCK);
           tma_load_2d(ab + stage * A_STAGE + half * A_BLOCK, &p.tm[e & 15u], full0 + 8 * stage,
                       (int)((e >> 4) & 15u) * 64, (int)(e >> 8));
-          ++issued;
-          if (++half == 2) {
-            half = 0;
-            if (++stage == (uint32_t)p.nst) {
-              stage = 0;
-              phase ^= 1u;
-            }
+        }
+        __syncwarp();
+        ++issued;
+        if (++half == 2) {
+          half = 0;
+          if (++stage == (uint32_t)p.nst) {
+            stage = 0;
+            phase ^= 1u;
           }
         }
       }
-      if (!ok) {
-        // let the copies already issued land before the CTA can exit
-        volatile int never = 0;
-        const int used = (issued + 1) / 2;
-        for (int k = 0; k < p.nst && k < used; ++k) {
-          const int i = used - 1 - k;
-          mbar_wait(full0 + 8 * (i % p.nst), (uint32_t)((i / p.nst) & 1), &never, DRAIN_NS);
-        }
+    }
+    if (!ok) {
+      // let the copies already issued land before the CTA can exit
+      volatile int never = 0;
+      const int used = (issued + 1) / 2;
+      for (int k = 0; k < p.nst && k < used; ++k) {
+        const int i = used - 1 - k;
+        mbar_wait(full0 + 8 * (i % p.nst), (uint32_t)((i / p.nst) & 1), &never, DRAIN_NS);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // MMA issuer: per stage (two blocks) one full-barrier wait and one
-      // release; per block 2 or 4 MMAs with descriptors advanced by adds; a
-      // group end commits the accumulator to the epilogue and waits for its
-      // next hand-over.
-      uint32_t stage = 0, phase = 0, e_phase = 0;
-      bool ok = true, need_e = true;
-      int half = 0, consumed = 0, my_tiles = 0;
-      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
-      const int total = my_tiles * p.n_sched;
-      const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
-      const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
-      constexpr uint32_t BSTEP = (2 * B_SBO) >> 4;
-      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-        const uint32_t* sm_tab = sched_s + MAX_SCHED;
-        uint32_t e_next = sm_tab[0];
-        for (int i = 0; i < p.n_sched; ++i) {
-          const uint32_t e = e_next;
-          if (i + 1 < p.n_sched) e_next = sm_tab[i + 1];
-          if (need_e) {
-            if (!mbar_wait_spin(e_bar, e_phase, abort, WAIT_NS)) {
-              set_abort(m, p.err);
-              ok = false;
-              break;
-            }
-            e_phase ^= 1u;
-            need_e = false;
-            tc_fence_after();
-          }
-          if (half == 0) {
-            if (!mbar_wait(full0 + 8 * stage, phase, abort, WAIT_NS)) {
-              set_abort(m, p.err);
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-          }
-          const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE + half * A_BLOCK) >> 4);
-          const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
-          const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
+    // MMA issuer, run by the whole warp with one elected lane issuing: per
+    // stage (two blocks) one full-barrier wait and one release; per block 2 or 4
+    // MMAs with descriptors advanced by adds; the block's flags say which
+    // epilogue hand-over to wait for first and which barrier to commit after.
+    uint32_t stage = 0, phase = 0, e_phase = 0, eh_phase = 0;
+    bool ok = true;
+    int half = 0, consumed = 0, my_tiles = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
+    const int total = my_tiles * p.n_sched;
+    const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
+    const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
+    constexpr uint32_t BSTEP = (2 * B_SBO) >> 4;
+    const uint32_t* sm_tab = sched_s + MAX_SCHED;
+    auto wait_bar = [&](uint32_t bar, uint32_t& ph, bool spin) -> bool {
+      const bool got = spin ? mbar_wait_spin(bar, ph, abort, WAIT_NS) : mbar_wait(bar, ph, abort, WAIT_NS);
+      if (!__all_sync(0xffffffffu, got)) {
+        if (lane == 0) set_abort(m, p.err);
+        return false;
+      }
+      ph ^= 1u;
+      return true;
+    };
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      for (int i = 0; i < p.n_sched; ++i) {
+        const uint32_t e = sm_tab[i];
+        if (e & (S_W_E | S_W_H)) {
+          if (!(ok = wait_bar((e & S_W_E) ? e_bar : eh_bar, (e & S_W_E) ? e_phase : eh_phase, true))) break;
+          tc_fence_after();
+        }
+        if (half == 0) {
+          uint32_t ph = phase;
+          if (!(ok = wait_bar(full0 + 8 * stage, ph, false))) break;
+          tc_fence_after();
+        }
+        const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE + half * A_BLOCK) >> 4);
+        const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
+        const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
+        const bool release = half == 1 || consumed + 1 == total;
+        if (elect_one()) {
           const uint32_t idesc = p.idesc;
-          umma_f16(d, ad, bd, idesc, (e >> 17) & 1u);
+          umma_f16(d, ad, bd, idesc, (e & S_ACC) ? 1u : 0u);
           umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
-          if (e & (1u << 16)) {
+          if (e & S_NK4) {
             umma_f16(d, ad + 4, bd + 2 * BSTEP, idesc, 1u);
             umma_f16(d, ad + 6, bd + 3 * BSTEP, idesc, 1u);
           }
-          if (e & (1u << 18)) {
-            umma_commit(acc_bar);
-            need_e = true;
+          if (e & S_C_ACC) umma_commit(acc_bar);
+          if (e & S_C_HB) umma_commit(hb_bar);
+          if (release) umma_commit(empty0 + 8 * stage);
+        }
+        __syncwarp();
+        ++consumed;
+        if (release) {
+          half = 0;
+          if (++stage == (uint32_t)p.nst) {
+            stage = 0;
+            phase ^= 1u;
           }
-          ++consumed;
-          if (++half == 2 || consumed == total) {
-            umma_commit(empty0 + 8 * stage);
-            half = 0;
-            if (++stage == (uint32_t)p.nst) {
-              stage = 0;
-              phase ^= 1u;
-            }
-          }
+        } else {
+          half = 1;
         }
       }
-      // no MMA may still run when TMEM is released
-      umma_commit(drain_bar);
-      volatile int never = 0;
-      mbar_wait(drain_bar, 0, &never, DRAIN_NS);
     }
+    // no MMA may still run when TMEM is released (the elected lane is the one
+    // that issued them)
+    if (elect_one()) umma_commit(drain_bar);
+    __syncwarp();
+    volatile int never = 0;
+    mbar_wait(drain_bar, 0, &never, DRAIN_NS);
   } else {
     ECtx x;
     x.p = &p;
@@ -776,31 +807,34 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     // the pooled vectors in the HB region (d_model 128)
     x.w2s = (p.D * 256 >= (MAX_TRK_TILE + p.Q) * 128 * 4) ? x.hid + MAX_TRK_TILE * 128
                                                            : x.pooled + MAX_TRK_TILE * p.D;
-    uint32_t acc_phase = 0;
+    uint32_t acc_phase = 0, hb_phase = 0;
     // Every thread makes its shared-memory operand writes visible to the async
     // proxy and orders its TMEM reads, the named barrier collects them, then a
-    // single arrival hands the phase to the MMA issuer.
-    auto signal = [&]() {
+    // single arrival hands the phase to the MMA issuer (e_bar, or eh_bar for
+    // the scan states in HB).
+    auto signal_to = [&](uint32_t bar) {
       fence_proxy_async_smem();
       tc_fence_before();
       ebar_sync();
-      if (x.te == 0) mbar_arrive(e_bar);
+      if (x.te == 0) mbar_arrive(bar);
     };
+    auto signal = [&]() { signal_to(e_bar); };
     // One elected epilogue thread polls the barrier; the others wait in the
     // hardware named barrier (no shared-memory polling traffic competing with
     // the tensor core's operand reads).  The vote makes the outcome uniform; the
     // barrier also orders the shared-memory view for all participants.
-    auto wait_acc = [&]() -> bool {
+    auto wait_on = [&](uint32_t bar, uint32_t& ph) -> bool {
       bool mine = true;
-      if (x.te == 0) mine = mbar_wait_spin(acc_bar, acc_phase, abort, WAIT_NS);
+      if (x.te == 0) mine = mbar_wait_spin(bar, ph, abort, WAIT_NS);
       if (!ebar_all(mine)) {
         set_abort(m, p.err);
         return false;
       }
-      acc_phase ^= 1u;
+      ph ^= 1u;
       tc_fence_after();
       return true;
     };
+    auto wait_acc = [&]() -> bool { return wait_on(acc_bar, acc_phase); };
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
       ep_setup<FP16>(x, t, n_slabs);
       signal();
@@ -817,8 +851,15 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           const size_t rb = (size_t)l * p.ROWS_IN + dc * 256;
           const float bz = p.b_in[rb + x.c], bn = p.b_in[rb + 128 + x.c];
           if (!(ok = wait_acc())) break;
-          ep_scan<FP16>(x, dc, bz, bn);
-          signal();
+          float z[2][32], n[2][32];
+          scan_load(x, z, n);
+          signal();   // the z/n columns are free for the next chunk
+          scan_run(x, z, n, bz, bn);
+          // HB still feeds the merge of the previous chunk (the gate hand-over
+          // covers the last merge of the previous layer)
+          if (dc > 0 && !(ok = wait_on(hb_bar, hb_phase))) break;
+          scan_store<FP16>(x, z);
+          signal_to(eh_bar);
         }
         if (!ok || !(ok = wait_acc())) break;
         ep_gate<FP16>(x, l);
@@ -849,11 +890,12 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
 // producer and the MMA issuer (identical for every tile).
 __global__ void build_schedule(const __grid_constant__ TcParams p, uint32_t* sp, uint32_t* sm, int* count) {
   int n = 0;
-  walk_tile(p, [&](int map, int row, int col, int nk, int tcol, int bsel, int bk, int acc, int end) {
+  walk_tile(p, [&](int map, int row, int col, int nk, int tcol, int bsel, int bk, int acc, int wait, int commit) {
     if (n < MAX_SCHED) {
       sp[n] = (uint32_t)map | ((uint32_t)(col >> 6) << 4) | ((uint32_t)row << 8);
       sm[n] = (uint32_t)(((bk >> 3) * B_SBO) >> 4) | ((uint32_t)bsel << 13) | ((uint32_t)(tcol >> 7) << 14) |
-              ((uint32_t)(nk == 4) << 16) | ((uint32_t)acc << 17) | ((uint32_t)end << 18);
+              (nk == 4 ? S_NK4 : 0u) | (acc ? S_ACC : 0u) | (commit == C_ACC ? S_C_ACC : 0u) |
+              (commit == C_HB ? S_C_HB : 0u) | (wait == W_E ? S_W_E : 0u) | (wait == W_H ? S_W_H : 0u);
     }
     ++n;
   });
