@@ -331,7 +331,7 @@ def main():
             "path": tf.path, "roofline": roofline, "clocks": clk,
             "e2e": {"value": e2e_value, "unit": "tracks/s", "h2d_bytes_per_step": int(tb.hits.nbytes + tb.n_hits.nbytes),
                     "d2h_bytes_per_step": int(B * 5 * 4), "matches_device_result": same},
-            "gpu_launches": int(4 * math.ceil(B / 4194304) * args.steps) if tf.path.startswith("tcgen05") else None,
+            "gpu_launches": int(5 * math.ceil(B / 4194304) * args.steps) if tf.path.startswith("tcgen05") else None,
             "device_errors": {"status": st, "bad_tracks": nbad}}
     if not args.no_cpu_baseline and world == 1:
         v, idx, ref, dt = run_oracle_sample(w, blob, tb, args.cpu_budget)

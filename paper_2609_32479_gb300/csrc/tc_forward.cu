@@ -75,7 +75,7 @@ struct TcParams {
   const int32_t* n_hits;
   float* out;
   float* out_q;
-  float* out_pool;
+  float* pool;   // [B][D] pooled means (the caller's buffer or an internal one)
   float* xs;
   const int32_t* slab_start;
   const int32_t* n_slabs;
@@ -89,11 +89,6 @@ struct TcParams {
   const float* b_m;
   const float* b_1;
   const float* b_2;
-  const float* head_g;
-  const float* head_w1t;
-  const float* head_b1;
-  const float* head_w2;
-  const float* head_b2;
   unsigned long long* err;
   int T, D, H, L, NDC, ROWS_IN, NQ, Q, nst;
   uint32_t idesc;
@@ -264,9 +259,6 @@ struct ECtx {
   Misc* m;
   uint32_t xb, hb, tq;
   float* xs;
-  float* pooled;
-  float* hid;
-  float* w2s;   // staged W_h2 [Q][128]
   int q, lane, half, c, col0, te, e, MT;
 };
 
@@ -325,7 +317,7 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
           run = (fl & F_FIRST) ? val : run + val;
           if (fl & F_LAST) {
             const int s = x.m->col_slot[col];
-            x.pooled[s * D + ch_g] = run / (float)x.m->slot_n[s];
+            p.pool[(size_t)x.m->slot_track[s] * D + ch_g] = run / (float)x.m->slot_n[s];
           }
         }
       }
@@ -532,95 +524,6 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
   }
 }
 
-// Pooled vectors -> RMSNorm -> 2-layer head -> outputs (fp32 CUDA cores).
-// pooled: [32][D] in the HB region; the XB region holds the hidden layer
-// [32][128] and a copy of W_h2 [Q][128] staged with coalesced loads.
-__device__ __forceinline__ void ep_head(const ECtx& x) {
-  const TcParams& p = *x.p;
-  Misc* m = x.m;
-  const int D = p.D, ns = m->n_slots;
-  float* w2s = x.w2s;
-  for (int i = x.te; i < p.Q * 32; i += NE)   // stage W_h2 as float4s
-    reinterpret_cast<float4*>(w2s)[i] = reinterpret_cast<const float4*>(p.head_w2)[i];
-  for (int s = x.e; s < ns; s += 8) {
-    const size_t trk = (size_t)m->slot_track[s];
-    const bool bad = m->slot_bad[s] != 0;
-    float ss = 0.0f;
-    for (int cc = x.lane; cc < D; cc += 32) {
-      const float v = x.pooled[s * D + cc];
-      ss = fmaf(v, v, ss);
-      if (p.out_pool) p.out_pool[trk * D + cc] = bad ? __int_as_float(0x7fc00000) : v;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-    const float r = 1.0f / sqrtf(ss / (float)D + p.rms_eps);
-    for (int cc = x.lane; cc < D; cc += 32) x.pooled[s * D + cc] *= r * p.head_g[cc];
-  }
-  ebar_sync();
-  {
-    // thread: hidden unit j, slots sg, sg + 2, ... (only the tile's slots)
-    const int j = x.te & 127, sg = x.te >> 7;
-    const int nmine = (ns - sg + 1) >> 1;
-    float a[16];
-    const float b1 = p.head_b1[j];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) a[i] = b1;
-    float w[8], wn[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) w[u] = p.head_w1t[u * 128 + j];
-#pragma unroll 1
-    for (int c0 = 0; c0 < D; c0 += 8) {
-      if (c0 + 8 < D) {
-#pragma unroll
-        for (int u = 0; u < 8; ++u) wn[u] = p.head_w1t[(c0 + 8 + u) * 128 + j];
-      }
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        if (i < nmine) {
-          const float4* pv = reinterpret_cast<const float4*>(x.pooled + (size_t)(sg + 2 * i) * D + c0);
-          const float4 p0 = pv[0], p1 = pv[1];
-          a[i] = fmaf(w[0], p0.x, a[i]);
-          a[i] = fmaf(w[1], p0.y, a[i]);
-          a[i] = fmaf(w[2], p0.z, a[i]);
-          a[i] = fmaf(w[3], p0.w, a[i]);
-          a[i] = fmaf(w[4], p1.x, a[i]);
-          a[i] = fmaf(w[5], p1.y, a[i]);
-          a[i] = fmaf(w[6], p1.z, a[i]);
-          a[i] = fmaf(w[7], p1.w, a[i]);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) w[u] = wn[u];
-    }
-#pragma unroll
-    for (int i = 0; i < 16; ++i)
-      if (i < nmine) x.hid[(sg + 2 * i) * 128 + j] = silu(a[i]);
-  }
-  ebar_sync();
-  for (int idx = x.te; idx < ns * p.Q; idx += NE) {
-    const int s = idx / p.Q, o = idx - s * p.Q;
-    const float4* w = reinterpret_cast<const float4*>(w2s + o * 128);
-    const float4* hv = reinterpret_cast<const float4*>(x.hid + s * 128);
-    float acc = p.head_b2[o];
-#pragma unroll 8
-    for (int j4 = 0; j4 < 32; ++j4) {
-      const float4 a4 = w[j4], h4 = hv[j4];
-      acc = fmaf(a4.x, h4.x, acc);
-      acc = fmaf(a4.y, h4.y, acc);
-      acc = fmaf(a4.z, h4.z, acc);
-      acc = fmaf(a4.w, h4.w, acc);
-    }
-    const size_t trk = (size_t)m->slot_track[s];
-    if (m->slot_bad[s]) acc = __int_as_float(0x7fc00000);
-    if (p.out_q) p.out_q[trk * p.Q + o] = acc;
-    const int qi = o % p.NQ;
-    if (qi == p.NQ / 2) p.out[trk * 5 + o / p.NQ] = acc;
-  }
-  for (int s = x.te; s < ns; s += NE)
-    if (m->slot_bad[s]) atomicAdd(p.err, 1ull);
-  ebar_sync();
-}
-
 template <bool FP16>
 __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -801,12 +704,6 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     x.MT = p.D >> 7;
     x.tq = tmem + ((uint32_t)(32 * x.q) << 16);
     x.xs = p.xs + (size_t)blockIdx.x * TILE * p.D;
-    x.pooled = reinterpret_cast<float*>(gbase + p.off_hb);
-    x.hid = reinterpret_cast<float*>(gbase + p.off_xb);
-    // W_h2 goes after the hidden layer in XB when it fits (d_model 256), else after
-    // the pooled vectors in the HB region (d_model 128)
-    x.w2s = (p.D * 256 >= (MAX_TRK_TILE + p.Q) * 128 * 4) ? x.hid + MAX_TRK_TILE * 128
-                                                           : x.pooled + MAX_TRK_TILE * p.D;
     uint32_t acc_phase = 0, hb_phase = 0;
     // Every thread makes its shared-memory operand writes visible to the async
     // proxy and orders its TMEM reads, the named barrier collects them, then a
@@ -873,8 +770,6 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         if (!last) signal();
       }
       if (!ok) break;
-      ebar_sync();
-      ep_head(x);
     }
   }
   tc_fence_before();
@@ -1098,6 +993,139 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, boo
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// ------------------------------------------------------------------ head
+// Pooled vector -> RMSNorm (gain g_h) -> W_h1 (D -> 128) + SiLU -> W_h2 (128 -> Q)
+// for every track, fp32 on the CUDA cores (the head of Sec. 3.2).  One CTA per SM
+// walks blocks of HEAD_TRK tracks with both weight matrices staged in shared
+// memory once per CTA; the fused kernel leaves the pooled means in global memory.
+struct HeadParams {
+  const float* pool;   // [B][D] pooled means
+  const int32_t* n_hits;
+  int64_t B;
+  int T, D, Q, NQ;
+  float rms_eps;
+  const float* g;     // [D]
+  const float* w1t;   // [D][128]
+  const float* b1;    // [128]
+  const float* w2;    // [Q][128]
+  const float* b2;    // [Q]
+  float* out;         // [B][5]
+  float* out_q;       // [B][Q] or null
+  float* out_pool;    // the caller's pooled buffer (invalid tracks -> NaN) or null
+  unsigned long long* err;
+};
+constexpr int HEAD_TRK = 32, HEAD_NT = 256;
+size_t head_smem_bytes(int D, int Q) {
+  return ((size_t)D * 128 + (size_t)Q * 128 + (size_t)HEAD_TRK * D + (size_t)HEAD_TRK * 128 + D + 128 + Q +
+          HEAD_TRK) * 4;
+}
+
+__global__ void __launch_bounds__(HEAD_NT, 1) head_kernel(const __grid_constant__ HeadParams hp) {
+  extern __shared__ float4 hsm4[];
+  const int D = hp.D, Q = hp.Q;
+  float* w1t = reinterpret_cast<float*>(hsm4);   // [D][128]
+  float* w2 = w1t + D * 128;                      // [Q][128]
+  float* xv = w2 + Q * 128;                       // [HEAD_TRK][D]
+  float* hid = xv + HEAD_TRK * D;                 // [HEAD_TRK][128]
+  float* gs = hid + HEAD_TRK * 128;               // [D]
+  float* b1s = gs + D;                            // [128]
+  float* b2s = b1s + 128;                         // [Q]
+  int* bad_s = reinterpret_cast<int*>(b2s + Q);   // [HEAD_TRK]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  for (int i = tid; i < D * 32; i += HEAD_NT) reinterpret_cast<float4*>(w1t)[i] = reinterpret_cast<const float4*>(hp.w1t)[i];
+  for (int i = tid; i < Q * 32; i += HEAD_NT) reinterpret_cast<float4*>(w2)[i] = reinterpret_cast<const float4*>(hp.w2)[i];
+  for (int i = tid; i < D; i += HEAD_NT) gs[i] = hp.g[i];
+  for (int i = tid; i < 128; i += HEAD_NT) b1s[i] = hp.b1[i];
+  for (int i = tid; i < Q; i += HEAD_NT) b2s[i] = hp.b2[i];
+  __syncthreads();
+  const float qnan = __int_as_float(0x7fc00000);
+  const int64_t nblk = (hp.B + HEAD_TRK - 1) / HEAD_TRK;
+  for (int64_t blk = blockIdx.x; blk < nblk; blk += gridDim.x) {
+    const int64_t t0 = blk * HEAD_TRK;
+    const int nt = (int)((hp.B - t0) < HEAD_TRK ? (hp.B - t0) : HEAD_TRK);
+    // RMSNorm of each pooled vector (one warp per track); padding rows and
+    // invalid tracks become zero rows whose outputs are replaced by NaN
+    for (int i = warp; i < HEAD_TRK; i += HEAD_NT / 32) {
+      float* row = xv + i * D;
+      bool bad = true;
+      if (i < nt) {
+        const int n = hp.n_hits[t0 + i];
+        bad = n < 1 || n > hp.T;
+      }
+      if (bad) {
+        for (int c = lane; c < D; c += 32) row[c] = 0.0f;
+        if (i < nt && hp.out_pool)
+          for (int c = lane; c < D; c += 32) hp.out_pool[(t0 + i) * D + c] = qnan;
+      } else {
+        const float4* src = reinterpret_cast<const float4*>(hp.pool + (t0 + i) * D);
+        float ss = 0.0f;
+        for (int c4 = lane; c4 < D / 4; c4 += 32) {
+          const float4 v = src[c4];
+          reinterpret_cast<float4*>(row)[c4] = v;
+          ss = fmaf(v.x, v.x, ss);
+          ss = fmaf(v.y, v.y, ss);
+          ss = fmaf(v.z, v.z, ss);
+          ss = fmaf(v.w, v.w, ss);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        const float r = 1.0f / sqrtf(ss / (float)D + hp.rms_eps);
+        for (int c = lane; c < D; c += 32) row[c] *= r * gs[c];
+      }
+      if (lane == 0) bad_s[i] = bad;
+    }
+    __syncthreads();
+    {   // hidden unit j of tracks sg, sg + 2, ...
+      const int j = tid & 127, sg = tid >> 7;
+      float a[HEAD_TRK / 2];
+#pragma unroll
+      for (int i = 0; i < HEAD_TRK / 2; ++i) a[i] = b1s[j];
+#pragma unroll 2
+      for (int c = 0; c < D; c += 4) {
+        const float w0 = w1t[c * 128 + j], w1 = w1t[(c + 1) * 128 + j], w2v = w1t[(c + 2) * 128 + j],
+                    w3 = w1t[(c + 3) * 128 + j];
+#pragma unroll
+        for (int i = 0; i < HEAD_TRK / 2; ++i) {
+          const float4 v = *reinterpret_cast<const float4*>(xv + (sg + 2 * i) * D + c);
+          a[i] = fmaf(w0, v.x, a[i]);
+          a[i] = fmaf(w1, v.y, a[i]);
+          a[i] = fmaf(w2v, v.z, a[i]);
+          a[i] = fmaf(w3, v.w, a[i]);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < HEAD_TRK / 2; ++i) hid[(sg + 2 * i) * 128 + j] = silu(a[i]);
+    }
+    __syncthreads();
+    // outputs; the dot product for output o starts at column 4o (mod 128), so the
+    // rows of W_h2 read by one warp fall in different banks while the
+    // summation order stays a function of o alone (results do not depend on a
+    // track's position in the batch)
+    for (int idx = tid; idx < nt * Q; idx += HEAD_NT) {
+      const int i = idx / Q, o = idx - i * Q;
+      const float4* w = reinterpret_cast<const float4*>(w2 + o * 128);
+      const float4* hv = reinterpret_cast<const float4*>(hid + i * 128);
+      float acc = 0.0f;
+#pragma unroll 8
+      for (int u = 0; u < 32; ++u) {
+        const int j4 = (u + o) & 31;
+        const float4 a4 = w[j4], h4 = hv[j4];
+        acc = fmaf(a4.x, h4.x, acc);
+        acc = fmaf(a4.y, h4.y, acc);
+        acc = fmaf(a4.z, h4.z, acc);
+        acc = fmaf(a4.w, h4.w, acc);
+      }
+      acc += b2s[o];
+      const int64_t trk = t0 + i;
+      if (bad_s[i]) acc = qnan;
+      if (hp.out_q) hp.out_q[trk * Q + o] = acc;
+      if (o % hp.NQ == hp.NQ / 2) hp.out[trk * 5 + o / hp.NQ] = acc;
+    }
+    if (tid < nt && bad_s[tid]) atomicAdd(hp.err, 1ull);
+    __syncthreads();
+  }
+}
+
 }  // namespace
 
 struct tf_tc_state {
@@ -1113,6 +1141,9 @@ struct tf_tc_state {
   uint32_t* sched = nullptr;   // [2][MAX_SCHED]: producer entries, then MMA entries
   int n_sched = 0;
   float* xs = nullptr;
+  float* pool = nullptr;   // pooled means when the caller passes no buffer, grown on demand
+  int64_t pool_tracks = 0;
+  size_t head_smem = 0;
   CUtensorMap tm[NMAPS];
 };
 
@@ -1127,6 +1158,7 @@ void tf_tc_destroy(trackfit_ctx* h) {
   cudaFree(t->dev);
   cudaFree(t->seg_count);
   cudaFree(t->xs);
+  cudaFree(t->pool);
   cudaFree(t->sched);
   delete t;
   h->tc = nullptr;
@@ -1158,10 +1190,8 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   if (t->nst < 2) return TRACKFIT_ERR_UNSUPPORTED;
   t->off_misc = t->off_a + t->nst * A_STAGE;
   t->smem = (size_t)t->off_misc + MISC_BYTES + SCHED_BYTES + 1024;
-  const bool w2_in_xb = D * 256 >= (MAX_TRK_TILE + s.Q) * 128 * 4;
-  if (MAX_TRK_TILE * 128 * 4 > D * 256 ||
-      (size_t)(MAX_TRK_TILE * D + (w2_in_xb ? 0 : s.Q * 128)) * 4 > (size_t)EB_BYTES)
-    return TRACKFIT_ERR_UNSUPPORTED;
+  t->head_smem = head_smem_bytes(D, s.Q);
+  if (t->head_smem > (size_t)smem_optin) return TRACKFIT_ERR_UNSUPPORTED;
 
   // ---- repack weights (bf16 GEMM operands, fp32 biases/head)
   const size_t n_e1 = (size_t)D * E, n_e2 = (size_t)D * D, n_in = (size_t)L * t->ROWS_IN * D,
@@ -1279,6 +1309,8 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   if (cudaFuncSetAttribute(tc_forward_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
           cudaSuccess ||
       cudaFuncSetAttribute(tc_forward_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->smem) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)t->head_smem) !=
           cudaSuccess)
     return TRACKFIT_ERR_CUDA;
   return TRACKFIT_OK;
@@ -1304,11 +1336,6 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   p.b_m = t->b_m;
   p.b_1 = t->b_1;
   p.b_2 = t->b_2;
-  p.head_g = t->hg;
-  p.head_w1t = t->hw1t;
-  p.head_b1 = t->hb1;
-  p.head_w2 = t->hw2;
-  p.head_b2 = t->hb2;
   p.err = h->d_err;
   p.T = s.T;
   p.D = s.D;
@@ -1333,6 +1360,29 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
     p.feat_inv_lo[f] = (float)(inv - (double)p.feat_inv_hi[f]);
   }
   for (int k = 0; k < 16; ++k) p.scale[k] = s.scale[k];
+  HeadParams hp;
+  std::memset(&hp, 0, sizeof(hp));
+  hp.T = s.T;
+  hp.D = s.D;
+  hp.Q = s.Q;
+  hp.NQ = s.NQ;
+  hp.rms_eps = s.rms_eps;
+  hp.g = t->hg;
+  hp.w1t = t->hw1t;
+  hp.b1 = t->hb1;
+  hp.w2 = t->hw2;
+  hp.b2 = t->hb2;
+  hp.err = h->d_err;
+  if (!out_pool) {   // internal pooled-mean buffer for one launch chunk
+    const int64_t need = B < MAXB ? B : MAXB;
+    if (t->pool_tracks < need) {
+      cudaFree(t->pool);
+      t->pool = nullptr;
+      t->pool_tracks = 0;
+      if (cudaMalloc(&t->pool, (size_t)need * s.D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
+      t->pool_tracks = need;
+    }
+  }
   for (int64_t c0 = 0; c0 < B; c0 += MAXB) {
     const int64_t nb = (B - c0 < MAXB) ? B - c0 : MAXB;
     const int nseg = (int)((nb + SEG - 1) / SEG);
@@ -1343,13 +1393,20 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
     p.n_hits = n_hits + c0;
     p.out = out + c0 * 5;
     p.out_q = out_q ? out_q + c0 * s.Q : nullptr;
-    p.out_pool = out_pool ? out_pool + c0 * s.P : nullptr;
+    p.pool = out_pool ? out_pool + c0 * s.P : t->pool;
     tf_prof_begin(h, st);
     if (p.fp16)
       tc_forward_kernel<true><<<t->nsm, NT, t->smem, st>>>(p);
     else
       tc_forward_kernel<false><<<t->nsm, NT, t->smem, st>>>(p);
     tf_prof_end(h, st);
+    hp.pool = p.pool;
+    hp.n_hits = p.n_hits;
+    hp.B = nb;
+    hp.out = p.out;
+    hp.out_q = p.out_q;
+    hp.out_pool = out_pool ? p.pool : nullptr;
+    head_kernel<<<t->nsm, HEAD_NT, t->head_smem, st>>>(hp);
     if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
   }
   return TRACKFIT_OK;
