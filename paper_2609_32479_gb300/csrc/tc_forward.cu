@@ -619,19 +619,22 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       }
     }
   } else if (warp == 1) {
-    // MMA issuer, run by the whole warp with one elected lane issuing: per
-    // stage (two blocks) one full-barrier wait and one release; per block 2 or 4
-    // MMAs with descriptors advanced by adds; the block's flags say which
-    // epilogue hand-over to wait for first and which barrier to commit after.
+    // MMA issuer, run by the whole warp with one elected lane issuing.  One
+    // iteration per stage (two consecutive schedule blocks, 8 MMAs): the stage's
+    // barrier is tested without blocking first, and both blocks go out in one
+    // elected run unless an epilogue hand-over falls between them, so the
+    // per-iteration bookkeeping stays short next to the tensor pipe's queue.
     uint32_t stage = 0, phase = 0, e_phase = 0, eh_phase = 0;
     bool ok = true;
-    int half = 0, consumed = 0, my_tiles = 0;
+    int my_tiles = 0;
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
     const int total = my_tiles * p.n_sched;
+    const int n_stages = (total + 1) >> 1;
     const uint64_t a_desc0 = sdesc_sw128(ab, 16, 1024);
     const uint64_t b_desc_xb = sdesc_sw128(xb, B_LBO, B_SBO), b_desc_hb = sdesc_sw128(hb, B_LBO, B_SBO);
     constexpr uint32_t BSTEP = (2 * B_SBO) >> 4;
     const uint32_t* sm_tab = sched_s + MAX_SCHED;
+    const uint32_t idesc = p.idesc;
     auto wait_bar = [&](uint32_t bar, uint32_t& ph, bool spin) -> bool {
       const bool got = spin ? mbar_wait_spin(bar, ph, abort, WAIT_NS) : mbar_wait(bar, ph, abort, WAIT_NS);
       if (!__all_sync(0xffffffffu, got)) {
@@ -641,45 +644,60 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       ph ^= 1u;
       return true;
     };
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-      for (int i = 0; i < p.n_sched; ++i) {
-        const uint32_t e = sm_tab[i];
-        if (e & (S_W_E | S_W_H)) {
-          if (!(ok = wait_bar((e & S_W_E) ? e_bar : eh_bar, (e & S_W_E) ? e_phase : eh_phase, true))) break;
-          tc_fence_after();
-        }
-        if (half == 0) {
-          uint32_t ph = phase;
-          if (!(ok = wait_bar(full0 + 8 * stage, ph, false))) break;
-          tc_fence_after();
-        }
-        const uint64_t ad = a_desc0 + (uint64_t)((stage * A_STAGE + half * A_BLOCK) >> 4);
-        const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
-        const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
-        const bool release = half == 1 || consumed + 1 == total;
+    auto handover = [&](uint32_t e) -> bool {
+      if (!wait_bar((e & S_W_E) ? e_bar : eh_bar, (e & S_W_E) ? e_phase : eh_phase, true)) return false;
+      tc_fence_after();
+      return true;
+    };
+    // the MMAs and group commits of one block (elected lane only)
+    auto issue = [&](uint32_t e, uint64_t ad) {
+      const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
+      const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
+      const uint32_t nk4 = e & S_NK4;
+      umma_f16(d, ad, bd, idesc, e & S_ACC);
+      umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
+      umma_f16_if(d, ad + 4, bd + 2 * BSTEP, idesc, 1u, nk4);
+      umma_f16_if(d, ad + 6, bd + 3 * BSTEP, idesc, 1u, nk4);
+      umma_commit_if(acc_bar, e & S_C_ACC);
+      umma_commit_if(hb_bar, e & S_C_HB);
+    };
+    int i0 = 0;   // schedule index of the stage's first block
+    for (int sg = 0; sg < n_stages; ++sg) {
+      int i1 = i0 + 1;
+      if (i1 == p.n_sched) i1 = 0;
+      const bool two = 2 * sg + 1 < total;
+      const uint32_t e0 = sm_tab[i0], e1 = two ? sm_tab[i1] : 0u;
+      i0 = i1 + 1;
+      if (i0 >= p.n_sched) i0 -= p.n_sched;
+      if ((e0 & (S_W_E | S_W_H)) && !(ok = handover(e0))) break;
+      if (!mbar_test_wait(full0 + 8 * stage, phase)) {
+        uint32_t ph = phase;
+        if (!(ok = wait_bar(full0 + 8 * stage, ph, false))) break;
+      }
+      tc_fence_after();
+      const uint64_t ad0 = a_desc0 + (uint64_t)((stage * A_STAGE) >> 4);
+      const uint64_t ad1 = ad0 + (uint64_t)(A_BLOCK >> 4);
+      const uint32_t empty = empty0 + 8 * stage;
+      if (e1 & (S_W_E | S_W_H)) {   // a hand-over between the two blocks
+        if (elect_one()) issue(e0, ad0);
+        __syncwarp();
+        if (!(ok = handover(e1))) break;
         if (elect_one()) {
-          const uint32_t idesc = p.idesc;
-          umma_f16(d, ad, bd, idesc, (e & S_ACC) ? 1u : 0u);
-          umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
-          if (e & S_NK4) {
-            umma_f16(d, ad + 4, bd + 2 * BSTEP, idesc, 1u);
-            umma_f16(d, ad + 6, bd + 3 * BSTEP, idesc, 1u);
-          }
-          if (e & S_C_ACC) umma_commit(acc_bar);
-          if (e & S_C_HB) umma_commit(hb_bar);
-          if (release) umma_commit(empty0 + 8 * stage);
+          issue(e1, ad1);
+          umma_commit(empty);
         }
         __syncwarp();
-        ++consumed;
-        if (release) {
-          half = 0;
-          if (++stage == (uint32_t)p.nst) {
-            stage = 0;
-            phase ^= 1u;
-          }
-        } else {
-          half = 1;
+      } else {
+        if (elect_one()) {
+          issue(e0, ad0);
+          if (two) issue(e1, ad1);
+          umma_commit(empty);
         }
+        __syncwarp();
+      }
+      if (++stage == (uint32_t)p.nst) {
+        stage = 0;
+        phase ^= 1u;
       }
     }
     // no MMA may still run when TMEM is released (the elected lane is the one
