@@ -108,12 +108,26 @@ struct Misc {
   int slot_track[MAX_TRK_TILE], slot_n[MAX_TRK_TILE], slot_bad[MAX_TRK_TILE];
   uint8_t col_flags[TILE], col_slot[TILE], col_tpos[TILE], pad2_[128];
   float part[4][TILE];
+  // per column half h, 32-column word w: bit j = column 64h + 32w + j starts a
+  // track (first) or ends one (last)
+  uint32_t m_first[2][2], m_last[2][2];
   float rinv[TILE];
   float hs[TILE][5];
 };
 static_assert(sizeof(Misc) <= MISC_BYTES, "misc region too small");
 
 __device__ __forceinline__ float sigm(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+constexpr float LOG2E_F = 1.4426950408889634f;
 __device__ __forceinline__ float silu(float x) { return x * sigm(x); }
 
 // Operand conversion (round to nearest even): bf16, or fp16 when FP16 is set.
@@ -407,33 +421,42 @@ __device__ __forceinline__ void scan_load(const ECtx& x, float (&z)[2][32], floa
   tmem_ld_wait();
 }
 // Eq. 2 per channel over the packed hits of this thread's 64 columns; the states
-// (zero at padding) replace z.
-__device__ __forceinline__ void scan_run(const ECtx& x, float (&z)[2][32], const float (&n)[2][32], float bz,
-                                         float bn) {
-  const uint8_t* flags = x.m->col_flags + x.col0;
+// replace z.  Tracks fill a slab from its first column, so padding only trails
+// the last track: the forward state is never read after it, and in reverse the
+// last track's end restarts the state.  Values left in padding columns stay in
+// padding columns (every product and norm is per column, every residual masks
+// them), so they need no clearing here.  z = sigma(a + b_z) is evaluated as
+// 1 / (1 + 2^(-(a + b_z) log2 e)).
+__device__ __forceinline__ void scan_run(const ECtx& x, float (&z)[2][32], float (&n)[2][32], float bz, float bn) {
+  // gates in place (independent across hits), then the serial recurrence
+  const float cz = -bz * LOG2E_F;
+  const uint32_t(&rmw)[2] = x.q < 2 ? x.m->m_first[x.half] : x.m->m_last[x.half];
+  const uint32_t rm[2] = {rmw[0], rmw[1]};
+#pragma unroll
+  for (int j = 0; j < 64; ++j) {
+    z[j >> 5][j & 31] = rcp_approx(1.0f + ex2_approx(fmaf(z[j >> 5][j & 31], -LOG2E_F, cz)));
+    n[j >> 5][j & 31] += bn;
+  }
   float h = 0.0f;
   if (x.q < 2) {
 #pragma unroll
     for (int j = 0; j < 64; ++j) {
-      const int fl = flags[j];
-      const float zz = sigm(z[j >> 5][j & 31] + bz), nn = n[j >> 5][j & 31] + bn;
-      h = (fl & F_FIRST) ? 0.0f : h;
-      const float hn = fmaf(zz, nn - h, h);
-      h = (fl & F_VALID) ? hn : h;
-      z[j >> 5][j & 31] = (fl & F_VALID) ? h : 0.0f;
+      const uint32_t bit = 1u << (j & 31);
+      h = (rm[j >> 5] & bit) ? 0.0f : h;
+      h = fmaf(z[j >> 5][j & 31], n[j >> 5][j & 31] - h, h);
+      z[j >> 5][j & 31] = h;
     }
   } else {
 #pragma unroll
     for (int j = 63; j >= 0; --j) {
-      const int fl = flags[j];
-      const float zz = sigm(z[j >> 5][j & 31] + bz), nn = n[j >> 5][j & 31] + bn;
-      h = (fl & F_LAST) ? 0.0f : h;
-      const float hn = fmaf(zz, nn - h, h);
-      h = (fl & F_VALID) ? hn : h;
-      z[j >> 5][j & 31] = (fl & F_VALID) ? h : 0.0f;
+      const uint32_t bit = 1u << (j & 31);
+      h = (rm[j >> 5] & bit) ? 0.0f : h;
+      h = fmaf(z[j >> 5][j & 31], n[j >> 5][j & 31] - h, h);
+      z[j >> 5][j & 31] = h;
     }
   }
 }
+
 template <bool FP16>
 __device__ __forceinline__ void scan_store(const ECtx& x, const float (&hv)[2][32]) {
   store_row32<FP16>(x.hb, x.c, x.col0, hv[0]);
@@ -484,6 +507,17 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
     if (x.lane == 0) m->n_slots = ns;
   }
   ebar_sync();
+  if (x.te < 4) {   // column bitmasks for the scans (read after later barriers)
+    const int hf = x.te >> 1, w = x.te & 1;
+    uint32_t fm = 0, lm = 0;
+    for (int j = 0; j < 32; ++j) {
+      const int f = m->col_flags[SLAB * hf + 32 * w + j];
+      fm |= (uint32_t)((f & F_FIRST) != 0) << j;
+      lm |= (uint32_t)((f & F_LAST) != 0) << j;
+    }
+    m->m_first[hf][w] = fm;
+    m->m_last[hf][w] = lm;
+  }
   for (int idx = x.te; idx < TILE * 5; idx += NE) {
     const int col = idx / 5, f = idx - col * 5;
     float v = 0.0f;
