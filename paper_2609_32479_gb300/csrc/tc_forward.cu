@@ -250,16 +250,34 @@ __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
             f(MAP_IN, rb + p.NDC * 256 + mt * 128, kc * 64, 4, 256 + mt * 128, BSEL_XB, kc * 64, kc > 0,
               (mt == 0 && kc == 0) ? W_E : W_NONE, C_NONE);
       }
-      // merge of chunk k: M[D] += W_m[:, chunk] * h(k); the last one also
-      // completes the gate product for the epilogue
+      // merge of chunk k: M[D] += W_m[:, chunk] * h(k).  The last one completes
+      // the gate epilogue's inputs one 128-channel tile at a time.
+      const bool last = k + 1 == p.NDC;
       for (int mt = 0; mt < MT; ++mt)
         for (int kc = 0; kc < 2; ++kc)
           f(MAP_M, l * p.D + mt * 128, k * 128 + kc * 64, 4, mt * 128, BSEL_HB, kc * 64, k > 0 || kc > 0,
             (mt == 0 && kc == 0) ? W_H : W_NONE,
-            (mt == MT - 1 && kc == 1) ? (k + 1 < p.NDC ? C_HB : C_ACC) : C_NONE);
+            kc == 1 && (last || mt == MT - 1) ? (last ? C_ACC : C_HB) : C_NONE);
     }
-    dense(MAP_1, l * p.D);
-    dense(MAP_2, l * p.D);
+    if (MT == 1) {
+      dense(MAP_1, l * p.D);
+      dense(MAP_2, l * p.D);
+    } else {
+      // d_model 256, pipelined by 128-channel tile: MLP1's first K half (x' of
+      // tile 0, XB rows 0-127) starts once the gate epilogue of tile 0 is out,
+      // the rest once tile 1 is; MLP2's K rows 0-127 (SiLU of tile 0) come from
+      // HB, rows 128-255 (SiLU of tile 1) from XB.
+      const int r1 = l * p.D;
+      for (int kc = 0; kc < 4; ++kc)
+        f(MAP_1, r1, kc * 64, 4, 0, BSEL_XB, kc * 64, kc > 0, (kc & 1) ? W_NONE : W_E, kc == 3 ? C_ACC : C_NONE);
+      for (int kc = 0; kc < 4; ++kc)
+        f(MAP_1, r1 + 128, kc * 64, 4, 128, BSEL_XB, kc * 64, kc > 0, W_NONE, kc == 3 ? C_ACC : C_NONE);
+      for (int kc = 0; kc < 4; ++kc)
+        f(MAP_2, r1, kc * 64, 4, 0, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, kc > 0, (kc & 1) ? W_NONE : W_E, C_NONE);
+      for (int kc = 0; kc < 4; ++kc)
+        f(MAP_2, r1 + 128, kc * 64, 4, 128, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, kc > 0, W_NONE,
+          kc == 3 ? C_ACC : C_NONE);
+    }
   }
 }
 
@@ -276,21 +294,26 @@ struct ECtx {
   int q, lane, half, c, col0, te, e, MT;
 };
 
+// silu(acc + bias) of the 128-channel tile mt -> k-rows row0 + c of buf
+template <bool FP16>
+__device__ __forceinline__ void ep_silu_mt(const ECtx& x, const float* bias, int mt, uint32_t buf, int row0) {
+  float v[2][32];   // both 32-column groups in one TMEM round trip
+  tmem_ld32(x.tq + mt * 128 + x.col0, v[0]);
+  tmem_ld32(x.tq + mt * 128 + x.col0 + 32, v[1]);
+  const float b = bias[mt * 128 + x.c];
+  tmem_ld_wait();
+#pragma unroll
+  for (int ch = 0; ch < 2; ++ch) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[ch][i] = silu(v[ch][i] + b);
+    store_row32<FP16>(buf, row0 + x.c, x.col0 + 32 * ch, v[ch]);
+  }
+}
 // silu(acc + bias) -> XB rows [mt*128 + c]
 template <bool FP16>
 __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
-  for (int mt = 0; mt < x.MT; ++mt) {
-    const float b = bias[mt * 128 + x.c];
 #pragma unroll 1
-    for (int ch = 0; ch < 2; ++ch) {
-      float v[32];
-      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, v);
-      tmem_ld_wait();
-#pragma unroll
-      for (int i = 0; i < 32; ++i) v[i] = silu(v[i] + b);
-      store_row32<FP16>(x.xb, mt * 128 + x.c, x.col0 + 32 * ch, v);
-    }
-  }
+  for (int mt = 0; mt < x.MT; ++mt) ep_silu_mt<FP16>(x, bias, mt, x.xb, mt * 128);
 }
 
 // X = acc + bias [+ x'], zero on pad columns.  x' (the gated residual of this
@@ -378,31 +401,29 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
   }
 }
 
-// x' = X + (M + b_m) * sigma(p_g + b_g) -> TMEM columns 256.. (in place of the gate
-// projection) and XB.  X is read back from the scratch with one batch of loads.
+// x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> TMEM columns
+// 256 + 128 mt.. (in place of the gate projection) and XB rows 128 mt + c.  X is
+// read back from the scratch.
 template <bool FP16>
-__device__ __forceinline__ void ep_gate(const ECtx& x, int l) {
+__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt) {
   const TcParams& p = *x.p;
   const int D = p.D;
+  const int ch_g = mt * 128 + x.c;
+  const float bm = p.b_m[l * D + ch_g];
+  const float bg = p.b_in[(size_t)l * p.ROWS_IN + p.NDC * 256 + ch_g];
 #pragma unroll 1
-  for (int mt = 0; mt < x.MT; ++mt) {
-    const int ch_g = mt * 128 + x.c;
-    const float bm = p.b_m[l * D + ch_g];
-    const float bg = p.b_in[(size_t)l * p.ROWS_IN + p.NDC * 256 + ch_g];
-#pragma unroll 1
-    for (int ch = 0; ch < 2; ++ch) {
-      float xv[32], mv[32], gv[32];
-      const float* xp = x.xs + (size_t)(x.col0 + 32 * ch) * D + ch_g;
+  for (int ch = 0; ch < 2; ++ch) {
+    float xv[32], mv[32], gv[32];
+    const float* xp = x.xs + (size_t)(x.col0 + 32 * ch) * D + ch_g;
 #pragma unroll
-      for (int i = 0; i < 32; ++i) xv[i] = xp[(size_t)i * D];
-      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, mv);
-      tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, gv);
-      tmem_ld_wait();
+    for (int i = 0; i < 32; ++i) xv[i] = xp[(size_t)i * D];
+    tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, mv);
+    tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, gv);
+    tmem_ld_wait();
 #pragma unroll
-      for (int i = 0; i < 32; ++i) mv[i] = xv[i] + (mv[i] + bm) * sigm(gv[i] + bg);
-      tmem_st32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, mv);
-      store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, mv);
-    }
+    for (int i = 0; i < 32; ++i) mv[i] = fmaf(mv[i] + bm, sigm(gv[i] + bg), xv[i]);
+    tmem_st32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, mv);
+    store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, mv);
   }
   tmem_st_wait();
 }
@@ -761,13 +782,13 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     // proxy and orders its TMEM reads, the named barrier collects them, then a
     // single arrival hands the phase to the MMA issuer (e_bar, or eh_bar for
     // the scan states in HB).
-    auto signal_to = [&](uint32_t bar) {
-      fence_proxy_async_smem();
+    auto signal_to = [&](uint32_t bar, bool wrote_operands) {
+      if (wrote_operands) fence_proxy_async_smem();   // costly: only after operand writes
       tc_fence_before();
       ebar_sync();
       if (x.te == 0) mbar_arrive(bar);
     };
-    auto signal = [&]() { signal_to(e_bar); };
+    auto signal = [&]() { signal_to(e_bar, true); };
     // One elected epilogue thread polls the barrier; the others wait in the
     // hardware named barrier (no shared-memory polling traffic competing with
     // the tensor core's operand reads).  The vote makes the outcome uniform; the
@@ -802,20 +823,36 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           if (!(ok = wait_acc())) break;
           float z[2][32], n[2][32];
           scan_load(x, z, n);
-          signal();   // the z/n columns are free for the next chunk
+          signal_to(e_bar, false);   // the z/n columns are free for the next chunk
           scan_run(x, z, n, bz, bn);
           // HB still feeds the merge of the previous chunk (the gate hand-over
           // covers the last merge of the previous layer)
           if (dc > 0 && !(ok = wait_on(hb_bar, hb_phase))) break;
           scan_store<FP16>(x, z);
-          signal_to(eh_bar);
+          signal_to(eh_bar, true);
         }
+        // gate and MLP1 epilogues one 128-channel tile at a time (the issuer
+        // pipelines the next tile's products behind each); with d_model 256 the
+        // SiLU of tile 0 goes to HB (MLP1 still reads XB rows 0-127 then)
+        const float* b1 = p.b_1 + (size_t)l * p.D;
         if (!ok || !(ok = wait_acc())) break;
-        ep_gate<FP16>(x, l);
+        ep_gate<FP16>(x, l, 0);
         signal();
-        if (!(ok = wait_acc())) break;
-        ep_silu<FP16>(x, p.b_1 + (size_t)l * p.D);
-        signal();
+        if (x.MT == 2) {
+          if (!(ok = wait_acc())) break;
+          ep_gate<FP16>(x, l, 1);
+          signal();
+          if (!(ok = wait_acc())) break;
+          ep_silu_mt<FP16>(x, b1, 0, x.hb, 0);
+          signal();
+          if (!(ok = wait_acc())) break;
+          ep_silu_mt<FP16>(x, b1, 1, x.xb, 128);
+          signal();
+        } else {
+          if (!(ok = wait_acc())) break;
+          ep_silu_mt<FP16>(x, b1, 0, x.xb, 0);
+          signal();
+        }
         if (!(ok = wait_acc())) break;
         const bool last = l == p.L - 1;
         ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, true, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
