@@ -37,8 +37,9 @@ using namespace sm100;
 
 namespace {
 
-constexpr int NT = 320;                   // warp 0 TMA, warp 1 MMA issuer, warps 2..9 epilogue
-constexpr int NE = 256;
+constexpr int NT = 576;                   // warp 0 TMA, warp 1 MMA issuer, warps 2..17 epilogue
+constexpr int NE = 512;                   // epilogue threads
+constexpr int SEGW = 32;                  // hit columns per epilogue thread (half a slab)
 constexpr int TILE = 128;
 constexpr int SLAB = 64;
 constexpr int MAX_TRK_SLAB = 16;
@@ -47,7 +48,7 @@ constexpr int A_BLOCK = 128 * 64 * 2;     // one 128-row x 64-k 16-bit weight bl
 constexpr int A_STAGE = 2 * A_BLOCK;      // a pipeline stage holds two consecutive blocks
 constexpr int MAX_SCHED = 2048;           // schedule entries per tile
 constexpr int EB_BYTES = 160 * 256;       // Fourier operand: 160 k-rows x 128 hits bf16
-constexpr int MISC_BYTES = 8192;
+constexpr int MISC_BYTES = 10240;
 constexpr int SCHED_BYTES = 2 * MAX_SCHED * 4;   // both schedule tables, copied to shared memory
 constexpr int MAX_STAGES = 8;
 constexpr int SEG = 1024;                 // tracks per packing segment
@@ -111,6 +112,7 @@ struct Misc {
   // per column half h, 32-column word w: bit j = column 64h + 32w + j starts a
   // track (first) or ends one (last)
   uint32_t m_first[2][2], m_last[2][2];
+  float carry[2][2][128];   // [slab][slot][channel]: states or pool sums between column segments
   float rinv[TILE];
   float hs[TILE][5];
 };
@@ -177,12 +179,22 @@ __device__ __forceinline__ void store_row32(uint32_t buf, int k, int n0, const f
   }
 }
 
-__device__ __forceinline__ void ebar_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+template <bool FP16>
+__device__ __forceinline__ void store_row16(uint32_t buf, int k, int n0, const float (&v)[16]) {
+#pragma unroll
+  for (int c = 0; c < 2; ++c) {
+    st_shared_v4(buf + bchunk(k, (n0 >> 3) + c), pack2<FP16>(v[8 * c + 0], v[8 * c + 1]),
+                 pack2<FP16>(v[8 * c + 2], v[8 * c + 3]), pack2<FP16>(v[8 * c + 4], v[8 * c + 5]),
+                 pack2<FP16>(v[8 * c + 6], v[8 * c + 7]));
+  }
+}
+
+__device__ __forceinline__ void ebar_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
 // Named-barrier vote over the 256 epilogue threads: true iff every thread passes true.
 __device__ __forceinline__ bool ebar_all(bool ok) {
   uint32_t r;
   asm volatile(
-      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, 1, 256, p;\n\t"
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, 1, 512, p;\n\t"
       "selp.u32 %0, 1, 0, q;\n\t}"
       : "=r"(r)
       : "r"((uint32_t)ok)
@@ -291,23 +303,32 @@ struct ECtx {
   Misc* m;
   uint32_t xb, hb, tq;
   float* xs;
-  int q, lane, half, c, col0, te, e, MT;
+  // quadrant q (TMEM lanes / channels 32q..), column segment seg = 32-column
+  // quarter of the tile (slab half = seg / 2, position in the slab sub = seg % 2)
+  int q, lane, seg, half, sub, c, col0, te, e, MT;
 };
+
+// The two epilogue warps that share a quadrant and a slab hand a recurrence state
+// (or a running pool sum) from the slab's first 32 columns to the second, or back
+// in the reverse direction: barrier 2 + 2q + half, 64 threads, one arrival by the
+// leading warp and one wait by the other per hand-over.
+__device__ __forceinline__ void carry_pass(const ECtx& x) {
+  asm volatile("bar.arrive %0, 64;" ::"r"(2 + 2 * x.q + x.half) : "memory");
+}
+__device__ __forceinline__ void carry_wait(const ECtx& x) {
+  asm volatile("bar.sync %0, 64;" ::"r"(2 + 2 * x.q + x.half) : "memory");
+}
 
 // silu(acc + bias) of the 128-channel tile mt -> k-rows row0 + c of buf
 template <bool FP16>
 __device__ __forceinline__ void ep_silu_mt(const ECtx& x, const float* bias, int mt, uint32_t buf, int row0) {
-  float v[2][32];   // both 32-column groups in one TMEM round trip
-  tmem_ld32(x.tq + mt * 128 + x.col0, v[0]);
-  tmem_ld32(x.tq + mt * 128 + x.col0 + 32, v[1]);
+  float v[32];
+  tmem_ld32(x.tq + mt * 128 + x.col0, v);
   const float b = bias[mt * 128 + x.c];
   tmem_ld_wait();
 #pragma unroll
-  for (int ch = 0; ch < 2; ++ch) {
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[ch][i] = silu(v[ch][i] + b);
-    store_row32<FP16>(buf, row0 + x.c, x.col0 + 32 * ch, v[ch]);
-  }
+  for (int i = 0; i < 32; ++i) v[i] = silu(v[i] + b);
+  store_row32<FP16>(buf, row0 + x.c, x.col0, v);
 }
 // silu(acc + bias) -> XB rows [mt*128 + c]
 template <bool FP16>
@@ -326,30 +347,38 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
   const TcParams& p = *x.p;
   const int D = p.D;
   const uint8_t* flags = x.m->col_flags;
-  float run0 = 0.0f, run1 = 0.0f;
-#pragma unroll 1
-  for (int ch = 0; ch < 2; ++ch) {
-    float sq[32];
+  float sq[32];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
+  for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
+  // mean pool: the slab's second column segment continues the running sums of
+  // the first (the same sequential sum as one thread walking the whole slab)
+  float run0 = 0.0f, run1 = 0.0f;
+  if (pool && x.sub == 1) {
+    carry_wait(x);
+    run0 = x.m->carry[x.half][0][x.c];
+    run1 = x.m->carry[x.half][1][x.c];
+  }
 #pragma unroll 1
-    for (int mt = 0; mt < x.MT; ++mt) {
-      float run = mt ? run1 : run0;
-      const int ch_g = mt * 128 + x.c;
-      const float b = bias[ch_g];
-      float v[32], r[32];
-      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, v);
-      if (add_x1) tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, r);
+  for (int mt = 0; mt < x.MT; ++mt) {
+    float run = mt ? run1 : run0;
+    const int ch_g = mt * 128 + x.c;
+    const float b = bias[ch_g];
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      const int c0 = x.col0 + 16 * hh;
+      float v[16], r[16];
+      tmem_ld16(x.tq + mt * 128 + c0, v);
+      if (add_x1) tmem_ld16(x.tq + 256 + mt * 128 + c0, r);
       tmem_ld_wait();
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int col = x.col0 + 32 * ch + i;
+      for (int i = 0; i < 16; ++i) {
+        const int col = c0 + i;
         float val = v[i] + b;
         if (add_x1) val += r[i];
         const int fl = flags[col];
         val = (fl & F_VALID) ? val : 0.0f;
         v[i] = val;
-        sq[i] = fmaf(val, val, sq[i]);
+        sq[16 * hh + i] = fmaf(val, val, sq[16 * hh + i]);
         if (pool) {
           run = (fl & F_FIRST) ? val : run + val;
           if (fl & F_LAST) {
@@ -358,19 +387,23 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
           }
         }
       }
-      if (mt) run1 = run; else run0 = run;
       if (!pool) {
-        float* xp = x.xs + (size_t)(x.col0 + 32 * ch) * D + ch_g;
+        float* xp = x.xs + (size_t)c0 * D + ch_g;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) xp[(size_t)i * D] = v[i];
+        for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
       }
     }
-    if (!pool) {
-      const float s = reduce_scatter32(sq, x.lane);
-      x.m->part[x.q][x.col0 + 32 * ch + x.lane] = s;
-    }
+    if (mt) run1 = run; else run0 = run;
   }
-  if (pool) return;
+  if (pool) {
+    if (x.sub == 0) {
+      x.m->carry[x.half][0][x.c] = run0;
+      x.m->carry[x.half][1][x.c] = run1;
+      carry_pass(x);
+    }
+    return;
+  }
+  x.m->part[x.q][x.col0 + x.lane] = reduce_scatter32(sq, x.lane);
   ebar_sync();
   if (x.te < TILE) {
     const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
@@ -382,21 +415,22 @@ __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bo
     const int ch_g = mt * 128 + x.c;
     const float b = bias[ch_g];
     const float g = gain[ch_g];
-#pragma unroll 1
-    for (int ch = 0; ch < 2; ++ch) {
-      float v[32], r[32];
-      tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, v);
-      if (add_x1) tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, r);
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      const int c0 = x.col0 + 16 * hh;
+      float v[16], r[16];
+      tmem_ld16(x.tq + mt * 128 + c0, v);
+      if (add_x1) tmem_ld16(x.tq + 256 + mt * 128 + c0, r);
       tmem_ld_wait();
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int col = x.col0 + 32 * ch + i;
+      for (int i = 0; i < 16; ++i) {
+        const int col = c0 + i;
         float val = v[i] + b;
         if (add_x1) val += r[i];
         val = (flags[col] & F_VALID) ? val : 0.0f;
         v[i] = val * g * x.m->rinv[col];
       }
-      store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, v);
+      store_row16<FP16>(x.xb, ch_g, c0, v);
     }
   }
 }
@@ -412,76 +446,82 @@ __device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt) {
   const float bm = p.b_m[l * D + ch_g];
   const float bg = p.b_in[(size_t)l * p.ROWS_IN + p.NDC * 256 + ch_g];
 #pragma unroll 1
-  for (int ch = 0; ch < 2; ++ch) {
-    float xv[32], mv[32], gv[32];
-    const float* xp = x.xs + (size_t)(x.col0 + 32 * ch) * D + ch_g;
+  for (int hh = 0; hh < 2; ++hh) {
+    const int c0 = x.col0 + 16 * hh;
+    float xv[16], mv[16], gv[16];
+    const float* xp = x.xs + (size_t)c0 * D + ch_g;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) xv[i] = xp[(size_t)i * D];
-    tmem_ld32(x.tq + mt * 128 + x.col0 + 32 * ch, mv);
-    tmem_ld32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, gv);
+    for (int i = 0; i < 16; ++i) xv[i] = xp[(size_t)i * D];
+    tmem_ld16(x.tq + mt * 128 + c0, mv);
+    tmem_ld16(x.tq + 256 + mt * 128 + c0, gv);
     tmem_ld_wait();
 #pragma unroll
-    for (int i = 0; i < 32; ++i) mv[i] = fmaf(mv[i] + bm, sigm(gv[i] + bg), xv[i]);
-    tmem_st32(x.tq + 256 + mt * 128 + x.col0 + 32 * ch, mv);
-    store_row32<FP16>(x.xb, ch_g, x.col0 + 32 * ch, mv);
+    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm(gv[i] + bg), xv[i]);
+    tmem_st16(x.tq + 256 + mt * 128 + c0, mv);
+    store_row16<FP16>(x.xb, ch_g, c0, mv);
   }
   tmem_st_wait();
 }
 
 // Scan chunk of one layer.  The chunk holds 64 channels of both directions:
 // TMEM lanes 0-63 (quadrants 0, 1) run the forward recurrence over the hits in
-// time order, lanes 64-127 (quadrants 2, 3) the reverse one.  The z/n
-// accumulators are first copied to registers (scan_load) so the issuer can
-// reuse their TMEM columns for the next chunk while the recurrence runs
-// (scan_run); the states then go to HB (scan_store).
-__device__ __forceinline__ void scan_load(const ECtx& x, float (&z)[2][32], float (&n)[2][32]) {
-  tmem_ld32(x.tq + 256 + x.col0, z[0]);
-  tmem_ld32(x.tq + 256 + x.col0 + 32, z[1]);
-  tmem_ld32(x.tq + 384 + x.col0, n[0]);
-  tmem_ld32(x.tq + 384 + x.col0 + 32, n[1]);
+// time order, lanes 64-127 (quadrants 2, 3) the reverse one.  Each thread owns a
+// 32-column segment; the two segments of a slab run one after the other, the
+// leading one handing its final state to the other (carry_pass / carry_wait).  The
+// z/n accumulators are first copied to registers (scan_load) so the issuer can
+// reuse their TMEM columns for the next chunk while the gates and the recurrence
+// run; the states then go to HB.
+__device__ __forceinline__ void scan_load(const ECtx& x, float (&z)[32], float (&n)[32]) {
+  tmem_ld32(x.tq + 256 + x.col0, z);
+  tmem_ld32(x.tq + 384 + x.col0, n);
   tmem_ld_wait();
 }
-// Eq. 2 per channel over the packed hits of this thread's 64 columns; the states
-// replace z.  Tracks fill a slab from its first column, so padding only trails
-// the last track: the forward state is never read after it, and in reverse the
-// last track's end restarts the state.  Values left in padding columns stay in
-// padding columns (every product and norm is per column, every residual masks
-// them), so they need no clearing here.  z = sigma(a + b_z) is evaluated as
-// 1 / (1 + 2^(-(a + b_z) log2 e)).
-__device__ __forceinline__ void scan_run(const ECtx& x, float (&z)[2][32], float (&n)[2][32], float bz, float bn) {
-  // gates in place (independent across hits), then the serial recurrence
+// The gates, independent across hits: z <- sigma(z + b_z), n <- n + b_n, with
+// sigma(a + b_z) = 1 / (1 + 2^(-(a + b_z) log2 e)).
+__device__ __forceinline__ void scan_gates(float (&z)[32], float (&n)[32], float bz, float bn) {
   const float cz = -bz * LOG2E_F;
-  const uint32_t(&rmw)[2] = x.q < 2 ? x.m->m_first[x.half] : x.m->m_last[x.half];
-  const uint32_t rm[2] = {rmw[0], rmw[1]};
 #pragma unroll
-  for (int j = 0; j < 64; ++j) {
-    z[j >> 5][j & 31] = rcp_approx(1.0f + ex2_approx(fmaf(z[j >> 5][j & 31], -LOG2E_F, cz)));
-    n[j >> 5][j & 31] += bn;
+  for (int j = 0; j < 32; ++j) {
+    z[j] = rcp_approx(1.0f + ex2_approx(fmaf(z[j], -LOG2E_F, cz)));
+    n[j] += bn;
   }
+}
+// Eq. 2 per channel over this thread's 32 columns, the states replacing z.
+// Tracks fill a slab from its first column, so padding only trails the last
+// track: the forward state is never read after it, and in reverse the last
+// track's end restarts the state.  Values left in padding columns stay in padding
+// columns (every product and norm is per column, every residual masks them), so
+// they need no clearing here.
+template <bool FP16>
+__device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&z)[32], const float (&n)[32]) {
+  const bool fwd = x.q < 2;
+  const bool leads = fwd ? x.sub == 0 : x.sub == 1;
+  const uint32_t rm = fwd ? x.m->m_first[x.half][x.sub] : x.m->m_last[x.half][x.sub];
   float h = 0.0f;
-  if (x.q < 2) {
+  if (!leads) {
+    carry_wait(x);
+    h = x.m->carry[x.half][0][x.c];
+  }
+  if (fwd) {
 #pragma unroll
-    for (int j = 0; j < 64; ++j) {
-      const uint32_t bit = 1u << (j & 31);
-      h = (rm[j >> 5] & bit) ? 0.0f : h;
-      h = fmaf(z[j >> 5][j & 31], n[j >> 5][j & 31] - h, h);
-      z[j >> 5][j & 31] = h;
+    for (int j = 0; j < 32; ++j) {
+      h = (rm & (1u << j)) ? 0.0f : h;
+      h = fmaf(z[j], n[j] - h, h);
+      z[j] = h;
     }
   } else {
 #pragma unroll
-    for (int j = 63; j >= 0; --j) {
-      const uint32_t bit = 1u << (j & 31);
-      h = (rm[j >> 5] & bit) ? 0.0f : h;
-      h = fmaf(z[j >> 5][j & 31], n[j >> 5][j & 31] - h, h);
-      z[j >> 5][j & 31] = h;
+    for (int j = 31; j >= 0; --j) {
+      h = (rm & (1u << j)) ? 0.0f : h;
+      h = fmaf(z[j], n[j] - h, h);
+      z[j] = h;
     }
   }
-}
-
-template <bool FP16>
-__device__ __forceinline__ void scan_store(const ECtx& x, const float (&hv)[2][32]) {
-  store_row32<FP16>(x.hb, x.c, x.col0, hv[0]);
-  store_row32<FP16>(x.hb, x.c, x.col0 + 32, hv[1]);
+  if (leads) {
+    x.m->carry[x.half][0][x.c] = h;
+    carry_pass(x);
+  }
+  store_row32<FP16>(x.hb, x.c, x.col0, z);
 }
 
 // Tile set-up: slot/column metadata, gather of the valid hits, Fourier operand.
@@ -489,6 +529,9 @@ template <bool FP16>
 __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
   const TcParams& p = *x.p;
   Misc* m = x.m;
+  // the previous tile's last epilogue (pooling) may still read the column
+  // metadata in other warps
+  ebar_sync();
   if (x.te < TILE) m->col_flags[x.te] = 0;
   ebar_sync();
   if (x.e == 0) {
@@ -617,7 +660,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   }
   if (warp == 0 && lane == 0)
     for (int i = 0; i < NMAPS; ++i) prefetch_tmap(&p.tm[i]);
-  static_assert(NT == 320, "warp roles assume 10 warps");
+  static_assert(NT == 576 && NE == 512 && SEGW == 32, "warp roles assume 18 warps");
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -769,10 +812,12 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     x.hb = hb;
     x.e = warp - 2;
     x.q = warp & 3;
-    x.half = x.e >> 2;
+    x.seg = x.e >> 2;
+    x.half = x.seg >> 1;
+    x.sub = x.seg & 1;
     x.lane = lane;
     x.c = 32 * x.q + lane;
-    x.col0 = SLAB * x.half;
+    x.col0 = SEGW * x.seg;
     x.te = threadIdx.x - 64;
     x.MT = p.D >> 7;
     x.tq = tmem + ((uint32_t)(32 * x.q) << 16);
@@ -821,14 +866,14 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           const size_t rb = (size_t)l * p.ROWS_IN + dc * 256;
           const float bz = p.b_in[rb + x.c], bn = p.b_in[rb + 128 + x.c];
           if (!(ok = wait_acc())) break;
-          float z[2][32], n[2][32];
+          float z[32], n[32];
           scan_load(x, z, n);
           signal_to(e_bar, false);   // the z/n columns are free for the next chunk
-          scan_run(x, z, n, bz, bn);
+          scan_gates(z, n, bz, bn);
           // HB still feeds the merge of the previous chunk (the gate hand-over
           // covers the last merge of the previous layer)
           if (dc > 0 && !(ok = wait_on(hb_bar, hb_phase))) break;
-          scan_store<FP16>(x, z);
+          scan_chain_store<FP16>(x, z, n);
           signal_to(eh_bar, true);
         }
         // gate and MLP1 epilogues one 128-channel tile at a time (the issuer
