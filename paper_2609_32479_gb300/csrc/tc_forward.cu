@@ -476,27 +476,32 @@ __device__ __forceinline__ void scan_load(const ECtx& x, float (&z)[32], float (
   tmem_ld32(x.tq + 384 + x.col0, n);
   tmem_ld_wait();
 }
-// The gates, independent across hits: z <- sigma(z + b_z), n <- n + b_n, with
-// sigma(a + b_z) = 1 / (1 + 2^(-(a + b_z) log2 e)).
-__device__ __forceinline__ void scan_gates(float (&z)[32], float (&n)[32], float bz, float bn) {
+// The gates, independent across hits, in the form h_t = a_t h_{t-1} + b_t of the
+// linear scan: with s = sigma(z + b_z) = 1 / (1 + e), e = 2^(-(z + b_z) log2 e),
+// a = 1 - s = e s (no cancellation as s -> 1) and b = s (n + b_n).  Where the
+// recurrence restarts (a track's first hit forward, its last in reverse) a = 0.
+// a replaces z, b replaces n.
+__device__ __forceinline__ void scan_gates(const ECtx& x, float (&z)[32], float (&n)[32], float bz, float bn) {
+  const uint32_t rm = x.q < 2 ? x.m->m_first[x.half][x.sub] : x.m->m_last[x.half][x.sub];
   const float cz = -bz * LOG2E_F;
 #pragma unroll
   for (int j = 0; j < 32; ++j) {
-    z[j] = rcp_approx(1.0f + ex2_approx(fmaf(z[j], -LOG2E_F, cz)));
-    n[j] += bn;
+    const float e = ex2_approx(fmaf(z[j], -LOG2E_F, cz));
+    const float sg = rcp_approx(1.0f + e);
+    z[j] = (rm & (1u << j)) ? 0.0f : e * sg;
+    n[j] = sg * (n[j] + bn);
   }
 }
-// Eq. 2 per channel over this thread's 32 columns, the states replacing z.
-// Tracks fill a slab from its first column, so padding only trails the last
-// track: the forward state is never read after it, and in reverse the last
-// track's end restarts the state.  Values left in padding columns stay in padding
-// columns (every product and norm is per column, every residual masks them), so
-// they need no clearing here.
+// Eq. 2 per channel over this thread's 32 columns (one FMA per hit on the serial
+// path), the states replacing z.  Tracks fill a slab from its first column, so
+// padding only trails the last track: the forward state is never read after it,
+// and in reverse the last track's end restarts the state.  Values left in
+// padding columns stay in padding columns (every product and norm is per
+// column, every residual masks them), so they need no clearing here.
 template <bool FP16>
-__device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&z)[32], const float (&n)[32]) {
+__device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&a)[32], const float (&b)[32]) {
   const bool fwd = x.q < 2;
   const bool leads = fwd ? x.sub == 0 : x.sub == 1;
-  const uint32_t rm = fwd ? x.m->m_first[x.half][x.sub] : x.m->m_last[x.half][x.sub];
   float h = 0.0f;
   if (!leads) {
     carry_wait(x);
@@ -505,23 +510,21 @@ __device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&z)[32], 
   if (fwd) {
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
-      h = (rm & (1u << j)) ? 0.0f : h;
-      h = fmaf(z[j], n[j] - h, h);
-      z[j] = h;
+      h = fmaf(a[j], h, b[j]);
+      a[j] = h;
     }
   } else {
 #pragma unroll
     for (int j = 31; j >= 0; --j) {
-      h = (rm & (1u << j)) ? 0.0f : h;
-      h = fmaf(z[j], n[j] - h, h);
-      z[j] = h;
+      h = fmaf(a[j], h, b[j]);
+      a[j] = h;
     }
   }
   if (leads) {
     x.m->carry[x.half][0][x.c] = h;
     carry_pass(x);
   }
-  store_row32<FP16>(x.hb, x.c, x.col0, z);
+  store_row32<FP16>(x.hb, x.c, x.col0, a);
 }
 
 // Tile set-up: slot/column metadata, gather of the valid hits, Fourier operand.
@@ -869,7 +872,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           float z[32], n[32];
           scan_load(x, z, n);
           signal_to(e_bar, false);   // the z/n columns are free for the next chunk
-          scan_gates(z, n, bz, bn);
+          scan_gates(x, z, n, bz, bn);
           // HB still feeds the merge of the previous chunk (the gate hand-over
           // covers the last merge of the previous layer)
           if (dc > 0 && !(ok = wait_on(hb_bar, hb_phase))) break;
