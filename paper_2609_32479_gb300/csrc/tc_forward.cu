@@ -202,22 +202,6 @@ __device__ __forceinline__ bool ebar_all(bool ok) {
   return r != 0;
 }
 
-// After a butterfly reduce-scatter of v[32] (one value per column per lane),
-// lane L returns the sum over the 32 lanes of column L.
-__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) {
-    const bool upper = (lane & off) != 0;
-#pragma unroll
-    for (int i = 0; i < off; ++i) {
-      const float send = upper ? v[i] : v[i + off];
-      const float keep = upper ? v[i + off] : v[i];
-      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
-    }
-  }
-  return v[0];
-}
-
 // The static sequence of 128x64 weight blocks of one tile, in the order the MMA
 // issuer consumes them.  f(map, row, col, nk, tmem_col, bsel, bk, acc, wait, commit):
 // nk MMAs of K=16 read the block, accumulate into TMEM columns tmem_col, with
@@ -236,13 +220,15 @@ __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
       f(MAP_E1, mt * 128, kc * 64, kc == 2 ? 2 : 4, mt * 128, BSEL_HB, kc * 64, kc > 0,
         (mt == 0 && kc == 0) ? W_E : W_NONE, (mt == MT - 1 && kc == 2) ? C_ACC : C_NONE);
   // a dense D x D product from XB into accumulator columns 0.. (MT tiles of 128 rows)
-  auto dense = [&](int map, int r0) {
+  // a dense D x D product from XB into accumulator columns tcol0 + 128 mt; with
+  // onto = true it accumulates onto what the columns hold (MLP2 onto x')
+  auto dense = [&](int map, int r0, int tcol0, bool onto) {
     for (int mt = 0; mt < MT; ++mt)
       for (int kc = 0; kc < KD; ++kc)
-        f(map, r0 + mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, (mt == 0 && kc == 0) ? W_E : W_NONE,
-          (mt == MT - 1 && kc == KD - 1) ? C_ACC : C_NONE);
+        f(map, r0 + mt * 128, kc * 64, 4, tcol0 + mt * 128, BSEL_XB, kc * 64, onto || kc > 0,
+          (mt == 0 && kc == 0) ? W_E : W_NONE, (mt == MT - 1 && kc == KD - 1) ? C_ACC : C_NONE);
   };
-  dense(MAP_E2, 0);
+  dense(MAP_E2, 0, 0, false);
   for (int l = 0; l < p.L; ++l) {
     const int rb = l * p.ROWS_IN;
     auto zn = [&](int k) {   // z and n of scan chunk k -> TMEM columns 256.. and 384..
@@ -272,22 +258,25 @@ __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
             kc == 1 && (last || mt == MT - 1) ? (last ? C_ACC : C_HB) : C_NONE);
     }
     if (MT == 1) {
-      dense(MAP_1, l * p.D);
-      dense(MAP_2, l * p.D);
+      dense(MAP_1, l * p.D, 256, false);   // MLP1 -> the z/n columns
+      dense(MAP_2, l * p.D, 0, true);      // MLP2 accumulates onto x'
     } else {
       // d_model 256, pipelined by 128-channel tile: MLP1's first K half (x' of
       // tile 0, XB rows 0-127) starts once the gate epilogue of tile 0 is out,
       // the rest once tile 1 is; MLP2's K rows 0-127 (SiLU of tile 0) come from
       // HB, rows 128-255 (SiLU of tile 1) from XB.
       const int r1 = l * p.D;
+      // MLP1 goes to the z/n columns (free once the gate epilogue of the tile has
+      // read them); MLP2 accumulates onto x', which the gate epilogue left in the
+      // merge columns
       for (int kc = 0; kc < 4; ++kc)
-        f(MAP_1, r1, kc * 64, 4, 0, BSEL_XB, kc * 64, kc > 0, (kc & 1) ? W_NONE : W_E, kc == 3 ? C_ACC : C_NONE);
+        f(MAP_1, r1, kc * 64, 4, 256, BSEL_XB, kc * 64, kc > 0, (kc & 1) ? W_NONE : W_E, kc == 3 ? C_ACC : C_NONE);
       for (int kc = 0; kc < 4; ++kc)
-        f(MAP_1, r1 + 128, kc * 64, 4, 128, BSEL_XB, kc * 64, kc > 0, W_NONE, kc == 3 ? C_ACC : C_NONE);
+        f(MAP_1, r1 + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, W_NONE, kc == 3 ? C_ACC : C_NONE);
       for (int kc = 0; kc < 4; ++kc)
-        f(MAP_2, r1, kc * 64, 4, 0, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, kc > 0, (kc & 1) ? W_NONE : W_E, C_NONE);
+        f(MAP_2, r1, kc * 64, 4, 0, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, true, (kc & 1) ? W_NONE : W_E, C_NONE);
       for (int kc = 0; kc < 4; ++kc)
-        f(MAP_2, r1 + 128, kc * 64, 4, 128, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, kc > 0, W_NONE,
+        f(MAP_2, r1 + 128, kc * 64, 4, 128, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, true, W_NONE,
           kc == 3 ? C_ACC : C_NONE);
     }
   }
@@ -321,146 +310,200 @@ __device__ __forceinline__ void carry_wait(const ECtx& x) {
 
 // silu(acc + bias) of the 128-channel tile mt -> k-rows row0 + c of buf
 template <bool FP16>
-__device__ __forceinline__ void ep_silu_mt(const ECtx& x, const float* bias, int mt, uint32_t buf, int row0) {
+__device__ __forceinline__ void ep_silu_mt(const ECtx& x, const float* bias, int mt, uint32_t tcol, uint32_t buf,
+                                           int row0) {
   float v[32];
-  tmem_ld32(x.tq + mt * 128 + x.col0, v);
+  tmem_ld32(x.tq + tcol + mt * 128 + x.col0, v);
   const float b = bias[mt * 128 + x.c];
   tmem_ld_wait();
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = silu(v[i] + b);
   store_row32<FP16>(buf, row0 + x.c, x.col0, v);
 }
-// silu(acc + bias) -> XB rows [mt*128 + c]
+// silu(acc + bias) of every tile (accumulator columns mt*128) -> XB rows
+// [mt*128 + c], all tiles' accumulators read under one TMEM wait
+template <bool FP16, int MT>
+__device__ __forceinline__ void ep_silu_t(const ECtx& x, const float* bias) {
+  float v[MT][32];
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) tmem_ld32(x.tq + mt * 128 + x.col0, v[mt]);
+  tmem_ld_wait();
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) {
+    const float b = bias[mt * 128 + x.c];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[mt][i] = silu(v[mt][i] + b);
+    store_row32<FP16>(x.xb, mt * 128 + x.c, x.col0, v[mt]);
+  }
+}
 template <bool FP16>
 __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
-#pragma unroll 1
-  for (int mt = 0; mt < x.MT; ++mt) ep_silu_mt<FP16>(x, bias, mt, x.xb, mt * 128);
+  if (x.MT == 2)
+    ep_silu_t<FP16, 2>(x, bias);
+  else
+    ep_silu_t<FP16, 1>(x, bias);
 }
 
 // X = acc + bias [+ x'], zero on pad columns.  x' (the gated residual of this
 // layer) sits in TMEM columns 256.. where the gate epilogue left it.  X goes to
 // the per-CTA scratch (read back once, by the next layer's gate epilogue), then
 // either the RMS-normalised x_hat -> XB (recomputing X from TMEM) or mean pooling.
-template <bool FP16>
-__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, bool add_x1, const float* gain,
-                                            bool pool) {
-  const TcParams& p = *x.p;
-  const int D = p.D;
-  const uint8_t* flags = x.m->col_flags;
-  float sq[32];
+// Sum of v over the 32 lanes for 16 columns at once: afterwards lane L holds the
+// total of column L & 15 (both halves of the warp hold the same 16 totals).
+__device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
 #pragma unroll
-  for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
+  for (int off = 8; off >= 1; off >>= 1) {
+    const bool upper = (lane & off) != 0;
+#pragma unroll
+    for (int i = 0; i < off; ++i) {
+      const float send = upper ? v[i] : v[i + off];
+      const float keep = upper ? v[i + off] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+    }
+  }
+  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
+}
+
+template <bool FP16, int MT, bool pool>
+__device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain) {
+  const TcParams& p = *x.p;
+  constexpr int D = 128 * MT;   // d_model (compile-time: strided scratch offsets become immediates)
+  const uint8_t* flags = x.m->col_flags;
+  // X = acc + bias (the accumulator already holds x' + MLP for a layer, the
+  // embedding product for the embedding), zero on pad columns; per 16-column
+  // half, every tile's accumulator is read under one TMEM wait
+  float bias_v[MT];
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) bias_v[mt] = bias[mt * 128 + x.c];
   // mean pool: the slab's second column segment continues the running sums of
   // the first (the same sequential sum as one thread walking the whole slab)
-  float run0 = 0.0f, run1 = 0.0f;
+  float run[MT];
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) run[mt] = 0.0f;
   if (pool && x.sub == 1) {
     carry_wait(x);
-    run0 = x.m->carry[x.half][0][x.c];
-    run1 = x.m->carry[x.half][1][x.c];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) run[mt] = x.m->carry[x.half][mt][x.c];
   }
-#pragma unroll 1
-  for (int mt = 0; mt < x.MT; ++mt) {
-    float run = mt ? run1 : run0;
-    const int ch_g = mt * 128 + x.c;
-    const float b = bias[ch_g];
 #pragma unroll
-    for (int hh = 0; hh < 2; ++hh) {
-      const int c0 = x.col0 + 16 * hh;
-      float v[16], r[16];
-      tmem_ld16(x.tq + mt * 128 + c0, v);
-      if (add_x1) tmem_ld16(x.tq + 256 + mt * 128 + c0, r);
-      tmem_ld_wait();
+  for (int hh = 0; hh < 2; ++hh) {
+    const int c0 = x.col0 + 16 * hh;
+    float v[MT][16];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int col = c0 + i;
-        float val = v[i] + b;
-        if (add_x1) val += r[i];
-        const int fl = flags[col];
-        val = (fl & F_VALID) ? val : 0.0f;
-        v[i] = val;
-        sq[16 * hh + i] = fmaf(val, val, sq[16 * hh + i]);
-        if (pool) {
-          run = (fl & F_FIRST) ? val : run + val;
+    for (int mt = 0; mt < MT; ++mt) tmem_ld16(x.tq + mt * 128 + c0, v[mt]);
+    tmem_ld_wait();
+    float sq[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int fl = flags[c0 + i];
+      sq[i] = 0.0f;
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        const float val = (fl & F_VALID) ? v[mt][i] + bias_v[mt] : 0.0f;
+        v[mt][i] = val;
+        sq[i] = fmaf(val, val, sq[i]);
+        if constexpr (pool) {
+          run[mt] = (fl & F_FIRST) ? val : run[mt] + val;
           if (fl & F_LAST) {
-            const int s = x.m->col_slot[col];
-            p.pool[(size_t)x.m->slot_track[s] * D + ch_g] = run / (float)x.m->slot_n[s];
+            const int s = x.m->col_slot[c0 + i];
+            p.pool[(size_t)x.m->slot_track[s] * D + mt * 128 + x.c] = run[mt] / (float)x.m->slot_n[s];
           }
         }
       }
-      if (!pool) {
-        float* xp = x.xs + (size_t)c0 * D + ch_g;
-#pragma unroll
-        for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
-      }
     }
-    if (mt) run1 = run; else run0 = run;
+    if constexpr (!pool) {
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[mt][i];
+      }
+      const float t = reduce_scatter16(sq, x.lane);
+      if (x.lane < 16) x.m->part[x.q][c0 + x.lane] = t;
+    }
   }
-  if (pool) {
+  if constexpr (pool) {
     if (x.sub == 0) {
-      x.m->carry[x.half][0][x.c] = run0;
-      x.m->carry[x.half][1][x.c] = run1;
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) x.m->carry[x.half][mt][x.c] = run[mt];
       carry_pass(x);
     }
-    return;
-  }
-  x.m->part[x.q][x.col0 + x.lane] = reduce_scatter32(sq, x.lane);
-  ebar_sync();
-  if (x.te < TILE) {
-    const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
-    x.m->rinv[x.te] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
-  }
-  ebar_sync();
-#pragma unroll 1
-  for (int mt = 0; mt < x.MT; ++mt) {
-    const int ch_g = mt * 128 + x.c;
-    const float b = bias[ch_g];
-    const float g = gain[ch_g];
+  } else {
+    ebar_sync();
+    if (x.te < TILE) {
+      const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
+      x.m->rinv[x.te] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
+    }
+    ebar_sync();
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
       const int c0 = x.col0 + 16 * hh;
-      float v[16], r[16];
-      tmem_ld16(x.tq + mt * 128 + c0, v);
-      if (add_x1) tmem_ld16(x.tq + 256 + mt * 128 + c0, r);
+      float v[MT][16];
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) tmem_ld16(x.tq + mt * 128 + c0, v[mt]);
       tmem_ld_wait();
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int col = c0 + i;
-        float val = v[i] + b;
-        if (add_x1) val += r[i];
-        val = (flags[col] & F_VALID) ? val : 0.0f;
-        v[i] = val * g * x.m->rinv[col];
+      for (int mt = 0; mt < MT; ++mt) {
+        const float g = gain[mt * 128 + x.c];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float val = (flags[c0 + i] & F_VALID) ? v[mt][i] + bias_v[mt] : 0.0f;
+          v[mt][i] = val * g * x.m->rinv[c0 + i];
+        }
+        store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v[mt]);
       }
-      store_row16<FP16>(x.xb, ch_g, c0, v);
     }
   }
 }
 
-// x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> TMEM columns
-// 256 + 128 mt.. (in place of the gate projection) and XB rows 128 mt + c.  X is
-// read back from the scratch.
 template <bool FP16>
-__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt) {
+__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, const float* gain, bool pool) {
+  if (x.MT == 2) {
+    if (pool)
+      ep_residual_t<FP16, 2, true>(x, bias, gain);
+    else
+      ep_residual_t<FP16, 2, false>(x, bias, gain);
+  } else {
+    if (pool)
+      ep_residual_t<FP16, 1, true>(x, bias, gain);
+    else
+      ep_residual_t<FP16, 1, false>(x, bias, gain);
+  }
+}
+
+// x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> TMEM columns
+// 128 mt.. (in place of the merge accumulator; MLP2 accumulates onto it) and XB
+// rows 128 mt + c.  X is read back from the scratch.
+template <bool FP16, int MT>
+__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt) {
   const TcParams& p = *x.p;
-  const int D = p.D;
+  constexpr int D = 128 * MT;
   const int ch_g = mt * 128 + x.c;
   const float bm = p.b_m[l * D + ch_g];
   const float bg = p.b_in[(size_t)l * p.ROWS_IN + p.NDC * 256 + ch_g];
-#pragma unroll 1
+#pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
     const int c0 = x.col0 + 16 * hh;
     float xv[16], mv[16], gv[16];
+    tmem_ld16(x.tq + mt * 128 + c0, mv);
+    tmem_ld16(x.tq + 256 + mt * 128 + c0, gv);
     const float* xp = x.xs + (size_t)c0 * D + ch_g;
 #pragma unroll
     for (int i = 0; i < 16; ++i) xv[i] = xp[(size_t)i * D];
-    tmem_ld16(x.tq + mt * 128 + c0, mv);
-    tmem_ld16(x.tq + 256 + mt * 128 + c0, gv);
     tmem_ld_wait();
 #pragma unroll
     for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm(gv[i] + bg), xv[i]);
-    tmem_st16(x.tq + 256 + mt * 128 + c0, mv);
+    tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
     store_row16<FP16>(x.xb, ch_g, c0, mv);
   }
   tmem_st_wait();
+}
+template <bool FP16>
+__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt) {
+  if (x.MT == 2)
+    ep_gate_t<FP16, 2>(x, l, mt);
+  else
+    ep_gate_t<FP16, 1>(x, l, mt);
 }
 
 // Scan chunk of one layer.  The chunk holds 64 channels of both directions:
@@ -860,7 +903,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       ep_silu<FP16>(x, p.b_e1);
       signal();
       if (!wait_acc()) break;
-      ep_residual<FP16>(x, p.b_e2, false, p.g, false);   // embedding output X0
+      ep_residual<FP16>(x, p.b_e2, p.g, false);   // embedding output X0
       signal();
       bool ok = true;
       for (int l = 0; l < p.L && ok; ++l) {
@@ -891,19 +934,19 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           ep_gate<FP16>(x, l, 1);
           signal();
           if (!(ok = wait_acc())) break;
-          ep_silu_mt<FP16>(x, b1, 0, x.hb, 0);
+          ep_silu_mt<FP16>(x, b1, 0, 256, x.hb, 0);
           signal();
           if (!(ok = wait_acc())) break;
-          ep_silu_mt<FP16>(x, b1, 1, x.xb, 128);
+          ep_silu_mt<FP16>(x, b1, 1, 256, x.xb, 128);
           signal();
         } else {
           if (!(ok = wait_acc())) break;
-          ep_silu_mt<FP16>(x, b1, 0, x.xb, 0);
+          ep_silu_mt<FP16>(x, b1, 0, 256, x.xb, 0);
           signal();
         }
         if (!(ok = wait_acc())) break;
         const bool last = l == p.L - 1;
-        ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, true, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
+        ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
         if (!last) signal();
       }
       if (!ok) break;
