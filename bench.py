@@ -309,20 +309,27 @@ def main():
     valid_hits = int(tb.n_hits.clip(0, m.max_hits).sum())
     flops = valid_hits * flops_per_hit(m) + B * flops_per_track_head(m)
     kern_avg_s = (kern_ms / max(kern_n, 1)) * 1e-3
+    # the library splits a step into launches (524,288 tracks each when, as here,
+    # no pooled output buffer is passed): per-launch work is the step's share
+    launches_per_step = max(kern_n // max(args.steps, 1), 1) if kern_n else 1
+    flops_launch = flops / launches_per_step
     dtype_tf = {1: "bf16_tflops", 2: "bf16_tflops"}.get(m.precision, "bf16_tflops")
     peak = float(peaks.get(dtype_tf, FALLBACK_PEAKS["bf16_tflops"]))
     peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-    achieved = flops / kern_avg_s / 1e12 if kern_n else None
+    achieved = flops_launch / kern_avg_s / 1e12 if kern_n else None
     traffic = traffic_for_kernel()
+    if traffic is not None:   # the summary scales its capture to 1,048,576 tracks
+        traffic *= (B / launches_per_step) / 1048576
     roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": (achieved / peak) if achieved else None, "traffic": traffic,
                 "peak_kind": f"{peak_kind} bf16 dense burst (fp16 runs at the bf16 rate)",
                 "frac_of_sustained": (achieved / peak_sus) if achieved else None,
                 "kernel": "tc_forward_kernel" if tf.path.startswith("tcgen05") else "simt layer sequence",
-                "kernel_ms_avg": kern_avg_s * 1e3, "flops_per_launch": flops,
-                "algorithmic_bytes_per_launch": B * bytes_per_track(m),
-                "hbm_frac_of_time": (B * bytes_per_track(m) / (peaks.get("hbm_gbs", 6800.0) * 1e9)) / kern_avg_s
-                if kern_n else None}
+                "kernel_ms_avg": kern_avg_s * 1e3, "launches_per_step": launches_per_step,
+                "flops_per_launch": flops_launch,
+                "algorithmic_bytes_per_launch": B * bytes_per_track(m) / launches_per_step,
+                "hbm_frac_of_time": (B * bytes_per_track(m) / launches_per_step /
+                                     (peaks.get("hbm_gbs", 6800.0) * 1e9)) / kern_avg_s if kern_n else None}
     line = {"metric": METRIC, "value": value, "unit": "tracks/s", "n_gpus": n_ranks, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
             "ms_per_step_min": float(min(step_ms)), "higher_is_better": True, "scaling": "weak",
@@ -331,7 +338,8 @@ def main():
             "path": tf.path, "roofline": roofline, "clocks": clk,
             "e2e": {"value": e2e_value, "unit": "tracks/s", "h2d_bytes_per_step": int(tb.hits.nbytes + tb.n_hits.nbytes),
                     "d2h_bytes_per_step": int(B * 5 * 4), "matches_device_result": same},
-            "gpu_launches": int(5 * math.ceil(B / 4194304) * args.steps) if tf.path.startswith("tcgen05") else None,
+            # per launch chunk: three packing kernels, the fused encoder, the head
+            "gpu_launches": int(5 * math.ceil(B / 524288) * args.steps) if tf.path.startswith("tcgen05") else None,
             "device_errors": {"status": st, "bad_tracks": nbad}}
     if not args.no_cpu_baseline and world == 1:
         v, idx, ref, dt = run_oracle_sample(w, blob, tb, args.cpu_budget)

@@ -53,6 +53,7 @@ constexpr int SCHED_BYTES = 2 * MAX_SCHED * 4;   // both schedule tables, copied
 constexpr int MAX_STAGES = 8;
 constexpr int SEG = 1024;                 // tracks per packing segment
 constexpr int64_t MAXB = 4194304;         // tracks per launch chunk
+constexpr int64_t POOL_TRACKS = 524288;   // tracks per launch chunk when the pooled means go to the internal buffer
 constexpr uint64_t WAIT_NS = 2000000000ull;
 constexpr uint64_t DRAIN_NS = 200000000ull;
 constexpr int B_SBO = 2048;               // k-group stride of the MN-major activation operand
@@ -1321,8 +1322,7 @@ struct tf_tc_state {
   uint32_t* sched = nullptr;   // [2][MAX_SCHED]: producer entries, then MMA entries
   int n_sched = 0;
   float* xs = nullptr;
-  float* pool = nullptr;   // pooled means when the caller passes no buffer, grown on demand
-  int64_t pool_tracks = 0;
+  float* pool = nullptr;   // pooled means when the caller passes no buffer [POOL_TRACKS][D]
   size_t head_smem = 0;
   CUtensorMap tm[NMAPS];
 };
@@ -1464,6 +1464,7 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   t->slab_start = t->seg_slabs + (size_t)nseg_max * (SEG + 1);
   t->n_slabs = t->slab_start + MAXB + 2;
   if (cudaMalloc(&t->xs, (size_t)t->nsm * TILE * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  if (cudaMalloc(&t->pool, (size_t)POOL_TRACKS * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
   // ---- tensor maps
   bool ok = make_map(&t->tm[MAP_E1], t->w_e1, D, E, fp16) && make_map(&t->tm[MAP_E2], t->w_e2, D, D, fp16) &&
             make_map(&t->tm[MAP_IN], t->w_in, (uint64_t)L * t->ROWS_IN, D, fp16) &&
@@ -1553,18 +1554,11 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   hp.w2 = t->hw2;
   hp.b2 = t->hb2;
   hp.err = h->d_err;
-  if (!out_pool) {   // internal pooled-mean buffer for one launch chunk
-    const int64_t need = B < MAXB ? B : MAXB;
-    if (t->pool_tracks < need) {
-      cudaFree(t->pool);
-      t->pool = nullptr;
-      t->pool_tracks = 0;
-      if (cudaMalloc(&t->pool, (size_t)need * s.D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
-      t->pool_tracks = need;
-    }
-  }
-  for (int64_t c0 = 0; c0 < B; c0 += MAXB) {
-    const int64_t nb = (B - c0 < MAXB) ? B - c0 : MAXB;
+  // without a caller buffer the pooled means go to the internal one, which
+  // bounds the launch chunk
+  const int64_t chunk = out_pool ? MAXB : POOL_TRACKS;
+  for (int64_t c0 = 0; c0 < B; c0 += chunk) {
+    const int64_t nb = (B - c0 < chunk) ? B - c0 : chunk;
     const int nseg = (int)((nb + SEG - 1) / SEG);
     plan_segments<<<nseg, 32, 0, st>>>(n_hits + c0, nb, s.T, t->seg_count, t->seg_slabs);
     plan_scan<<<1, 1024, 0, st>>>(t->seg_count, nseg, nb, t->seg_off, t->n_slabs, t->slab_start);
