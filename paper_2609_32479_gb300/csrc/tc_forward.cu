@@ -109,12 +109,12 @@ struct Misc {
   int pad_;
   int slot_track[MAX_TRK_TILE], slot_n[MAX_TRK_TILE], slot_bad[MAX_TRK_TILE];
   uint8_t col_flags[TILE], col_slot[TILE], col_tpos[TILE], pad2_[128];
-  float part[4][TILE];
+  alignas(16) float part[4][TILE];
   // per column half h, 32-column word w: bit j = column 64h + 32w + j starts a
-  // track (first) or ends one (last)
-  uint32_t m_first[2][2], m_last[2][2];
+  // track (first), ends one (last), holds a hit (valid)
+  uint32_t m_first[2][2], m_last[2][2], m_valid[2][2];
   float carry[2][2][128];   // [slab][slot][channel]: states or pool sums between column segments
-  float rinv[TILE];
+  alignas(16) float rinv[TILE];
   float hs[TILE][5];
 };
 static_assert(sizeof(Misc) <= MISC_BYTES, "misc region too small");
@@ -368,8 +368,9 @@ __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
 template <bool FP16, int MT, bool pool>
 __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain) {
   const TcParams& p = *x.p;
-  constexpr int D = 128 * MT;   // d_model (compile-time: strided scratch offsets become immediates)
+  constexpr int D = 128 * MT;   // d_model
   const uint8_t* flags = x.m->col_flags;
+  const uint32_t vm = x.m->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
   // X = acc + bias (the accumulator already holds x' + MLP for a layer, the
   // embedding product for the embedding), zero on pad columns; per 16-column
   // half, every tile's accumulator is read under one TMEM wait
@@ -396,14 +397,15 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
     float sq[16];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-      const int fl = flags[c0 + i];
+      const bool valid = (vm >> (16 * hh + i)) & 1u;
       sq[i] = 0.0f;
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
-        const float val = (fl & F_VALID) ? v[mt][i] + bias_v[mt] : 0.0f;
+        const float val = valid ? v[mt][i] + bias_v[mt] : 0.0f;
         v[mt][i] = val;
         sq[i] = fmaf(val, val, sq[i]);
         if constexpr (pool) {
+          const int fl = flags[c0 + i];
           run[mt] = (fl & F_FIRST) ? val : run[mt] + val;
           if (fl & F_LAST) {
             const int s = x.m->col_slot[c0 + i];
@@ -413,6 +415,8 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       }
     }
     if constexpr (!pool) {
+      // the residual stream to the scratch, column-major (a warp's store covers
+      // 32 consecutive channels: one 128-byte line)
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
         float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
@@ -442,14 +446,24 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       float v[MT][16];
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) tmem_ld16(x.tq + mt * 128 + c0, v[mt]);
+      float rv[16];
+      const float4* rp = reinterpret_cast<const float4*>(x.m->rinv + c0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float4 r4 = rp[i];
+        rv[4 * i] = r4.x;
+        rv[4 * i + 1] = r4.y;
+        rv[4 * i + 2] = r4.z;
+        rv[4 * i + 3] = r4.w;
+      }
       tmem_ld_wait();
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
         const float g = gain[mt * 128 + x.c];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const float val = (flags[c0 + i] & F_VALID) ? v[mt][i] + bias_v[mt] : 0.0f;
-          v[mt][i] = val * g * x.m->rinv[c0 + i];
+          const float val = ((vm >> (16 * hh + i)) & 1u) ? v[mt][i] + bias_v[mt] : 0.0f;
+          v[mt][i] = val * g * rv[i];
         }
         store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v[mt]);
       }
@@ -618,16 +632,18 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
     if (x.lane == 0) m->n_slots = ns;
   }
   ebar_sync();
-  if (x.te < 4) {   // column bitmasks for the scans (read after later barriers)
+  if (x.te < 4) {   // column bitmasks (read after later barriers)
     const int hf = x.te >> 1, w = x.te & 1;
-    uint32_t fm = 0, lm = 0;
+    uint32_t fm = 0, lm = 0, vm = 0;
     for (int j = 0; j < 32; ++j) {
       const int f = m->col_flags[SLAB * hf + 32 * w + j];
       fm |= (uint32_t)((f & F_FIRST) != 0) << j;
       lm |= (uint32_t)((f & F_LAST) != 0) << j;
+      vm |= (uint32_t)((f & F_VALID) != 0) << j;
     }
     m->m_first[hf][w] = fm;
     m->m_last[hf][w] = lm;
+    m->m_valid[hf][w] = vm;
   }
   for (int idx = x.te; idx < TILE * 5; idx += NE) {
     const int col = idx / 5, f = idx - col * 5;
