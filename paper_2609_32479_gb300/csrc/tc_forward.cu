@@ -191,17 +191,6 @@ __device__ __forceinline__ void store_row16(uint32_t buf, int k, int n0, const f
 }
 
 __device__ __forceinline__ void ebar_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
-// Named-barrier vote over the 256 epilogue threads: true iff every thread passes true.
-__device__ __forceinline__ bool ebar_all(bool ok) {
-  uint32_t r;
-  asm volatile(
-      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, 1, 512, p;\n\t"
-      "selp.u32 %0, 1, 0, q;\n\t}"
-      : "=r"(r)
-      : "r"((uint32_t)ok)
-      : "memory");
-  return r != 0;
-}
 
 // The static sequence of 128x64 weight blocks of one tile, in the order the MMA
 // issuer consumes them.  f(map, row, col, nk, tmem_col, bsel, bk, acc, wait, commit):
@@ -705,9 +694,9 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       mbar_init(empty0 + 8 * s, 1);
     }
     mbar_init(acc_bar, 1);
-    mbar_init(e_bar, 1);
+    mbar_init(e_bar, NE / 32);   // one arrival per epilogue warp
     mbar_init(hb_bar, 1);
-    mbar_init(eh_bar, 1);
+    mbar_init(eh_bar, NE / 32);
     mbar_init(drain_bar, 1);
     m->abort_flag = 0;
     fence_mbar_init();
@@ -886,56 +875,49 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     x.tq = tmem + ((uint32_t)(32 * x.q) << 16);
     x.xs = p.xs + (size_t)blockIdx.x * TILE * p.D;
     uint32_t acc_phase = 0, hb_phase = 0;
-    // Every thread makes its shared-memory operand writes visible to the async
-    // proxy and orders its TMEM reads, the named barrier collects them, then a
-    // single arrival hands the phase to the MMA issuer (e_bar, or eh_bar for
-    // the scan states in HB).
+    // The epilogue warps run decoupled: each makes its shared-memory operand
+    // writes visible to the async proxy, orders its TMEM reads and arrives on the
+    // hand-over barrier itself (e_bar and eh_bar count one arrival per warp), and
+    // each polls the MMA commits itself.  A failed wait sets the abort flag and
+    // every later wait fails fast, but no warp leaves the loop early: all warps
+    // keep taking the same sequence of named barriers (tile set-up, the norm
+    // reductions, the segment hand-overs), so none of them can be left waiting.
     auto signal_to = [&](uint32_t bar, bool wrote_operands) {
       if (wrote_operands) fence_proxy_async_smem();   // costly: only after operand writes
       tc_fence_before();
-      ebar_sync();
-      if (x.te == 0) mbar_arrive(bar);
+      __syncwarp();
+      if (x.lane == 0) mbar_arrive(bar);
     };
     auto signal = [&]() { signal_to(e_bar, true); };
-    // One elected epilogue thread polls the barrier; the others wait in the
-    // hardware named barrier (no shared-memory polling traffic competing with
-    // the tensor core's operand reads).  The vote makes the outcome uniform; the
-    // barrier also orders the shared-memory view for all participants.
-    auto wait_on = [&](uint32_t bar, uint32_t& ph) -> bool {
-      bool mine = true;
-      if (x.te == 0) mine = mbar_wait_spin(bar, ph, abort, WAIT_NS);
-      if (!ebar_all(mine)) {
-        set_abort(m, p.err);
-        return false;
-      }
+    auto wait_on = [&](uint32_t bar, uint32_t& ph) {
+      const bool got = mbar_wait(bar, ph, abort, WAIT_NS);   // try_wait: suspends instead of polling
+      if (!__all_sync(0xffffffffu, got) && x.lane == 0) set_abort(m, p.err);
       ph ^= 1u;
       tc_fence_after();
-      return true;
     };
-    auto wait_acc = [&]() -> bool { return wait_on(acc_bar, acc_phase); };
+    auto wait_acc = [&]() { wait_on(acc_bar, acc_phase); };
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
       ep_setup<FP16>(x, t, n_slabs);
       signal();
-      if (!wait_acc()) break;
+      wait_acc();
       ep_silu<FP16>(x, p.b_e1);
       signal();
-      if (!wait_acc()) break;
+      wait_acc();
       ep_residual<FP16>(x, p.b_e2, p.g, false);   // embedding output X0
       signal();
-      bool ok = true;
-      for (int l = 0; l < p.L && ok; ++l) {
+      for (int l = 0; l < p.L; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
           // biases are loaded before the wait so their latency hides behind it
           const size_t rb = (size_t)l * p.ROWS_IN + dc * 256;
           const float bz = p.b_in[rb + x.c], bn = p.b_in[rb + 128 + x.c];
-          if (!(ok = wait_acc())) break;
+          wait_acc();
           float z[32], n[32];
           scan_load(x, z, n);
           signal_to(e_bar, false);   // the z/n columns are free for the next chunk
           scan_gates(x, z, n, bz, bn);
           // HB still feeds the merge of the previous chunk (the gate hand-over
           // covers the last merge of the previous layer)
-          if (dc > 0 && !(ok = wait_on(hb_bar, hb_phase))) break;
+          if (dc > 0) wait_on(hb_bar, hb_phase);
           scan_chain_store<FP16>(x, z, n);
           signal_to(eh_bar, true);
         }
@@ -943,30 +925,29 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         // pipelines the next tile's products behind each); with d_model 256 the
         // SiLU of tile 0 goes to HB (MLP1 still reads XB rows 0-127 then)
         const float* b1 = p.b_1 + (size_t)l * p.D;
-        if (!ok || !(ok = wait_acc())) break;
+        wait_acc();
         ep_gate<FP16>(x, l, 0);
         signal();
         if (x.MT == 2) {
-          if (!(ok = wait_acc())) break;
+          wait_acc();
           ep_gate<FP16>(x, l, 1);
           signal();
-          if (!(ok = wait_acc())) break;
+          wait_acc();
           ep_silu_mt<FP16>(x, b1, 0, 256, x.hb, 0);
           signal();
-          if (!(ok = wait_acc())) break;
+          wait_acc();
           ep_silu_mt<FP16>(x, b1, 1, 256, x.xb, 128);
           signal();
         } else {
-          if (!(ok = wait_acc())) break;
+          wait_acc();
           ep_silu_mt<FP16>(x, b1, 0, 256, x.xb, 0);
           signal();
         }
-        if (!(ok = wait_acc())) break;
+        wait_acc();
         const bool last = l == p.L - 1;
         ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
         if (!last) signal();
       }
-      if (!ok) break;
     }
   }
   tc_fence_before();
