@@ -795,7 +795,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       return true;
     };
     auto handover = [&](uint32_t e) -> bool {
-      if (!wait_bar((e & S_W_E) ? e_bar : eh_bar, (e & S_W_E) ? e_phase : eh_phase, true)) return false;
+      if (!wait_bar((e & S_W_E) ? e_bar : eh_bar, (e & S_W_E) ? e_phase : eh_phase, false)) return false;
       tc_fence_after();
       return true;
     };
