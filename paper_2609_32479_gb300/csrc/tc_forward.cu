@@ -79,7 +79,8 @@ struct TcParams {
   float* out_q;
   float* pool;   // [B][D] pooled means (the caller's buffer or an internal one)
   float* xs;
-  const int32_t* slab_start;
+  const int32_t* slab_start;   // slab s = tracks order[slab_start[s] .. slab_start[s + 1])
+  const int32_t* order;        // tracks in packing order
   const int32_t* n_slabs;
   const uint32_t* sched_p;   // per block: map | col/64 << 4 | row << 8
   const uint32_t* sched_m;   // per block: b offset | bsel << 13 | tcol/128 << 14 | S_* flags
@@ -591,9 +592,10 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
       if (s >= n_slabs) break;
       const int b0 = p.slab_start[s];
       const int cnt = p.slab_start[s + 1] - b0;
-      int n = 0, bad = 0;
+      int n = 0, bad = 0, trk = 0;
       if (x.lane < cnt) {
-        n = p.n_hits[b0 + x.lane];
+        trk = p.order[b0 + x.lane];
+        n = p.n_hits[trk];
         bad = (n < 1 || n > p.T);
         if (bad) n = 0;
       }
@@ -606,7 +608,7 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
       if (x.lane < cnt) {
         const int slot = ns + x.lane;
         const int c0 = SLAB * hf + incl - n;
-        m->slot_track[slot] = b0 + x.lane;
+        m->slot_track[slot] = trk;
         m->slot_n[slot] = n;
         m->slot_bad[slot] = bad;
         for (int t = 0; t < n; ++t) {
@@ -978,34 +980,65 @@ __global__ void build_schedule(const __grid_constant__ TcParams p, uint32_t* sp,
 // ------------------------------------------------------------------ packing
 // One warp per segment of SEG tracks packs whole tracks greedily into slabs of
 // at most 64 hits and MAX_TRK_SLAB tracks; every segment starts a new slab.
-__global__ void plan_segments(const int32_t* __restrict__ n_hits, int64_t B, int T, int32_t* __restrict__ seg_count,
-                              int32_t* __restrict__ seg_slabs) {
+// Packing of one segment of up to SEG tracks into slabs of at most SLAB hits and
+// MAX_TRK_SLAB tracks (one warp per segment, decisions by lane 0 so the order is
+// deterministic): best fit over length buckets, each slab taking the longest
+// remaining track that still fits until none does; tracks with an invalid hit
+// count take a slot but no columns, at the end.  A track's results do not
+// depend on where it is packed.  Writes the segment's slice of the packing order
+// and the order positions where its slabs start.
+__global__ void __launch_bounds__(32) plan_pack(const int32_t* __restrict__ n_hits, int64_t B, int T,
+                                                int32_t* __restrict__ seg_count, int32_t* __restrict__ seg_slabs,
+                                                int32_t* __restrict__ order) {
+  __shared__ int32_t cnt[SLAB + 1], pos[SLAB + 2];
+  __shared__ int16_t len_of[SEG], items[SEG];
   const int seg = blockIdx.x, lane = threadIdx.x;
   const int64_t b0 = (int64_t)seg * SEG;
-  const int64_t b1 = (b0 + SEG < B) ? b0 + SEG : B;
-  int32_t* out = seg_slabs + (size_t)seg * (SEG + 1);
-  int cnt = 1, cur = 0, trk = 0;
-  if (lane == 0) out[0] = (int32_t)b0;
-  for (int64_t base = b0; base < b1; base += 32) {
-    int v = 0;
-    if (base + lane < b1) {
-      v = n_hits[base + lane];
-      if (v < 1 || v > T) v = 0;
-    }
-    const int lim = (int)((b1 - base) < 32 ? (b1 - base) : 32);
-    for (int i = 0; i < lim; ++i) {
-      const int ni = __shfl_sync(0xffffffffu, v, i);
-      if (trk == MAX_TRK_SLAB || cur + ni > SLAB) {
-        if (lane == 0) out[cnt] = (int32_t)(base + i);
-        ++cnt;
-        cur = 0;
-        trk = 0;
-      }
-      cur += ni;
-      ++trk;
-    }
+  const int nt = (int)((b0 + SEG < B) ? SEG : B - b0);
+  for (int i = lane; i <= SLAB; i += 32) cnt[i] = 0;
+  __syncwarp();
+  for (int i = lane; i < nt; i += 32) {
+    int v = n_hits[b0 + i];
+    if (v < 1 || v > T) v = 0;
+    len_of[i] = (int16_t)v;
   }
-  if (lane == 0) seg_count[seg] = cnt;
+  __syncwarp();
+  if (lane == 0) {
+    for (int i = 0; i < nt; ++i) ++cnt[len_of[i]];
+    pos[0] = 0;
+    for (int l = 0; l <= SLAB; ++l) pos[l + 1] = pos[l] + cnt[l];
+    for (int i = 0; i < nt; ++i) items[pos[len_of[i]]++] = (int16_t)i;   // pos[l] -> end of bucket l
+    int32_t* out = seg_slabs + (size_t)seg * (SEG + 1);
+    int o = 0, ns = 0, cap = SLAB, ntr = 0;
+    int remaining = nt - cnt[0];
+    out[ns++] = (int32_t)b0;
+    int top = T < SLAB ? T : SLAB;
+    while (remaining > 0) {
+      int l = cap < top ? cap : top;
+      while (l >= 1 && cnt[l] == 0) --l;
+      if (l >= 1 && ntr < MAX_TRK_SLAB) {
+        order[b0 + o++] = (int32_t)(b0 + items[pos[l] - cnt[l]]);   // bucket l, next in track order
+        --cnt[l];
+        cap -= l;
+        ++ntr;
+        --remaining;
+      } else {   // the slab is full: start the next one
+        out[ns++] = (int32_t)(b0 + o);
+        cap = SLAB;
+        ntr = 0;
+      }
+    }
+    for (int k = 0; k < cnt[0]; ++k) {   // invalid tracks
+      if (ntr == MAX_TRK_SLAB) {
+        out[ns++] = (int32_t)(b0 + o);
+        ntr = 0;
+      }
+      order[b0 + o++] = (int32_t)(b0 + items[pos[0] - cnt[0] + k]);
+      ++ntr;
+    }
+    if (o == 0) ns = 0;   // (an empty segment cannot occur: nt >= 1)
+    seg_count[seg] = ns;
+  }
 }
 
 // Exclusive scan of the per-segment slab counts (one block), total and sentinel.
@@ -1315,7 +1348,8 @@ struct tf_tc_state {
   uint16_t *w_e1 = nullptr, *w_e2 = nullptr, *w_in = nullptr, *w_m = nullptr, *w_1 = nullptr, *w_2 = nullptr;
   float *b_e1 = nullptr, *b_e2 = nullptr, *g = nullptr, *b_in = nullptr, *b_m = nullptr, *b_1 = nullptr,
         *b_2 = nullptr, *hg = nullptr, *hw1t = nullptr, *hb1 = nullptr, *hw2 = nullptr, *hb2 = nullptr;
-  int32_t *seg_count = nullptr, *seg_off = nullptr, *seg_slabs = nullptr, *slab_start = nullptr, *n_slabs = nullptr;
+  int32_t *seg_count = nullptr, *seg_off = nullptr, *seg_slabs = nullptr, *slab_start = nullptr, *n_slabs = nullptr,
+          *order = nullptr;
   uint32_t* sched = nullptr;   // [2][MAX_SCHED]: producer entries, then MMA entries
   int n_sched = 0;
   float* xs = nullptr;
@@ -1454,12 +1488,13 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   }
   // ---- packing buffers and the per-CTA residual scratch
   const int nseg_max = (int)((MAXB + SEG - 1) / SEG);
-  const size_t plan_ints = (size_t)nseg_max * 2 + (size_t)nseg_max * (SEG + 1) + (size_t)MAXB + 2 + 64;
+  const size_t plan_ints = (size_t)nseg_max * 2 + (size_t)nseg_max * (SEG + 1) + (size_t)MAXB + 2 + 64 + (size_t)MAXB;
   if (cudaMalloc(&t->seg_count, plan_ints * 4) != cudaSuccess) return TRACKFIT_ERR_OOM;
   t->seg_off = t->seg_count + nseg_max;
   t->seg_slabs = t->seg_off + nseg_max;
   t->slab_start = t->seg_slabs + (size_t)nseg_max * (SEG + 1);
   t->n_slabs = t->slab_start + MAXB + 2;
+  t->order = t->n_slabs + 64;
   if (cudaMalloc(&t->xs, (size_t)t->nsm * TILE * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
   if (cudaMalloc(&t->pool, (size_t)POOL_TRACKS * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
   // ---- tensor maps
@@ -1503,6 +1538,7 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   for (int i = 0; i < NMAPS; ++i) p.tm[i] = t->tm[i];
   p.xs = t->xs;
   p.slab_start = t->slab_start;
+  p.order = t->order;
   p.n_slabs = t->n_slabs;
   p.sched_p = t->sched;
   p.sched_m = t->sched + MAX_SCHED;
@@ -1557,7 +1593,7 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   for (int64_t c0 = 0; c0 < B; c0 += chunk) {
     const int64_t nb = (B - c0 < chunk) ? B - c0 : chunk;
     const int nseg = (int)((nb + SEG - 1) / SEG);
-    plan_segments<<<nseg, 32, 0, st>>>(n_hits + c0, nb, s.T, t->seg_count, t->seg_slabs);
+    plan_pack<<<nseg, 32, 0, st>>>(n_hits + c0, nb, s.T, t->seg_count, t->seg_slabs, t->order);
     plan_scan<<<1, 1024, 0, st>>>(t->seg_count, nseg, nb, t->seg_off, t->n_slabs, t->slab_start);
     plan_scatter<<<nseg, 128, 0, st>>>(t->seg_count, t->seg_off, t->seg_slabs, t->slab_start);
     p.hits = hits + c0 * s.T * 5;
