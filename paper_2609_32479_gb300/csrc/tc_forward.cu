@@ -1286,26 +1286,37 @@ __global__ void __launch_bounds__(HEAD_NT, 1) head_kernel(const __grid_constant_
       if (lane == 0) bad_s[i] = bad;
     }
     __syncthreads();
-    {   // hidden unit j of tracks sg, sg + 2, ...
-      const int j = tid & 127, sg = tid >> 7;
-      float a[HEAD_TRK / 2];
+    {   // hidden units 4*j4 .. 4*j4+3 of tracks 4*tg .. 4*tg+3 (16-byte loads of
+        // both operands: 8 loads per 64 FMAs); the sum over c runs in order
+      const int j4 = tid & 31, tg = tid >> 5;
+      float a[4][4];
 #pragma unroll
-      for (int i = 0; i < HEAD_TRK / 2; ++i) a[i] = b1s[j];
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) a[r][u] = b1s[4 * j4 + u];
 #pragma unroll 2
       for (int c = 0; c < D; c += 4) {
-        const float w0 = w1t[c * 128 + j], w1 = w1t[(c + 1) * 128 + j], w2v = w1t[(c + 2) * 128 + j],
-                    w3 = w1t[(c + 3) * 128 + j];
+        float4 w[4], xr[4];
 #pragma unroll
-        for (int i = 0; i < HEAD_TRK / 2; ++i) {
-          const float4 v = *reinterpret_cast<const float4*>(xv + (sg + 2 * i) * D + c);
-          a[i] = fmaf(w0, v.x, a[i]);
-          a[i] = fmaf(w1, v.y, a[i]);
-          a[i] = fmaf(w2v, v.z, a[i]);
-          a[i] = fmaf(w3, v.w, a[i]);
+        for (int k = 0; k < 4; ++k) w[k] = *reinterpret_cast<const float4*>(w1t + (c + k) * 128 + 4 * j4);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) xr[r] = *reinterpret_cast<const float4*>(xv + (4 * tg + r) * D + c);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const float xk[4] = {xr[r].x, xr[r].y, xr[r].z, xr[r].w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            a[r][0] = fmaf(w[k].x, xk[k], a[r][0]);
+            a[r][1] = fmaf(w[k].y, xk[k], a[r][1]);
+            a[r][2] = fmaf(w[k].z, xk[k], a[r][2]);
+            a[r][3] = fmaf(w[k].w, xk[k], a[r][3]);
+          }
         }
       }
 #pragma unroll
-      for (int i = 0; i < HEAD_TRK / 2; ++i) hid[(sg + 2 * i) * 128 + j] = silu(a[i]);
+      for (int r = 0; r < 4; ++r)
+        *reinterpret_cast<float4*>(hid + (4 * tg + r) * 128 + 4 * j4) =
+            make_float4(silu(a[r][0]), silu(a[r][1]), silu(a[r][2]), silu(a[r][3]));
     }
     __syncthreads();
     // outputs; the dot product for output o starts at column 4o (mod 128), so the
