@@ -99,6 +99,7 @@ struct TcParams {
   int fp16;
   float rms_eps;
   float feat_min[5], feat_inv_hi[5], feat_inv_lo[5], scale[16];
+  int scale_doubling;   // scale[k + 3] == 2 scale[k] for every k: Fourier by angle doubling
 };
 
 struct Misc {
@@ -649,29 +650,68 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
   // u = (v - min) / (max - min) and the argument s_k * u as unevaluated sums of
   // two floats (error-free TwoSum / TwoProduct with fma), reduced modulo 2
   // exactly, so sin(pi s_k u) carries only the final fp32 rounding.
-  for (int idx = x.te; idx < TILE * 5; idx += NE) {
-    const int col = idx & (TILE - 1), f = idx >> 7;
-    const bool valid = (m->col_flags[col] & F_VALID) != 0;
+  auto arg = [&](int col, int f, float sk) -> float {
     const float v = m->hs[col][f], mn = -p.feat_min[f];
     const float dh = v + mn;
     const float bv = dh - v;
     const float dl = (v - (dh - bv)) + (mn - bv);
     const float uh = dh * p.feat_inv_hi[f];
     const float ul = fmaf(dh, p.feat_inv_hi[f], -uh) + fmaf(dh, p.feat_inv_lo[f], dl * p.feat_inv_hi[f]);
-    const uint32_t cb = x.hb + (uint32_t)((col & 7) * 2);
-#pragma unroll 4
-    for (int k = 0; k < 16; ++k) {
-      const float sk = p.scale[k];
-      const float xh = uh * sk;
-      const float xl = fmaf(uh, sk, -xh) + ul * sk;
-      const float r = (xh - 2.0f * rintf(0.5f * xh)) + xl;
-      float sn = 0.0f, cs = 0.0f;
-      if (valid) {
-        sn = sinpif(r);
-        cs = cospif(r);
+    const float xh = uh * sk;
+    const float xl = fmaf(uh, sk, -xh) + ul * sk;
+    return (xh - 2.0f * rintf(0.5f * xh)) + xl;
+  };
+  if (p.scale_doubling) {
+    // s_{k+3} = 2 s_k: sin/cos evaluated for the scales k = 0-2, 6-8, 12-14 and
+    // the others by one step of the double angle identities (2 s c, (c - s)(c + s)),
+    // so no value is more than one doubling (a few ulp) from an evaluated one;
+    // one work item = 8 columns of one feature and one evaluated scale, stored as
+    // 16-byte chunks of the operand
+    for (int it = x.te; it < (TILE / 8) * 5 * 9; it += NE) {
+      const int g = it % (TILE / 8), fk = it / (TILE / 8), f = fk % 5, bi = fk / 5;
+      const int kb = (bi / 3) * 6 + bi % 3;
+      float sn[8], cs[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int col = 8 * g + j;
+        sn[j] = 0.0f;
+        cs[j] = 0.0f;
+        if (m->col_flags[col] & F_VALID) {
+          const float r = arg(col, f, p.scale[kb]);
+          sn[j] = sinpif(r);
+          cs[j] = cospif(r);
+        }
       }
-      st_shared_u16(cb + bchunk(f * 32 + k, col >> 3), to16<FP16>(sn));
-      st_shared_u16(cb + bchunk(f * 32 + 16 + k, col >> 3), to16<FP16>(cs));
+#pragma unroll 1
+      for (int k = kb; k < 16 && k <= kb + 3; k += 3) {
+        st_shared_v4(x.hb + bchunk(f * 32 + k, g), pack2<FP16>(sn[0], sn[1]), pack2<FP16>(sn[2], sn[3]),
+                     pack2<FP16>(sn[4], sn[5]), pack2<FP16>(sn[6], sn[7]));
+        st_shared_v4(x.hb + bchunk(f * 32 + 16 + k, g), pack2<FP16>(cs[0], cs[1]), pack2<FP16>(cs[2], cs[3]),
+                     pack2<FP16>(cs[4], cs[5]), pack2<FP16>(cs[6], cs[7]));
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float s2 = 2.0f * sn[j] * cs[j], c2 = (cs[j] - sn[j]) * (cs[j] + sn[j]);
+          sn[j] = s2;
+          cs[j] = c2;
+        }
+      }
+    }
+  } else {
+    for (int idx = x.te; idx < TILE * 5; idx += NE) {
+      const int col = idx & (TILE - 1), f = idx >> 7;
+      const bool valid = (m->col_flags[col] & F_VALID) != 0;
+      const uint32_t cb = x.hb + (uint32_t)((col & 7) * 2);
+#pragma unroll 4
+      for (int k = 0; k < 16; ++k) {
+        float sn = 0.0f, cs = 0.0f;
+        if (valid) {
+          const float r = arg(col, f, p.scale[k]);
+          sn = sinpif(r);
+          cs = cospif(r);
+        }
+        st_shared_u16(cb + bchunk(f * 32 + k, col >> 3), to16<FP16>(sn));
+        st_shared_u16(cb + bchunk(f * 32 + 16 + k, col >> 3), to16<FP16>(cs));
+      }
     }
   }
 }
@@ -1585,6 +1625,9 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
     p.feat_inv_lo[f] = (float)(inv - (double)p.feat_inv_hi[f]);
   }
   for (int k = 0; k < 16; ++k) p.scale[k] = s.scale[k];
+  p.scale_doubling = 1;
+  for (int k = 0; k + 3 < 16; ++k)
+    if (s.scale[k + 3] != 2.0f * s.scale[k]) p.scale_doubling = 0;
   HeadParams hp;
   std::memset(&hp, 0, sizeof(hp));
   hp.T = s.T;
