@@ -309,8 +309,8 @@ def main():
     valid_hits = int(tb.n_hits.clip(0, m.max_hits).sum())
     flops = valid_hits * flops_per_hit(m) + B * flops_per_track_head(m)
     kern_avg_s = (kern_ms / max(kern_n, 1)) * 1e-3
-    # the library splits a step into launches (524,288 tracks each when, as here,
-    # no pooled output buffer is passed): per-launch work is the step's share
+    # the library splits a step into launches (1,048,576 tracks each when, as
+    # here, no pooled output buffer is passed): per-launch work is the step's share
     launches_per_step = max(kern_n // max(args.steps, 1), 1) if kern_n else 1
     flops_launch = flops / launches_per_step
     dtype_tf = {1: "bf16_tflops", 2: "bf16_tflops"}.get(m.precision, "bf16_tflops")
@@ -339,7 +339,7 @@ def main():
             "e2e": {"value": e2e_value, "unit": "tracks/s", "h2d_bytes_per_step": int(tb.hits.nbytes + tb.n_hits.nbytes),
                     "d2h_bytes_per_step": int(B * 5 * 4), "matches_device_result": same},
             # per launch chunk: three packing kernels, the fused encoder, the head
-            "gpu_launches": int(5 * math.ceil(B / 524288) * args.steps) if tf.path.startswith("tcgen05") else None,
+            "gpu_launches": int(5 * math.ceil(B / 1048576) * args.steps) if tf.path.startswith("tcgen05") else None,
             "device_errors": {"status": st, "bad_tracks": nbad}}
     if not args.no_cpu_baseline and world == 1:
         v, idx, ref, dt = run_oracle_sample(w, blob, tb, args.cpu_budget)

@@ -53,7 +53,7 @@ constexpr int SCHED_BYTES = 2 * MAX_SCHED * 4;   // both schedule tables, copied
 constexpr int MAX_STAGES = 8;
 constexpr int SEG = 1024;                 // tracks per packing segment
 constexpr int64_t MAXB = 4194304;         // tracks per launch chunk
-constexpr int64_t POOL_TRACKS = 524288;   // tracks per launch chunk when the pooled means go to the internal buffer
+constexpr int64_t POOL_TRACKS = 1048576;  // tracks per launch chunk when the pooled means go to the internal buffer
 constexpr uint64_t WAIT_NS = 2000000000ull;
 constexpr uint64_t DRAIN_NS = 200000000ull;
 constexpr int B_SBO = 2048;               // k-group stride of the MN-major activation operand
