@@ -220,7 +220,14 @@ __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
         f(map, r0 + mt * 128, kc * 64, 4, tcol0 + mt * 128, BSEL_XB, kc * 64, onto || kc > 0,
           (mt == 0 && kc == 0) ? W_E : W_NONE, (mt == MT - 1 && kc == KD - 1) ? C_ACC : C_NONE);
   };
-  dense(MAP_E2, 0, 0, false);
+  if (MT == 1) {
+    dense(MAP_E2, 0, 0, false);
+  } else {   // committed per 128-channel tile, like MLP2
+    for (int mt = 0; mt < 2; ++mt)
+      for (int kc = 0; kc < KD; ++kc)
+        f(MAP_E2, mt * 128, kc * 64, 4, mt * 128, BSEL_XB, kc * 64, kc > 0, (mt == 0 && kc == 0) ? W_E : W_NONE,
+          kc == KD - 1 ? C_ACC : C_NONE);
+  }
   for (int l = 0; l < p.L; ++l) {
     const int rb = l * p.ROWS_IN;
     auto zn = [&](int k) {   // z and n of scan chunk k -> TMEM columns 256.. and 384..
@@ -230,7 +237,17 @@ __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
         f(MAP_IN, rb + k * 256 + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, W_NONE,
           kc == KD - 1 ? C_ACC : C_NONE);
     };
-    zn(0);
+    if (MT == 1) {
+      zn(0);
+    } else {   // x_hat arrives one 128-channel tile at a time (K rows 0-127, then 128-255)
+      for (int kh = 0; kh < 2; ++kh) {
+        for (int kc = 2 * kh; kc < 2 * kh + 2; ++kc)
+          f(MAP_IN, rb, kc * 64, 4, 256, BSEL_XB, kc * 64, kc > 0, kc == 2 * kh ? W_E : W_NONE, C_NONE);
+        for (int kc = 2 * kh; kc < 2 * kh + 2; ++kc)
+          f(MAP_IN, rb + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, W_NONE,
+            kc == KD - 1 ? C_ACC : C_NONE);
+      }
+    }
     for (int k = 0; k < p.NDC; ++k) {
       if (k + 1 < p.NDC) {
         zn(k + 1);
@@ -265,8 +282,9 @@ __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
         f(MAP_1, r1, kc * 64, 4, 256, BSEL_XB, kc * 64, kc > 0, (kc & 1) ? W_NONE : W_E, kc == 3 ? C_ACC : C_NONE);
       for (int kc = 0; kc < 4; ++kc)
         f(MAP_1, r1 + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, W_NONE, kc == 3 ? C_ACC : C_NONE);
-      for (int kc = 0; kc < 4; ++kc)
-        f(MAP_2, r1, kc * 64, 4, 0, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, true, (kc & 1) ? W_NONE : W_E, C_NONE);
+      for (int kc = 0; kc < 4; ++kc)   // tile 0 of MLP2 completes first (the residual starts on it)
+        f(MAP_2, r1, kc * 64, 4, 0, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, true, (kc & 1) ? W_NONE : W_E,
+          kc == 3 ? C_ACC : C_NONE);
       for (int kc = 0; kc < 4; ++kc)
         f(MAP_2, r1 + 128, kc * 64, 4, 128, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, true, W_NONE,
           kc == 3 ? C_ACC : C_NONE);
@@ -356,15 +374,18 @@ __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
   return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
 }
 
-template <bool FP16, int MT, bool pool>
-__device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain) {
+template <bool FP16, int MT, bool pool, class W, class S>
+__device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
+                                              S&& signal_tile) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;   // d_model
   const uint8_t* flags = x.m->col_flags;
   const uint32_t vm = x.m->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
   // X = acc + bias (the accumulator already holds x' + MLP for a layer, the
-  // embedding product for the embedding), zero on pad columns; per 16-column
-  // half, every tile's accumulator is read under one TMEM wait
+  // embedding product for the embedding), zero on pad columns.  The products
+  // complete one 128-channel tile at a time: tile 0 is processed while tile 1 is
+  // still being computed (wait_tile), and x_hat is handed over per tile
+  // (signal_tile) so the next products can start on its K rows.
   float bias_v[MT];
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) bias_v[mt] = bias[mt * 128 + x.c];
@@ -378,23 +399,23 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) run[mt] = x.m->carry[x.half][mt][x.c];
   }
+  float sq[32];
 #pragma unroll
-  for (int hh = 0; hh < 2; ++hh) {
-    const int c0 = x.col0 + 16 * hh;
-    float v[MT][16];
+  for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt) tmem_ld16(x.tq + mt * 128 + c0, v[mt]);
-    tmem_ld_wait();
-    float sq[16];
+  for (int mt = 0; mt < MT; ++mt) {
+    if (mt > 0) wait_tile();
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const bool valid = (vm >> (16 * hh + i)) & 1u;
-      sq[i] = 0.0f;
+    for (int hh = 0; hh < 2; ++hh) {
+      const int c0 = x.col0 + 16 * hh;
+      float v[16];
+      tmem_ld16(x.tq + mt * 128 + c0, v);
+      tmem_ld_wait();
 #pragma unroll
-      for (int mt = 0; mt < MT; ++mt) {
-        const float val = valid ? v[mt][i] + bias_v[mt] : 0.0f;
-        v[mt][i] = val;
-        sq[i] = fmaf(val, val, sq[i]);
+      for (int i = 0; i < 16; ++i) {
+        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
+        v[i] = val;
+        sq[16 * hh + i] = fmaf(val, val, sq[16 * hh + i]);
         if constexpr (pool) {
           const int fl = flags[c0 + i];
           run[mt] = (fl & F_FIRST) ? val : run[mt] + val;
@@ -404,18 +425,11 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
           }
         }
       }
-    }
-    if constexpr (!pool) {
-      // the residual stream to the scratch, column-major (a warp's store covers
-      // 32 consecutive channels: one 128-byte line)
-#pragma unroll
-      for (int mt = 0; mt < MT; ++mt) {
+      if constexpr (!pool) {   // the residual stream to the scratch (a warp's store: one 128-byte line)
         float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[mt][i];
+        for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
       }
-      const float t = reduce_scatter16(sq, x.lane);
-      if (x.lane < 16) x.m->part[x.q][c0 + x.lane] = t;
     }
   }
   if constexpr (pool) {
@@ -425,6 +439,14 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       carry_pass(x);
     }
   } else {
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      float h16[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) h16[i] = sq[16 * hh + i];
+      const float t = reduce_scatter16(h16, x.lane);
+      if (x.lane < 16) x.m->part[x.q][x.col0 + 16 * hh + x.lane] = t;
+    }
     ebar_sync();
     if (x.te < TILE) {
       const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
@@ -432,48 +454,48 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
     }
     ebar_sync();
 #pragma unroll
-    for (int hh = 0; hh < 2; ++hh) {
-      const int c0 = x.col0 + 16 * hh;
-      float v[MT][16];
+    for (int mt = 0; mt < MT; ++mt) {
+      const float g = gain[mt * 128 + x.c];
 #pragma unroll
-      for (int mt = 0; mt < MT; ++mt) tmem_ld16(x.tq + mt * 128 + c0, v[mt]);
-      float rv[16];
-      const float4* rp = reinterpret_cast<const float4*>(x.m->rinv + c0);
+      for (int hh = 0; hh < 2; ++hh) {
+        const int c0 = x.col0 + 16 * hh;
+        float v[16], rv[16];
+        tmem_ld16(x.tq + mt * 128 + c0, v);
+        const float4* rp = reinterpret_cast<const float4*>(x.m->rinv + c0);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float4 r4 = rp[i];
-        rv[4 * i] = r4.x;
-        rv[4 * i + 1] = r4.y;
-        rv[4 * i + 2] = r4.z;
-        rv[4 * i + 3] = r4.w;
-      }
-      tmem_ld_wait();
-#pragma unroll
-      for (int mt = 0; mt < MT; ++mt) {
-        const float g = gain[mt * 128 + x.c];
+        for (int i = 0; i < 4; ++i) {
+          const float4 r4 = rp[i];
+          rv[4 * i] = r4.x;
+          rv[4 * i + 1] = r4.y;
+          rv[4 * i + 2] = r4.z;
+          rv[4 * i + 3] = r4.w;
+        }
+        tmem_ld_wait();
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const float val = ((vm >> (16 * hh + i)) & 1u) ? v[mt][i] + bias_v[mt] : 0.0f;
-          v[mt][i] = val * g * rv[i];
+          const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
+          v[i] = val * g * rv[i];
         }
-        store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v[mt]);
+        store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v);
       }
+      signal_tile();   // x_hat of this tile is in XB
     }
   }
 }
 
-template <bool FP16>
-__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, const float* gain, bool pool) {
+template <bool FP16, class W, class S>
+__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, const float* gain, bool pool,
+                                            W&& wait_tile, S&& signal_tile) {
   if (x.MT == 2) {
     if (pool)
-      ep_residual_t<FP16, 2, true>(x, bias, gain);
+      ep_residual_t<FP16, 2, true>(x, bias, gain, wait_tile, signal_tile);
     else
-      ep_residual_t<FP16, 2, false>(x, bias, gain);
+      ep_residual_t<FP16, 2, false>(x, bias, gain, wait_tile, signal_tile);
   } else {
     if (pool)
-      ep_residual_t<FP16, 1, true>(x, bias, gain);
+      ep_residual_t<FP16, 1, true>(x, bias, gain, wait_tile, signal_tile);
     else
-      ep_residual_t<FP16, 1, false>(x, bias, gain);
+      ep_residual_t<FP16, 1, false>(x, bias, gain, wait_tile, signal_tile);
   }
 }
 
@@ -945,8 +967,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       ep_silu<FP16>(x, p.b_e1);
       signal();
       wait_acc();
-      ep_residual<FP16>(x, p.b_e2, p.g, false);   // embedding output X0
-      signal();
+      ep_residual<FP16>(x, p.b_e2, p.g, false, wait_acc, signal);   // embedding output X0
       for (int l = 0; l < p.L; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
           // biases are loaded before the wait so their latency hides behind it
@@ -987,8 +1008,8 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         }
         wait_acc();
         const bool last = l == p.L - 1;
-        ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last);
-        if (!last) signal();
+        ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last, wait_acc,
+                          signal);
       }
     }
   }
