@@ -12,12 +12,14 @@
 // cross-thread exchange.
 //
 // Tile: 128 hit columns = two 64-column slabs; each slab holds whole tracks
-// (packed greedily, unpadded).  Warp roles (320 threads):
-//   warp 0      TMA producer of weight blocks (warp-wide loop, one elected lane issues)
-//   warp 1      tcgen05.mma issuer (warp-wide loop, one elected lane issues), TMEM owner
-//   warps 2..9  epilogue: TMEM lane quadrant = warp % 4, column half = (warp-2)/4
-// TMEM (512 columns): R0,R1 = merge / MLP accumulators (d_model rows), R2,R3 =
-// z and n of one scan chunk, then the output-gate projection.
+// (packed by best fit, unpadded).  Warp roles (608 threads):
+//   warp 0       TMA producer of weight blocks (warp-wide loop, one elected lane issues)
+//   warp 1       tcgen05.mma issuer (warp-wide loop, one elected lane issues), TMEM owner
+//   warps 2..17  epilogue: TMEM lane quadrant = warp % 4, 32-column segment = (warp-2)/4
+//   warp 18      loader: column metadata and Fourier operand of the next tile
+// TMEM (512 columns): R0,R1 = merge accumulators, then x' with the MLP2 product
+// accumulated onto it (d_model rows); R2,R3 = z and n of one scan chunk, then the
+// output-gate projection, then MLP1 (and the embedding's first product).
 // The fp32 residual stream of the tile lives in a per-CTA global scratch slab
 // (L2-resident), never in HBM-sized intermediates.
 #include <cuda.h>
@@ -37,7 +39,7 @@ using namespace sm100;
 
 namespace {
 
-constexpr int NT = 576;                   // warp 0 TMA, warp 1 MMA issuer, warps 2..17 epilogue
+constexpr int NT = 608;                   // warp 0 TMA, warp 1 MMA issuer, warps 2..17 epilogue, warp 18 loader
 constexpr int NE = 512;                   // epilogue threads
 constexpr int SEGW = 32;                  // hit columns per epilogue thread (half a slab)
 constexpr int TILE = 128;
@@ -100,24 +102,30 @@ struct TcParams {
   float rms_eps;
   float feat_min[5], feat_inv_hi[5], feat_inv_lo[5], scale[16];
   int scale_doubling;   // scale[k + 3] == 2 scale[k] for every k: Fourier by angle doubling
+  uint8_t* fbuf;        // per CTA two Fourier operands (HB byte images) written by the loader warp
 };
 
-struct Misc {
-  uint64_t full[MAX_STAGES], empty[MAX_STAGES];
-  uint64_t acc_bar, e_bar, hb_bar, eh_bar, drain_bar;
-  uint32_t tmem_base;
-  int abort_flag;
-  int n_slots;
-  int pad_;
-  int slot_track[MAX_TRK_TILE], slot_n[MAX_TRK_TILE], slot_bad[MAX_TRK_TILE];
-  uint8_t col_flags[TILE], col_slot[TILE], col_tpos[TILE], pad2_[128];
-  alignas(16) float part[4][TILE];
+// Column metadata of one tile, written by the loader warp one tile ahead (two
+// buffers, alternating by tile).
+struct TileMeta {
+  int slot_track[MAX_TRK_TILE], slot_n[MAX_TRK_TILE];
+  uint8_t col_flags[TILE], col_slot[TILE];
   // per column half h, 32-column word w: bit j = column 64h + 32w + j starts a
   // track (first), ends one (last), holds a hit (valid)
   uint32_t m_first[2][2], m_last[2][2], m_valid[2][2];
+};
+struct Misc {
+  uint64_t full[MAX_STAGES], empty[MAX_STAGES];
+  uint64_t acc_bar, e_bar, hb_bar, eh_bar, drain_bar;
+  uint64_t meta_full[2], meta_free[2];   // loader -> epilogue, epilogue -> loader
+  uint32_t tmem_base;
+  int abort_flag;
+  TileMeta meta[2];
+  uint8_t col_tpos[TILE];   // the loader's own
+  alignas(16) float part[4][TILE];
   float carry[2][2][128];   // [slab][slot][channel]: states or pool sums between column segments
   alignas(16) float rinv[TILE];
-  float hs[TILE][5];
+  float hs[TILE][5];   // the loader's own
 };
 static_assert(sizeof(Misc) <= MISC_BYTES, "misc region too small");
 
@@ -146,16 +154,6 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {   // a -> low half
     return *reinterpret_cast<uint32_t*>(&v);
   }
 }
-template <bool FP16>
-__device__ __forceinline__ uint16_t to16(float a) {
-  if constexpr (FP16) {
-    __half v = __float2half_rn(a);
-    return *reinterpret_cast<uint16_t*>(&v);
-  } else {
-    __nv_bfloat16 v = __float2bfloat16_rn(a);
-    return *reinterpret_cast<uint16_t*>(&v);
-  }
-}
 
 // Byte offset, inside an MN-major 128-byte-swizzled operand with 128 columns, of
 // the 16-byte chunk that holds columns [8*n8, 8*n8+8) of k-row k.  Atoms are 8
@@ -166,9 +164,6 @@ __device__ __forceinline__ uint32_t bchunk(int k, int n8) {
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
-}
-__device__ __forceinline__ void st_shared_u16(uint32_t addr, uint16_t v) {
-  asm volatile("st.shared.u16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
 }
 
 // Write 32 consecutive columns [n0, n0+32) of k-row k (n0 % 32 == 0) as 16-bit operands.
@@ -207,9 +202,11 @@ __device__ __forceinline__ void ebar_sync() { asm volatile("bar.sync 1, 512;" ::
 template <class F>
 __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
   const int MT = p.D >> 7, KD = p.D >> 6;
+  // the embedding's first product goes to the z/n columns, so it can run while
+  // the epilogue still pools the previous tile from columns 0..
   for (int mt = 0; mt < MT; ++mt)
     for (int kc = 0; kc < 3; ++kc)
-      f(MAP_E1, mt * 128, kc * 64, kc == 2 ? 2 : 4, mt * 128, BSEL_HB, kc * 64, kc > 0,
+      f(MAP_E1, mt * 128, kc * 64, kc == 2 ? 2 : 4, 256 + mt * 128, BSEL_HB, kc * 64, kc > 0,
         (mt == 0 && kc == 0) ? W_E : W_NONE, (mt == MT - 1 && kc == 2) ? C_ACC : C_NONE);
   // a dense D x D product from XB into accumulator columns 0.. (MT tiles of 128 rows)
   // a dense D x D product from XB into accumulator columns tcol0 + 128 mt; with
@@ -300,6 +297,7 @@ __device__ __forceinline__ void set_abort(Misc* m, unsigned long long* err) {
 struct ECtx {
   const TcParams* p;
   Misc* m;
+  const TileMeta* md;   // metadata of the tile being processed
   uint32_t xb, hb, tq;
   float* xs;
   // quadrant q (TMEM lanes / channels 32q..), column segment seg = 32-column
@@ -336,7 +334,7 @@ template <bool FP16, int MT>
 __device__ __forceinline__ void ep_silu_t(const ECtx& x, const float* bias) {
   float v[MT][32];
 #pragma unroll
-  for (int mt = 0; mt < MT; ++mt) tmem_ld32(x.tq + mt * 128 + x.col0, v[mt]);
+  for (int mt = 0; mt < MT; ++mt) tmem_ld32(x.tq + 256 + mt * 128 + x.col0, v[mt]);
   tmem_ld_wait();
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
@@ -379,8 +377,8 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
                                               S&& signal_tile) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;   // d_model
-  const uint8_t* flags = x.m->col_flags;
-  const uint32_t vm = x.m->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
+  const uint8_t* flags = x.md->col_flags;
+  const uint32_t vm = x.md->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
   // X = acc + bias (the accumulator already holds x' + MLP for a layer, the
   // embedding product for the embedding), zero on pad columns.  The products
   // complete one 128-channel tile at a time: tile 0 is processed while tile 1 is
@@ -420,8 +418,8 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
           const int fl = flags[c0 + i];
           run[mt] = (fl & F_FIRST) ? val : run[mt] + val;
           if (fl & F_LAST) {
-            const int s = x.m->col_slot[c0 + i];
-            p.pool[(size_t)x.m->slot_track[s] * D + mt * 128 + x.c] = run[mt] / (float)x.m->slot_n[s];
+            const int s = x.md->col_slot[c0 + i];
+            p.pool[(size_t)x.md->slot_track[s] * D + mt * 128 + x.c] = run[mt] / (float)x.md->slot_n[s];
           }
         }
       }
@@ -553,7 +551,7 @@ __device__ __forceinline__ void scan_load(const ECtx& x, float (&z)[32], float (
 // recurrence restarts (a track's first hit forward, its last in reverse) a = 0.
 // a replaces z, b replaces n.
 __device__ __forceinline__ void scan_gates(const ECtx& x, float (&z)[32], float (&n)[32], float bz, float bn) {
-  const uint32_t rm = x.q < 2 ? x.m->m_first[x.half][x.sub] : x.m->m_last[x.half][x.sub];
+  const uint32_t rm = x.q < 2 ? x.md->m_first[x.half][x.sub] : x.md->m_last[x.half][x.sub];
   const float cz = -bz * LOG2E_F;
 #pragma unroll
   for (int j = 0; j < 32; ++j) {
@@ -598,77 +596,72 @@ __device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&a)[32], 
   store_row32<FP16>(x.hb, x.c, x.col0, a);
 }
 
-// Tile set-up: slot/column metadata, gather of the valid hits, Fourier operand.
+// Tile set-up, run one tile ahead by the loader warp while the epilogue warps
+// work on the current tile: the column metadata of the tile's two slabs (into
+// the metadata buffer md), the features of its hits, and the Fourier operand
+// (the B operand of the embedding's first product) as the byte image of HB in
+// the CTA's global buffer fb, from which the epilogue copies it at tile start.
 template <bool FP16>
-__device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
-  const TcParams& p = *x.p;
-  Misc* m = x.m;
-  // the previous tile's last epilogue (pooling) may still read the column
-  // metadata in other warps
-  ebar_sync();
-  if (x.te < TILE) m->col_flags[x.te] = 0;
-  ebar_sync();
-  if (x.e == 0) {
-    int ns = 0;
-    for (int hf = 0; hf < 2; ++hf) {
-      const int s = 2 * tile + hf;
-      if (s >= n_slabs) break;
-      const int b0 = p.slab_start[s];
-      const int cnt = p.slab_start[s + 1] - b0;
-      int n = 0, bad = 0, trk = 0;
-      if (x.lane < cnt) {
-        trk = p.order[b0 + x.lane];
-        n = p.n_hits[trk];
-        bad = (n < 1 || n > p.T);
-        if (bad) n = 0;
-      }
-      int incl = n;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (x.lane >= o) incl += y;
-      }
-      if (x.lane < cnt) {
-        const int slot = ns + x.lane;
-        const int c0 = SLAB * hf + incl - n;
-        m->slot_track[slot] = trk;
-        m->slot_n[slot] = n;
-        m->slot_bad[slot] = bad;
-        for (int t = 0; t < n; ++t) {
-          const int col = c0 + t;
-          m->col_flags[col] = (uint8_t)(F_VALID | (t == 0 ? F_FIRST : 0) | (t == n - 1 ? F_LAST : 0));
-          m->col_slot[col] = (uint8_t)slot;
-          m->col_tpos[col] = (uint8_t)t;
-        }
-      }
-      ns += cnt;
+__device__ __forceinline__ void load_tile(const TcParams& p, Misc* m, TileMeta* md, uint8_t* fb, int tile,
+                                          int n_slabs, int lane) {
+  for (int c = lane; c < TILE; c += 32) md->col_flags[c] = 0;
+  __syncwarp();
+  int ns = 0;
+  for (int hf = 0; hf < 2; ++hf) {
+    const int s = 2 * tile + hf;
+    if (s >= n_slabs) break;
+    const int b0 = p.slab_start[s];
+    const int cnt = p.slab_start[s + 1] - b0;
+    int n = 0, trk = 0;
+    if (lane < cnt) {
+      trk = p.order[b0 + lane];
+      n = p.n_hits[trk];
+      if (n < 1 || n > p.T) n = 0;   // rejected by the packer's validity check: no columns
     }
-    if (x.lane == 0) m->n_slots = ns;
+    int incl = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane < cnt) {
+      const int slot = ns + lane;
+      const int c0 = SLAB * hf + incl - n;
+      md->slot_track[slot] = trk;
+      md->slot_n[slot] = n;
+      for (int t = 0; t < n; ++t) {
+        const int col = c0 + t;
+        md->col_flags[col] = (uint8_t)(F_VALID | (t == 0 ? F_FIRST : 0) | (t == n - 1 ? F_LAST : 0));
+        md->col_slot[col] = (uint8_t)slot;
+        m->col_tpos[col] = (uint8_t)t;
+      }
+    }
+    ns += cnt;
   }
-  ebar_sync();
-  if (x.te < 4) {   // column bitmasks (read after later barriers)
-    const int hf = x.te >> 1, w = x.te & 1;
+  __syncwarp();
+  if (lane < 4) {   // column bitmasks
+    const int hf = lane >> 1, w = lane & 1;
     uint32_t fm = 0, lm = 0, vm = 0;
     for (int j = 0; j < 32; ++j) {
-      const int f = m->col_flags[SLAB * hf + 32 * w + j];
+      const int f = md->col_flags[SLAB * hf + 32 * w + j];
       fm |= (uint32_t)((f & F_FIRST) != 0) << j;
       lm |= (uint32_t)((f & F_LAST) != 0) << j;
       vm |= (uint32_t)((f & F_VALID) != 0) << j;
     }
-    m->m_first[hf][w] = fm;
-    m->m_last[hf][w] = lm;
-    m->m_valid[hf][w] = vm;
+    md->m_first[hf][w] = fm;
+    md->m_last[hf][w] = lm;
+    md->m_valid[hf][w] = vm;
   }
-  for (int idx = x.te; idx < TILE * 5; idx += NE) {
+  for (int idx = lane; idx < TILE * 5; idx += 32) {
     const int col = idx / 5, f = idx - col * 5;
     float v = 0.0f;
-    if (m->col_flags[col] & F_VALID) {
-      const size_t trk = (size_t)m->slot_track[m->col_slot[col]];
+    if (md->col_flags[col] & F_VALID) {
+      const size_t trk = (size_t)md->slot_track[md->col_slot[col]];
       v = p.hits[(trk * p.T + m->col_tpos[col]) * 5 + f];
     }
     m->hs[col][f] = v;
   }
-  ebar_sync();
+  __syncwarp();
   // u = (v - min) / (max - min) and the argument s_k * u as unevaluated sums of
   // two floats (error-free TwoSum / TwoProduct with fma), reduced modulo 2
   // exactly, so sin(pi s_k u) carries only the final fp32 rounding.
@@ -683,59 +676,55 @@ __device__ __forceinline__ void ep_setup(const ECtx& x, int tile, int n_slabs) {
     const float xl = fmaf(uh, sk, -xh) + ul * sk;
     return (xh - 2.0f * rintf(0.5f * xh)) + xl;
   };
-  if (p.scale_doubling) {
-    // s_{k+3} = 2 s_k: sin/cos evaluated for the scales k = 0-2, 6-8, 12-14 and
-    // the others by one step of the double angle identities (2 s c, (c - s)(c + s)),
-    // so no value is more than one doubling (a few ulp) from an evaluated one;
-    // one work item = 8 columns of one feature and one evaluated scale, stored as
-    // 16-byte chunks of the operand
-    for (int it = x.te; it < (TILE / 8) * 5 * 9; it += NE) {
-      const int g = it % (TILE / 8), fk = it / (TILE / 8), f = fk % 5, bi = fk / 5;
-      const int kb = (bi / 3) * 6 + bi % 3;
-      float sn[8], cs[8];
+  auto put = [&](int row, int g, const float (&v)[8]) {
+    *reinterpret_cast<uint4*>(fb + bchunk(row, g)) =
+        make_uint4(pack2<FP16>(v[0], v[1]), pack2<FP16>(v[2], v[3]), pack2<FP16>(v[4], v[5]), pack2<FP16>(v[6], v[7]));
+  };
+  // one work item = 8 columns of one feature and one evaluated scale, stored as
+  // 16-byte chunks of the operand.  With s_{k+3} = 2 s_k, sin/cos are evaluated
+  // for the scales k = 0-2, 6-8, 12-14 only and the others follow by one step of
+  // the double angle identities (2 s c, (c - s)(c + s)), so no value is more than
+  // one doubling (a few ulp) from an evaluated one.
+  const int n_eval = p.scale_doubling ? 9 : 16;
+  for (int it = lane; it < (TILE / 8) * 5 * n_eval; it += 32) {
+    const int g = it % (TILE / 8), fk = it / (TILE / 8), f = fk % 5, bi = fk / 5;
+    const int kb = p.scale_doubling ? (bi / 3) * 6 + bi % 3 : bi;
+    float sn[8], cs[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int col = 8 * g + j;
+      sn[j] = 0.0f;
+      cs[j] = 0.0f;
+      if (md->col_flags[col] & F_VALID) {
+        const float r = arg(col, f, p.scale[kb]);
+        sn[j] = sinpif(r);
+        cs[j] = cospif(r);
+      }
+    }
+    put(f * 32 + kb, g, sn);
+    put(f * 32 + 16 + kb, g, cs);
+    if (p.scale_doubling && kb + 3 < 16) {
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        const int col = 8 * g + j;
-        sn[j] = 0.0f;
-        cs[j] = 0.0f;
-        if (m->col_flags[col] & F_VALID) {
-          const float r = arg(col, f, p.scale[kb]);
-          sn[j] = sinpif(r);
-          cs[j] = cospif(r);
-        }
+        const float s2 = 2.0f * sn[j] * cs[j], c2 = (cs[j] - sn[j]) * (cs[j] + sn[j]);
+        sn[j] = s2;
+        cs[j] = c2;
       }
-#pragma unroll 1
-      for (int k = kb; k < 16 && k <= kb + 3; k += 3) {
-        st_shared_v4(x.hb + bchunk(f * 32 + k, g), pack2<FP16>(sn[0], sn[1]), pack2<FP16>(sn[2], sn[3]),
-                     pack2<FP16>(sn[4], sn[5]), pack2<FP16>(sn[6], sn[7]));
-        st_shared_v4(x.hb + bchunk(f * 32 + 16 + k, g), pack2<FP16>(cs[0], cs[1]), pack2<FP16>(cs[2], cs[3]),
-                     pack2<FP16>(cs[4], cs[5]), pack2<FP16>(cs[6], cs[7]));
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float s2 = 2.0f * sn[j] * cs[j], c2 = (cs[j] - sn[j]) * (cs[j] + sn[j]);
-          sn[j] = s2;
-          cs[j] = c2;
-        }
-      }
-    }
-  } else {
-    for (int idx = x.te; idx < TILE * 5; idx += NE) {
-      const int col = idx & (TILE - 1), f = idx >> 7;
-      const bool valid = (m->col_flags[col] & F_VALID) != 0;
-      const uint32_t cb = x.hb + (uint32_t)((col & 7) * 2);
-#pragma unroll 4
-      for (int k = 0; k < 16; ++k) {
-        float sn = 0.0f, cs = 0.0f;
-        if (valid) {
-          const float r = arg(col, f, p.scale[k]);
-          sn = sinpif(r);
-          cs = cospif(r);
-        }
-        st_shared_u16(cb + bchunk(f * 32 + k, col >> 3), to16<FP16>(sn));
-        st_shared_u16(cb + bchunk(f * 32 + 16 + k, col >> 3), to16<FP16>(cs));
-      }
+      put(f * 32 + kb + 3, g, sn);
+      put(f * 32 + 16 + kb + 3, g, cs);
     }
   }
+}
+
+// Tile start on the epilogue side: the Fourier operand from the CTA's global
+// buffer into HB (five 16-byte chunks per thread, all loads in flight at once).
+__device__ __forceinline__ void ep_fourier_in(const ECtx& x, const uint8_t* fb) {
+  static_assert(EB_BYTES == 5 * 16 * NE, "one chunk per thread per round");
+  uint4 v[5];
+#pragma unroll
+  for (int r = 0; r < 5; ++r) v[r] = reinterpret_cast<const uint4*>(fb)[r * NE + x.te];
+#pragma unroll
+  for (int r = 0; r < 5; ++r) st_shared_v4(x.hb + 16 * (r * NE + x.te), v[r].x, v[r].y, v[r].z, v[r].w);
 }
 
 template <bool FP16>
@@ -762,6 +751,10 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     mbar_init(hb_bar, 1);
     mbar_init(eh_bar, NE / 32);
     mbar_init(drain_bar, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&m->meta_full[b]), 1);
+      mbar_init(smem_u32(&m->meta_free[b]), NE / 32);
+    }
     m->abort_flag = 0;
     fence_mbar_init();
   }
@@ -776,7 +769,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   }
   if (warp == 0 && lane == 0)
     for (int i = 0; i < NMAPS; ++i) prefetch_tmap(&p.tm[i]);
-  static_assert(NT == 576 && NE == 512 && SEGW == 32, "warp roles assume 18 warps");
+  static_assert(NT == 608 && NE == 512 && SEGW == 32, "warp roles assume 19 warps");
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -920,7 +913,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     __syncwarp();
     volatile int never = 0;
     mbar_wait(drain_bar, 0, &never, DRAIN_NS);
-  } else {
+  } else if (warp < 2 + NE / 32) {
     ECtx x;
     x.p = &p;
     x.m = m;
@@ -960,9 +953,19 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       tc_fence_after();
     };
     auto wait_acc = [&]() { wait_on(acc_bar, acc_phase); };
-    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
-      ep_setup<FP16>(x, t, n_slabs);
+    const uint8_t* fbuf = p.fbuf + (size_t)blockIdx.x * 2 * EB_BYTES;
+    uint32_t meta_ph[2] = {0u, 0u};
+    // tile start: the loader's metadata and Fourier operand of the CTA's i-th tile
+    auto tile_in = [&](int i) {
+      const int b = i & 1;
+      wait_on(smem_u32(&m->meta_full[b]), meta_ph[b]);
+      ep_fourier_in(x, fbuf + b * EB_BYTES);
       signal();
+    };
+    if ((int)blockIdx.x < n_tiles) tile_in(0);
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+      x.md = &m->meta[i & 1];
       wait_acc();
       ep_silu<FP16>(x, p.b_e1);
       signal();
@@ -1007,10 +1010,35 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           signal();
         }
         wait_acc();
-        const bool last = l == p.L - 1;
-        ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, last ? nullptr : p.g + (size_t)(l + 1) * p.D, last, wait_acc,
-                          signal);
+        if (l + 1 < p.L) {
+          ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, false, wait_acc, signal);
+        } else {
+          // both output tiles of the last MLP2 have completed, so HB and XB are
+          // free: the next tile's Fourier operand goes in and its first product
+          // (into the z/n columns) runs while this tile is pooled
+          if (x.MT == 2) wait_acc();
+          if (t + (int)gridDim.x < n_tiles) tile_in(i + 1);
+          ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, nullptr, true, [] {}, signal);
+          signal_to(smem_u32(&m->meta_free[i & 1]), false);   // this tile's metadata is no longer read
+        }
       }
+    }
+  } else {
+    // loader warp: tile set-up one tile ahead of the epilogue
+    uint8_t* fbuf = p.fbuf + (size_t)blockIdx.x * 2 * EB_BYTES;
+    uint32_t free_ph[2] = {0u, 0u};
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+      const int b = i & 1;
+      if (i >= 2) {   // buffer b last held the metadata of tile i - 2
+        const bool got = mbar_wait(smem_u32(&m->meta_free[b]), free_ph[b], abort, WAIT_NS);
+        if (!__all_sync(0xffffffffu, got) && lane == 0) set_abort(m, p.err);
+        free_ph[b] ^= 1u;
+      }
+      load_tile<FP16>(p, m, &m->meta[b], fbuf + b * EB_BYTES, t, n_slabs, lane);
+      __threadfence_block();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&m->meta_full[b]));
     }
   }
   tc_fence_before();
@@ -1039,8 +1067,6 @@ __global__ void build_schedule(const __grid_constant__ TcParams p, uint32_t* sp,
 }
 
 // ------------------------------------------------------------------ packing
-// One warp per segment of SEG tracks packs whole tracks greedily into slabs of
-// at most 64 hits and MAX_TRK_SLAB tracks; every segment starts a new slab.
 // Packing of one segment of up to SEG tracks into slabs of at most SLAB hits and
 // MAX_TRK_SLAB tracks (one warp per segment, decisions by lane 0 so the order is
 // deterministic): best fit over length buckets, each slab taking the longest
@@ -1425,6 +1451,7 @@ struct tf_tc_state {
   uint32_t* sched = nullptr;   // [2][MAX_SCHED]: producer entries, then MMA entries
   int n_sched = 0;
   float* xs = nullptr;
+  uint8_t* fbuf = nullptr;
   float* pool = nullptr;   // pooled means when the caller passes no buffer [POOL_TRACKS][D]
   size_t head_smem = 0;
   CUtensorMap tm[NMAPS];
@@ -1441,6 +1468,7 @@ void tf_tc_destroy(trackfit_ctx* h) {
   cudaFree(t->dev);
   cudaFree(t->seg_count);
   cudaFree(t->xs);
+  cudaFree(t->fbuf);
   cudaFree(t->pool);
   cudaFree(t->sched);
   delete t;
@@ -1568,6 +1596,7 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   t->n_slabs = t->slab_start + MAXB + 2;
   t->order = t->n_slabs + 64;
   if (cudaMalloc(&t->xs, (size_t)t->nsm * TILE * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  if (cudaMalloc(&t->fbuf, (size_t)t->nsm * 2 * EB_BYTES) != cudaSuccess) return TRACKFIT_ERR_OOM;
   if (cudaMalloc(&t->pool, (size_t)POOL_TRACKS * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
   // ---- tensor maps
   bool ok = make_map(&t->tm[MAP_E1], t->w_e1, D, E, fp16) && make_map(&t->tm[MAP_E2], t->w_e2, D, D, fp16) &&
@@ -1609,6 +1638,7 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   std::memset(&p, 0, sizeof(p));
   for (int i = 0; i < NMAPS; ++i) p.tm[i] = t->tm[i];
   p.xs = t->xs;
+  p.fbuf = t->fbuf;
   p.slab_start = t->slab_start;
   p.order = t->order;
   p.n_slabs = t->n_slabs;
