@@ -123,7 +123,7 @@ struct Misc {
   TileMeta meta[2];
   uint8_t col_tpos[TILE];   // the loader's own
   alignas(16) float part[4][TILE];
-  float carry[2][2][128];   // [slab][slot][channel]: states or pool sums between column segments
+  float carry[2][128];   // [slab][channel]: scan states between a slab's column segments
   alignas(16) float rinv[TILE];
   float hs[TILE][5];   // the loader's own
 };
@@ -306,9 +306,9 @@ struct ECtx {
 };
 
 // The two epilogue warps that share a quadrant and a slab hand a recurrence state
-// (or a running pool sum) from the slab's first 32 columns to the second, or back
-// in the reverse direction: barrier 2 + 2q + half, 64 threads, one arrival by the
-// leading warp and one wait by the other per hand-over.
+// from the slab's first 32 columns to the second, or back in the reverse
+// direction: barrier 2 + 2q + half, 64 threads, one arrival by the leading warp
+// and one wait by the other per hand-over.
 __device__ __forceinline__ void carry_pass(const ECtx& x) {
   asm volatile("bar.arrive %0, 64;" ::"r"(2 + 2 * x.q + x.half) : "memory");
 }
@@ -352,10 +352,10 @@ __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
     ep_silu_t<FP16, 1>(x, bias);
 }
 
-// X = acc + bias [+ x'], zero on pad columns.  x' (the gated residual of this
-// layer) sits in TMEM columns 256.. where the gate epilogue left it.  X goes to
-// the per-CTA scratch (read back once, by the next layer's gate epilogue), then
-// either the RMS-normalised x_hat -> XB (recomputing X from TMEM) or mean pooling.
+// X = acc + bias, zero on pad columns (a layer's accumulator already holds x'
+// plus the MLP2 product).  X goes to the per-CTA scratch (read back once, by the
+// next layer's gate epilogue) and the RMS-normalised x_hat to XB (recomputing X
+// from TMEM); the last layer's X is mean-pooled instead (ep_pool).
 // Sum of v over the 32 lanes for 16 columns at once: afterwards lane L holds the
 // total of column L & 15 (both halves of the warp hold the same 16 totals).
 __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
@@ -372,12 +372,11 @@ __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
   return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
 }
 
-template <bool FP16, int MT, bool pool, class W, class S>
+template <bool FP16, int MT, class W, class S>
 __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
                                               S&& signal_tile) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;   // d_model
-  const uint8_t* flags = x.md->col_flags;
   const uint32_t vm = x.md->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
   // X = acc + bias (the accumulator already holds x' + MLP for a layer, the
   // embedding product for the embedding), zero on pad columns.  The products
@@ -387,16 +386,6 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
   float bias_v[MT];
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) bias_v[mt] = bias[mt * 128 + x.c];
-  // mean pool: the slab's second column segment continues the running sums of
-  // the first (the same sequential sum as one thread walking the whole slab)
-  float run[MT];
-#pragma unroll
-  for (int mt = 0; mt < MT; ++mt) run[mt] = 0.0f;
-  if (pool && x.sub == 1) {
-    carry_wait(x);
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt) run[mt] = x.m->carry[x.half][mt][x.c];
-  }
   float sq[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
@@ -414,86 +403,95 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
         const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
         v[i] = val;
         sq[16 * hh + i] = fmaf(val, val, sq[16 * hh + i]);
-        if constexpr (pool) {
-          const int fl = flags[c0 + i];
-          run[mt] = (fl & F_FIRST) ? val : run[mt] + val;
-          if (fl & F_LAST) {
-            const int s = x.md->col_slot[c0 + i];
-            p.pool[(size_t)x.md->slot_track[s] * D + mt * 128 + x.c] = run[mt] / (float)x.md->slot_n[s];
-          }
-        }
       }
-      if constexpr (!pool) {   // the residual stream to the scratch (a warp's store: one 128-byte line)
-        float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
+      // the residual stream to the scratch (a warp's store: one 128-byte line)
+      float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
-      }
+      for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
     }
   }
-  if constexpr (pool) {
-    if (x.sub == 0) {
 #pragma unroll
-      for (int mt = 0; mt < MT; ++mt) x.m->carry[x.half][mt][x.c] = run[mt];
-      carry_pass(x);
-    }
-  } else {
+  for (int hh = 0; hh < 2; ++hh) {
+    float h16[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) h16[i] = sq[16 * hh + i];
+    const float t = reduce_scatter16(h16, x.lane);
+    if (x.lane < 16) x.m->part[x.q][x.col0 + 16 * hh + x.lane] = t;
+  }
+  ebar_sync();
+  if (x.te < TILE) {
+    const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
+    x.m->rinv[x.te] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
+  }
+  ebar_sync();
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) {
+    const float g = gain[mt * 128 + x.c];
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
-      float h16[16];
+      const int c0 = x.col0 + 16 * hh;
+      float v[16], rv[16];
+      tmem_ld16(x.tq + mt * 128 + c0, v);
+      const float4* rp = reinterpret_cast<const float4*>(x.m->rinv + c0);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) h16[i] = sq[16 * hh + i];
-      const float t = reduce_scatter16(h16, x.lane);
-      if (x.lane < 16) x.m->part[x.q][x.col0 + 16 * hh + x.lane] = t;
-    }
-    ebar_sync();
-    if (x.te < TILE) {
-      const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
-      x.m->rinv[x.te] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
-    }
-    ebar_sync();
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt) {
-      const float g = gain[mt * 128 + x.c];
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
-        const int c0 = x.col0 + 16 * hh;
-        float v[16], rv[16];
-        tmem_ld16(x.tq + mt * 128 + c0, v);
-        const float4* rp = reinterpret_cast<const float4*>(x.m->rinv + c0);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float4 r4 = rp[i];
-          rv[4 * i] = r4.x;
-          rv[4 * i + 1] = r4.y;
-          rv[4 * i + 2] = r4.z;
-          rv[4 * i + 3] = r4.w;
-        }
-        tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
-          v[i] = val * g * rv[i];
-        }
-        store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v);
+      for (int i = 0; i < 4; ++i) {
+        const float4 r4 = rp[i];
+        rv[4 * i] = r4.x;
+        rv[4 * i + 1] = r4.y;
+        rv[4 * i + 2] = r4.z;
+        rv[4 * i + 3] = r4.w;
       }
-      signal_tile();   // x_hat of this tile is in XB
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
+        v[i] = val * g * rv[i];
+      }
+      store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v);
     }
+    signal_tile();   // x_hat of this tile is in XB
   }
 }
 
 template <bool FP16, class W, class S>
-__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, const float* gain, bool pool,
-                                            W&& wait_tile, S&& signal_tile) {
-  if (x.MT == 2) {
-    if (pool)
-      ep_residual_t<FP16, 2, true>(x, bias, gain, wait_tile, signal_tile);
-    else
-      ep_residual_t<FP16, 2, false>(x, bias, gain, wait_tile, signal_tile);
-  } else {
-    if (pool)
-      ep_residual_t<FP16, 1, true>(x, bias, gain, wait_tile, signal_tile);
-    else
-      ep_residual_t<FP16, 1, false>(x, bias, gain, wait_tile, signal_tile);
+__device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
+                                            S&& signal_tile) {
+  if (x.MT == 2)
+    ep_residual_t<FP16, 2>(x, bias, gain, wait_tile, signal_tile);
+  else
+    ep_residual_t<FP16, 1>(x, bias, gain, wait_tile, signal_tile);
+}
+
+// Masked mean pooling of the last layer's output X = acc + bias.  The warp of
+// quadrant q, slab half and segment sub pools channel tile mt = sub (channels
+// 128 mt + 32 q + lane) over all 64 columns of the slab, each track's hits summed
+// in order from its first; with d_model 128 the sub = 1 warps have no tile.
+// The column loops stay rolled: this runs once per tile, and its code is cold.
+__device__ __forceinline__ void ep_pool(const ECtx& x, const float* bias) {
+  const TcParams& p = *x.p;
+  const int mt = x.sub;
+  if (mt >= x.MT) return;
+  const int D = p.D, ch = mt * 128 + x.c;
+  const float bv = bias[ch];
+  const uint8_t* flags = x.md->col_flags;
+  float run = 0.0f;
+#pragma unroll 1
+  for (int k = 0; k < 4; ++k) {   // 16-column groups of the slab
+    const int c0 = SLAB * x.half + 16 * k;
+    const uint32_t vm = x.md->m_valid[x.half][k >> 1] >> (16 * (k & 1));
+    float v[16];
+    tmem_ld16(x.tq + mt * 128 + c0, v);
+    tmem_ld_wait();
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float val = ((vm >> i) & 1u) ? v[i] + bv : 0.0f;
+      const int fl = flags[c0 + i];
+      run = (fl & F_FIRST) ? val : run + val;
+      if (fl & F_LAST) {
+        const int s = x.md->col_slot[c0 + i];
+        p.pool[(size_t)x.md->slot_track[s] * D + ch] = run / (float)x.md->slot_n[s];
+      }
+    }
   }
 }
 
@@ -574,7 +572,7 @@ __device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&a)[32], 
   float h = 0.0f;
   if (!leads) {
     carry_wait(x);
-    h = x.m->carry[x.half][0][x.c];
+    h = x.m->carry[x.half][x.c];
   }
   if (fwd) {
 #pragma unroll
@@ -590,7 +588,7 @@ __device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&a)[32], 
     }
   }
   if (leads) {
-    x.m->carry[x.half][0][x.c] = h;
+    x.m->carry[x.half][x.c] = h;
     carry_pass(x);
   }
   store_row32<FP16>(x.hb, x.c, x.col0, a);
@@ -970,7 +968,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       ep_silu<FP16>(x, p.b_e1);
       signal();
       wait_acc();
-      ep_residual<FP16>(x, p.b_e2, p.g, false, wait_acc, signal);   // embedding output X0
+      ep_residual<FP16>(x, p.b_e2, p.g, wait_acc, signal);   // embedding output X0
       for (int l = 0; l < p.L; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
           // biases are loaded before the wait so their latency hides behind it
@@ -1011,14 +1009,14 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         }
         wait_acc();
         if (l + 1 < p.L) {
-          ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, false, wait_acc, signal);
+          ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, wait_acc, signal);
         } else {
           // both output tiles of the last MLP2 have completed, so HB and XB are
           // free: the next tile's Fourier operand goes in and its first product
           // (into the z/n columns) runs while this tile is pooled
           if (x.MT == 2) wait_acc();
           if (t + (int)gridDim.x < n_tiles) tile_in(i + 1);
-          ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, nullptr, true, [] {}, signal);
+          ep_pool(x, p.b_2 + (size_t)l * p.D);
           signal_to(smem_u32(&m->meta_free[i & 1]), false);   // this tile's metadata is no longer read
         }
       }
