@@ -187,7 +187,9 @@ __device__ __forceinline__ void store_row16(uint32_t buf, int k, int n0, const f
   }
 }
 
-__device__ __forceinline__ void ebar_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
+// The four epilogue warps of one 32-column segment (one per TMEM quadrant):
+// barrier 10 + seg, 128 threads.
+__device__ __forceinline__ void seg_sync(int seg) { asm volatile("bar.sync %0, 128;" ::"r"(10 + seg) : "memory"); }
 
 // The static sequence of 128x64 weight blocks of one tile, in the order the MMA
 // issuer consumes them.  f(map, row, col, nk, tmem_col, bsel, bk, acc, wait, commit):
@@ -279,12 +281,13 @@ __device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
         f(MAP_1, r1, kc * 64, 4, 256, BSEL_XB, kc * 64, kc > 0, (kc & 1) ? W_NONE : W_E, kc == 3 ? C_ACC : C_NONE);
       for (int kc = 0; kc < 4; ++kc)
         f(MAP_1, r1 + 128, kc * 64, 4, 384, BSEL_XB, kc * 64, kc > 0, W_NONE, kc == 3 ? C_ACC : C_NONE);
-      for (int kc = 0; kc < 4; ++kc)   // tile 0 of MLP2 completes first (the residual starts on it)
-        f(MAP_2, r1, kc * 64, 4, 0, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, true, (kc & 1) ? W_NONE : W_E,
-          kc == 3 ? C_ACC : C_NONE);
-      for (int kc = 0; kc < 4; ++kc)
-        f(MAP_2, r1 + 128, kc * 64, 4, 128, kc < 2 ? BSEL_HB : BSEL_XB, kc * 64, true, W_NONE,
-          kc == 3 ? C_ACC : C_NONE);
+      // MLP2: K rows 0-127 (HB) of both output tiles once the SiLU of tile 0 is
+      // in, then rows 128-255 (XB), tile 0 first (the residual starts on it)
+      for (int kh = 0; kh < 2; ++kh)
+        for (int mt = 0; mt < 2; ++mt)
+          for (int kc = 2 * kh; kc < 2 * kh + 2; ++kc)
+            f(MAP_2, r1 + mt * 128, kc * 64, 4, mt * 128, kh == 0 ? BSEL_HB : BSEL_XB, kc * 64, true,
+              (mt == 0 && kc == 2 * kh) ? W_E : W_NONE, kc == 3 ? C_ACC : C_NONE);
     }
   }
 }
@@ -418,12 +421,15 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
     const float t = reduce_scatter16(h16, x.lane);
     if (x.lane < 16) x.m->part[x.q][x.col0 + 16 * hh + x.lane] = t;
   }
-  ebar_sync();
-  if (x.te < TILE) {
-    const float t = x.m->part[0][x.te] + x.m->part[1][x.te] + x.m->part[2][x.te] + x.m->part[3][x.te];
-    x.m->rinv[x.te] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
+  // the column sums over all channels: the four quadrants' partial sums of this
+  // segment's columns
+  seg_sync(x.seg);
+  if (x.q == 0) {
+    const int c = x.col0 + x.lane;
+    const float t = x.m->part[0][c] + x.m->part[1][c] + x.m->part[2][c] + x.m->part[3][c];
+    x.m->rinv[c] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
   }
-  ebar_sync();
+  seg_sync(x.seg);
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
     const float g = gain[mt * 128 + x.c];
@@ -495,11 +501,20 @@ __device__ __forceinline__ void ep_pool(const ECtx& x, const float* bias) {
   }
 }
 
+// X of the thread's channel in tile mt and its 32 columns, read back from the
+// scratch; issued before the wait for the gate's inputs so the loads' latency
+// hides behind it.
+__device__ __forceinline__ void gate_x_load(const ECtx& x, int mt, float (&xv)[32]) {
+  const int D = x.p->D;
+  const float* xp = x.xs + (size_t)x.col0 * D + mt * 128 + x.c;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) xv[i] = xp[(size_t)i * D];
+}
 // x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> TMEM columns
 // 128 mt.. (in place of the merge accumulator; MLP2 accumulates onto it) and XB
-// rows 128 mt + c.  X is read back from the scratch.
+// rows 128 mt + c.
 template <bool FP16, int MT>
-__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt) {
+__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const float (&xv)[32]) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;
   const int ch_g = mt * 128 + x.c;
@@ -508,26 +523,23 @@ __device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt) {
 #pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
     const int c0 = x.col0 + 16 * hh;
-    float xv[16], mv[16], gv[16];
+    float mv[16], gv[16];
     tmem_ld16(x.tq + mt * 128 + c0, mv);
     tmem_ld16(x.tq + 256 + mt * 128 + c0, gv);
-    const float* xp = x.xs + (size_t)c0 * D + ch_g;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) xv[i] = xp[(size_t)i * D];
     tmem_ld_wait();
 #pragma unroll
-    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm(gv[i] + bg), xv[i]);
+    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm(gv[i] + bg), xv[16 * hh + i]);
     tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
     store_row16<FP16>(x.xb, ch_g, c0, mv);
   }
   tmem_st_wait();
 }
 template <bool FP16>
-__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt) {
+__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt, const float (&xv)[32]) {
   if (x.MT == 2)
-    ep_gate_t<FP16, 2>(x, l, mt);
+    ep_gate_t<FP16, 2>(x, l, mt, xv);
   else
-    ep_gate_t<FP16, 1>(x, l, mt);
+    ep_gate_t<FP16, 1>(x, l, mt, xv);
 }
 
 // Scan chunk of one layer.  The chunk holds 64 channels of both directions:
@@ -989,12 +1001,15 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         // pipelines the next tile's products behind each); with d_model 256 the
         // SiLU of tile 0 goes to HB (MLP1 still reads XB rows 0-127 then)
         const float* b1 = p.b_1 + (size_t)l * p.D;
+        float xg[32];
+        gate_x_load(x, 0, xg);
         wait_acc();
-        ep_gate<FP16>(x, l, 0);
+        ep_gate<FP16>(x, l, 0, xg);
         signal();
         if (x.MT == 2) {
+          gate_x_load(x, 1, xg);
           wait_acc();
-          ep_gate<FP16>(x, l, 1);
+          ep_gate<FP16>(x, l, 1, xg);
           signal();
           wait_acc();
           ep_silu_mt<FP16>(x, b1, 0, 256, x.hb, 0);
