@@ -142,6 +142,21 @@ __device__ __forceinline__ float rcp_approx(float x) {
 }
 constexpr float LOG2E_F = 1.4426950408889634f;
 __device__ __forceinline__ float silu(float x) { return x * sigm(x); }
+// The output gate and the MLP's SiLU inside the fused kernel use one MUFU
+// operation per value instead of two (ex2 and rcp), from sigma(x) =
+// (1 + tanh(x / 2)) / 2: tanh.approx has a relative error of about 2^-11, below
+// the rounding of the 16-bit operands these values feed.  (The scan gates keep
+// ex2 and rcp: a = 1 - sigma there needs relative accuracy as sigma -> 1.)
+__device__ __forceinline__ float tanh_approx(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float sigm_t(float x) { return fmaf(0.5f, tanh_approx(0.5f * x), 0.5f); }
+__device__ __forceinline__ float silu_t(float x) {
+  const float h = 0.5f * x;
+  return fmaf(h, tanh_approx(h), h);
+}
 
 // Operand conversion (round to nearest even): bf16, or fp16 when FP16 is set.
 template <bool FP16>
@@ -328,7 +343,7 @@ __device__ __forceinline__ void ep_silu_mt(const ECtx& x, const float* bias, int
   const float b = bias[mt * 128 + x.c];
   tmem_ld_wait();
 #pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = silu(v[i] + b);
+  for (int i = 0; i < 32; ++i) v[i] = silu_t(v[i] + b);
   store_row32<FP16>(buf, row0 + x.c, x.col0, v);
 }
 // silu(acc + bias) of every tile (accumulator columns mt*128) -> XB rows
@@ -528,7 +543,7 @@ __device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const fl
     tmem_ld16(x.tq + 256 + mt * 128 + c0, gv);
     tmem_ld_wait();
 #pragma unroll
-    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm(gv[i] + bg), xv[16 * hh + i]);
+    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm_t(gv[i] + bg), xv[16 * hh + i]);
     tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
     store_row16<FP16>(x.xb, ch_g, c0, mv);
   }
