@@ -53,7 +53,9 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0) {
+    // a try_wait may suspend the thread for a while, so the abort flag is read
+    // often: once a wait has failed, the others give up promptly
+    if ((i & 7u) == 0) {
       if (*abort) return false;
       if (globaltimer() - t0 > limit_ns) return false;
     }
@@ -77,7 +79,7 @@ __device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity, vo
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
     if (mbar_test_wait(bar, parity)) return true;
-    if ((i & 1023u) == 0) {
+    if ((i & 63u) == 0) {
       if (*abort) return false;
       if (globaltimer() - t0 > limit_ns) return false;
     }

@@ -52,7 +52,8 @@ def full(raw, tracks, out_md, out_json, cmd):
     hdr, units, vals = rows[0], rows[1], rows[2]
     d = dict(zip(hdr, vals))
     u = dict(zip(hdr, units))
-    lines = [f"# tc_forward_kernel, large workload ({tracks} tracks) — ncu --set full", "",
+    how = "ncu --set full" if "--set full" in cmd else "ncu, the metrics below"
+    lines = [f"# tc_forward_kernel, large workload ({tracks} tracks) — {how}", "",
              f"Command: `{cmd}`", "", "| metric | value |", "|---|---|"]
     for k, name in KEYS:
         if k in d:
