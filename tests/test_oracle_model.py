@@ -253,6 +253,62 @@ def test_mean_pool_divides_by_hit_count():
     np.testing.assert_allclose(out[:, :4], np.tile(hn / (1 + np.exp(-hn)), (3, 1)), rtol=1e-13)
 
 
+def test_prenorm_makes_the_scans_scale_invariant():
+    """The projections read the RMS-normalised input (pre-norm, the reading of
+    Sec. 3.2 taken here): scaling a hit's input vector by 8 leaves the gates,
+    candidates and so both scans unchanged, up to the eps term (~1e-7 here)."""
+    m = small_model(T=7, D=8, H=12, L=1)
+    W = O.split_blob(cfg_dict(m), Wl.gen_weights(m, 4))
+    x = rng.standard_normal((3, 7, 8))
+    valid = np.arange(7)[None, :] < np.array([7, 4, 1])[:, None]
+    _, hf1, hb1 = O.encoder_layer(x, W, 0, cfg_dict(m), valid, False)
+    _, hf8, hb8 = O.encoder_layer(8.0 * x, W, 0, cfg_dict(m), valid, False)
+    np.testing.assert_allclose(hf8, hf1, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(hb8, hb1, rtol=1e-5, atol=1e-6)
+
+
+def test_mlp_reads_the_gated_residual():
+    """The MLP acts on x' = x + merge * gate, not on the layer input: with the gate
+    open, W_m = 0 and b_m = c, x' = x + c, and with W_1 = W_2 = I the output is
+    x' + SiLU(x')."""
+    D, H, T = 3, 3, 4
+    m = small_model(T=T, D=D, H=H, L=1)
+    W = zero_weights(m)
+    W["layer0.g"] = np.ones(D)
+    W["layer0.b_in"][4 * H:] = 40.0
+    c = np.array([0.5, -1.25, 2.0])
+    W["layer0.b_m"] = c
+    W["layer0.w1"] = np.eye(D)
+    W["layer0.w2"] = np.eye(D)
+    x = rng.standard_normal((2, T, D))
+    valid = np.ones((2, T), bool)
+    x2, _, _ = O.encoder_layer(x, W, 0, cfg_dict(m), valid, False)
+    x1 = x + c / (1 + math.exp(-40.0))
+    np.testing.assert_allclose(x2, x1 + x1 / (1 + np.exp(-x1)), rtol=1e-13, atol=1e-15)
+
+
+def test_padded_hits_are_zero_in_the_layer_output():
+    """Padded hits leave a layer as zero vectors (the layer's last step), whatever
+    the biases would put there."""
+    m = small_model(T=6, D=8, H=12, L=1)
+    W = O.split_blob(cfg_dict(m), Wl.gen_weights(m, 6))
+    x = rng.standard_normal((3, 6, 8))
+    valid = np.arange(6)[None, :] < np.array([6, 2, 5])[:, None]
+    x2, _, _ = O.encoder_layer(x, W, 0, cfg_dict(m), valid, False)
+    assert np.all(x2[~valid] == 0.0)
+    assert np.all(x2[valid] != 0.0)
+
+
+def test_mean_pool_reads_valid_hits_only():
+    """Masked mean pooling (Sec. 3.2): values in padded rows do not enter the mean."""
+    x = rng.standard_normal((3, 5, 4))
+    n = np.array([5, 1, 3])
+    valid = np.arange(5)[None, :] < n[:, None]
+    got = O.pool(x, None, None, n, valid, 0)
+    for i in range(3):
+        np.testing.assert_allclose(got[i], x[i, :n[i]].mean(axis=0), rtol=1e-14)
+
+
 def test_bf16_mode_is_close_but_not_identical():
     m = small_model(D=16, H=24)
     hits, n = random_tracks(m, 32)
