@@ -64,8 +64,8 @@ constexpr int B_LBO = 1024;               // 64-hit atom stride
 enum { MAP_E1 = 0, MAP_E2, MAP_IN, MAP_M, MAP_1, MAP_2, NMAPS };
 enum { BSEL_XB = 0, BSEL_HB = 1 };
 // Hand-overs around a schedule block: before its first MMA the issuer waits for
-// the epilogue's next arrival on e_bar (W_E) or eh_bar (W_H); after its last MMA
-// it commits to acc_bar (C_ACC) or hb_bar (C_HB).
+// the epilogue's next hand-over on e_bar (W_E; two barriers used alternately) or
+// eh_bar (W_H); after its last MMA it commits to acc_bar (C_ACC) or hb_bar (C_HB).
 enum { W_NONE = 0, W_E = 1, W_H = 2 };
 enum { C_NONE = 0, C_ACC = 1, C_HB = 2 };
 // bits of an MMA schedule entry
@@ -116,7 +116,7 @@ struct TileMeta {
 };
 struct Misc {
   uint64_t full[MAX_STAGES], empty[MAX_STAGES];
-  uint64_t acc_bar, e_bar, hb_bar, eh_bar, drain_bar;
+  uint64_t acc_bar, e_bar[2], hb_bar, eh_bar, drain_bar;
   uint64_t meta_full[2], meta_free[2];   // loader -> epilogue, epilogue -> loader
   uint32_t tmem_base;
   int abort_flag;
@@ -743,11 +743,14 @@ __device__ __forceinline__ void load_tile(const TcParams& p, Misc* m, TileMeta* 
 
 // Tile start on the epilogue side: the Fourier operand from the CTA's global
 // buffer into HB (five 16-byte chunks per thread, all loads in flight at once).
+// The loads bypass L1 (ld.global.cg): the buffer is rewritten by the loader warp
+// every other tile, and a line of an earlier tile's operand must not be served
+// from L1.
 __device__ __forceinline__ void ep_fourier_in(const ECtx& x, const uint8_t* fb) {
   static_assert(EB_BYTES == 5 * 16 * NE, "one chunk per thread per round");
   uint4 v[5];
 #pragma unroll
-  for (int r = 0; r < 5; ++r) v[r] = reinterpret_cast<const uint4*>(fb)[r * NE + x.te];
+  for (int r = 0; r < 5; ++r) v[r] = __ldcg(reinterpret_cast<const uint4*>(fb) + r * NE + x.te);
 #pragma unroll
   for (int r = 0; r < 5; ++r) st_shared_v4(x.hb + 16 * (r * NE + x.te), v[r].x, v[r].y, v[r].z, v[r].w);
 }
@@ -762,7 +765,8 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   Misc* m = reinterpret_cast<Misc*>(gbase + p.off_misc);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t full0 = smem_u32(&m->full[0]), empty0 = smem_u32(&m->empty[0]);
-  const uint32_t acc_bar = smem_u32(&m->acc_bar), e_bar = smem_u32(&m->e_bar);
+  const uint32_t acc_bar = smem_u32(&m->acc_bar);
+  const uint32_t e_bar0 = smem_u32(&m->e_bar[0]), e_bar1 = smem_u32(&m->e_bar[1]);
   const uint32_t hb_bar = smem_u32(&m->hb_bar), eh_bar = smem_u32(&m->eh_bar);
   const uint32_t drain_bar = smem_u32(&m->drain_bar);
 
@@ -772,7 +776,8 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       mbar_init(empty0 + 8 * s, 1);
     }
     mbar_init(acc_bar, 1);
-    mbar_init(e_bar, NE / 32);   // one arrival per epilogue warp
+    mbar_init(e_bar0, NE / 32);   // one arrival per epilogue warp
+    mbar_init(e_bar1, NE / 32);
     mbar_init(hb_bar, 1);
     mbar_init(eh_bar, NE / 32);
     mbar_init(drain_bar, 1);
@@ -856,7 +861,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     // barrier is tested without blocking first, and both blocks go out in one
     // elected run unless an epilogue hand-over falls between them, so the
     // per-iteration bookkeeping stays short next to the tensor pipe's queue.
-    uint32_t stage = 0, phase = 0, e_phase = 0, eh_phase = 0;
+    uint32_t stage = 0, phase = 0, eh_phase = 0, e_k = 0, e_phase0 = 0, e_phase1 = 0;
     bool ok = true;
     int my_tiles = 0;
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) ++my_tiles;
@@ -877,7 +882,13 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       return true;
     };
     auto handover = [&](uint32_t e) -> bool {
-      if (!wait_bar((e & S_W_E) ? e_bar : eh_bar, (e & S_W_E) ? e_phase : eh_phase, false)) return false;
+      if (e & S_W_E) {   // the k-th W_E hand-over arrives on e_bar[k % 2]
+        const bool got = (e_k & 1u) ? wait_bar(e_bar1, e_phase1, false) : wait_bar(e_bar0, e_phase0, false);
+        if (!got) return false;
+        ++e_k;
+      } else if (!wait_bar(eh_bar, eh_phase, false)) {
+        return false;
+      }
       tc_fence_after();
       return true;
     };
@@ -960,7 +971,13 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     // The epilogue warps run decoupled: each makes its shared-memory operand
     // writes visible to the async proxy, orders its TMEM reads and arrives on the
     // hand-over barrier itself (e_bar and eh_bar count one arrival per warp), and
-    // each polls the MMA commits itself.  A failed wait sets the abort flag and
+    // each polls the MMA commits itself.  Some consecutive hand-overs do not wait
+    // for the issuer in between (gate tile 0 then 1, SiLU 0 then 1, x_hat 0 then
+    // 1), so a warp can arrive for the next one before a slower warp has arrived
+    // for the current one; on a single counting barrier that arrival would
+    // complete the current phase early.  The W_E hand-overs therefore alternate
+    // between two barriers: a warp is never more than one hand-over ahead of
+    // another (the one after a pair waits for a product that needs both).  A failed wait sets the abort flag and
     // every later wait fails fast, but no warp leaves the loop early: all warps
     // keep taking the same sequence of named barriers (tile set-up, the norm
     // reductions, the segment hand-overs), so none of them can be left waiting.
@@ -970,7 +987,12 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       __syncwarp();
       if (x.lane == 0) mbar_arrive(bar);
     };
-    auto signal = [&]() { signal_to(e_bar, true); };
+    uint32_t e_k = 0;   // W_E hand-overs so far: the next goes to e_bar[e_k % 2]
+    auto signal_e = [&](bool wrote_operands) {
+      signal_to((e_k & 1u) ? e_bar1 : e_bar0, wrote_operands);
+      ++e_k;
+    };
+    auto signal = [&]() { signal_e(true); };
     auto wait_on = [&](uint32_t bar, uint32_t& ph) {
       const bool got = mbar_wait(bar, ph, abort, WAIT_NS);   // try_wait: suspends instead of polling
       if (!__all_sync(0xffffffffu, got) && x.lane == 0) set_abort(m, p.err);
@@ -1004,7 +1026,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           wait_acc();
           float z[32], n[32];
           scan_load(x, z, n);
-          signal_to(e_bar, false);   // the z/n columns are free for the next chunk
+          signal_e(false);   // the z/n columns are free for the next chunk
           scan_gates(x, z, n, bz, bn);
           // HB still feeds the merge of the previous chunk (the gate hand-over
           // covers the last merge of the previous layer)
