@@ -176,6 +176,16 @@ int trackfit_debug_scan(const float* a, const float* b, const float* x, const in
                         int64_t n_tracks, int32_t T, int32_t C, float* h_fwd, float* h_bwd,
                         void* stream);
 
+/* Test hook, host only (no GPU needed): per-tile totals of the tensor-core
+ * path's block schedule for cfg, from the same expansion the fused kernel uses.
+ * counts (host, n_counts >= 6): [0] 128 x 64 weight blocks, [1] MMA instructions
+ * (128 x 128 x 16 each), [2] operand hand-overs the issuer waits for from the
+ * epilogue (W_E), [3] state hand-overs (W_H), [4] accumulator commits the
+ * epilogue waits for (C_ACC), [5] state-buffer commits (C_HB).  Returns
+ * TRACKFIT_ERR_UNSUPPORTED when cfg does not run on the tensor-core path,
+ * TRACKFIT_ERR_INVALID_ARG for NULL pointers or n_counts < 6. */
+int trackfit_debug_schedule(const trackfit_config_t* cfg, int64_t* counts, int32_t n_counts);
+
 /* Test hook for the tensor-core operand layouts: D = A * B on one 128 x 128
  * tile through the same TMA, shared-memory descriptor and tensor-memory path as
  * the fused kernel.  A device bf16 bits [128][K] row-major (K-major), Bkn device

@@ -217,7 +217,7 @@ __device__ __forceinline__ void seg_sync(int seg) { asm volatile("bar.sync %0, 1
 // issuer computes z/n of chunk k+1 into the same TMEM columns, and the merge
 // product of chunk k follows once its states h(k) are in shared memory.
 template <class F>
-__device__ __forceinline__ void walk_tile(const TcParams& p, F&& f) {
+__host__ __device__ inline void walk_tile(const TcParams& p, F&& f) {
   const int MT = p.D >> 7, KD = p.D >> 6;
   // the embedding's first product goes to the z/n columns, so it can run while
   // the epilogue still pools the previous tile from columns 0..
@@ -1506,6 +1506,36 @@ struct tf_tc_state {
   size_t head_smem = 0;
   CUtensorMap tm[NMAPS];
 };
+
+struct ScheduleCounter {   // a callable for walk_tile on either side
+  int64_t c[6] = {0, 0, 0, 0, 0, 0};
+  __host__ __device__ void operator()(int, int, int, int nk, int, int, int, int, int wait, int commit) {
+    ++c[0];
+    c[1] += nk;
+    c[2] += wait == W_E;
+    c[3] += wait == W_H;
+    c[4] += commit == C_ACC;
+    c[5] += commit == C_HB;
+  }
+};
+
+// Per-tile totals of the fused kernel's block schedule, from the same walk_tile
+// the kernel expands (host only, no device needed): counts[0] blocks, [1] MMA
+// instructions (128 x 128 x 16 each), [2] W_E and [3] W_H hand-over waits, [4]
+// C_ACC and [5] C_HB commits.
+int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n) {
+  if (n < 6) return TRACKFIT_ERR_INVALID_ARG;
+  TcParams q;
+  memset(&q, 0, sizeof(q));
+  q.D = s.D;
+  q.L = s.L;
+  q.NDC = s.H / 64;
+  q.ROWS_IN = q.NDC * 256 + s.D;
+  ScheduleCounter c;
+  walk_tile(q, c);
+  for (int i = 0; i < 6; ++i) counts[i] = c.c[i];
+  return TRACKFIT_OK;
+}
 
 bool tf_tc_supported(const tf_shape& s) {
   return (s.precision == TRACKFIT_BF16_PROJ || s.precision == TRACKFIT_FP16_PROJ) && s.pool == TRACKFIT_POOL_MEAN && (s.D == 128 || s.D == 256) &&

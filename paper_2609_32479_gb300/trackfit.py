@@ -24,7 +24,8 @@ ABI_VERSION = 1
 EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trackfit_forward_ex",
            "trackfit_forward_host", "trackfit_device_errors", "trackfit_path_name", "trackfit_set_path",
            "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma",
-           "trackfit_profile", "trackfit_profile_read", "trackfit_forward_noalloc")
+           "trackfit_profile", "trackfit_profile_read", "trackfit_forward_noalloc",
+           "trackfit_debug_schedule")
 
 
 class Config(ctypes.Structure):
@@ -86,6 +87,8 @@ def load() -> ctypes.CDLL:
     lib.trackfit_profile_read.restype = ctypes.c_int
     lib.trackfit_forward_noalloc.argtypes = [ctypes.POINTER(Config), vp, vp, vp, i64, vp, vp]
     lib.trackfit_forward_noalloc.restype = ctypes.c_int
+    lib.trackfit_debug_schedule.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32]
+    lib.trackfit_debug_schedule.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -112,6 +115,19 @@ def make_config(m: W.ModelConfig) -> Config:
 def weight_count(m: W.ModelConfig) -> int:
     c = make_config(m)
     return int(load().trackfit_weight_count(ctypes.byref(c)))
+
+
+def schedule_counts(m: W.ModelConfig):
+    """Per-tile totals of the tensor-core path's block schedule (host only): dict
+    with blocks, mmas, w_e, w_h, c_acc, c_hb; None when m does not run on that path."""
+    c = make_config(m)
+    out = (ctypes.c_int64 * 6)()
+    st = load().trackfit_debug_schedule(ctypes.byref(c), out, 6)
+    if st == ERR_UNSUPPORTED:
+        return None
+    if st != OK:
+        raise TrackfitError(st, "trackfit_debug_schedule")
+    return dict(zip(("blocks", "mmas", "w_e", "w_h", "c_acc", "c_hb"), (int(v) for v in out)))
 
 
 def _stream_handle(stream) -> Optional[int]:

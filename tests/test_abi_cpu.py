@@ -70,3 +70,44 @@ def test_null_and_count_errors_on_host(lib):
     for s in range(7):
         assert T.strerror(s) and T.strerror(s) != "unknown status"
     assert lib.trackfit_path_name(None) == b"none"
+
+
+def _epilogue_handovers(m):
+    """Per-tile hand-overs of the fused kernel's epilogue warps, restated from
+    their loop: the tile's Fourier operand, the embedding's SiLU, then x_hat one
+    128-channel tile at a time; per layer one release of the z/n columns per scan
+    chunk, the output gate and the MLP's SiLU per channel tile, and x_hat per
+    channel tile except after the last layer (mean pooling instead).  The waits:
+    the embedding's two products (the second per channel tile), per layer the
+    z/n products of every chunk, the last merge, MLP1 and MLP2 per channel tile."""
+    MT, NDC, L = m.d_model // 128, m.d_hidden // 64, m.n_layers
+    signals = 2 + MT + sum(NDC + 2 * MT + (MT if l + 1 < L else 0) for l in range(L))
+    waits = 1 + MT + L * (NDC + 3 * MT)
+    return signals, waits
+
+
+@pytest.mark.parametrize("D,H,L,prec", [(128, 192, 6, W.PRECISION_BF16), (256, 384, 8, W.PRECISION_BF16),
+                                        (128, 192, 1, W.PRECISION_FP16), (256, 384, 1, W.PRECISION_FP16),
+                                        (256, 384, 2, W.PRECISION_BF16), (128, 192, 16, W.PRECISION_BF16)])
+def test_schedule_handovers_match_the_epilogue(lib, D, H, L, prec):
+    """The issuer's hand-over waits and commits pair one to one with the epilogue's
+    arrivals and waits (a mismatch would stall a wait until its time limit, or let
+    one side run ahead), and the MMAs cover exactly the per-hit work of the model."""
+    m = W.ModelConfig(max_hits=24, d_model=D, d_hidden=H, n_layers=L, precision=prec)
+    c = T.schedule_counts(m)
+    assert c is not None
+    signals, waits = _epilogue_handovers(m)
+    NDC = H // 64
+    assert c["w_e"] == signals
+    assert c["c_acc"] == waits
+    assert c["w_h"] == L * NDC
+    assert c["c_hb"] == L * (NDC - 1)
+    E = 2 * m.n_features * m.n_fourier
+    flops_per_column = 2 * (D * E + D * D) + L * (2 * D * (4 * H + D) + 4 * H * D + 4 * D * D)
+    assert c["mmas"] * 128 * 128 * 16 * 2 == 128 * flops_per_column
+    assert c["blocks"] * 4 >= c["mmas"]
+
+
+def test_schedule_hook_rejects_cuda_core_configs(lib):
+    assert T.schedule_counts(W.workload("tiny").model) is None
+    assert T.schedule_counts(W.workload("large").model.with_(precision=W.PRECISION_FP32)) is None
