@@ -1,0 +1,161 @@
+"""Oracle for the analytic seed of Sec. 3.1 (plain, slow, fp64).
+
+TEST INFRASTRUCTURE ONLY: imported by tests/ (and, like trackfit_oracle, by
+nothing on the product path).  Not used by the CUDA kernels yet: the seed is the
+next step on the path, and this module fixes what it computes first.
+
+What it computes (Sec. 3.1): from three hits of a track, the circle through their
+transverse positions by the conformal (inversion) map of Karimaki (1991), which
+turns "circle through three points" into "line through two points" with no fit
+or iteration; the circle's radius and turning direction give p_T and the charge;
+the direction at the point of closest approach to the beam line gives phi; the z
+positions against the transverse arc length give theta; the closest-approach
+point gives d0 and z0.  Everything in fp64 (the paper computes the seed in fp64
+to avoid a cancellation in the transport to the beam line).
+
+Conventions (those of the synthetic track generator, against which the tests pin
+the functions): B along +z; a positive charge turns clockwise seen from +z; at
+turning angle a from the perigee the direction angle is phi0 - q a, the
+transverse arc length R a, and z = z0 + R a cot(theta); the perigee point is
+(-d0 sin phi0, d0 cos phi0); p_T = C R B / 1000 GeV for R in mm and B in T, with
+C = 0.299792458; q/p = q sin(theta) / p_T in 1/GeV.
+
+Readings where the paper is silent (listed in the design doc as well):
+- the seed triplet: hits taken in path order, each seed hit the first later hit
+  more than 10 mm (3-D) from the previous seed hit, so that overlap hits on the
+  same layer (1.5 mm apart) never form a pair; the slope uses the first and the
+  third seed hit (the longer lever arm);
+- with fewer than three hits so spaced the seed is undefined (NaN row).
+
+Parity status: pinned in tests/test_oracle_seed.py (closed-form recovery of
+generated helices to fp64 rounding, invariances under rotation about and
+translation along the beam line, charge reversal, hit order).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+C_LIGHT = 0.299792458          # GeV / (T m)
+SEED_MIN_SEPARATION_MM = 10.0
+
+__all__ = ["circle_through_three", "seed_perigee", "seed_triplet", "seed_from_hits", "helix_point",
+           "C_LIGHT", "SEED_MIN_SEPARATION_MM"]
+
+
+def circle_through_three(p0, p1, p2):
+    """Centre and radius of the circle through three transverse points [..., 2].
+
+    With p0 moved to the origin, the inversion (u, v) = (x, y) / (x^2 + y^2) maps a
+    circle through the origin with centre c onto the straight line
+    2 c_x u + 2 c_y v = 1 (divide x^2 + y^2 = 2 c.x by x^2 + y^2); the images of
+    p1 and p2 fix that line, i.e. two linear equations in c.  Collinear points give
+    an infinite radius."""
+    p0, p1, p2 = (np.asarray(p, dtype=np.float64) for p in (p0, p1, p2))
+    a = p1 - p0
+    b = p2 - p0
+    na = np.sum(a * a, axis=-1)
+    nb = np.sum(b * b, axis=-1)
+    u1, v1 = a[..., 0] / na, a[..., 1] / na
+    u2, v2 = b[..., 0] / nb, b[..., 1] / nb
+    det = u1 * v2 - u2 * v1
+    with np.errstate(divide="ignore", invalid="ignore"):
+        cx = (v2 - v1) / (2.0 * det)
+        cy = (u1 - u2) / (2.0 * det)
+    centre = np.stack([p0[..., 0] + cx, p0[..., 1] + cy], axis=-1)
+    return centre, np.hypot(cx, cy)
+
+
+def _wrap(a):
+    return (a + np.pi) % (2.0 * np.pi) - np.pi
+
+
+def seed_perigee(h0, h1, h2, b_field):
+    """Perigee parameters (d0, z0, phi0, theta, q/p) [..., 5] of the helix through
+    three hits h0, h1, h2 [..., 3] (x, y, z in mm), given in path order.
+
+    Charge: moving h0 -> h1 -> h2 the track turns left (counter-clockwise) for a
+    negative charge: q = -sign((h1 - h0) x (h2 - h0)).  The closest transverse
+    point of the circle to the beam line is P = C - R C/|C|; there the direction
+    has the centre on its right for q > 0, i.e. t = q (-C_y, C_x)/|C| rotated to
+    the direction of motion, and d0 = P . (-sin phi0, cos phi0).  The turning
+    angle from P to a hit is the angle swept clockwise (q > 0) or
+    counter-clockwise (q < 0) around C; with the transverse arc lengths s0, s2 of
+    h0, h2, cot(theta) = (z2 - z0h) / (s2 - s0) and z0 = z0h - s0 cot(theta)."""
+    h0, h1, h2 = (np.asarray(h, dtype=np.float64) for h in (h0, h1, h2))
+    centre, R = circle_through_three(h0[..., :2], h1[..., :2], h2[..., :2])
+    a = h1[..., :2] - h0[..., :2]
+    b = h2[..., :2] - h0[..., :2]
+    cross = a[..., 0] * b[..., 1] - a[..., 1] * b[..., 0]
+    q = -np.sign(cross)
+    dc = np.hypot(centre[..., 0], centre[..., 1])
+    ux, uy = centre[..., 0] / dc, centre[..., 1] / dc          # unit vector beam line -> centre
+    px, py = centre[..., 0] - R * ux, centre[..., 1] - R * uy  # closest point to the beam line
+    # direction of motion at P: perpendicular to (C - P) = R u, centre on the right for q > 0
+    tx, ty = -q * uy, q * ux
+    phi0 = np.arctan2(ty, tx)
+    d0 = -px * np.sin(phi0) + py * np.cos(phi0)
+
+    def turning(h):
+        # angle of (h - C) measured from (P - C), positive in the direction of motion
+        g_p = np.arctan2(py - centre[..., 1], px - centre[..., 0])
+        g_h = np.arctan2(h[..., 1] - centre[..., 1], h[..., 0] - centre[..., 0])
+        return np.mod(-q * (g_h - g_p), 2.0 * np.pi)
+
+    s0 = R * turning(h0)
+    s2 = R * turning(h2)
+    cot = (h2[..., 2] - h0[..., 2]) / (s2 - s0)
+    z0 = h0[..., 2] - s0 * cot
+    theta = np.arctan2(1.0, cot)
+    pt = C_LIGHT * b_field * R / 1000.0
+    qop = q * np.sin(theta) / pt
+    return np.stack([d0, z0, phi0, theta, qop], axis=-1)
+
+
+def seed_triplet(hits, n_hits, min_sep=SEED_MIN_SEPARATION_MM):
+    """Indices [B, 3] of the seed hits of every track (the reading stated in the
+    module docstring), -1 where a track has fewer than three such hits.  hits
+    [B, T, >=3] with x, y, z first, in path order; n_hits [B]."""
+    hits = np.asarray(hits, dtype=np.float64)
+    B = hits.shape[0]
+    out = np.full((B, 3), -1, dtype=np.int64)
+    for b in range(B):
+        picked = [0] if n_hits[b] >= 1 else []
+        for t in range(1, int(n_hits[b])):
+            if len(picked) == 3:
+                break
+            if np.linalg.norm(hits[b, t, :3] - hits[b, picked[-1], :3]) > min_sep:
+                picked.append(t)
+        if len(picked) == 3:
+            out[b] = picked
+    return out
+
+
+def seed_from_hits(hits, n_hits, b_field, min_sep=SEED_MIN_SEPARATION_MM):
+    """Seed perigee [B, 5] of every track from its seed triplet; NaN rows where the
+    triplet does not exist."""
+    hits = np.asarray(hits, dtype=np.float64)
+    idx = seed_triplet(hits, n_hits, min_sep)
+    ok = idx[:, 0] >= 0
+    out = np.full((hits.shape[0], 5), np.nan)
+    if np.any(ok):
+        rows = np.nonzero(ok)[0]
+        h = [hits[rows, idx[ok, k], :3] for k in range(3)]
+        out[rows] = seed_perigee(h[0], h[1], h[2], b_field)
+    return out
+
+
+def helix_point(perigee, alpha, b_field):
+    """Position (x, y, z) [..., 3] at turning angle alpha >= 0 from the perigee, for
+    perigee parameters (d0, z0, phi0, theta, q/p) [..., 5]: the forward map the
+    seed inverts, written from the conventions in the module docstring."""
+    d0, z0, phi0, theta, qop = (np.asarray(perigee, dtype=np.float64)[..., k] for k in range(5))
+    q = np.sign(qop)
+    pt = np.sin(theta) / np.abs(qop)
+    R = 1000.0 * pt / (C_LIGHT * b_field)
+    x0, y0 = -d0 * np.sin(phi0), d0 * np.cos(phi0)
+    cx, cy = x0 + q * R * np.sin(phi0), y0 - q * R * np.cos(phi0)
+    phi = phi0 - q * alpha
+    x = cx - q * R * np.sin(phi)
+    y = cy + q * R * np.cos(phi)
+    z = z0 + R * alpha / np.tan(theta)
+    return np.stack([x, y, z], axis=-1)

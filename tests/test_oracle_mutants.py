@@ -4,15 +4,18 @@ Each mutant rewrites one expression of one oracle function: a dropped term, a wr
 sign, a swapped operand, an index off by one, the kinds of slip a restatement of
 Sec. 3.2 / Eq. 2 can make.  The rewritten function is installed in the oracle
 module for the duration of the test (CPU only, nothing else is touched) and every
-pin of tests/test_oracle_units.py and tests/test_oracle_model.py runs against it;
-at least one pin must fail.  A mutant that survives marks a gap in the pins."""
+pin of tests/test_oracle_units.py and tests/test_oracle_model.py (for the
+analytic-seed oracle: tests/test_oracle_seed.py) runs against it; at least one pin
+must fail.  A mutant that survives marks a gap in the pins."""
 import inspect
 import textwrap
 
 import pytest
 
+from oracle import seed_oracle as SO
 from oracle import trackfit_oracle as O
 from tests import test_oracle_model as PM
+from tests import test_oracle_seed as PS
 from tests import test_oracle_units as PU
 
 # mutants may overflow or cast NaN on the way to failing a pin
@@ -68,10 +71,28 @@ MUTANTS = [
 ]
 
 
-def _pins():
-    """Every pin of the two oracle test modules, parametrised cases expanded."""
+# mutants of the analytic-seed oracle (Sec. 3.1), caught by tests/test_oracle_seed.py
+SEED_MUTANTS = [
+    ("circle-centre-sign", "circle_through_three", "cy = (u1 - u2) / (2.0 * det)", "cy = (u2 - u1) / (2.0 * det)"),
+    ("circle-no-inversion", "circle_through_three", "u1, v1 = a[..., 0] / na, a[..., 1] / na", "u1, v1 = a[..., 0], a[..., 1]"),
+    ("seed-charge-sign", "seed_perigee", "q = -np.sign(cross)", "q = np.sign(cross)"),
+    ("seed-perigee-far-side", "seed_perigee", "px, py = centre[..., 0] - R * ux, centre[..., 1] - R * uy",
+     "px, py = centre[..., 0] + R * ux, centre[..., 1] + R * uy"),
+    ("seed-d0-sign", "seed_perigee", "d0 = -px * np.sin(phi0) + py * np.cos(phi0)", "d0 = px * np.sin(phi0) + py * np.cos(phi0)"),
+    ("seed-turning-reversed", "seed_perigee", "np.mod(-q * (g_h - g_p)", "np.mod(q * (g_h - g_p)"),
+    ("seed-z0-from-h2", "seed_perigee", "z0 = h0[..., 2] - s0 * cot", "z0 = h0[..., 2] - s2 * cot"),
+    ("seed-theta-complement", "seed_perigee", "theta = np.arctan2(1.0, cot)", "theta = np.arctan2(cot, 1.0)"),
+    ("seed-pt-units", "seed_perigee", "pt = C_LIGHT * b_field * R / 1000.0", "pt = C_LIGHT * b_field * R / 100.0"),
+    ("seed-qop-no-sin", "seed_perigee", "qop = q * np.sin(theta) / pt", "qop = q / pt"),
+    ("triplet-no-separation", "seed_triplet", "> min_sep", "> -1.0"),
+    ("helix-turns-wrong-way", "helix_point", "phi = phi0 - q * alpha", "phi = phi0 + q * alpha"),
+]
+
+
+def _pins(mods=None):
+    """Every pin of the oracle test modules, parametrised cases expanded."""
     out = []
-    for mod in (PU, PM):
+    for mod in (mods or (PU, PM)):
         for name, fn in sorted(vars(mod).items()):
             if not (name.startswith("test_") and callable(fn)):
                 continue
@@ -86,12 +107,12 @@ def _pins():
     return out
 
 
-def _install(monkeypatch, fname, old, new):
-    src = textwrap.dedent(inspect.getsource(getattr(O, fname)))
+def _install(monkeypatch, fname, old, new, mod=O):
+    src = textwrap.dedent(inspect.getsource(getattr(mod, fname)))
     assert src.count(old) == 1, f"mutation text not found once in {fname}: {old}"
     ns = {}
-    exec(compile(src.replace(old, new, 1), f"<mutant of {fname}>", "exec"), vars(O), ns)
-    monkeypatch.setattr(O, fname, ns[fname])
+    exec(compile(src.replace(old, new, 1), f"<mutant of {fname}>", "exec"), vars(mod), ns)
+    monkeypatch.setattr(mod, fname, ns[fname])
 
 
 @pytest.mark.parametrize("mid,fname,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
@@ -110,3 +131,14 @@ def test_pins_catch_mutant(monkeypatch, mid, fname, old, new):
 def test_unmutated_oracle_passes_every_pin():
     for pid, fn, kw in _pins():
         fn(**kw)
+
+
+@pytest.mark.parametrize("mid,fname,old,new", SEED_MUTANTS, ids=[m[0] for m in SEED_MUTANTS])
+def test_seed_pins_catch_mutant(monkeypatch, mid, fname, old, new):
+    _install(monkeypatch, fname, old, new, mod=SO)
+    for pid, fn, kw in _pins((PS,)):
+        try:
+            fn(**kw)
+        except Exception:
+            return
+    raise AssertionError(f"mutant {mid} passes every seed pin")
