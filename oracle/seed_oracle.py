@@ -25,11 +25,20 @@ Readings where the paper is silent (listed in the design doc as well):
   more than 10 mm (3-D) from the previous seed hit, so that overlap hits on the
   same layer (1.5 mm apart) never form a pair; the slope uses the first and the
   third seed hit (the longer lever arm);
-- with fewer than three hits so spaced the seed is undefined (NaN row).
+- with fewer than three hits so spaced the seed is undefined (NaN row);
+- the per-hit features: the foot point is the helix point whose normal plane
+  holds the hit, du and dv the hit's coordinates there along U = z x t / |z x t|
+  and V = t x U, s_helix the 3-D path length from the perigee to the foot point,
+  the asinh scale 1 mm;
+- the decode: d0, z0, phi, theta add the heads' corrections (phi wrapped), q/p
+  adds r (|q/p_seed| + 0.02 / GeV) (Sec. 3.3 states the residuals, not how the
+  heads' outputs are scaled; the corrections here are taken as given).
 
 Parity status: pinned in tests/test_oracle_seed.py (closed-form recovery of
 generated helices to fp64 rounding, invariances under rotation about and
-translation along the beam line, charge reversal, hit order).
+translation along the beam line, charge reversal, hit order; zero residuals of
+points on the helix and exact recovery of displacements in the normal plane;
+the decode's closed forms).
 """
 from __future__ import annotations
 
@@ -39,7 +48,8 @@ C_LIGHT = 0.299792458          # GeV / (T m)
 SEED_MIN_SEPARATION_MM = 10.0
 
 __all__ = ["circle_through_three", "seed_perigee", "seed_triplet", "seed_from_hits", "helix_point",
-           "C_LIGHT", "SEED_MIN_SEPARATION_MM"]
+           "helix_tangent", "curvilinear_residuals", "seed_features", "decode", "C_LIGHT",
+           "SEED_MIN_SEPARATION_MM", "QOP_EPS"]
 
 
 def circle_through_three(p0, p1, p2):
@@ -159,3 +169,102 @@ def helix_point(perigee, alpha, b_field):
     y = cy + q * R * np.cos(phi)
     z = z0 + R * alpha / np.tan(theta)
     return np.stack([x, y, z], axis=-1)
+
+
+# ---------------------------------------------------------------------------
+# per-hit residual features against the seed helix (Sec. 3.1)
+# ---------------------------------------------------------------------------
+
+def helix_tangent(perigee, alpha):
+    """Unit 3-D direction of motion [..., 3] at turning angle alpha: transverse
+    direction angle phi0 - q alpha, polar angle theta."""
+    perigee = np.asarray(perigee, dtype=np.float64)
+    phi0, theta, qop = perigee[..., 2], perigee[..., 3], perigee[..., 4]
+    phi = phi0 - np.sign(qop) * alpha
+    st = np.sin(theta)
+    return np.stack([st * np.cos(phi), st * np.sin(phi), np.cos(theta)], axis=-1)
+
+
+def curvilinear_residuals(perigee, hit, b_field, iters=60):
+    """(du, dv, s) of one hit [..., 3] against the helix of perigee [..., 5].
+
+    The foot point is the helix point whose normal plane holds the hit:
+    (hit - p(a)) . t(a) = 0, solved for the turning angle a by Newton's method from
+    the transverse angle of the hit around the circle's centre (a few steps reach
+    fp64 rounding; the iteration stops when a no longer changes).  In that plane
+    the curvilinear axes are U = z x t / |z x t| and V = t x U (the frame of the
+    linearised Kalman filter); du, dv are the hit's coordinates along them and s
+    the 3-D path length R a / sin(theta) from the perigee to the foot point.
+    Readings: the foot point as defined here, s measured from the perigee."""
+    perigee = np.asarray(perigee, dtype=np.float64)
+    hit = np.asarray(hit, dtype=np.float64)
+    d0, z0, phi0, theta, qop = (perigee[..., k] for k in range(5))
+    q = np.sign(qop)
+    R = 1000.0 * np.sin(theta) / np.abs(qop) / (C_LIGHT * b_field)
+    x0, y0 = -d0 * np.sin(phi0), d0 * np.cos(phi0)
+    cx, cy = x0 + q * R * np.sin(phi0), y0 - q * R * np.cos(phi0)
+    g0 = np.arctan2(y0 - cy, x0 - cx)
+    gh = np.arctan2(hit[..., 1] - cy, hit[..., 0] - cx)
+    a = np.mod(-q * (gh - g0), 2.0 * np.pi)
+    for _ in range(iters):
+        p = helix_point(perigee, a, b_field)
+        t = helix_tangent(perigee, a)
+        r = hit - p
+        g = np.sum(r * t, axis=-1)
+        # d/da of (hit - p) . t = -|dp/da|^2 / ... : dp/da = (R / sin theta) t, and
+        # dt/da = -q sin(theta) (-sin phi, cos phi, 0)
+        phi = phi0 - q * a
+        dt = np.stack([q * np.sin(theta) * np.sin(phi), -q * np.sin(theta) * np.cos(phi), 0.0 * phi], axis=-1)
+        dg = -R / np.sin(theta) + np.sum(r * dt, axis=-1)
+        step = g / dg
+        a_new = a - step
+        if np.all(np.abs(a_new - a) <= 1e-15 * np.maximum(1.0, np.abs(a))):
+            a = a_new
+            break
+        a = a_new
+    p = helix_point(perigee, a, b_field)
+    t = helix_tangent(perigee, a)
+    zhat = np.zeros_like(t)
+    zhat[..., 2] = 1.0
+    U = np.cross(zhat, t)
+    U = U / np.linalg.norm(U, axis=-1, keepdims=True)
+    V = np.cross(t, U)
+    r = hit - p
+    return np.sum(r * U, axis=-1), np.sum(r * V, axis=-1), R * a / np.sin(theta)
+
+
+def seed_features(perigee, hits, n_hits, b_field, scale_mm=1.0):
+    """The three seed features of every hit (Sec. 3.1): asinh(du / scale),
+    asinh(dv / scale) and s_helix [B, T, 3], zero on padded hits and on tracks
+    without a seed.  Reading: the asinh scale is 1 mm."""
+    perigee = np.asarray(perigee, dtype=np.float64)
+    hits = np.asarray(hits, dtype=np.float64)
+    B, T = hits.shape[:2]
+    out = np.zeros((B, T, 3))
+    valid = (np.arange(T)[None, :] < np.asarray(n_hits)[:, None]) & np.all(np.isfinite(perigee), axis=1)[:, None]
+    for t in range(T):
+        rows = np.nonzero(valid[:, t])[0]
+        if rows.size == 0:
+            continue
+        du, dv, s = curvilinear_residuals(perigee[rows], hits[rows, t, :3], b_field)
+        out[rows, t] = np.stack([np.arcsinh(du / scale_mm), np.arcsinh(dv / scale_mm), s], axis=-1)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# decode of the heads' median outputs against the seed (Sec. 3.3)
+# ---------------------------------------------------------------------------
+
+QOP_EPS = 0.02   # 1/GeV, the floor of the scale-free q/p residual
+
+
+def decode(seed, delta):
+    """Track parameters [..., 5] from the seed perigee and the heads' corrections:
+    d0, z0, theta additive, phi additive and wrapped to (-pi, pi], and q/p from
+    the scale-free residual r = (q/p - q/p_seed) / (|q/p_seed| + 0.02 / GeV)."""
+    seed = np.asarray(seed, dtype=np.float64)
+    delta = np.asarray(delta, dtype=np.float64)
+    out = seed + delta
+    out[..., 2] = np.pi - np.mod(np.pi - out[..., 2], 2.0 * np.pi)
+    out[..., 4] = seed[..., 4] + delta[..., 4] * (np.abs(seed[..., 4]) + QOP_EPS)
+    return out

@@ -86,6 +86,17 @@ SEED_MUTANTS = [
     ("seed-qop-no-sin", "seed_perigee", "qop = q * np.sin(theta) / pt", "qop = q / pt"),
     ("triplet-no-separation", "seed_triplet", "> min_sep", "> -1.0"),
     ("helix-turns-wrong-way", "helix_point", "phi = phi0 - q * alpha", "phi = phi0 + q * alpha"),
+    ("tangent-no-polar-angle", "helix_tangent", "st = np.sin(theta)", "st = 1.0"),
+    ("residual-axes-swapped", "curvilinear_residuals", "return np.sum(r * U, axis=-1), np.sum(r * V, axis=-1)",
+     "return np.sum(r * V, axis=-1), np.sum(r * U, axis=-1)"),
+    ("residual-v-sign", "curvilinear_residuals", "V = np.cross(t, U)", "V = np.cross(U, t)"),
+    ("residual-no-foot-search", "curvilinear_residuals", "a_new = a - step", "a_new = a"),
+    ("residual-transverse-path", "curvilinear_residuals", "R * a / np.sin(theta)", "R * a"),
+    ("features-no-asinh", "seed_features", "np.arcsinh(du / scale_mm)", "du / scale_mm"),
+    ("decode-phi-unwrapped", "decode", "out[..., 2] = np.pi - np.mod(np.pi - out[..., 2], 2.0 * np.pi)",
+     "out[..., 2] = out[..., 2]"),
+    ("decode-qop-absolute", "decode", "delta[..., 4] * (np.abs(seed[..., 4]) + QOP_EPS)", "delta[..., 4]"),
+    ("decode-qop-no-floor", "decode", "(np.abs(seed[..., 4]) + QOP_EPS)", "np.abs(seed[..., 4])"),
 ]
 
 

@@ -143,3 +143,74 @@ def test_seed_triplet_skips_close_hits():
     assert idx[1].tolist() == [-1, -1, -1]
     out = S.seed_from_hits(hits, np.array([6, 3]), B_FIELD)
     assert np.all(np.isnan(out[1]))
+
+
+# ---------------------------------------------------------------- per-hit features
+
+def _frame(truth, alpha):
+    """Tangent and curvilinear axes at turning angle alpha, written directly from
+    the generator's helix: direction angle phi0 - q alpha, polar angle theta."""
+    q = np.sign(truth[:, 4])
+    phi = truth[:, 2] - q * alpha
+    st, ct = np.sin(truth[:, 3]), np.cos(truth[:, 3])
+    t = np.stack([st * np.cos(phi), st * np.sin(phi), ct], axis=-1)
+    U = np.stack([-np.sin(phi), np.cos(phi), 0.0 * phi], axis=-1)       # z x t / |z x t|
+    V = np.cross(t, U)
+    return t, U, V
+
+
+def test_points_on_the_helix_have_zero_residuals():
+    pts, truth, alphas = _helices(500, seed=21)
+    for p, al in zip(pts, alphas):
+        du, dv, s = S.curvilinear_residuals(truth, p, B_FIELD)
+        assert np.all(np.abs(du) < 1e-8) and np.all(np.abs(dv) < 1e-8)
+        R = 1000.0 * np.sin(truth[:, 3]) / np.abs(truth[:, 4]) / (W.C_LIGHT * B_FIELD)
+        np.testing.assert_allclose(s, R * al / np.sin(truth[:, 3]), rtol=1e-12)
+
+
+def test_displacements_in_the_normal_plane_are_recovered():
+    """A hit moved by du U + dv V off a helix point keeps that point as its foot
+    point; the residuals give back (du, dv), signs included."""
+    pts, truth, alphas = _helices(800, seed=22)
+    for p, al in zip(pts, alphas):
+        _, U, V = _frame(truth, al)
+        du = rng.uniform(-5.0, 5.0, len(al))
+        dv = rng.uniform(-5.0, 5.0, len(al))
+        h = p + du[:, None] * U + dv[:, None] * V
+        gu, gv, s = S.curvilinear_residuals(truth, h, B_FIELD)
+        np.testing.assert_allclose(gu, du, rtol=0, atol=1e-9)
+        np.testing.assert_allclose(gv, dv, rtol=0, atol=1e-9)
+
+
+def test_seed_features_layout_and_padding():
+    pts, truth, alphas = _helices(20, seed=23)
+    B = len(truth)
+    hits = np.zeros((B + 1, 4, 5))
+    for k in range(3):
+        hits[:B, k, :3] = pts[k]
+    _, U, V = _frame(truth, alphas[1])
+    hits[:B, 1, :3] += 2.0 * U - 0.5 * V
+    n = np.array([3] * B + [3])
+    per = np.concatenate([truth, np.full((1, 5), np.nan)])
+    f = S.seed_features(per, hits, n, B_FIELD)
+    assert f.shape == (B + 1, 4, 3)
+    np.testing.assert_allclose(f[:B, 1, 0], np.arcsinh(2.0), rtol=1e-9)
+    np.testing.assert_allclose(f[:B, 1, 1], np.arcsinh(-0.5), rtol=1e-9)
+    assert np.all(np.abs(f[:B, [0, 2], :2]) < 1e-8)
+    assert np.all(f[:B, 3] == 0.0) and np.all(f[B] == 0.0)
+    assert np.all(np.diff(f[:B, :3, 2], axis=1) > 0.0)        # path length grows along the track
+
+
+# ---------------------------------------------------------------- decode
+
+def test_decode_closed_forms():
+    seed = np.array([[0.1, -3.0, 3.1, 1.2, -0.5], [0.0, 0.0, -1.0, 0.4, 0.01]])
+    zero = np.zeros((2, 5))
+    np.testing.assert_allclose(S.decode(seed, zero), seed, rtol=0, atol=1e-15)
+    delta = np.array([[0.2, 1.0, 0.1, -0.05, 0.1], [-0.1, 0.5, 0.2, 0.01, -0.5]])
+    out = S.decode(seed, delta)
+    np.testing.assert_allclose(out[:, [0, 1, 3]], seed[:, [0, 1, 3]] + delta[:, [0, 1, 3]], rtol=1e-15)
+    np.testing.assert_allclose(out[0, 2], 3.2 - 2.0 * np.pi, rtol=1e-14)      # wrapped into (-pi, pi]
+    np.testing.assert_allclose(out[1, 2], -0.8, rtol=1e-14)
+    np.testing.assert_allclose(out[0, 4], -0.5 + 0.1 * (0.5 + 0.02), rtol=1e-15)
+    np.testing.assert_allclose(out[1, 4], 0.01 - 0.5 * (0.01 + 0.02), rtol=1e-14)
