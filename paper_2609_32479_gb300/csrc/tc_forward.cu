@@ -977,10 +977,11 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     // for the current one; on a single counting barrier that arrival would
     // complete the current phase early.  The W_E hand-overs therefore alternate
     // between two barriers: a warp is never more than one hand-over ahead of
-    // another (the one after a pair waits for a product that needs both).  A failed wait sets the abort flag and
-    // every later wait fails fast, but no warp leaves the loop early: all warps
-    // keep taking the same sequence of named barriers (tile set-up, the norm
-    // reductions, the segment hand-overs), so none of them can be left waiting.
+    // another (the one after a pair waits for a product that needs both).
+    // A failed wait sets the abort flag and every later wait fails fast, but no
+    // warp leaves the loop early: all warps keep taking the same sequence of named
+    // barriers (the column-norm exchanges, the segment hand-overs), so none of
+    // them can be left waiting.
     auto signal_to = [&](uint32_t bar, bool wrote_operands) {
       if (wrote_operands) fence_proxy_async_smem();   // costly: only after operand writes
       tc_fence_before();
