@@ -1,5 +1,6 @@
 // tcgen05 path: one persistent, warp-specialised kernel runs the whole encoder
-// forward (embedding, every minGRU layer, pooling, head) for BF16_PROJ configs.
+// forward (embedding, every minGRU layer, pooling) for the 16-bit-operand
+// configs; head_kernel then applies the regression head to the pooled vectors.
 //
 // Orientation: every per-hit matrix product is computed transposed,
 //   D[channel][hit] = W[channel][k] * Act[k][hit],
@@ -225,7 +226,6 @@ __host__ __device__ inline void walk_tile(const TcParams& p, F&& f) {
     for (int kc = 0; kc < 3; ++kc)
       f(MAP_E1, mt * 128, kc * 64, kc == 2 ? 2 : 4, 256 + mt * 128, BSEL_HB, kc * 64, kc > 0,
         (mt == 0 && kc == 0) ? W_E : W_NONE, (mt == MT - 1 && kc == 2) ? C_ACC : C_NONE);
-  // a dense D x D product from XB into accumulator columns 0.. (MT tiles of 128 rows)
   // a dense D x D product from XB into accumulator columns tcol0 + 128 mt; with
   // onto = true it accumulates onto what the columns hold (MLP2 onto x')
   auto dense = [&](int map, int r0, int tcol0, bool onto) {
@@ -346,8 +346,8 @@ __device__ __forceinline__ void ep_silu_mt(const ECtx& x, const float* bias, int
   for (int i = 0; i < 32; ++i) v[i] = silu_t(v[i] + b);
   store_row32<FP16>(buf, row0 + x.c, x.col0, v);
 }
-// silu(acc + bias) of every tile (accumulator columns mt*128) -> XB rows
-// [mt*128 + c], all tiles' accumulators read under one TMEM wait
+// silu(acc + bias) of the embedding's first product (accumulator columns
+// 256 + mt*128) -> XB rows [mt*128 + c], all tiles read under one TMEM wait
 template <bool FP16, int MT>
 __device__ __forceinline__ void ep_silu_t(const ECtx& x, const float* bias) {
   float v[MT][32];
