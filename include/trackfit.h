@@ -181,10 +181,14 @@ int trackfit_debug_scan(const float* a, const float* b, const float* x, const in
  * counts (host, n_counts >= 6): [0] 128 x 64 weight blocks, [1] MMA instructions
  * (128 x 128 x 16 each), [2] operand hand-overs the issuer waits for from the
  * epilogue (W_E), [3] state hand-overs (W_H), [4] accumulator commits the
- * epilogue waits for (C_ACC), [5] state-buffer commits (C_HB).  Returns
- * TRACKFIT_ERR_UNSUPPORTED when cfg does not run on the tensor-core path,
- * TRACKFIT_ERR_INVALID_ARG for NULL pointers or n_counts < 6. */
-int trackfit_debug_schedule(const trackfit_config_t* cfg, int64_t* counts, int32_t n_counts);
+ * epilogue waits for (C_ACC), [5] state-buffer commits (C_HB).  codes (host,
+ * optional, NULL when codes_cap is 0): the first codes_cap blocks' hand-overs in
+ * issue order, one byte each: wait (0 none, 1 W_E, 2 W_H) | commit (0 none,
+ * 1 C_ACC, 2 C_HB) << 2.  Returns TRACKFIT_ERR_UNSUPPORTED when cfg does not run
+ * on the tensor-core path, TRACKFIT_ERR_INVALID_ARG for NULL pointers, n_counts
+ * < 6, or codes_cap > 0 with codes NULL. */
+int trackfit_debug_schedule(const trackfit_config_t* cfg, int64_t* counts, int32_t n_counts, uint8_t* codes,
+                            int64_t codes_cap);
 
 /* Test hook for the tensor-core operand layouts: D = A * B on one 128 x 128
  * tile through the same TMA, shared-memory descriptor and tensor-memory path as

@@ -285,13 +285,14 @@ extern "C" int trackfit_debug_scan(const float* a, const float* b, const float* 
                             reinterpret_cast<cudaStream_t>(stream));
 }
 
-extern "C" int trackfit_debug_schedule(const trackfit_config_t* cfg, int64_t* counts, int32_t n_counts) {
+extern "C" int trackfit_debug_schedule(const trackfit_config_t* cfg, int64_t* counts, int32_t n_counts,
+                                       uint8_t* codes, int64_t codes_cap) {
   if (!cfg || !counts) return TRACKFIT_ERR_INVALID_ARG;
   tf_shape s;
   tf_blob_off o;
   if (!derive(cfg, &s, &o)) return TRACKFIT_ERR_UNSUPPORTED;
   if (!tf_tc_supported(s)) return TRACKFIT_ERR_UNSUPPORTED;
-  return tf_tc_schedule_counts(s, counts, n_counts);
+  return tf_tc_schedule_counts(s, counts, n_counts, codes, codes_cap);
 }
 
 extern "C" int trackfit_debug_umma(trackfit_t h, const uint16_t* A, const uint16_t* Bkn, int32_t K, float* D,

@@ -1510,7 +1510,10 @@ struct tf_tc_state {
 
 struct ScheduleCounter {   // a callable for walk_tile on either side
   int64_t c[6] = {0, 0, 0, 0, 0, 0};
+  uint8_t* codes = nullptr;   // optional: per block wait | commit << 2, in order
+  int64_t cap = 0;
   __host__ __device__ void operator()(int, int, int, int nk, int, int, int, int, int wait, int commit) {
+    if (c[0] < cap) codes[c[0]] = (uint8_t)(wait | (commit << 2));
     ++c[0];
     c[1] += nk;
     c[2] += wait == W_E;
@@ -1523,9 +1526,10 @@ struct ScheduleCounter {   // a callable for walk_tile on either side
 // Per-tile totals of the fused kernel's block schedule, from the same walk_tile
 // the kernel expands (host only, no device needed): counts[0] blocks, [1] MMA
 // instructions (128 x 128 x 16 each), [2] W_E and [3] W_H hand-over waits, [4]
-// C_ACC and [5] C_HB commits.
-int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n) {
-  if (n < 6) return TRACKFIT_ERR_INVALID_ARG;
+// C_ACC and [5] C_HB commits; with codes, also each block's wait | commit << 2
+// in issue order (at most cap blocks).
+int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n, uint8_t* codes, int64_t cap) {
+  if (n < 6 || (cap > 0 && !codes)) return TRACKFIT_ERR_INVALID_ARG;
   TcParams q;
   memset(&q, 0, sizeof(q));
   q.D = s.D;
@@ -1533,6 +1537,8 @@ int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n) {
   q.NDC = s.H / 64;
   q.ROWS_IN = q.NDC * 256 + s.D;
   ScheduleCounter c;
+  c.codes = codes;
+  c.cap = cap;
   walk_tile(q, c);
   for (int i = 0; i < 6; ++i) counts[i] = c.c[i];
   return TRACKFIT_OK;

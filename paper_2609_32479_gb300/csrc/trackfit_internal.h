@@ -72,7 +72,7 @@ int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int
 
 // tc_forward.cu
 bool tf_tc_supported(const tf_shape& s);
-int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n);
+int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n, uint8_t* codes, int64_t cap);
 int tf_tc_create(trackfit_ctx* h, const float* host_w);
 void tf_tc_destroy(trackfit_ctx* h);
 int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,

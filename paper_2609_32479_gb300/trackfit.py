@@ -87,7 +87,7 @@ def load() -> ctypes.CDLL:
     lib.trackfit_profile_read.restype = ctypes.c_int
     lib.trackfit_forward_noalloc.argtypes = [ctypes.POINTER(Config), vp, vp, vp, i64, vp, vp]
     lib.trackfit_forward_noalloc.restype = ctypes.c_int
-    lib.trackfit_debug_schedule.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32]
+    lib.trackfit_debug_schedule.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32, vp, i64]
     lib.trackfit_debug_schedule.restype = ctypes.c_int
     _lib = lib
     return lib
@@ -117,17 +117,26 @@ def weight_count(m: W.ModelConfig) -> int:
     return int(load().trackfit_weight_count(ctypes.byref(c)))
 
 
-def schedule_counts(m: W.ModelConfig):
+def schedule_counts(m: W.ModelConfig, with_codes: bool = False):
     """Per-tile totals of the tensor-core path's block schedule (host only): dict
-    with blocks, mmas, w_e, w_h, c_acc, c_hb; None when m does not run on that path."""
+    with blocks, mmas, w_e, w_h, c_acc, c_hb (and, with_codes, "codes": each block's
+    wait | commit << 2 in issue order); None when m does not run on that path."""
     c = make_config(m)
     out = (ctypes.c_int64 * 6)()
-    st = load().trackfit_debug_schedule(ctypes.byref(c), out, 6)
+    lib = load()
+    st = lib.trackfit_debug_schedule(ctypes.byref(c), out, 6, None, 0)
     if st == ERR_UNSUPPORTED:
         return None
     if st != OK:
         raise TrackfitError(st, "trackfit_debug_schedule")
-    return dict(zip(("blocks", "mmas", "w_e", "w_h", "c_acc", "c_hb"), (int(v) for v in out)))
+    res = dict(zip(("blocks", "mmas", "w_e", "w_h", "c_acc", "c_hb"), (int(v) for v in out)))
+    if with_codes:
+        codes = (ctypes.c_uint8 * res["blocks"])()
+        st = lib.trackfit_debug_schedule(ctypes.byref(c), out, 6, codes, res["blocks"])
+        if st != OK:
+            raise TrackfitError(st, "trackfit_debug_schedule")
+        res["codes"] = list(codes)
+    return res
 
 
 def _stream_handle(stream) -> Optional[int]:

@@ -111,3 +111,54 @@ def test_schedule_handovers_match_the_epilogue(lib, D, H, L, prec):
 def test_schedule_hook_rejects_cuda_core_configs(lib):
     assert T.schedule_counts(W.workload("tiny").model) is None
     assert T.schedule_counts(W.workload("large").model.with_(precision=W.PRECISION_FP32)) is None
+
+
+def _epilogue_events(m, tiles=2):
+    """The epilogue warps' hand-over events in program order for `tiles` tiles:
+    'S' = an operand hand-over (W_E arrival), 'W' = a wait for an accumulator
+    commit (C_ACC), restated from the epilogue loop."""
+    MT, NDC, L = m.d_model // 128, m.d_hidden // 64, m.n_layers
+    ev = ["S"]                                   # the first tile's Fourier operand
+    for _ in range(tiles):
+        ev += ["W", "S"]                         # embedding product 1 -> its SiLU
+        ev += ["W"] * MT + ["S"] * MT            # embedding product 2 -> x_hat per channel tile
+        for l in range(L):
+            ev += ["W", "S"] * NDC               # z/n of each chunk -> columns released
+            ev += ["W", "S"] * MT                # last merge tile -> output gate of that tile
+            ev += ["W", "S"] * MT                # MLP1 tile -> its SiLU
+            ev += ["W"] * MT                     # MLP2 tiles
+            ev += ["S"] * MT if l + 1 < L else ["S"]   # x_hat per tile, or the next tile's operand
+    return ev
+
+
+@pytest.mark.parametrize("D,H,L", [(128, 192, 6), (256, 384, 8), (256, 384, 1), (128, 192, 1)])
+def test_no_epilogue_warp_runs_two_hand_overs_ahead(lib, D, H, L):
+    """The operand hand-overs alternate between two barriers, which is enough only
+    if no warp can arrive for hand-over k + 2 before every warp has arrived for k:
+    hand-over k + 2 must come after a wait for an accumulator commit that the
+    issuer makes only after consuming hand-over k.  Checked on the issuer's block
+    order against the epilogue's event order over two tiles."""
+    m = W.ModelConfig(max_hits=24, d_model=D, d_hidden=H, n_layers=L, precision=W.PRECISION_BF16)
+    codes = T.schedule_counts(m, with_codes=True)["codes"] * 3
+    w_before_commit = []                       # W_E hand-overs the issuer consumed before commit c
+    n_we = 0
+    for code in codes:
+        if code & 3 == 1:
+            n_we += 1
+        if (code >> 2) == 1:
+            w_before_commit.append(n_we)
+    ev = _epilogue_events(m)
+    n_sig = sum(e == "S" for e in ev)
+    assert sum(e == "W" for e in ev) <= len(w_before_commit)
+    waits = 0
+    s = 0
+    for e in ev:
+        if e == "W":
+            waits += 1
+            continue
+        # a warp reaching hand-over s has seen commit waits - 1, which needs hand-overs
+        # 0 .. w_before_commit[waits - 1] - 1 from every warp
+        done_by_all = w_before_commit[waits - 1] if waits else 0
+        assert s - done_by_all <= 1, f"hand-over {s} can run {s - done_by_all} ahead"
+        s += 1
+    assert s == n_sig
