@@ -162,3 +162,14 @@ def test_no_epilogue_warp_runs_two_hand_overs_ahead(lib, D, H, L):
         assert s - done_by_all <= 1, f"hand-over {s} can run {s - done_by_all} ahead"
         s += 1
     assert s == n_sig
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """No CPU fallback: without the built library the binding raises instead of
+    computing anything."""
+    monkeypatch.setattr(T, "_lib", None)
+    monkeypatch.setattr(T, "LIB_PATH", str(tmp_path / "libtrackfit.so"))
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        T.load()
+    with pytest.raises(RuntimeError):
+        T.weight_count(W.workload("tiny").model)
