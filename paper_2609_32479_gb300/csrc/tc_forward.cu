@@ -66,7 +66,8 @@ enum { MAP_E1 = 0, MAP_E2, MAP_IN, MAP_M, MAP_1, MAP_2, NMAPS };
 enum { BSEL_XB = 0, BSEL_HB = 1 };
 // Hand-overs around a schedule block: before its first MMA the issuer waits for
 // the epilogue's next hand-over on e_bar (W_E; two barriers used alternately) or
-// eh_bar (W_H); after its last MMA it commits to acc_bar (C_ACC) or hb_bar (C_HB).
+// eh_bar (W_H); after its last MMA it commits to acc_bar (C_ACC; two barriers
+// used alternately) or hb_bar (C_HB).
 enum { W_NONE = 0, W_E = 1, W_H = 2 };
 enum { C_NONE = 0, C_ACC = 1, C_HB = 2 };
 // bits of an MMA schedule entry
@@ -117,7 +118,7 @@ struct TileMeta {
 };
 struct Misc {
   uint64_t full[MAX_STAGES], empty[MAX_STAGES];
-  uint64_t acc_bar, e_bar[2], hb_bar, eh_bar, drain_bar;
+  uint64_t acc_bar[2], e_bar[2], hb_bar, eh_bar, drain_bar;
   uint64_t meta_full[2], meta_free[2];   // loader -> epilogue, epilogue -> loader
   uint32_t tmem_base;
   int abort_flag;
@@ -765,7 +766,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
   Misc* m = reinterpret_cast<Misc*>(gbase + p.off_misc);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t full0 = smem_u32(&m->full[0]), empty0 = smem_u32(&m->empty[0]);
-  const uint32_t acc_bar = smem_u32(&m->acc_bar);
+  const uint32_t acc_bar0 = smem_u32(&m->acc_bar[0]), acc_bar1 = smem_u32(&m->acc_bar[1]);
   const uint32_t e_bar0 = smem_u32(&m->e_bar[0]), e_bar1 = smem_u32(&m->e_bar[1]);
   const uint32_t hb_bar = smem_u32(&m->hb_bar), eh_bar = smem_u32(&m->eh_bar);
   const uint32_t drain_bar = smem_u32(&m->drain_bar);
@@ -775,7 +776,8 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
-    mbar_init(acc_bar, 1);
+    mbar_init(acc_bar0, 1);
+    mbar_init(acc_bar1, 1);
     mbar_init(e_bar0, NE / 32);   // one arrival per epilogue warp
     mbar_init(e_bar1, NE / 32);
     mbar_init(hb_bar, 1);
@@ -892,8 +894,18 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       tc_fence_after();
       return true;
     };
+    // The k-th accumulator commit goes to acc_bar[k % 2] (some commits come in
+    // pairs with no epilogue hand-over between them; see the epilogue).  The
+    // count is kept by the whole warp: the barrier of a block's commit, and the
+    // count advanced past it.
+    uint32_t acc_k = 0;
+    auto acc_for = [&](uint32_t e) -> uint32_t {
+      const uint32_t b = (acc_k & 1u) ? acc_bar1 : acc_bar0;
+      if (e & S_C_ACC) ++acc_k;
+      return b;
+    };
     // the MMAs and group commits of one block (elected lane only)
-    auto issue = [&](uint32_t e, uint64_t ad) {
+    auto issue = [&](uint32_t e, uint64_t ad, uint32_t acc_b) {
       const uint64_t bd = ((e >> 13) & 1u ? b_desc_hb : b_desc_xb) + (uint64_t)(e & 0x1FFFu);
       const uint32_t d = tmem + ((e >> 14) & 3u) * 128u;
       const uint32_t nk4 = e & S_NK4;
@@ -901,7 +913,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       umma_f16(d, ad + 2, bd + BSTEP, idesc, 1u);
       umma_f16_if(d, ad + 4, bd + 2 * BSTEP, idesc, 1u, nk4);
       umma_f16_if(d, ad + 6, bd + 3 * BSTEP, idesc, 1u, nk4);
-      umma_commit_if(acc_bar, e & S_C_ACC);
+      umma_commit_if(acc_b, e & S_C_ACC);
       umma_commit_if(hb_bar, e & S_C_HB);
     };
     int i0 = 0;   // schedule index of the stage's first block
@@ -912,6 +924,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       const uint32_t e0 = sm_tab[i0], e1 = two ? sm_tab[i1] : 0u;
       i0 = i1 + 1;
       if (i0 >= p.n_sched) i0 -= p.n_sched;
+      const uint32_t ab0 = acc_for(e0), ab1 = acc_for(e1);   // (e1 = 0 commits nothing)
       if ((e0 & (S_W_E | S_W_H)) && !(ok = handover(e0))) break;
       if (!mbar_test_wait(full0 + 8 * stage, phase)) {
         uint32_t ph = phase;
@@ -922,18 +935,18 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       const uint64_t ad1 = ad0 + (uint64_t)(A_BLOCK >> 4);
       const uint32_t empty = empty0 + 8 * stage;
       if (e1 & (S_W_E | S_W_H)) {   // a hand-over between the two blocks
-        if (elect_one()) issue(e0, ad0);
+        if (elect_one()) issue(e0, ad0, ab0);
         __syncwarp();
         if (!(ok = handover(e1))) break;
         if (elect_one()) {
-          issue(e1, ad1);
+          issue(e1, ad1, ab1);
           umma_commit(empty);
         }
         __syncwarp();
       } else {
         if (elect_one()) {
-          issue(e0, ad0);
-          if (two) issue(e1, ad1);
+          issue(e0, ad0, ab0);
+          if (two) issue(e1, ad1, ab1);
           umma_commit(empty);
         }
         __syncwarp();
@@ -967,7 +980,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     x.MT = p.D >> 7;
     x.tq = tmem + ((uint32_t)(32 * x.q) << 16);
     x.xs = p.xs + (size_t)blockIdx.x * TILE * p.D;
-    uint32_t acc_phase = 0, hb_phase = 0;
+    uint32_t acc_ph0 = 0, acc_ph1 = 0, hb_phase = 0;
     // The epilogue warps run decoupled: each makes its shared-memory operand
     // writes visible to the async proxy, orders its TMEM reads and arrives on the
     // hand-over barrier itself (e_bar and eh_bar count one arrival per warp), and
@@ -977,7 +990,13 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     // for the current one; on a single counting barrier that arrival would
     // complete the current phase early.  The W_E hand-overs therefore alternate
     // between two barriers: a warp is never more than one hand-over ahead of
-    // another (the one after a pair waits for a product that needs both).
+    // another (the one after a pair waits for a product that needs both).  The
+    // accumulator commits come in such pairs too (the last merge's two channel
+    // tiles, MLP1's, MLP2's, the embedding's second product): a warp that starts
+    // its wait for the first of a pair after the second has landed would see the
+    // phase parity flipped twice, so they alternate between two barriers as
+    // well (a warp is never two commits behind: the issuer makes commit k + 2
+    // only after a hand-over that every warp gives after its wait for commit k).
     // A failed wait sets the abort flag and every later wait fails fast, but no
     // warp leaves the loop early: all warps keep taking the same sequence of named
     // barriers (the column-norm exchanges, the segment hand-overs), so none of
@@ -1000,7 +1019,14 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       ph ^= 1u;
       tc_fence_after();
     };
-    auto wait_acc = [&]() { wait_on(acc_bar, acc_phase); };
+    uint32_t acc_k = 0;   // accumulator commits waited for so far: the next is on acc_bar[acc_k % 2]
+    auto wait_acc = [&]() {
+      if (acc_k & 1u)
+        wait_on(acc_bar1, acc_ph1);
+      else
+        wait_on(acc_bar0, acc_ph0);
+      ++acc_k;
+    };
     const uint8_t* fbuf = p.fbuf + (size_t)blockIdx.x * 2 * EB_BYTES;
     uint32_t meta_ph[2] = {0u, 0u};
     // tile start: the loader's metadata and Fourier operand of the CTA's i-th tile

@@ -113,17 +113,21 @@ def test_schedule_hook_rejects_cuda_core_configs(lib):
     assert T.schedule_counts(W.workload("large").model.with_(precision=W.PRECISION_FP32)) is None
 
 
-def _epilogue_events(m, tiles=2):
+def _epilogue_events(m, tiles=2, states=False):
     """The epilogue warps' hand-over events in program order for `tiles` tiles:
     'S' = an operand hand-over (W_E arrival), 'W' = a wait for an accumulator
-    commit (C_ACC), restated from the epilogue loop."""
+    commit (C_ACC), restated from the epilogue loop; with states, also 'B' = a
+    wait for a state-buffer commit (C_HB) and 'H' = a state hand-over (W_H)."""
     MT, NDC, L = m.d_model // 128, m.d_hidden // 64, m.n_layers
     ev = ["S"]                                   # the first tile's Fourier operand
     for _ in range(tiles):
         ev += ["W", "S"]                         # embedding product 1 -> its SiLU
         ev += ["W"] * MT + ["S"] * MT            # embedding product 2 -> x_hat per channel tile
         for l in range(L):
-            ev += ["W", "S"] * NDC               # z/n of each chunk -> columns released
+            for dc in range(NDC):                # z/n of each chunk -> columns released
+                ev += ["W", "S"]                 # (-> previous merge done -> states handed over)
+                if states:
+                    ev += (["B"] if dc > 0 else []) + ["H"]
             ev += ["W", "S"] * MT                # last merge tile -> output gate of that tile
             ev += ["W", "S"] * MT                # MLP1 tile -> its SiLU
             ev += ["W"] * MT                     # MLP2 tiles
@@ -173,3 +177,45 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
         T.load()
     with pytest.raises(RuntimeError):
         T.weight_count(W.workload("tiny").model)
+
+
+@pytest.mark.parametrize("D,H,L", [(128, 192, 6), (256, 384, 8), (256, 384, 1), (128, 192, 1), (128, 192, 16)])
+def test_no_epilogue_warp_falls_two_commits_behind(lib, D, H, L):
+    """The accumulator commits alternate between two barriers, which is enough only
+    if no warp can still be waiting for commit k when commit k + 2 (same barrier)
+    lands: the issuer must make commit k + 2 only after some hand-over (operand or
+    state) that every warp gives after its wait for commit k.  Checked on the
+    issuer's block order against the epilogue's event order over three tiles."""
+    m = W.ModelConfig(max_hits=24, d_model=D, d_hidden=H, n_layers=L, precision=W.PRECISION_BF16)
+    tiles = 3
+    codes = T.schedule_counts(m, with_codes=True)["codes"] * tiles
+    ev = _epilogue_events(m, tiles=tiles, states=True)
+    # accumulator waits completed by a warp before it gives its k-th W_E / W_H hand-over
+    done_before = {"S": [], "H": []}
+    waits = 0
+    for e in ev:
+        if e == "W":
+            waits += 1
+        elif e in done_before:
+            done_before[e].append(waits)
+    n_commits = sum(1 for c in codes if (c >> 2) == 1)
+    assert n_commits >= waits                    # every epilogue wait has its commit
+    # walk the issuer: gate[j] = the most accumulator waits that every warp has
+    # certainly completed when commit j is issued
+    n_s = n_h = 0
+    gate = 0
+    j = 0
+    for c in codes:
+        if c & 3 == 1:
+            if n_s < len(done_before["S"]):
+                gate = max(gate, done_before["S"][n_s])
+            n_s += 1
+        elif c & 3 == 2:
+            if n_h < len(done_before["H"]):
+                gate = max(gate, done_before["H"][n_h])
+            n_h += 1
+        if (c >> 2) == 1:
+            if j >= 2 and j < waits:
+                assert gate >= j - 1, f"commit {j} can land while a warp still waits for commit {j - 2}"
+            j += 1
+    assert n_s >= len(done_before["S"]) - 1 and n_h >= len(done_before["H"])
