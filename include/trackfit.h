@@ -86,7 +86,8 @@ typedef struct {
 
 typedef struct trackfit_ctx* trackfit_t;
 
-/* Number of fp32 values in the weight blob for cfg (0 if cfg is NULL or
+/* Size of the encoder of Sec. 3.2 for cfg (the paper's model: 0.64 M parameters).
+ * Number of fp32 values in the weight blob for cfg (0 if cfg is NULL or
  * unsupported).  Blob order, every matrix in PyTorch [out][in] row-major order,
  * with D = d_model, H = d_hidden, E = 2 * n_features * n_fourier,
  * P = D (mean pooling) or 2H (endpoints), Hh = head_hidden, Q = 5 * n_quantiles:
@@ -97,7 +98,11 @@ typedef struct trackfit_ctx* trackfit_t;
  *   g_h[P] W_h1[Hh][P] b_h1[Hh] W_h2[Q][Hh] b_h2[Q]   (Q rows parameter-major: [5][7]) */
 size_t trackfit_weight_count(const trackfit_config_t* cfg);
 
-/* Validate cfg, copy the host fp32 weights to the device (converted and repacked
+/* Load a trained encoder (Sec. 3.2: Fourier featurisation, dense embedding,
+ * bidirectional minGRU layers, RMSNorm and the quantile head) for inference.
+ * With 16-bit operand precision the weights of the per-hit products are
+ * converted once here (Sec. 3.5: reduced-precision projection weights).
+ * Validate cfg, copy the host fp32 weights to the device (converted and repacked
  * for the kernels) and allocate the handle's workspace.  Synchronous; launches no
  * work on any user stream.  The caller keeps ownership of `weights` and may free
  * it on return.  Errors: INVALID_ARG (NULL, n_weights != trackfit_weight_count),
@@ -106,7 +111,13 @@ size_t trackfit_weight_count(const trackfit_config_t* cfg);
 int trackfit_create(const trackfit_config_t* cfg, const float* weights, size_t n_weights,
                     trackfit_t* out);
 
-/* Run the encoder on n_tracks tracks, asynchronously on `stream` (a cudaStream_t;
+/* The fit itself (Sec. 3, problem statement): each track's hit sequence, in
+ * measurement-time order, to its five perigee parameters, for a batch of
+ * independent tracks in one call (Sec. 4: the fit is embarrassingly parallel
+ * across tracks; Sec. 3.5: tracks run packed, without padding, inside the
+ * kernels).  The output is the median of the 7 quantiles of each parameter
+ * (Sec. 3.3).
+ * Run the encoder on n_tracks tracks, asynchronously on `stream` (a cudaStream_t;
  * NULL = the legacy default stream).  No host synchronisation, no allocation.
  *   hits       device, [n_tracks][max_hits][5] fp32, row-major, 16-byte aligned;
  *              hit t of track b is valid for t < n_hits[b]; padded entries are
@@ -120,23 +131,34 @@ int trackfit_create(const trackfit_config_t* cfg, const float* weights, size_t n
 int trackfit_forward(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
                      float* out_params, void* stream);
 
-/* As trackfit_forward, and optionally also writes (each pointer may be NULL):
+/* As trackfit_forward, and optionally also writes (each pointer may be NULL)
+ * the head's full quantile output (Sec. 3.3: 7 quantiles per parameter) and the
+ * pooled track vector it reads (Sec. 3.2):
  *   out_quantiles device [n_tracks][5][7] fp32: all head outputs (Sec. 3.2-3.3);
  *   out_pooled    device [n_tracks][P] fp32: the pooled vector before the head. */
 int trackfit_forward_ex(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
                         float* out_params, float* out_quantiles, float* out_pooled, void* stream);
 
-/* End-to-end variant with HOST buffers: copies hits [n_tracks][max_hits][5] and
+/* The fit of trackfit_forward with the data movement a deployment pays (Sec. 4.2
+ * times the whole forward from the hits to the parameters).
+ * End-to-end variant with HOST buffers: copies hits [n_tracks][max_hits][5] and
  * n_hits [n_tracks] to the device, runs the encoder and copies out_params
  * [n_tracks][5] back, all on `stream`, and returns after the stream has finished
  * this work (synchronous).  Pinned (page-locked) host memory makes the copies
  * asynchronous and faster; pageable memory works too.  The device staging
  * buffers are owned by the handle and grow on demand (this call may allocate).
- * Errors as trackfit_forward, plus OOM. */
+ * Errors as trackfit_forward, plus OOM.  Before returning it reads and resets the
+ * device error counters (as trackfit_device_errors): TRACKFIT_ERR_BAD_HITS when
+ * tracks had hit counts outside [1, max_hits] (their rows are NaN, the others
+ * valid), TRACKFIT_ERR_TIMEOUT when a bounded device wait expired (the output is
+ * not valid). */
 int trackfit_forward_host(trackfit_t h, const float* hits_host, const int32_t* n_hits_host,
                           int64_t n_tracks, float* out_params_host, void* stream);
 
-/* Read and reset the device error counters: synchronises `stream`, returns the
+/* Validity of a batch's results.  The problem statement (Sec. 3) defines a
+ * track by its hits; a track with no hit, or with more hits than max_hits, has
+ * no defined fit and gets a NaN row, counted here.
+ * Read and reset the device error counters: synchronises `stream`, returns the
  * number of tracks with invalid n_hits since the last call in *n_bad, and
  * returns TRACKFIT_ERR_TIMEOUT if a bounded device wait expired (else OK or
  * BAD_HITS when *n_bad > 0). */
@@ -160,7 +182,9 @@ int trackfit_set_path(trackfit_t h, int path);
 int trackfit_profile(trackfit_t h, int enable);
 int trackfit_profile_read(trackfit_t h, double* kernel_ms, int64_t* launches);
 
-/* Free everything the handle owns.  Accepts NULL.  The caller must make sure no
+/* Release a loaded encoder (the counterpart of trackfit_create; the paper's
+ * model lives for the whole job, Sec. 4.2).
+ * Free everything the handle owns.  Accepts NULL.  The caller must make sure no
  * work using the handle is still running on any stream. */
 void trackfit_destroy(trackfit_t h);
 
@@ -168,7 +192,7 @@ void trackfit_destroy(trackfit_t h);
 const char* trackfit_strerror(int status);
 
 /* Test hook: masked bidirectional linear recurrence h_t = a_t h_{t-1} + b_t x_t
- * (the spec form of Eq. 2 with a = 1 - z, b = z, x = n) on the device.
+ * (Eq. 2 written as a linear recurrence, with a = 1 - z, b = z, x = n) on the device.
  * a, b, x, h_fwd, h_bwd: device [n_tracks][T][C] fp32; n_hits device [n_tracks].
  * Steps t >= n_hits[b] carry the state and output 0; the reverse scan starts at
  * t = n_hits[b] - 1.  Asynchronous on `stream`. */

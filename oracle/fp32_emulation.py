@@ -1,0 +1,132 @@
+"""fp32 emulation of the oracle's forward: the same steps in the same order, in
+fp32 arithmetic instead of fp64.
+
+TEST INFRASTRUCTURE, like the rest of this package: only the tests, the smoke
+check, the bench's CPU leg and the script under tests/golden/ that writes the
+stored tolerance bars may use it.  It shares no code with the CUDA path.
+
+Why it exists.  On the reduced-precision configs the paper's recipe (Sec. 3.5:
+16-bit projection operands, fp32 accumulation and recurrence) rounds every
+operand of the per-hit matrix products to 16 bits.  Two correct implementations
+that accumulate in different precisions (fp64 here, fp32 on the GPU) round a few
+operands to different neighbouring 16-bit values, and the random-init network
+amplifies those flips.  The spread between this emulation and the fp64 oracle
+on the same inputs is therefore the error a correct fp32-accumulating
+implementation is expected to show; the GPU parity bars for bf16 operands are
+derived from it (tests/golden/make_bf16_bars.py).
+
+Arithmetic: hit features normalised and featurised in fp64 then rounded to fp32
+(the GPU forms the Fourier argument without rounding error); every product,
+bias, gate, norm, scan step, residual, pooling sum and head operation in fp32
+(numpy float32; matmul accumulates in fp32); the 16-bit operand rounding of the
+oracle (round to nearest even) applied to the same operands.
+"""
+from __future__ import annotations
+
+from typing import Optional
+
+import numpy as np
+
+from . import trackfit_oracle as O
+
+F32 = np.float32
+
+
+def _op(x, prec):
+    """Operand of a per-hit product, rounded to bf16 (1) or fp16 (2); fp32 result.
+    Both formats embed exactly in fp32, so the round trip through fp64 is exact."""
+    x = np.asarray(x, dtype=F32)
+    if prec == 1:
+        return O.bf16_round(x.astype(np.float64)).astype(F32)
+    if prec == 2:
+        return O.fp16_round(x.astype(np.float64)).astype(F32)
+    return x
+
+
+def _lin(x, w, b, prec):
+    return (_op(x, prec) @ _op(w, prec).T + b.astype(F32)).astype(F32)
+
+
+def sigmoid(x):
+    with np.errstate(over="ignore"):
+        return (F32(1.0) / (F32(1.0) + np.exp(-x, dtype=F32))).astype(F32)
+
+
+def silu(x):
+    return (x * sigmoid(x)).astype(F32)
+
+
+def rmsnorm(x, g, eps):
+    ms = np.mean(x * x, axis=-1, keepdims=True, dtype=F32)
+    return (x / np.sqrt(ms + F32(eps)) * g.astype(F32)).astype(F32)
+
+
+def linear_scan(a, b, x, valid, reverse=False):
+    """h_t = a_t h_{t-1} + b_t x_t along axis 1 in fp32 (masked as the oracle's)."""
+    B, T, C = x.shape
+    h = np.zeros((B, C), dtype=F32)
+    out = np.zeros((B, T, C), dtype=F32)
+    steps = range(T - 1, -1, -1) if reverse else range(T)
+    for t in steps:
+        v = valid[:, t, None]
+        h = np.where(v, (a[:, t] * h + b[:, t] * x[:, t]).astype(F32), h)
+        out[:, t] = np.where(v, h, F32(0.0))
+    return out
+
+
+def encoder_layer(x, W, l, cfg, valid, prec):
+    """One layer, the oracle's encoder_layer in fp32 (mean-pooling form)."""
+    D, H = cfg["d_model"], cfg["d_hidden"]
+    p = f"layer{l}."
+    xh = rmsnorm(x, W[p + "g"], cfg["rms_eps"])
+    proj = _lin(xh, W[p + "w_in"], W[p + "b_in"], prec)
+    z_f = sigmoid(proj[..., 0:H])
+    n_f = proj[..., H:2 * H]
+    z_b = sigmoid(proj[..., 2 * H:3 * H])
+    n_b = proj[..., 3 * H:4 * H]
+    gate = sigmoid(proj[..., 4 * H:4 * H + D])
+    one = F32(1.0)
+    h_f = linear_scan((one - z_f).astype(F32), z_f, n_f, valid)
+    h_b = linear_scan((one - z_b).astype(F32), z_b, n_b, valid, reverse=True)
+    y = np.concatenate([h_f, h_b], axis=-1)
+    m = _lin(y, W[p + "w_m"], W[p + "b_m"], prec)
+    x1 = (x + m * gate).astype(F32)
+    u = silu(_lin(x1, W[p + "w1"], W[p + "b1"], prec))
+    x2 = (x1 + _lin(u, W[p + "w2"], W[p + "b2"], prec)).astype(F32)
+    return np.where(valid[..., None], x2, F32(0.0)), h_f, h_b
+
+
+def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
+    """Track parameters [B, 5] (returned as fp64 holding fp32 values) for mean
+    pooling; with capture, also the pooled vector after every layer
+    (capture["pooled_by_layer"][l], fp64 holding fp32 values)."""
+    if int(cfg["pool"]) != 0:
+        raise ValueError("the fp32 emulation covers mean pooling only")
+    Wd = O.split_blob(cfg, blob)
+    W = {k: v.astype(F32) for k, v in Wd.items()}
+    prec = int(cfg["precision"])
+    hits = np.asarray(hits)
+    n_hits = np.asarray(n_hits).astype(np.int64)
+    B, T, _ = hits.shape
+    bad = (n_hits < 1) | (n_hits > T)
+    n_ok = np.where(bad, 1, n_hits)
+    valid = np.arange(T)[None, :] < n_ok[:, None]
+    e = O.fourier(O.normalise(hits, cfg["feat_min"], cfg["feat_max"]), cfg["fourier_scale"]).astype(F32)
+    hdn = silu(_lin(e, W["emb.w1"], W["emb.b1"], prec))
+    x = np.where(valid[..., None], _lin(hdn, W["emb.w2"], W["emb.b2"], prec), F32(0.0))
+    nf = n_ok[:, None].astype(F32)
+    by_layer = []
+    for l in range(cfg["n_layers"]):
+        x, _, _ = encoder_layer(x, W, l, cfg, valid, prec)
+        if capture is not None:
+            by_layer.append((np.sum(x, axis=1, dtype=F32) / nf).astype(np.float64))
+    pv = (np.sum(x, axis=1, dtype=F32) / nf).astype(F32)
+    hn = rmsnorm(pv, W["head.g"], cfg["rms_eps"])
+    hid = silu((hn @ W["head.w1"].T + W["head.b1"]).astype(F32))
+    q = (hid @ W["head.w2"].T + W["head.b2"]).astype(F32)
+    nq = cfg["n_quantiles"]
+    q = q.reshape(B, q.shape[1] // nq, nq)
+    out = np.where(bad[:, None], np.nan, q[:, :, nq // 2].astype(np.float64))
+    if capture is not None:
+        capture.update(pooled=pv.astype(np.float64), pooled_by_layer=by_layer)
+    return out

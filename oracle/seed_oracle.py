@@ -20,7 +20,7 @@ transverse arc length R a, and z = z0 + R a cot(theta); the perigee point is
 (-d0 sin phi0, d0 cos phi0); p_T = C R B / 1000 GeV for R in mm and B in T, with
 C = 0.299792458; q/p = q sin(theta) / p_T in 1/GeV.
 
-Readings where the paper is silent (listed in the design doc as well):
+Readings where the paper is silent:
 - the seed triplet: hits taken in path order, each seed hit the first later hit
   more than 10 mm (3-D) from the previous seed hit, so that overlap hits on the
   same layer (1.5 mm apart) never form a pair; the slope uses the first and the

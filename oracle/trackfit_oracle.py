@@ -9,7 +9,7 @@ Everything is computed in fp64 with plain numpy: elementwise formulas and
 matmul as the only library step.  Each function states the passage of the paper
 it follows ("Fast and Precise Learned Charged-Particle Trajectory Regression at
 the LHC").  Where the paper is silent, the reading taken is stated in the
-function and collected in DESIGN.md.
+function that takes it.
 
 Reduced-precision modes (precision = 1: bf16, precision = 2: fp16): the paper
 runs the encoder GEMMs in fp16 with fp32 recurrence state (Sec. 3.5).  The oracle

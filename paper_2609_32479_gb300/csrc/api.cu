@@ -259,7 +259,11 @@ extern "C" int trackfit_forward_host(trackfit_t h, const float* hits_host, const
   if (r != TRACKFIT_OK) return r;
   e = cudaMemcpyAsync(out_host, h->st_out, n_tracks * 5 * sizeof(float), cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
-  return tf_status_from_cuda(e);
+  if (e != cudaSuccess) return tf_status_from_cuda(e);
+  // the results are only as good as the device's own checks: read (and reset)
+  // the error counters, as trackfit_device_errors does
+  int64_t n_bad = 0;
+  return trackfit_device_errors(h, stream, &n_bad);
 }
 
 extern "C" int trackfit_device_errors(trackfit_t h, void* stream, int64_t* n_bad) {

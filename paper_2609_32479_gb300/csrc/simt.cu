@@ -281,17 +281,18 @@ int tf_simt_workspace(trackfit_ctx* h) {
   return tf_status_from_cuda(cudaMalloc(&h->ws, h->ws_bytes));
 }
 
-int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out,
-                    float* out_q, float* out_pool, cudaStream_t st) {
-  const tf_shape& s = h->s;
-  const float* W = h->d_w;
-  const tf_blob_off& o = h->off;
+// The whole SIMT forward over chunks of ws_tracks tracks, with the workspace and
+// the device error counter supplied by the caller.  prof (may be null) is the
+// handle whose timing hook brackets each chunk's kernels.
+int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* ws, int64_t ws_tracks,
+                unsigned long long* err, const float* hits, const int32_t* n_hits, int64_t B, float* out,
+                float* out_q, float* out_pool, cudaStream_t st, trackfit_ctx* prof) {
   const int rnd = s.precision;   // TRACKFIT_FP32 = 0, BF16_PROJ = 1, FP16_PROJ = 2
   const int D = s.D, H = s.H, PD = 4 * s.H + s.D;
-  for (int64_t c0 = 0; c0 < B; c0 += h->ws_tracks) {
-    const int64_t nb = (B - c0 < h->ws_tracks) ? B - c0 : h->ws_tracks;
+  for (int64_t c0 = 0; c0 < B; c0 += ws_tracks) {
+    const int64_t nb = (B - c0 < ws_tracks) ? B - c0 : ws_tracks;
     const int64_t R = nb * s.T;
-    float* EB = h->ws;
+    float* EB = ws;
     float* U = EB + R * s.E;
     float* X = U + R * D;
     float* XH = X + R * D;
@@ -300,7 +301,7 @@ int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, i
     float* X1 = Y + R * 2 * H;
     const float* hc = hits + c0 * s.T * 5;
     const int32_t* nc = n_hits + c0;
-    tf_prof_begin(h, st);
+    if (prof) tf_prof_begin(prof, st);
     int64_t nthreads = R * s.F;
     fourier_kernel<<<(unsigned)((nthreads + 255) / 256), 256, 0, st>>>(hc, R, EB, s);
     GemmArgs g{};
@@ -338,11 +339,17 @@ int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, i
     pool_head_kernel<<<(unsigned)nb, 128, 0, st>>>(X, Y, nc, nb, s, W + o.head_g, W + o.head_w1, W + o.head_b1,
                                                     W + o.head_w2, W + o.head_b2, out + c0 * 5,
                                                     out_q ? out_q + c0 * s.Q : nullptr,
-                                                    out_pool ? out_pool + c0 * s.P : nullptr, h->d_err);
-    tf_prof_end(h, st);
+                                                    out_pool ? out_pool + c0 * s.P : nullptr, err);
+    if (prof) tf_prof_end(prof, st);
     if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
   }
   return TRACKFIT_OK;
+}
+
+int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out,
+                    float* out_q, float* out_pool, cudaStream_t st) {
+  return tf_simt_run(h->s, h->off, h->d_w, h->ws, h->ws_tracks, h->d_err, hits, n_hits, B, out, out_q, out_pool, st,
+                     h);
 }
 
 int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits, int64_t B, int T,
@@ -352,64 +359,12 @@ int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int
   return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
 }
 
-// Same layer sequence as tf_simt_forward, with the workspace and the device
-// error counter supplied by the caller instead of a handle (used by the
-// no-allocation entry point; the handle path above is unchanged).
+// The forward with caller-supplied workspace and error counter (the
+// no-allocation entry point): no quantile or pooled export, no timing hook.
 int tf_simt_forward_explicit(const tf_shape& s, const tf_blob_off& o, const float* W, float* ws, int64_t ws_tracks,
                              unsigned long long* err, const float* hits, const int32_t* n_hits, int64_t B,
                              float* out, cudaStream_t st) {
-  const int rnd = s.precision;
-  const int D = s.D, H = s.H, PD = 4 * s.H + s.D;
-  for (int64_t c0 = 0; c0 < B; c0 += ws_tracks) {
-    const int64_t nb = (B - c0 < ws_tracks) ? B - c0 : ws_tracks;
-    const int64_t R = nb * s.T;
-    float* EB = ws;
-    float* U = EB + R * s.E;
-    float* X = U + R * D;
-    float* XH = X + R * D;
-    float* PR = XH + R * D;
-    float* Y = PR + R * PD;
-    float* X1 = Y + R * 2 * H;
-    const float* hc = hits + c0 * s.T * 5;
-    const int32_t* nc = n_hits + c0;
-    int64_t nthreads = R * s.F;
-    fourier_kernel<<<(unsigned)((nthreads + 255) / 256), 256, 0, st>>>(hc, R, EB, s);
-    GemmArgs g{};
-    g.R = (int)R;
-    g.rnd = rnd;
-    g.n_hits = nc;
-    g.T = s.T;
-    g.H = H;
-    g.A = EB; g.lda = s.E; g.W = W + o.emb_w1; g.bias = W + o.emb_b1; g.C = U; g.ldc = D;
-    g.N = D; g.K = s.E; g.epi = EPI_SILU;
-    if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
-    g.A = U; g.lda = D; g.W = W + o.emb_w2; g.bias = W + o.emb_b2; g.C = X; g.ldc = D;
-    g.N = D; g.K = D; g.epi = EPI_MASK;
-    if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
-    for (int l = 0; l < s.L; ++l) {
-      const tf_layer_off& lo = o.layer[l];
-      rmsnorm_kernel<<<(unsigned)((R + 7) / 8), 256, 0, st>>>(X, R, D, W + lo.g, s.rms_eps, XH);
-      g.A = XH; g.lda = D; g.W = W + lo.w_in; g.bias = W + lo.b_in; g.C = PR; g.ldc = PD;
-      g.N = PD; g.K = D; g.epi = EPI_PROJ;
-      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
-      dim3 sg((H + 127) / 128, (unsigned)nb);
-      mingru_scan_kernel<<<sg, 128, 0, st>>>(PR, PD, nc, nb, s.T, H, Y);
-      if (s.pool == TRACKFIT_POOL_ENDPOINTS && l == s.L - 1) break;
-      g.A = Y; g.lda = 2 * H; g.W = W + lo.w_m; g.bias = W + lo.b_m; g.C = X1; g.ldc = D;
-      g.N = D; g.K = 2 * H; g.epi = EPI_GATE_RES; g.res = X; g.ldr = D; g.gate = PR + 4 * H; g.ldg = PD;
-      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
-      g.A = X1; g.lda = D; g.W = W + lo.w1; g.bias = W + lo.b1; g.C = U; g.ldc = D;
-      g.N = D; g.K = D; g.epi = EPI_SILU;
-      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
-      g.A = U; g.lda = D; g.W = W + lo.w2; g.bias = W + lo.b2; g.C = X; g.ldc = D;
-      g.N = D; g.K = D; g.epi = EPI_RES_MASK; g.res = X1; g.ldr = D;
-      if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
-    }
-    pool_head_kernel<<<(unsigned)nb, 128, 0, st>>>(X, Y, nc, nb, s, W + o.head_g, W + o.head_w1, W + o.head_b1,
-                                                    W + o.head_w2, W + o.head_b2, out + c0 * 5, nullptr, nullptr, err);
-    if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
-  }
-  return TRACKFIT_OK;
+  return tf_simt_run(s, o, W, ws, ws_tracks, err, hits, n_hits, B, out, nullptr, nullptr, st, nullptr);
 }
 
 size_t tf_simt_bytes_per_track(const tf_shape& s) { return ws_floats_per_track(s) * sizeof(float); }

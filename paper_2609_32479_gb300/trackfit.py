@@ -267,6 +267,15 @@ def debug_umma(tf: "Trackfit", A, Bkn, D, stream=None) -> None:
 def forward_noalloc(model: W.ModelConfig, weights, hits, n_hits, out, stream=None) -> None:
     """No-allocation forward: device fp32 weight blob, hits, n_hits and out as
     torch CUDA tensors; the library's static device scratch supplies the workspace."""
+    B = int(n_hits.shape[0])
+    if tuple(n_hits.shape) != (B,):
+        raise ValueError(f"n_hits must be [B], got {tuple(n_hits.shape)}")
+    if tuple(hits.shape) != (B, model.max_hits, model.n_features):
+        raise ValueError(f"hits must be [{B}, {model.max_hits}, {model.n_features}], got {tuple(hits.shape)}")
+    if tuple(out.shape) != (B, 5):
+        raise ValueError(f"out must be [{B}, 5], got {tuple(out.shape)}")
+    if int(weights.numel()) != weight_count(model):
+        raise ValueError(f"weights hold {int(weights.numel())} values, the model needs {weight_count(model)}")
     cfg = make_config(model)
     st = load().trackfit_forward_noalloc(ctypes.byref(cfg), _dev(weights, "torch.float32"),
                                          _dev(hits, "torch.float32"), _dev(n_hits, "torch.int32"),

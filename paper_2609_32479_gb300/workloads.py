@@ -12,7 +12,7 @@ measurement time, 6-20 hits per track, 13 on average (Sec. 3.5).  Those samples
 and the trained weights are not available, so every workload here is seeded
 synthetic helix tracks in a uniform solenoid field, with random-init weights.
 
-Readings (every one also listed in the design doc):
+Readings of the paper's detector and sample description:
   * field B_z = 2 T; helix radius R[mm] = 1000 * pT[GeV] / (0.299792458 * B[T]);
   * 10 barrel layers at radii linspace(33, 1000); tiny/small/sweep barrels are
     unbounded cylinders, medium/large barrels have half-length 600 mm plus 7

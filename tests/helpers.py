@@ -21,6 +21,11 @@ def normalised_errors(got, ref):
     return np.abs(got - ref) / np.maximum(np.abs(ref), rms[None, :])
 
 
+def track_errors(got, ref):
+    """Per track: the largest normalised error over its output columns."""
+    return np.max(normalised_errors(got, ref), axis=1)
+
+
 def parity_error(got, ref):
     """Max over tracks of the normalised error, per output column."""
     return np.max(normalised_errors(got, ref), axis=0)
