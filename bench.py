@@ -204,7 +204,7 @@ def parity_block(w: W.Workload, blob, tb, gpu_out, idx, ref, emul_max_tracks: in
     runs on the first tracks of the sample, giving the spread a correct
     fp32-accumulating implementation shows on the same tracks; the 2e-3 bar on
     every track is reported as its own pass/fail."""
-    from tests.helpers import track_errors
+    from tests.helpers import bf16_bars, track_errors
     e = track_errors(gpu_out[idx], ref)
     out = {"tracks": int(idx.size), "metric": "per track: max over the 5 outputs of |g - r| / max(|r|, column RMS)",
            "p90": float(np.percentile(e, 90)), "p99": float(np.percentile(e, 99)), "max": float(e.max()),
@@ -213,12 +213,16 @@ def parity_block(w: W.Workload, blob, tb, gpu_out, idx, ref, emul_max_tracks: in
         from oracle import fp32_emulation as E
         k = min(emul_max_tracks, idx.size)
         sub = idx[:k]
-        em = E.forward(dataclasses.asdict(w.model), blob, tb.hits[sub], tb.n_hits[sub])
-        e_em = track_errors(em, ref[:k])
+        ems = [E.forward(dataclasses.asdict(w.model), blob, tb.hits[sub], tb.n_hits[sub], order=o) for o in E.ORDERS]
+        e_ems = [track_errors(em, ref[:k]) for em in ems]
         e_g = track_errors(gpu_out[sub], ref[:k])
+        b90, bmx = bf16_bars(ref[:k], ems)
         out["same_tracks_vs_fp32_emulation"] = {
             "tracks": int(k), "gpu_p90": float(np.percentile(e_g, 90)), "gpu_max": float(e_g.max()),
-            "emulation_p90": float(np.percentile(e_em, 90)), "emulation_max": float(e_em.max())}
+            "emulation_p90": [float(np.percentile(x, 90)) for x in e_ems],
+            "emulation_max": [float(x.max()) for x in e_ems], "orders": list(E.ORDERS),
+            "bar_p90": b90, "bar_max": bmx,
+            "gate_ok": bool(np.percentile(e_g, 90) <= b90 and e_g.max() <= bmx)}
     return out
 
 

@@ -43,8 +43,27 @@ def _op(x, prec):
     return x
 
 
-def _lin(x, w, b, prec):
-    return (_op(x, prec) @ _op(w, prec).T + b.astype(F32)).astype(F32)
+# Accumulation order of the fp32 matrix products: "blas" = numpy's float32
+# matmul (the BLAS library's blocking); "k16" = the K axis in consecutive blocks
+# of 16 products, each block summed and added to a running fp32 accumulator (the
+# step of one tensor-core instruction).  Both are correct fp32 evaluations of the
+# same product; their spread against the fp64 oracle is what the tolerance covers.
+ORDERS = ("blas", "k16")
+
+
+def _matmul(a, bt, order):
+    if order == "blas":
+        return (a @ bt).astype(F32)
+    if order == "k16":
+        acc = np.zeros(a.shape[:-1] + (bt.shape[1],), dtype=F32)
+        for k0 in range(0, a.shape[-1], 16):
+            acc = (acc + (a[..., k0:k0 + 16] @ bt[k0:k0 + 16]).astype(F32)).astype(F32)
+        return acc
+    raise ValueError(order)
+
+
+def _lin(x, w, b, prec, order="blas"):
+    return (_matmul(_op(x, prec), _op(w, prec).T, order) + b.astype(F32)).astype(F32)
 
 
 def sigmoid(x):
@@ -74,12 +93,12 @@ def linear_scan(a, b, x, valid, reverse=False):
     return out
 
 
-def encoder_layer(x, W, l, cfg, valid, prec):
+def encoder_layer(x, W, l, cfg, valid, prec, order="blas"):
     """One layer, the oracle's encoder_layer in fp32 (mean-pooling form)."""
     D, H = cfg["d_model"], cfg["d_hidden"]
     p = f"layer{l}."
     xh = rmsnorm(x, W[p + "g"], cfg["rms_eps"])
-    proj = _lin(xh, W[p + "w_in"], W[p + "b_in"], prec)
+    proj = _lin(xh, W[p + "w_in"], W[p + "b_in"], prec, order)
     z_f = sigmoid(proj[..., 0:H])
     n_f = proj[..., H:2 * H]
     z_b = sigmoid(proj[..., 2 * H:3 * H])
@@ -89,14 +108,14 @@ def encoder_layer(x, W, l, cfg, valid, prec):
     h_f = linear_scan((one - z_f).astype(F32), z_f, n_f, valid)
     h_b = linear_scan((one - z_b).astype(F32), z_b, n_b, valid, reverse=True)
     y = np.concatenate([h_f, h_b], axis=-1)
-    m = _lin(y, W[p + "w_m"], W[p + "b_m"], prec)
+    m = _lin(y, W[p + "w_m"], W[p + "b_m"], prec, order)
     x1 = (x + m * gate).astype(F32)
-    u = silu(_lin(x1, W[p + "w1"], W[p + "b1"], prec))
-    x2 = (x1 + _lin(u, W[p + "w2"], W[p + "b2"], prec)).astype(F32)
+    u = silu(_lin(x1, W[p + "w1"], W[p + "b1"], prec, order))
+    x2 = (x1 + _lin(u, W[p + "w2"], W[p + "b2"], prec, order)).astype(F32)
     return np.where(valid[..., None], x2, F32(0.0)), h_f, h_b
 
 
-def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
+def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None, order: str = "blas"):
     """Track parameters [B, 5] (returned as fp64 holding fp32 values) for mean
     pooling; with capture, also the pooled vector after every layer
     (capture["pooled_by_layer"][l], fp64 holding fp32 values)."""
@@ -112,12 +131,12 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
     n_ok = np.where(bad, 1, n_hits)
     valid = np.arange(T)[None, :] < n_ok[:, None]
     e = O.fourier(O.normalise(hits, cfg["feat_min"], cfg["feat_max"]), cfg["fourier_scale"]).astype(F32)
-    hdn = silu(_lin(e, W["emb.w1"], W["emb.b1"], prec))
-    x = np.where(valid[..., None], _lin(hdn, W["emb.w2"], W["emb.b2"], prec), F32(0.0))
+    hdn = silu(_lin(e, W["emb.w1"], W["emb.b1"], prec, order))
+    x = np.where(valid[..., None], _lin(hdn, W["emb.w2"], W["emb.b2"], prec, order), F32(0.0))
     nf = n_ok[:, None].astype(F32)
     by_layer = []
     for l in range(cfg["n_layers"]):
-        x, _, _ = encoder_layer(x, W, l, cfg, valid, prec)
+        x, _, _ = encoder_layer(x, W, l, cfg, valid, prec, order)
         if capture is not None:
             by_layer.append((np.sum(x, axis=1, dtype=F32) / nf).astype(np.float64))
     pv = (np.sum(x, axis=1, dtype=F32) / nf).astype(F32)
@@ -128,5 +147,5 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
     q = q.reshape(B, q.shape[1] // nq, nq)
     out = np.where(bad[:, None], np.nan, q[:, :, nq // 2].astype(np.float64))
     if capture is not None:
-        capture.update(pooled=pv.astype(np.float64), pooled_by_layer=by_layer)
+        capture.update(pooled=pv.astype(np.float64), pooled_by_layer=by_layer, quantiles=q.astype(np.float64))
     return out

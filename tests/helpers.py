@@ -31,20 +31,50 @@ def parity_error(got, ref):
     return np.max(normalised_errors(got, ref), axis=0)
 
 
-FP32_TOL = 1e-5
-BF16_TOL = 2e-3          # bulk bar (90th percentile of tracks) for bf16 operands
-BF16_TAIL_TOL = 1e-2     # every track, bf16 operands (rounding-boundary flips)
-FP16_TOL = 2e-3          # every track, fp16 operands
+FP32_TOL = 1e-5         # every track, fp32 path
+FP16_TOL = 2e-3         # every track, fp16 operands
+# bf16 operands: the bars come from the fp32 emulation of the oracle on the same
+# tracks (oracle/fp32_emulation.py), in both of its accumulation orders.  Per
+# track error e_b = max over the outputs of the normalised error; the GPU's 90th
+# percentile and maximum of e_b may exceed the worse emulation's by these factors
+# (measured spread between correct fp32 evaluations, see the design notes), and
+# never need to be below BF16_FLOOR.
+BF16_P90_FACTOR = 1.3
+BF16_MAX_FACTOR = 1.5
+BF16_FLOOR = 2e-4
+EVERY_TRACK_BAR = 2e-3  # the stated bar for every track, reported beside the gate
 
 
-def parity_ok(got, ref, precision):
-    """The parity gate of one precision; returns (ok, summary string)."""
-    e = normalised_errors(got, ref)
-    mx = e.max()
+def emulations(model, blob, hits, n_hits):
+    """The fp32 emulation of the oracle in each accumulation order (mean pooling)."""
+    from oracle import fp32_emulation as E
+    cfg = dataclasses.asdict(model)
+    return [E.forward(cfg, blob, hits, n_hits, order=o) for o in E.ORDERS]
+
+
+def bf16_bars(ref, emuls):
+    """(p90 bar, max bar) of the per-track error, from emulation outputs on the same tracks."""
+    es = [track_errors(e, ref) for e in emuls]
+    p90 = max(float(np.percentile(e, 90)) for e in es)
+    mx = max(float(e.max()) for e in es)
+    return max(BF16_P90_FACTOR * p90, BF16_FLOOR), max(BF16_MAX_FACTOR * mx, BF16_FLOOR)
+
+
+def parity_ok(got, ref, precision, emul=None):
+    """The parity gate of one precision; returns (ok, summary string).  For bf16
+    operands emul must hold the fp32 emulation's outputs on the same tracks (one
+    array or a list, see emulations())."""
+    e = track_errors(got, ref)
+    mx = float(e.max())
     if precision == 0:
         return bool(mx <= FP32_TOL), f"max {mx:.3e} (tol {FP32_TOL})"
     if precision == 2:
         return bool(mx <= FP16_TOL), f"max {mx:.3e} (tol {FP16_TOL})"
-    p90 = np.percentile(e, 90)
-    return bool(p90 <= BF16_TOL and mx <= BF16_TAIL_TOL), \
-        f"p90 {p90:.3e} (tol {BF16_TOL}), max {mx:.3e} (tol {BF16_TAIL_TOL})"
+    if emul is None:
+        raise ValueError("the bf16 gate needs the fp32 emulation's outputs on the same tracks")
+    emuls = list(emul) if isinstance(emul, (list, tuple)) else [emul]
+    b90, bmx = bf16_bars(ref, emuls)
+    p90 = float(np.percentile(e, 90))
+    return bool(p90 <= b90 and mx <= bmx), \
+        (f"per-track p90 {p90:.3e} (bar {b90:.3e}), max {mx:.3e} (bar {bmx:.3e}); "
+         f"every track within {EVERY_TRACK_BAR}: {'yes' if mx <= EVERY_TRACK_BAR else 'no'}")

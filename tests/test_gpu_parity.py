@@ -7,7 +7,7 @@ import pytest
 
 from oracle import trackfit_oracle as O
 from paper_2609_32479_gb300 import workloads as W
-from tests.helpers import parity_error, parity_ok
+from tests.helpers import emulations, parity_error, parity_ok
 
 pytestmark = pytest.mark.gpu
 
@@ -53,6 +53,14 @@ def oracle(model, blob, hits, n_hits, capture=None):
     return O.forward(dataclasses.asdict(model), blob, hits, n_hits, capture=capture)
 
 
+def emul(model, blob, hits, n_hits):
+    """The fp32 emulation's outputs on the same tracks (the bf16 gate's reference
+    spread); None for the other precisions."""
+    if model.precision != W.PRECISION_BF16:
+        return None
+    return emulations(model, blob, hits, n_hits)
+
+
 CASES = [("tiny", None), ("small", None), ("medium", 1000), ("large", 300), ("sweep8", 515), ("sweep16", 300),
          ("sweep32", 200), ("sweep64", 130)]
 FP16_CASES = [("medium", 1000), ("large", 300), ("sweep8", 515), ("sweep64", 130)]
@@ -68,7 +76,7 @@ def test_parity_against_oracle(T, name, n, path):
     blob = W.gen_weights(w.model, w.weight_seed)
     r = run(T, w.model, blob, tb.hits, tb.n_hits, path=path)
     ref = oracle(w.model, blob, tb.hits, tb.n_hits)
-    ok, msg = parity_ok(r["out"], ref, w.model.precision)
+    ok, msg = parity_ok(r["out"], ref, w.model.precision, emul=emul(w.model, blob, tb.hits, tb.n_hits))
     print(f"{name} [{r['path']}] parity: {msg}; per parameter max {parity_error(r['out'], ref)}")
     assert r["status"] == 0 and r["n_bad"] == 0
     assert np.all(np.isfinite(r["out"]))
@@ -105,7 +113,7 @@ def test_full_size_sampled_parity(T, name):
     idx += [0, w.n_tracks - 1]
     idx = np.array(sorted(set(int(i) for i in idx)))
     ref = oracle(w.model, blob, tb.hits[idx], tb.n_hits[idx])
-    ok, msg = parity_ok(r["out"][idx], ref, w.model.precision)
+    ok, msg = parity_ok(r["out"][idx], ref, w.model.precision, emul=emul(w.model, blob, tb.hits[idx], tb.n_hits[idx]))
     print(f"{name} full batch [{r['path']}], {idx.size} sampled tracks: {msg}")
     assert np.all(np.isfinite(r["out"]))
     assert ok, msg
@@ -156,8 +164,18 @@ def test_quantile_and_pooled_exports(T, name):
     np.testing.assert_array_equal(r["out"], r["q"][:, :, w.model.n_quantiles // 2])
     cap = {}
     oracle(w.model, blob, tb.hits, tb.n_hits, capture=cap)
-    for got, ref in ((r["pooled"], cap["pooled"]), (r["q"].reshape(200, -1), cap["quantiles"].reshape(200, -1))):
-        ok, msg = parity_ok(got, ref, w.model.precision)
+    caps = []
+    if w.model.precision == W.PRECISION_BF16:
+        from oracle import fp32_emulation as E
+        for o in E.ORDERS:
+            c = {}
+            E.forward(dataclasses.asdict(w.model), blob, tb.hits, tb.n_hits, capture=c, order=o)
+            caps.append(c)
+    for key in ("pooled", "quantiles"):
+        got = r["pooled"] if key == "pooled" else r["q"].reshape(200, -1)
+        em = [c[key].reshape(200, -1) for c in caps] or None
+        ok, msg = parity_ok(got, cap[key].reshape(200, -1), w.model.precision, emul=em)
+        print(f"{name} {key}: {msg}")
         assert ok, msg
 
 
