@@ -223,6 +223,70 @@ int trackfit_debug_schedule(const trackfit_config_t* cfg, int64_t* counts, int32
 int trackfit_debug_umma(trackfit_t h, const uint16_t* A, const uint16_t* Bkn, int32_t K, float* D,
                         void* stream);
 
+/* The analytic seed of Sec. 3.1, on the device in fp64 (the paper keeps the seed
+ * in float64 to avoid a cancellation in the beam-line transport at high
+ * momentum).  Per track: the seed triplet (the first hit, then each first later
+ * hit more than 10 mm (3-D) from the previous seed hit: there are no
+ * detector-volume identifiers in these inputs, and the distance keeps two hits
+ * of one surface out of a triplet), the circle through the triplet's transverse
+ * points by the conformal map, its point closest to the beam line, the charge
+ * from the turning direction, theta from the first and third seed hit, and the
+ * perigee (d0, z0, phi0, theta, q/p) with p_T = 0.299792458 B R / 1000 GeV.  Per
+ * hit: the three residual features of Sec. 3.1 against that helix, asinh(du),
+ * asinh(dv) and s_helix, where the foot point is the helix point whose normal
+ * plane holds the hit (Newton's method), du and dv the hit's coordinates there
+ * along U = z x t / |z x t| and V = t x U (the curvilinear frame), s the 3-D
+ * path length from the perigee, lengths in mm (asinh scale 1 mm).
+ *   hits         device [n_tracks][max_hits][5] fp32 (x, y, z first), as trackfit_forward.
+ *   n_hits       device [n_tracks] int32.
+ *   b_field      the solenoid field B_z in tesla (> 0).
+ *   seed_out     device [n_tracks][5] fp64: the seed perigee; a NaN row where a
+ *                track has fewer than three hits so spaced, or n_hits outside
+ *                [0, max_hits].
+ *   features_out device [n_tracks][max_hits][3] fp32 or NULL: the residual
+ *                features, zero on padded hits and on tracks without a seed.
+ * All pointers 16-byte aligned; the caller owns every buffer.  Asynchronous on
+ * `stream`; allocates nothing.  Errors: INVALID_ARG (NULL, n_tracks <= 0,
+ * max_hits outside [1, 64], b_field not > 0, misalignment), CUDA. */
+int trackfit_seed(const float* hits, const int32_t* n_hits, int64_t n_tracks, int32_t max_hits, double b_field,
+                  double* seed_out, float* features_out, void* stream);
+
+/* Decode of the heads' corrections against the seed (Sec. 3.3): d0, z0, theta
+ * additive, phi additive and wrapped to (-pi, pi], q/p from the scale-free
+ * residual r: q/p = q/p_seed + r (|q/p_seed| + 0.02 / GeV).
+ *   seed         device [n_tracks][5] fp64 (trackfit_seed's output).
+ *   corrections  device [n_tracks][5] fp32 (the heads' median outputs).
+ *   out_params   device [n_tracks][5] fp32 (computed in fp64, then rounded).
+ * 16-byte aligned; asynchronous on `stream`; allocates nothing.  Errors:
+ * INVALID_ARG (NULL, n_tracks <= 0, misalignment), CUDA. */
+int trackfit_decode(const double* seed, const float* corrections, int64_t n_tracks, float* out_params,
+                    void* stream);
+
+/* Test hook for the failure path of the fused tensor-core kernel's bounded
+ * waits (every wait for a hand-over inside that kernel gives up after a time
+ * limit, records TRACKFIT_ERR_TIMEOUT in the handle's device error counters,
+ * and the kernel drains its copies and products and returns instead of
+ * hanging).  For this handle's later forwards: limit_ns > 0 replaces the 2 s
+ * limit (0 restores it); hold_tile >= 0 makes the loader warp of the first CTA
+ * hold back its hand-over of the metadata of its hold_tile-th tile for twice the
+ * limit (or until a wait has given up), so that the epilogue's wait for it
+ * expires; -1 holds nothing.  The outputs of a forward that timed out are not
+ * valid; trackfit_device_errors reports TRACKFIT_ERR_TIMEOUT and resets the
+ * counters, after which the handle is usable again.  Host side only; launches
+ * nothing.  Errors: INVALID_ARG (NULL handle, limit_ns < 0, hold_tile < -1),
+ * UNSUPPORTED (the handle runs the CUDA-core path, which has no waits). */
+int trackfit_debug_wait_limit(trackfit_t h, int64_t limit_ns, int32_t hold_tile);
+
+/* Test hook for allocation failures (host side, not thread-safe): every device
+ * allocation the library makes for a handle (trackfit_create, the staging
+ * buffers of trackfit_forward_host) is counted.  fail_nth > 0 makes the
+ * fail_nth-th allocation from now on fail as if the device were out of memory
+ * (the call then returns TRACKFIT_ERR_OOM after freeing what it had allocated);
+ * 0 arms nothing.  Returns the number of device allocations the library holds
+ * now; *attempted (may be NULL) receives the allocations attempted since the
+ * previous call. */
+int64_t trackfit_debug_alloc(int64_t fail_nth, int64_t* attempted);
+
 /* Forward pass that allocates no device memory, for callers that cannot call
  * cudaMalloc (code whose device memory is owned by an outer framework or pool,
  * or that must not let an allocation synchronise the device).  The paper has no

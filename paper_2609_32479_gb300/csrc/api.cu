@@ -14,6 +14,38 @@ int tf_status_from_cuda(cudaError_t e) {
   return TRACKFIT_ERR_CUDA;
 }
 
+// Allocation bookkeeping for the test hook trackfit_debug_alloc (host side; the
+// counters are not meant for concurrent use).
+static int64_t g_live_allocs = 0, g_attempted = 0, g_fail_countdown = 0;
+
+cudaError_t tf_malloc(void** p, size_t bytes) {
+  ++g_attempted;
+  if (g_fail_countdown > 0 && --g_fail_countdown == 0) {
+    *p = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  const cudaError_t e = cudaMalloc(p, bytes);
+  if (e == cudaSuccess) ++g_live_allocs;
+  return e;
+}
+
+void tf_free(void* p) {
+  if (!p) return;
+  if (cudaFree(p) == cudaSuccess) --g_live_allocs;
+}
+
+extern "C" int64_t trackfit_debug_alloc(int64_t fail_nth, int64_t* attempted) {
+  if (attempted) *attempted = g_attempted;
+  g_attempted = 0;
+  g_fail_countdown = fail_nth > 0 ? fail_nth : 0;
+  return g_live_allocs;
+}
+
+extern "C" int trackfit_debug_wait_limit(trackfit_t h, int64_t limit_ns, int32_t hold_tile) {
+  if (!h) return TRACKFIT_ERR_INVALID_ARG;
+  return tf_tc_wait_limit(h, limit_ns, hold_tile);
+}
+
 static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Fill the shape summary and blob offsets; false if cfg is outside the supported set.
@@ -156,12 +188,12 @@ extern "C" void trackfit_destroy(trackfit_t h) {
   if (!h) return;
   if (h->prof_on) trackfit_profile(h, 0);
   tf_tc_destroy(h);
-  cudaFree(h->d_w);
-  cudaFree(h->d_err);
-  cudaFree(h->ws);
-  cudaFree(h->st_hits);
-  cudaFree(h->st_n);
-  cudaFree(h->st_out);
+  tf_free(h->d_w);
+  tf_free(h->d_err);
+  tf_free(h->ws);
+  tf_free(h->st_hits);
+  tf_free(h->st_n);
+  tf_free(h->st_out);
   delete h;
 }
 
@@ -179,9 +211,9 @@ extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weight
   h->s = s;
   h->off = o;
   h->path = TF_PATH_SIMT;
-  int st = tf_status_from_cuda(cudaMalloc(&h->d_w, o.total * sizeof(float)));
+  int st = tf_status_from_cuda(tf_malloc((void**)&h->d_w, o.total * sizeof(float)));
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(h->d_w, weights, o.total * sizeof(float), cudaMemcpyHostToDevice));
-  if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMalloc(&h->d_err, 4 * sizeof(unsigned long long)));
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(tf_malloc((void**)&h->d_err, 4 * sizeof(unsigned long long)));
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemset(h->d_err, 0, 4 * sizeof(unsigned long long)));
   if (st == TRACKFIT_OK) st = tf_simt_workspace(h);
   if (st == TRACKFIT_OK && tf_tc_supported(s)) {
@@ -239,17 +271,25 @@ extern "C" int trackfit_forward_host(trackfit_t h, const float* hits_host, const
   const size_t row = (size_t)h->s.T * 5;
   if (n_tracks > h->st_cap) {
     cudaStreamSynchronize(st);
-    cudaFree(h->st_hits);
-    cudaFree(h->st_n);
-    cudaFree(h->st_out);
+    tf_free(h->st_hits);
+    tf_free(h->st_n);
+    tf_free(h->st_out);
     h->st_hits = nullptr;
     h->st_n = nullptr;
     h->st_out = nullptr;
     h->st_cap = 0;
-    int s1 = tf_status_from_cuda(cudaMalloc(&h->st_hits, n_tracks * row * sizeof(float)));
-    if (s1 == TRACKFIT_OK) s1 = tf_status_from_cuda(cudaMalloc(&h->st_n, ((n_tracks + 3) / 4) * 4 * sizeof(int32_t)));
-    if (s1 == TRACKFIT_OK) s1 = tf_status_from_cuda(cudaMalloc(&h->st_out, n_tracks * 5 * sizeof(float)));
-    if (s1 != TRACKFIT_OK) return s1;
+    int s1 = tf_status_from_cuda(tf_malloc((void**)&h->st_hits, n_tracks * row * sizeof(float)));
+    if (s1 == TRACKFIT_OK) s1 = tf_status_from_cuda(tf_malloc((void**)&h->st_n, ((n_tracks + 3) / 4) * 4 * sizeof(int32_t)));
+    if (s1 == TRACKFIT_OK) s1 = tf_status_from_cuda(tf_malloc((void**)&h->st_out, n_tracks * 5 * sizeof(float)));
+    if (s1 != TRACKFIT_OK) {   // keep nothing of a failed set-up
+      tf_free(h->st_hits);
+      tf_free(h->st_n);
+      tf_free(h->st_out);
+      h->st_hits = nullptr;
+      h->st_n = nullptr;
+      h->st_out = nullptr;
+      return s1;
+    }
     h->st_cap = n_tracks;
   }
   cudaError_t e = cudaMemcpyAsync(h->st_hits, hits_host, n_tracks * row * sizeof(float), cudaMemcpyHostToDevice, st);

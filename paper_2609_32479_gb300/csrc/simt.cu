@@ -278,7 +278,7 @@ int tf_simt_workspace(trackfit_ctx* h) {
   if (n * h->s.T > 65535LL * 64) n = 65535LL * 64 / h->s.T;   // grid.y limit of the GEMM
   h->ws_tracks = n;
   h->ws_bytes = per * (size_t)n;
-  return tf_status_from_cuda(cudaMalloc(&h->ws, h->ws_bytes));
+  return tf_status_from_cuda(tf_malloc((void**)&h->ws, h->ws_bytes));
 }
 
 // The whole SIMT forward over chunks of ws_tracks tracks, with the workspace and

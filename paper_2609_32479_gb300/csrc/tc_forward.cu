@@ -57,7 +57,7 @@ constexpr int MAX_STAGES = 8;
 constexpr int SEG = 1024;                 // tracks per packing segment
 constexpr int64_t MAXB = 4194304;         // tracks per launch chunk
 constexpr int64_t POOL_TRACKS = 1048576;  // tracks per launch chunk when the pooled means go to the internal buffer
-constexpr uint64_t WAIT_NS = 2000000000ull;
+constexpr uint64_t WAIT_NS = 2000000000ull;   // bounded-wait limit (a handle's test hook may lower it)
 constexpr uint64_t DRAIN_NS = 200000000ull;
 constexpr int B_SBO = 2048;               // k-group stride of the MN-major activation operand
 constexpr int B_LBO = 1024;               // 64-hit atom stride
@@ -97,6 +97,8 @@ struct TcParams {
   const float* b_1;
   const float* b_2;
   unsigned long long* err;
+  uint64_t wait_ns;     // limit of every bounded wait
+  int hold_tile;        // test hook: CTA 0's loader holds this tile's metadata hand-over (-1: none)
   int T, D, H, L, NDC, ROWS_IN, NQ, Q, nst;
   uint32_t idesc;
   int off_xb, off_hb, off_a, off_misc;
@@ -144,17 +146,20 @@ __device__ __forceinline__ float rcp_approx(float x) {
 }
 constexpr float LOG2E_F = 1.4426950408889634f;
 __device__ __forceinline__ float silu(float x) { return x * sigm(x); }
-// The output gate and the MLP's SiLU inside the fused kernel use one MUFU
-// operation per value instead of two (ex2 and rcp), from sigma(x) =
-// (1 + tanh(x / 2)) / 2: tanh.approx has a relative error of about 2^-11, below
-// the rounding of the 16-bit operands these values feed.  (The scan gates keep
-// ex2 and rcp: a = 1 - sigma there needs relative accuracy as sigma -> 1.)
+// The MLP's SiLU inside the fused kernel uses one MUFU operation per value
+// instead of two (ex2 and rcp), from SiLU(x) = (x / 2)(1 + tanh(x / 2)):
+// tanh.approx has a relative error of about 2^-11, and the result is rounded
+// to a 16-bit operand right away (measured: no change in the error against the
+// oracle).  The output gate does not: its value scales the merge into the fp32
+// residual stream, where that error showed up on every track, so it takes the
+// two-operation sigmoid, as do the scan gates (a = 1 - sigma there also needs
+// relative accuracy as sigma -> 1).
+__device__ __forceinline__ float sigm_acc(float x) { return rcp_approx(1.0f + ex2_approx(-x * LOG2E_F)); }
 __device__ __forceinline__ float tanh_approx(float x) {
   float y;
   asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-__device__ __forceinline__ float sigm_t(float x) { return fmaf(0.5f, tanh_approx(0.5f * x), 0.5f); }
 __device__ __forceinline__ float silu_t(float x) {
   const float h = 0.5f * x;
   return fmaf(h, tanh_approx(h), h);
@@ -281,9 +286,17 @@ __host__ __device__ inline void walk_tile(const TcParams& p, F&& f) {
             (mt == 0 && kc == 0) ? W_H : W_NONE,
             kc == 1 && (last || mt == MT - 1) ? (last ? C_ACC : C_HB) : C_NONE);
     }
+    // MLP2 goes to the merge columns.  It starts a fresh accumulator: the
+    // residual epilogue adds x' (kept in the fp32 scratch) in fp32 with
+    // round-to-nearest, because the tensor core's fp32 accumulation truncates
+    // and, accumulating onto the large x', would shrink the residual stream by a
+    // few ulps per layer.  In the last layer it still accumulates onto x' (left
+    // there by the gate epilogue): its pooling reads the tile's columns across
+    // warps, which the scratch path does not synchronise.
+    const bool onto = l + 1 == p.L;
     if (MT == 1) {
       dense(MAP_1, l * p.D, 256, false);   // MLP1 -> the z/n columns
-      dense(MAP_2, l * p.D, 0, true);      // MLP2 accumulates onto x'
+      dense(MAP_2, l * p.D, 0, onto);
     } else {
       // d_model 256, pipelined by 128-channel tile: MLP1's first K half (x' of
       // tile 0, XB rows 0-127) starts once the gate epilogue of tile 0 is out,
@@ -302,7 +315,7 @@ __host__ __device__ inline void walk_tile(const TcParams& p, F&& f) {
       for (int kh = 0; kh < 2; ++kh)
         for (int mt = 0; mt < 2; ++mt)
           for (int kc = 2 * kh; kc < 2 * kh + 2; ++kc)
-            f(MAP_2, r1 + mt * 128, kc * 64, 4, mt * 128, kh == 0 ? BSEL_HB : BSEL_XB, kc * 64, true,
+            f(MAP_2, r1 + mt * 128, kc * 64, 4, mt * 128, kh == 0 ? BSEL_HB : BSEL_XB, kc * 64, onto || kc > 0,
               (mt == 0 && kc == 2 * kh) ? W_E : W_NONE, kc == 3 ? C_ACC : C_NONE);
     }
   }
@@ -326,10 +339,17 @@ struct ECtx {
 
 // The two epilogue warps that share a quadrant and a slab hand a recurrence state
 // from the slab's first 32 columns to the second, or back in the reverse
-// direction: barrier 2 + 2q + half, 64 threads, one arrival by the leading warp
-// and one wait by the other per hand-over.
+// direction: barrier 2 + 2q + half, 64 threads, both warps synchronising once
+// per hand-over.  (The leading warp must not merely arrive: a warp that could
+// arrive twice before its partner synchronises would complete a barrier
+// instance on its own and leave the partner's last one unmatched.  In normal
+// operation the state-buffer wait keeps the leader within one hand-over, but
+// after an expired wait every wait fails fast and that bound is gone; with a
+// synchronisation on both sides the two warps pair up whatever the waits do.
+// The partner reaches its side before its own scan, so the leader, which
+// scans first, seldom waits.)
 __device__ __forceinline__ void carry_pass(const ECtx& x) {
-  asm volatile("bar.arrive %0, 64;" ::"r"(2 + 2 * x.q + x.half) : "memory");
+  asm volatile("bar.sync %0, 64;" ::"r"(2 + 2 * x.q + x.half) : "memory");
 }
 __device__ __forceinline__ void carry_wait(const ECtx& x) {
   asm volatile("bar.sync %0, 64;" ::"r"(2 + 2 * x.q + x.half) : "memory");
@@ -371,10 +391,14 @@ __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
     ep_silu_t<FP16, 1>(x, bias);
 }
 
-// X = acc + bias, zero on pad columns (a layer's accumulator already holds x'
-// plus the MLP2 product).  X goes to the per-CTA scratch (read back once, by the
-// next layer's gate epilogue) and the RMS-normalised x_hat to XB (recomputing X
-// from TMEM); the last layer's X is mean-pooled instead (ep_pool).
+// X = acc + bias, zero on pad columns: for the embedding the accumulator holds
+// its second product; for a layer (ADD_XS) it holds the MLP2 product and
+// X = x' + (acc + bias), with x' read from the per-CTA scratch where the gate
+// epilogue left it (xr holds tile 0's, loaded by the caller before its wait).
+// X goes to the scratch (read back once, by the next layer's gate epilogue) and
+// the RMS-normalised x_hat to XB, recomputing X from TMEM (for a layer X is
+// stored into the accumulator columns for that); the last layer's X is
+// mean-pooled instead (ep_pool).
 // Sum of v over the 32 lanes for 16 columns at once: afterwards lane L holds the
 // total of column L & 15 (both halves of the warp hold the same 16 totals).
 __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
@@ -391,9 +415,11 @@ __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
   return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
 }
 
-template <bool FP16, int MT, class W, class S>
+__device__ __forceinline__ void xs_load(const ECtx& x, int mt, float (&xv)[32]);
+
+template <bool FP16, int MT, bool ADD_XS, class W, class S>
 __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
-                                              S&& signal_tile) {
+                                              S&& signal_tile, float (&xr)[32]) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;   // d_model
   const uint32_t vm = x.md->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
@@ -410,7 +436,10 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
   for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
-    if (mt > 0) wait_tile();
+    if (mt > 0) {
+      if (ADD_XS) xs_load(x, mt, xr);
+      wait_tile();
+    }
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
       const int c0 = x.col0 + 16 * hh;
@@ -419,7 +448,8 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
+        const float a = v[i] + bias_v[mt];
+        const float val = ((vm >> (16 * hh + i)) & 1u) ? (ADD_XS ? xr[16 * hh + i] + a : a) : 0.0f;
         v[i] = val;
         sq[16 * hh + i] = fmaf(val, val, sq[16 * hh + i]);
       }
@@ -427,8 +457,10 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
 #pragma unroll
       for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
+      if (ADD_XS) tmem_st16(x.tq + mt * 128 + c0, v);
     }
   }
+  if (ADD_XS) tmem_st_wait();
 #pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
     float h16[16];
@@ -466,7 +498,7 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
+        const float val = ADD_XS ? v[i] : (((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f);
         v[i] = val * g * rv[i];
       }
       store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v);
@@ -475,13 +507,13 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
   }
 }
 
-template <bool FP16, class W, class S>
+template <bool FP16, bool ADD_XS, class W, class S>
 __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
-                                            S&& signal_tile) {
+                                            S&& signal_tile, float (&xr)[32]) {
   if (x.MT == 2)
-    ep_residual_t<FP16, 2>(x, bias, gain, wait_tile, signal_tile);
+    ep_residual_t<FP16, 2, ADD_XS>(x, bias, gain, wait_tile, signal_tile, xr);
   else
-    ep_residual_t<FP16, 1>(x, bias, gain, wait_tile, signal_tile);
+    ep_residual_t<FP16, 1, ADD_XS>(x, bias, gain, wait_tile, signal_tile, xr);
 }
 
 // Masked mean pooling of the last layer's output X = acc + bias.  The warp of
@@ -493,6 +525,9 @@ __device__ __forceinline__ void ep_pool(const ECtx& x, const float* bias) {
   const TcParams& p = *x.p;
   const int mt = x.sub;
   if (mt >= x.MT) return;
+  // after an expired wait the tile's metadata may not have been handed over:
+  // no stores indexed by it
+  if (*reinterpret_cast<volatile int*>(&x.m->abort_flag)) return;
   const int D = p.D, ch = mt * 128 + x.c;
   const float bv = bias[ch];
   const uint8_t* flags = x.md->col_flags;
@@ -517,20 +552,22 @@ __device__ __forceinline__ void ep_pool(const ECtx& x, const float* bias) {
   }
 }
 
-// X of the thread's channel in tile mt and its 32 columns, read back from the
-// scratch; issued before the wait for the gate's inputs so the loads' latency
-// hides behind it.
-__device__ __forceinline__ void gate_x_load(const ECtx& x, int mt, float (&xv)[32]) {
+// The residual stream of the thread's channel in tile mt and its 32 columns
+// (X before the gate epilogue, x' after it), read back from the scratch; issued
+// before the wait for the accumulator it is combined with, so the loads'
+// latency hides behind it.
+__device__ __forceinline__ void xs_load(const ECtx& x, int mt, float (&xv)[32]) {
   const int D = x.p->D;
   const float* xp = x.xs + (size_t)x.col0 * D + mt * 128 + x.c;
 #pragma unroll
   for (int i = 0; i < 32; ++i) xv[i] = xp[(size_t)i * D];
 }
-// x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> TMEM columns
-// 128 mt.. (in place of the merge accumulator; MLP2 accumulates onto it) and XB
-// rows 128 mt + c.
+// x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> XB rows
+// 128 mt + c (the MLP's operand) and, in fp32, the scratch (in place of X, read
+// back by the residual epilogue) or, in the last layer (to_tmem), the merge
+// accumulator's TMEM columns 128 mt.. (MLP2 accumulates onto it there).
 template <bool FP16, int MT>
-__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const float (&xv)[32]) {
+__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const float (&xv)[32], bool to_tmem) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;
   const int ch_g = mt * 128 + x.c;
@@ -544,18 +581,24 @@ __device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const fl
     tmem_ld16(x.tq + 256 + mt * 128 + c0, gv);
     tmem_ld_wait();
 #pragma unroll
-    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm_t(gv[i] + bg), xv[16 * hh + i]);
-    tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
+    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm_acc(gv[i] + bg), xv[16 * hh + i]);
+    if (to_tmem) {
+      tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
+    } else {
+      float* xp = x.xs + (size_t)c0 * D + ch_g;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = mv[i];
+    }
     store_row16<FP16>(x.xb, ch_g, c0, mv);
   }
-  tmem_st_wait();
+  if (to_tmem) tmem_st_wait();
 }
 template <bool FP16>
-__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt, const float (&xv)[32]) {
+__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt, const float (&xv)[32], bool to_tmem) {
   if (x.MT == 2)
-    ep_gate_t<FP16, 2>(x, l, mt, xv);
+    ep_gate_t<FP16, 2>(x, l, mt, xv, to_tmem);
   else
-    ep_gate_t<FP16, 1>(x, l, mt, xv);
+    ep_gate_t<FP16, 1>(x, l, mt, xv, to_tmem);
 }
 
 // Scan chunk of one layer.  The chunk holds 64 channels of both directions:
@@ -825,7 +868,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       for (int i = 0; i < p.n_sched; ++i) {
         const uint32_t e = sched_s[i];
         if (half == 0) {
-          const bool got = mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, WAIT_NS);
+          const bool got = mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort, p.wait_ns);
           if (!__all_sync(0xffffffffu, got)) {
             if (lane == 0) set_abort(m, p.err);
             ok = false;
@@ -875,7 +918,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     const uint32_t* sm_tab = sched_s + MAX_SCHED;
     const uint32_t idesc = p.idesc;
     auto wait_bar = [&](uint32_t bar, uint32_t& ph, bool spin) -> bool {
-      const bool got = spin ? mbar_wait_spin(bar, ph, abort, WAIT_NS) : mbar_wait(bar, ph, abort, WAIT_NS);
+      const bool got = spin ? mbar_wait_spin(bar, ph, abort, p.wait_ns) : mbar_wait(bar, ph, abort, p.wait_ns);
       if (!__all_sync(0xffffffffu, got)) {
         if (lane == 0) set_abort(m, p.err);
         return false;
@@ -1014,7 +1057,7 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     };
     auto signal = [&]() { signal_e(true); };
     auto wait_on = [&](uint32_t bar, uint32_t& ph) {
-      const bool got = mbar_wait(bar, ph, abort, WAIT_NS);   // try_wait: suspends instead of polling
+      const bool got = mbar_wait(bar, ph, abort, p.wait_ns);   // try_wait: suspends instead of polling
       if (!__all_sync(0xffffffffu, got) && x.lane == 0) set_abort(m, p.err);
       ph ^= 1u;
       tc_fence_after();
@@ -1043,8 +1086,9 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       wait_acc();
       ep_silu<FP16>(x, p.b_e1);
       signal();
+      float xr[32];   // the residual stream of one channel tile (x' for a layer's residual)
       wait_acc();
-      ep_residual<FP16>(x, p.b_e2, p.g, wait_acc, signal);   // embedding output X0
+      ep_residual<FP16, false>(x, p.b_e2, p.g, wait_acc, signal, xr);   // embedding output X0
       for (int l = 0; l < p.L; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
           // biases are loaded before the wait so their latency hides behind it
@@ -1065,15 +1109,15 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         // pipelines the next tile's products behind each); with d_model 256 the
         // SiLU of tile 0 goes to HB (MLP1 still reads XB rows 0-127 then)
         const float* b1 = p.b_1 + (size_t)l * p.D;
-        float xg[32];
-        gate_x_load(x, 0, xg);
+        const bool last = l + 1 == p.L;
+        xs_load(x, 0, xr);
         wait_acc();
-        ep_gate<FP16>(x, l, 0, xg);
+        ep_gate<FP16>(x, l, 0, xr, last);
         signal();
         if (x.MT == 2) {
-          gate_x_load(x, 1, xg);
+          xs_load(x, 1, xr);
           wait_acc();
-          ep_gate<FP16>(x, l, 1, xg);
+          ep_gate<FP16>(x, l, 1, xr, last);
           signal();
           wait_acc();
           ep_silu_mt<FP16>(x, b1, 0, 256, x.hb, 0);
@@ -1086,9 +1130,10 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           ep_silu_mt<FP16>(x, b1, 0, 256, x.xb, 0);
           signal();
         }
+        if (!last) xs_load(x, 0, xr);   // x' of channel tile 0, before the wait for MLP2
         wait_acc();
-        if (l + 1 < p.L) {
-          ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, wait_acc, signal);
+        if (!last) {
+          ep_residual<FP16, true>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, wait_acc, signal, xr);
         } else {
           // both output tiles of the last MLP2 have completed, so HB and XB are
           // free: the next tile's Fourier operand goes in and its first product
@@ -1108,12 +1153,21 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
       const int b = i & 1;
       if (i >= 2) {   // buffer b last held the metadata of tile i - 2
-        const bool got = mbar_wait(smem_u32(&m->meta_free[b]), free_ph[b], abort, WAIT_NS);
+        const bool got = mbar_wait(smem_u32(&m->meta_free[b]), free_ph[b], abort, p.wait_ns);
         if (!__all_sync(0xffffffffu, got) && lane == 0) set_abort(m, p.err);
         free_ph[b] ^= 1u;
       }
       load_tile<FP16>(p, m, &m->meta[b], fbuf + b * EB_BYTES, t, n_slabs, lane);
       __threadfence_block();
+      __syncwarp();
+      if (i == p.hold_tile && blockIdx.x == 0) {
+        // test hook: hold this hand-over past the waiters' limit (at most twice
+        // the limit, and no longer once a wait has given up), so that the
+        // epilogue's wait for it expires; the metadata itself is complete
+        const uint64_t t0 = globaltimer();
+        while (!*abort && globaltimer() - t0 < 2 * p.wait_ns) {
+        }
+      }
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&m->meta_full[b]));
     }
@@ -1531,6 +1585,8 @@ struct tf_tc_state {
   uint8_t* fbuf = nullptr;
   float* pool = nullptr;   // pooled means when the caller passes no buffer [POOL_TRACKS][D]
   size_t head_smem = 0;
+  uint64_t wait_ns = WAIT_NS;   // test hook (trackfit_debug_wait_limit)
+  int hold_tile = -1;
   CUtensorMap tm[NMAPS];
 };
 
@@ -1570,6 +1626,14 @@ int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n, uint8_t* co
   return TRACKFIT_OK;
 }
 
+int tf_tc_wait_limit(trackfit_ctx* h, int64_t limit_ns, int hold_tile) {
+  if (!h->tc) return TRACKFIT_ERR_UNSUPPORTED;
+  if (limit_ns < 0 || hold_tile < -1) return TRACKFIT_ERR_INVALID_ARG;
+  h->tc->wait_ns = limit_ns > 0 ? (uint64_t)limit_ns : WAIT_NS;
+  h->tc->hold_tile = hold_tile;
+  return TRACKFIT_OK;
+}
+
 bool tf_tc_supported(const tf_shape& s) {
   return (s.precision == TRACKFIT_BF16_PROJ || s.precision == TRACKFIT_FP16_PROJ) && s.pool == TRACKFIT_POOL_MEAN && (s.D == 128 || s.D == 256) &&
          s.H % 64 == 0 && s.T <= 64 && s.Hh == 128 && s.Q <= 75 && s.F == 5 && s.K == 16;
@@ -1578,12 +1642,12 @@ bool tf_tc_supported(const tf_shape& s) {
 void tf_tc_destroy(trackfit_ctx* h) {
   if (!h || !h->tc) return;
   tf_tc_state* t = h->tc;
-  cudaFree(t->dev);
-  cudaFree(t->seg_count);
-  cudaFree(t->xs);
-  cudaFree(t->fbuf);
-  cudaFree(t->pool);
-  cudaFree(t->sched);
+  tf_free(t->dev);
+  tf_free(t->seg_count);
+  tf_free(t->xs);
+  tf_free(t->fbuf);
+  tf_free(t->pool);
+  tf_free(t->sched);
   delete t;
   h->tc = nullptr;
 }
@@ -1692,7 +1756,7 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   };
   size_t total = 0;
   for (auto& pt : parts) total += (pt.bytes + 255) & ~(size_t)255;
-  if (cudaMalloc(&t->dev, total) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  if (tf_malloc((void**)&t->dev, total) != cudaSuccess) return TRACKFIT_ERR_OOM;
   size_t off = 0;
   for (auto& pt : parts) {
     *pt.dst = static_cast<char*>(t->dev) + off;
@@ -1702,15 +1766,15 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
   // ---- packing buffers and the per-CTA residual scratch
   const int nseg_max = (int)((MAXB + SEG - 1) / SEG);
   const size_t plan_ints = (size_t)nseg_max * 2 + (size_t)nseg_max * (SEG + 1) + (size_t)MAXB + 2 + 64 + (size_t)MAXB;
-  if (cudaMalloc(&t->seg_count, plan_ints * 4) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  if (tf_malloc((void**)&t->seg_count, plan_ints * 4) != cudaSuccess) return TRACKFIT_ERR_OOM;
   t->seg_off = t->seg_count + nseg_max;
   t->seg_slabs = t->seg_off + nseg_max;
   t->slab_start = t->seg_slabs + (size_t)nseg_max * (SEG + 1);
   t->n_slabs = t->slab_start + MAXB + 2;
   t->order = t->n_slabs + 64;
-  if (cudaMalloc(&t->xs, (size_t)t->nsm * TILE * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
-  if (cudaMalloc(&t->fbuf, (size_t)t->nsm * 2 * EB_BYTES) != cudaSuccess) return TRACKFIT_ERR_OOM;
-  if (cudaMalloc(&t->pool, (size_t)POOL_TRACKS * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  if (tf_malloc((void**)&t->xs, (size_t)t->nsm * TILE * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  if (tf_malloc((void**)&t->fbuf, (size_t)t->nsm * 2 * EB_BYTES) != cudaSuccess) return TRACKFIT_ERR_OOM;
+  if (tf_malloc((void**)&t->pool, (size_t)POOL_TRACKS * D * sizeof(float)) != cudaSuccess) return TRACKFIT_ERR_OOM;
   // ---- tensor maps
   bool ok = make_map(&t->tm[MAP_E1], t->w_e1, D, E, fp16) && make_map(&t->tm[MAP_E2], t->w_e2, D, D, fp16) &&
             make_map(&t->tm[MAP_IN], t->w_in, (uint64_t)L * t->ROWS_IN, D, fp16) &&
@@ -1727,7 +1791,7 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
     q.NDC = t->NDC;
     q.ROWS_IN = t->ROWS_IN;
     int* d_count = nullptr;
-    if (cudaMalloc(&t->sched, 2 * MAX_SCHED * sizeof(uint32_t) + 16) != cudaSuccess) return TRACKFIT_ERR_OOM;
+    if (tf_malloc((void**)&t->sched, 2 * MAX_SCHED * sizeof(uint32_t) + 16) != cudaSuccess) return TRACKFIT_ERR_OOM;
     d_count = reinterpret_cast<int*>(t->sched + 2 * MAX_SCHED);
     build_schedule<<<1, 1>>>(q, t->sched, t->sched + MAX_SCHED, d_count);
     if (cudaMemcpy(&t->n_sched, d_count, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return TRACKFIT_ERR_CUDA;
@@ -1766,6 +1830,8 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
   p.b_1 = t->b_1;
   p.b_2 = t->b_2;
   p.err = h->d_err;
+  p.wait_ns = t->wait_ns;
+  p.hold_tile = t->hold_tile;
   p.T = s.T;
   p.D = s.D;
   p.H = s.H;

@@ -78,7 +78,13 @@ void tf_tc_destroy(trackfit_ctx* h);
 int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,
                   float* out, float* out_q, float* out_pool, cudaStream_t st);
 
+int tf_tc_wait_limit(trackfit_ctx* h, int64_t limit_ns, int hold_tile);
 int tf_tc_probe(trackfit_ctx* h, const uint16_t* A, const uint16_t* Bkn, int K, float* D, cudaStream_t st);
 
 // api.cu
 int tf_status_from_cuda(cudaError_t e);
+// Every device allocation of a handle goes through these two (counted; a test
+// hook can make one fail as if the device were out of memory).  tf_free
+// accepts null.
+cudaError_t tf_malloc(void** p, size_t bytes);
+void tf_free(void* p);

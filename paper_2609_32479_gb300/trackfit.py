@@ -25,7 +25,8 @@ EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trac
            "trackfit_forward_host", "trackfit_device_errors", "trackfit_path_name", "trackfit_set_path",
            "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma",
            "trackfit_profile", "trackfit_profile_read", "trackfit_forward_noalloc",
-           "trackfit_debug_schedule")
+           "trackfit_debug_schedule", "trackfit_debug_wait_limit", "trackfit_debug_alloc", "trackfit_seed",
+           "trackfit_decode")
 
 
 class Config(ctypes.Structure):
@@ -89,6 +90,14 @@ def load() -> ctypes.CDLL:
     lib.trackfit_forward_noalloc.restype = ctypes.c_int
     lib.trackfit_debug_schedule.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32, vp, i64]
     lib.trackfit_debug_schedule.restype = ctypes.c_int
+    lib.trackfit_debug_wait_limit.argtypes = [vp, i64, i32]
+    lib.trackfit_debug_wait_limit.restype = ctypes.c_int
+    lib.trackfit_debug_alloc.argtypes = [i64, ctypes.POINTER(i64)]
+    lib.trackfit_debug_alloc.restype = i64
+    lib.trackfit_seed.argtypes = [vp, vp, i64, i32, ctypes.c_double, vp, vp, vp]
+    lib.trackfit_seed.restype = ctypes.c_int
+    lib.trackfit_decode.argtypes = [vp, vp, i64, vp, vp]
+    lib.trackfit_decode.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -227,6 +236,12 @@ class Trackfit:
             raise TrackfitError(st, "trackfit_profile_read")
         return ms.value, n.value
 
+    def debug_wait_limit(self, limit_ns: int, hold_tile: int = -1) -> None:
+        """Test hook: bounded-wait limit of the fused kernel and a held hand-over."""
+        st = self.lib.trackfit_debug_wait_limit(self._h, int(limit_ns), int(hold_tile))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_debug_wait_limit")
+
     def close(self) -> None:
         if getattr(self, "_h", None) is not None and self._h.value:
             self.lib.trackfit_destroy(self._h)
@@ -282,3 +297,37 @@ def forward_noalloc(model: W.ModelConfig, weights, hits, n_hits, out, stream=Non
                                          int(n_hits.shape[0]), _dev(out, "torch.float32"), _stream_handle(stream))
     if st != OK:
         raise TrackfitError(st, "trackfit_forward_noalloc")
+
+
+def debug_alloc(fail_nth: int = 0):
+    """Test hook: (device allocations the library holds, allocations attempted
+    since the previous call); fail_nth > 0 makes that allocation from now fail."""
+    att = ctypes.c_int64(0)
+    live = load().trackfit_debug_alloc(int(fail_nth), ctypes.byref(att))
+    return int(live), int(att.value)
+
+
+def seed(hits, n_hits, b_field: float, seed_out, features_out=None, stream=None) -> None:
+    """Analytic fp64 seed (device tensors): hits [B, T, 5] f32, n_hits [B] i32 ->
+    seed_out [B, 5] f64, features_out [B, T, 3] f32 (optional)."""
+    B, T = int(hits.shape[0]), int(hits.shape[1])
+    if tuple(n_hits.shape) != (B,) or tuple(seed_out.shape) != (B, 5):
+        raise ValueError("seed: n_hits must be [B] and seed_out [B, 5]")
+    if features_out is not None and tuple(features_out.shape) != (B, T, 3):
+        raise ValueError("seed: features_out must be [B, T, 3]")
+    st = load().trackfit_seed(_dev(hits, "torch.float32"), _dev(n_hits, "torch.int32"), B, T, float(b_field),
+                              _dev(seed_out, "torch.float64"), _dev(features_out, "torch.float32"),
+                              _stream_handle(stream))
+    if st != OK:
+        raise TrackfitError(st, "trackfit_seed")
+
+
+def decode(seed_t, corrections, out, stream=None) -> None:
+    """Seed decode (device tensors): seed [B, 5] f64, corrections [B, 5] f32 -> out [B, 5] f32."""
+    B = int(seed_t.shape[0])
+    if tuple(seed_t.shape) != (B, 5) or tuple(corrections.shape) != (B, 5) or tuple(out.shape) != (B, 5):
+        raise ValueError("decode: seed, corrections and out must be [B, 5]")
+    st = load().trackfit_decode(_dev(seed_t, "torch.float64"), _dev(corrections, "torch.float32"), B,
+                                _dev(out, "torch.float32"), _stream_handle(stream))
+    if st != OK:
+        raise TrackfitError(st, "trackfit_decode")
