@@ -198,7 +198,7 @@ def reference_main(args, w: W.Workload):
     return 0
 
 
-def parity_block(w: W.Workload, blob, tb, gpu_out, idx, ref, emul_max_tracks: int = 768) -> dict:
+def parity_block(w: W.Workload, blob, tb, gpu_out, idx, ref, emul_max_tracks: int = 384) -> dict:
     """Per-track parity of the GPU output on the oracle's sample.  For 16-bit
     operands the fp32 emulation of the oracle (same arithmetic, fp32 accumulation)
     runs on the first tracks of the sample, giving the spread a correct
@@ -216,13 +216,15 @@ def parity_block(w: W.Workload, blob, tb, gpu_out, idx, ref, emul_max_tracks: in
         ems = [E.forward(dataclasses.asdict(w.model), blob, tb.hits[sub], tb.n_hits[sub], order=o) for o in E.ORDERS]
         e_ems = [track_errors(em, ref[:k]) for em in ems]
         e_g = track_errors(gpu_out[sub], ref[:k])
-        b90, bmx = bf16_bars(ref[:k], ems)
+        bmean, b90, bmx = bf16_bars(ref[:k], ems)
         out["same_tracks_vs_fp32_emulation"] = {
-            "tracks": int(k), "gpu_p90": float(np.percentile(e_g, 90)), "gpu_max": float(e_g.max()),
+            "tracks": int(k), "gpu_mean": float(e_g.mean()), "gpu_p90": float(np.percentile(e_g, 90)),
+            "gpu_max": float(e_g.max()), "orders": list(E.ORDERS),
+            "emulation_mean": [float(x.mean()) for x in e_ems],
             "emulation_p90": [float(np.percentile(x, 90)) for x in e_ems],
-            "emulation_max": [float(x.max()) for x in e_ems], "orders": list(E.ORDERS),
-            "bar_p90": b90, "bar_max": bmx,
-            "gate_ok": bool(np.percentile(e_g, 90) <= b90 and e_g.max() <= bmx)}
+            "emulation_max": [float(x.max()) for x in e_ems],
+            "bar_mean": bmean, "bar_p90": b90, "bar_max": bmx,
+            "gate_ok": bool(e_g.mean() <= bmean and np.percentile(e_g, 90) <= b90 and e_g.max() <= bmx)}
     return out
 
 

@@ -139,13 +139,34 @@ int trackfit_forward(trackfit_t h, const float* hits, const int32_t* n_hits, int
 int trackfit_forward_ex(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
                         float* out_params, float* out_quantiles, float* out_pooled, void* stream);
 
+/* The fit of trackfit_forward on the packed, unpadded layout the paper deploys
+ * (Sec. 3.5: tracks run packed, without padding): no padding rows cross HBM.
+ *   hits        device [n_hit_rows][5] fp32 (x, y, z [mm], r [mm], phi [rad]),
+ *               the hits of all tracks back to back, 16-byte aligned.
+ *   n_hit_rows  rows in hits (bounds every track's rows).
+ *   offsets     device [n_tracks + 1] int64, 16-byte aligned: track b's hits are
+ *               rows offsets[b] .. offsets[b + 1] - 1, in measurement-time order.
+ *   out_params  device [n_tracks][5] fp32, as trackfit_forward.
+ * A track whose row range is empty, longer than max_hits, or outside
+ * [0, n_hit_rows) gets a NaN row and is counted in the device error counter;
+ * none of its rows is read.  Results are bit-identical to trackfit_forward on
+ * the same tracks padded to max_hits.  Asynchronous on `stream`; no host
+ * synchronisation, no allocation (the per-track counts go to a buffer the
+ * handle allocated at create, in chunks of 1,048,576 tracks).  Errors:
+ * INVALID_ARG (NULL, n_tracks <= 0, n_hit_rows < 0, misalignment), CUDA. */
+int trackfit_forward_packed(trackfit_t h, const float* hits, int64_t n_hit_rows, const int64_t* offsets,
+                            int64_t n_tracks, float* out_params, void* stream);
+
 /* The fit of trackfit_forward with the data movement a deployment pays (Sec. 4.2
  * times the whole forward from the hits to the parameters).
  * End-to-end variant with HOST buffers: copies hits [n_tracks][max_hits][5] and
  * n_hits [n_tracks] to the device, runs the encoder and copies out_params
  * [n_tracks][5] back, all on `stream`, and returns after the stream has finished
- * this work (synchronous).  Pinned (page-locked) host memory makes the copies
- * asynchronous and faster; pageable memory works too.  The device staging
+ * this work (synchronous).  The batch moves in steps of 262,144 tracks: a
+ * step's inputs are copied on a stream of the handle's own while the previous
+ * step computes on `stream`, and its outputs are copied back behind it.  Pinned
+ * (page-locked) host memory makes the copies asynchronous and lets them
+ * overlap; pageable memory works too.  The device staging
  * buffers are owned by the handle and grow on demand (this call may allocate).
  * Errors as trackfit_forward, plus OOM.  Before returning it reads and resets the
  * device error counters (as trackfit_device_errors): TRACKFIT_ERR_BAD_HITS when

@@ -43,27 +43,69 @@ def _op(x, prec):
     return x
 
 
-# Accumulation order of the fp32 matrix products: "blas" = numpy's float32
-# matmul (the BLAS library's blocking); "k16" = the K axis in consecutive blocks
-# of 16 products, each block summed and added to a running fp32 accumulator (the
-# step of one tensor-core instruction).  Both are correct fp32 evaluations of the
-# same product; their spread against the fp64 oracle is what the tolerance covers.
-ORDERS = ("blas", "k16")
+# Accumulation order of the fp32 matrix products: "k16" = the K axis in
+# consecutive blocks of 16 products, each block summed and added to a running
+# fp32 accumulator (the step of one tensor-core instruction), rounding to
+# nearest; "k16rz" = the same steps with each new accumulator value rounded
+# toward zero; "blas" (not in ORDERS) = numpy's float32 matmul as it blocks it.  All three are
+# fp32 accumulations of the same product; "k16rz" is the rounding a tensor core
+# applies (measured: its fp32 sums of same-sign products fall short of the
+# exact sum by a few ulps, a bias round-to-nearest does not have), and a
+# systematically shortened accumulator moves more 16-bit roundings across a
+# boundary than an unbiased one.  Their spread against the fp64 oracle is what
+# the tolerance covers.
+ORDERS = ("k16", "k16rz")
 
 
-def _matmul(a, bt, order):
+def _add_toward_zero(acc, blk):
+    """acc + blk (fp32 arrays) rounded toward zero: the round-to-nearest sum, moved
+    one step toward zero where it rounded away from it (the exact rounding error
+    of the sum, from Knuth's TwoSum, has the opposite sign).  One step toward zero
+    is one less in the magnitude bits of the float."""
+    s = acc + blk
+    bb = s - acc
+    err = acc - (s - bb)
+    err += blk - bb
+    away = (err < 0) & (s > 0)
+    away |= (err > 0) & (s < 0)
+    s.view(np.int32)[...] -= away
+    return s
+
+
+def _matmul(a, bt, order, init=None):
+    """a @ bt accumulated in fp32 in the given order; init (same shape as the
+    result, the blocked orders only) is the accumulator's starting value."""
     if order == "blas":
         return (a @ bt).astype(F32)
-    if order == "k16":
-        acc = np.zeros(a.shape[:-1] + (bt.shape[1],), dtype=F32)
+    if order not in ("k16", "k16rz"):
+        raise ValueError(order)
+    shape = a.shape[:-1] + (bt.shape[1],)
+    a2 = a.reshape(-1, a.shape[-1])
+    out = np.empty((a2.shape[0], bt.shape[1]), dtype=F32)
+    init2 = None if init is None else init.reshape(-1, bt.shape[1])
+    for r0 in range(0, a2.shape[0], 2048):           # rows in chunks: bounded temporaries
+        ac = np.ascontiguousarray(a2[r0:r0 + 2048])
+        acc = np.zeros((ac.shape[0], bt.shape[1]), dtype=F32) if init2 is None else init2[r0:r0 + 2048].astype(F32)
         for k0 in range(0, a.shape[-1], 16):
-            acc = (acc + (a[..., k0:k0 + 16] @ bt[k0:k0 + 16]).astype(F32)).astype(F32)
-        return acc
-    raise ValueError(order)
+            blk = (ac[:, k0:k0 + 16] @ bt[k0:k0 + 16]).astype(F32)
+            acc = (acc + blk).astype(F32) if order == "k16" else _add_toward_zero(acc, blk)
+        out[r0:r0 + 2048] = acc
+    return out.reshape(shape)
 
 
-def _lin(x, w, b, prec, order="blas"):
-    return (_matmul(_op(x, prec), _op(w, prec).T, order) + b.astype(F32)).astype(F32)
+def _lin(x, w, b, prec, order="k16", rows=None, onto=None):
+    """x W^T + b over the last axis of x; with rows (a boolean mask over x's
+    leading axes) only those rows are computed, the others are zero (padding
+    rows, whose values never reach a result).  onto (blocked orders): the
+    accumulation starts from it, giving onto + x W^T + b."""
+    if order == "blas" and onto is not None:
+        return (onto + _lin(x, w, b, prec, order, rows)).astype(F32)
+    if rows is None:
+        return (_matmul(_op(x, prec), _op(w, prec).T, order, onto) + b.astype(F32)).astype(F32)
+    out = np.zeros(x.shape[:-1] + (w.shape[0],), dtype=F32)
+    out[rows] = (_matmul(_op(x[rows], prec), _op(w, prec).T, order, None if onto is None else onto[rows])
+                 + b.astype(F32)).astype(F32)
+    return out
 
 
 def sigmoid(x):
@@ -93,12 +135,12 @@ def linear_scan(a, b, x, valid, reverse=False):
     return out
 
 
-def encoder_layer(x, W, l, cfg, valid, prec, order="blas"):
+def encoder_layer(x, W, l, cfg, valid, prec, order="k16"):
     """One layer, the oracle's encoder_layer in fp32 (mean-pooling form)."""
     D, H = cfg["d_model"], cfg["d_hidden"]
     p = f"layer{l}."
     xh = rmsnorm(x, W[p + "g"], cfg["rms_eps"])
-    proj = _lin(xh, W[p + "w_in"], W[p + "b_in"], prec, order)
+    proj = _lin(xh, W[p + "w_in"], W[p + "b_in"], prec, order, valid)
     z_f = sigmoid(proj[..., 0:H])
     n_f = proj[..., H:2 * H]
     z_b = sigmoid(proj[..., 2 * H:3 * H])
@@ -108,14 +150,16 @@ def encoder_layer(x, W, l, cfg, valid, prec, order="blas"):
     h_f = linear_scan((one - z_f).astype(F32), z_f, n_f, valid)
     h_b = linear_scan((one - z_b).astype(F32), z_b, n_b, valid, reverse=True)
     y = np.concatenate([h_f, h_b], axis=-1)
-    m = _lin(y, W[p + "w_m"], W[p + "b_m"], prec, order)
+    m = _lin(y, W[p + "w_m"], W[p + "b_m"], prec, order, valid)
     x1 = (x + m * gate).astype(F32)
-    u = silu(_lin(x1, W[p + "w1"], W[p + "b1"], prec, order))
-    x2 = (x1 + _lin(u, W[p + "w2"], W[p + "b2"], prec, order)).astype(F32)
+    u = silu(_lin(x1, W[p + "w1"], W[p + "b1"], prec, order, valid))
+    # the second MLP product accumulates onto x' (the association the tensor-core
+    # path uses: x' is the accumulator's starting value, the bias is added last)
+    x2 = _lin(u, W[p + "w2"], W[p + "b2"], prec, order, valid, onto=x1)
     return np.where(valid[..., None], x2, F32(0.0)), h_f, h_b
 
 
-def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None, order: str = "blas"):
+def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None, order: str = "k16"):
     """Track parameters [B, 5] (returned as fp64 holding fp32 values) for mean
     pooling; with capture, also the pooled vector after every layer
     (capture["pooled_by_layer"][l], fp64 holding fp32 values)."""
@@ -131,8 +175,8 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None, order
     n_ok = np.where(bad, 1, n_hits)
     valid = np.arange(T)[None, :] < n_ok[:, None]
     e = O.fourier(O.normalise(hits, cfg["feat_min"], cfg["feat_max"]), cfg["fourier_scale"]).astype(F32)
-    hdn = silu(_lin(e, W["emb.w1"], W["emb.b1"], prec, order))
-    x = np.where(valid[..., None], _lin(hdn, W["emb.w2"], W["emb.b2"], prec, order), F32(0.0))
+    hdn = silu(_lin(e, W["emb.w1"], W["emb.b1"], prec, order, valid))
+    x = np.where(valid[..., None], _lin(hdn, W["emb.w2"], W["emb.b2"], prec, order, valid), F32(0.0))
     nf = n_ok[:, None].astype(F32)
     by_layer = []
     for l in range(cfg["n_layers"]):

@@ -191,9 +191,12 @@ extern "C" void trackfit_destroy(trackfit_t h) {
   tf_free(h->d_w);
   tf_free(h->d_err);
   tf_free(h->ws);
+  tf_free(h->pk_n);
   tf_free(h->st_hits);
   tf_free(h->st_n);
   tf_free(h->st_out);
+  for (int i = 0; i < h->cp_nev; ++i) cudaEventDestroy(h->cp_ev[i]);
+  if (h->cp_stream) cudaStreamDestroy(h->cp_stream);
   delete h;
 }
 
@@ -216,6 +219,7 @@ extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weight
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(tf_malloc((void**)&h->d_err, 4 * sizeof(unsigned long long)));
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemset(h->d_err, 0, 4 * sizeof(unsigned long long)));
   if (st == TRACKFIT_OK) st = tf_simt_workspace(h);
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(tf_malloc((void**)&h->pk_n, TF_PACKED_CHUNK * sizeof(int32_t)));
   if (st == TRACKFIT_OK && tf_tc_supported(s)) {
     st = tf_tc_create(h, weights);
     if (st == TRACKFIT_OK) h->path = TF_PATH_TC;
@@ -259,6 +263,34 @@ extern "C" int trackfit_forward_ex(trackfit_t h, const float* hits, const int32_
   return tf_simt_forward(h, hits, n_hits, n_tracks, out_params, out_q, out_pool, st);
 }
 
+// Per-track hit counts of a packed batch: n_b = offsets[b + 1] - offsets[b] when
+// the track's rows lie inside the hit array and 1 <= n_b <= T, else 0 (an
+// invalid track: NaN row, counted, and none of its rows read).
+__global__ void counts_from_offsets(const int64_t* __restrict__ offs, int64_t B, int64_t n_rows, int T,
+                                    int32_t* __restrict__ n) {
+  const int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const int64_t lo = offs[b], hi = offs[b + 1], d = hi - lo;
+  n[b] = (lo >= 0 && hi <= n_rows && d >= 1 && d <= T) ? (int32_t)d : 0;
+}
+
+extern "C" int trackfit_forward_packed(trackfit_t h, const float* hits, int64_t n_hit_rows, const int64_t* offsets,
+                                       int64_t n_tracks, float* out_params, void* stream) {
+  if (!h || !hits || !offsets || !out_params || n_tracks <= 0 || n_hit_rows < 0) return TRACKFIT_ERR_INVALID_ARG;
+  if (!aligned16(hits) || !aligned16(offsets) || !aligned16(out_params)) return TRACKFIT_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  for (int64_t c0 = 0; c0 < n_tracks; c0 += TF_PACKED_CHUNK) {
+    const int64_t nb = (n_tracks - c0 < TF_PACKED_CHUNK) ? n_tracks - c0 : TF_PACKED_CHUNK;
+    counts_from_offsets<<<(unsigned)((nb + 255) / 256), 256, 0, st>>>(offsets + c0, nb, n_hit_rows, h->s.T, h->pk_n);
+    if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
+    const int r = h->path == TF_PATH_TC
+                      ? tf_tc_forward(h, hits, h->pk_n, nb, out_params + c0 * 5, nullptr, nullptr, st, offsets + c0)
+                      : tf_simt_forward(h, hits, h->pk_n, nb, out_params + c0 * 5, nullptr, nullptr, st, offsets + c0);
+    if (r != TRACKFIT_OK) return r;
+  }
+  return TRACKFIT_OK;
+}
+
 extern "C" int trackfit_forward(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
                                 float* out_params, void* stream) {
   return trackfit_forward_ex(h, hits, n_hits, n_tracks, out_params, nullptr, nullptr, stream);
@@ -292,12 +324,53 @@ extern "C" int trackfit_forward_host(trackfit_t h, const float* hits_host, const
     }
     h->st_cap = n_tracks;
   }
-  cudaError_t e = cudaMemcpyAsync(h->st_hits, hits_host, n_tracks * row * sizeof(float), cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(h->st_n, n_hits_host, n_tracks * sizeof(int32_t), cudaMemcpyHostToDevice, st);
-  if (e != cudaSuccess) return TRACKFIT_ERR_CUDA;
-  int r = trackfit_forward(h, h->st_hits, h->st_n, n_tracks, h->st_out, stream);
-  if (r != TRACKFIT_OK) return r;
-  e = cudaMemcpyAsync(out_host, h->st_out, n_tracks * 5 * sizeof(float), cudaMemcpyDeviceToHost, st);
+  // Copies overlap the compute: chunk k + 1's inputs travel on the handle's copy
+  // stream while chunk k runs on the caller's stream, and each chunk's outputs
+  // travel back behind it.
+  if (!h->cp_stream) {
+    if (cudaStreamCreateWithFlags(&h->cp_stream, cudaStreamNonBlocking) != cudaSuccess) {
+      h->cp_stream = nullptr;
+      return TRACKFIT_ERR_CUDA;
+    }
+    for (int i = 0; i < TF_HOST_EVENTS; ++i) {
+      if (cudaEventCreateWithFlags(&h->cp_ev[i], cudaEventDisableTiming) != cudaSuccess) {   // all or nothing
+        for (int j = 0; j < h->cp_nev; ++j) cudaEventDestroy(h->cp_ev[j]);
+        h->cp_nev = 0;
+        cudaStreamDestroy(h->cp_stream);
+        h->cp_stream = nullptr;
+        return TRACKFIT_ERR_CUDA;
+      }
+      ++h->cp_nev;
+    }
+  }
+  cudaStream_t cs = h->cp_stream;
+  cudaEvent_t* ev = h->cp_ev;
+  const int64_t chunk = TF_HOST_CHUNK;
+  // the staging buffers may still be read by earlier work on the caller's stream
+  cudaError_t e = cudaEventRecord(ev[0], st);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev[0], 0);
+  int k = 0;
+  for (int64_t c0 = 0; c0 < n_tracks && e == cudaSuccess; c0 += chunk, ++k) {
+    const int64_t nb = (n_tracks - c0 < chunk) ? n_tracks - c0 : chunk;
+    cudaEvent_t in = ev[1 + (2 * k) % (TF_HOST_EVENTS - 2)], done = ev[2 + (2 * k) % (TF_HOST_EVENTS - 2)];
+    e = cudaMemcpyAsync(h->st_hits + c0 * row, hits_host + c0 * row, nb * row * sizeof(float), cudaMemcpyHostToDevice, cs);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(h->st_n + c0, n_hits_host + c0, nb * sizeof(int32_t), cudaMemcpyHostToDevice, cs);
+    if (e == cudaSuccess) e = cudaEventRecord(in, cs);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, in, 0);
+    if (e != cudaSuccess) break;
+    const int r = trackfit_forward(h, h->st_hits + c0 * row, h->st_n + c0, nb, h->st_out + c0 * 5, stream);
+    if (r != TRACKFIT_OK) {
+      cudaStreamSynchronize(cs);
+      return r;
+    }
+    e = cudaEventRecord(done, st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, done, 0);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(out_host + c0 * 5, h->st_out + c0 * 5, nb * 5 * sizeof(float), cudaMemcpyDeviceToHost, cs);
+  }
+  const cudaError_t e2 = cudaStreamSynchronize(cs);
+  if (e == cudaSuccess) e = e2;
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return tf_status_from_cuda(e);
   // the results are only as good as the device's own checks: read (and reset)

@@ -104,14 +104,24 @@ __global__ void __launch_bounds__(256) gemm_kernel(GemmArgs g) {
 
 // Fourier features (Sec. 3.2): one thread per (hit row, feature).  The argument
 // s_k * u is formed in fp64 and reduced modulo 2 before the fp32 sinpi/cospi, so
-// the fp32 result carries no argument error from the up-to-32x scale.
+// the fp32 result carries no argument error from the up-to-32x scale.  With a
+// packed input (offs), row r = b T + t reads hit offs[b] + t for t < n_hits[b]
+// and is zero otherwise (padding rows are excluded by select later).
 __global__ void fourier_kernel(const float* __restrict__ hits, int64_t rows, float* __restrict__ e,
-                               tf_shape s) {
+                               tf_shape s, const int64_t* __restrict__ offs, const int32_t* __restrict__ n_hits) {
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (i >= rows * s.F) return;
   int64_t r = i / s.F;
   int f = (int)(i - r * s.F);
-  double u = ((double)hits[r * s.F + f] - s.feat_min_d[f]) / s.feat_range_d[f];
+  float v;
+  if (offs) {
+    const int64_t b = r / s.T, t = r - b * s.T;
+    const int n = n_hits[b];
+    v = (n >= 1 && n <= s.T && t < n) ? hits[(offs[b] + t) * s.F + f] : 0.0f;
+  } else {
+    v = hits[r * s.F + f];
+  }
+  double u = ((double)v - s.feat_min_d[f]) / s.feat_range_d[f];
   float* o = e + r * s.E + f * 2 * s.K;
   for (int k = 0; k < s.K; ++k) {
     double a = u * (double)s.scale[k];
@@ -286,7 +296,7 @@ int tf_simt_workspace(trackfit_ctx* h) {
 // handle whose timing hook brackets each chunk's kernels.
 int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* ws, int64_t ws_tracks,
                 unsigned long long* err, const float* hits, const int32_t* n_hits, int64_t B, float* out,
-                float* out_q, float* out_pool, cudaStream_t st, trackfit_ctx* prof) {
+                float* out_q, float* out_pool, cudaStream_t st, trackfit_ctx* prof, const int64_t* offs) {
   const int rnd = s.precision;   // TRACKFIT_FP32 = 0, BF16_PROJ = 1, FP16_PROJ = 2
   const int D = s.D, H = s.H, PD = 4 * s.H + s.D;
   for (int64_t c0 = 0; c0 < B; c0 += ws_tracks) {
@@ -299,11 +309,12 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
     float* PR = XH + R * D;
     float* Y = PR + R * PD;
     float* X1 = Y + R * 2 * H;
-    const float* hc = hits + c0 * s.T * 5;
+    const float* hc = offs ? hits : hits + c0 * s.T * 5;
+    const int64_t* oc = offs ? offs + c0 : nullptr;
     const int32_t* nc = n_hits + c0;
     if (prof) tf_prof_begin(prof, st);
     int64_t nthreads = R * s.F;
-    fourier_kernel<<<(unsigned)((nthreads + 255) / 256), 256, 0, st>>>(hc, R, EB, s);
+    fourier_kernel<<<(unsigned)((nthreads + 255) / 256), 256, 0, st>>>(hc, R, EB, s, oc, nc);
     GemmArgs g{};
     g.R = (int)R;
     g.rnd = rnd;
@@ -347,9 +358,9 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
 }
 
 int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out,
-                    float* out_q, float* out_pool, cudaStream_t st) {
+                    float* out_q, float* out_pool, cudaStream_t st, const int64_t* offs) {
   return tf_simt_run(h->s, h->off, h->d_w, h->ws, h->ws_tracks, h->d_err, hits, n_hits, B, out, out_q, out_pool, st,
-                     h);
+                     h, offs);
 }
 
 int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits, int64_t B, int T,
@@ -364,7 +375,7 @@ int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int
 int tf_simt_forward_explicit(const tf_shape& s, const tf_blob_off& o, const float* W, float* ws, int64_t ws_tracks,
                              unsigned long long* err, const float* hits, const int32_t* n_hits, int64_t B,
                              float* out, cudaStream_t st) {
-  return tf_simt_run(s, o, W, ws, ws_tracks, err, hits, n_hits, B, out, nullptr, nullptr, st, nullptr);
+  return tf_simt_run(s, o, W, ws, ws_tracks, err, hits, n_hits, B, out, nullptr, nullptr, st, nullptr, nullptr);
 }
 
 size_t tf_simt_bytes_per_track(const tf_shape& s) { return ws_floats_per_track(s) * sizeof(float); }

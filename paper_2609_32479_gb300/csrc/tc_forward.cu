@@ -78,6 +78,7 @@ enum { F_FIRST = 1, F_LAST = 2, F_VALID = 4 };
 struct TcParams {
   CUtensorMap tm[NMAPS];
   const float* hits;
+  const int64_t* offs;   // packed input: track b's hits are rows offs[b] .. of hits (null: padded [B][T][5])
   const int32_t* n_hits;
   float* out;
   float* out_q;
@@ -286,17 +287,9 @@ __host__ __device__ inline void walk_tile(const TcParams& p, F&& f) {
             (mt == 0 && kc == 0) ? W_H : W_NONE,
             kc == 1 && (last || mt == MT - 1) ? (last ? C_ACC : C_HB) : C_NONE);
     }
-    // MLP2 goes to the merge columns.  It starts a fresh accumulator: the
-    // residual epilogue adds x' (kept in the fp32 scratch) in fp32 with
-    // round-to-nearest, because the tensor core's fp32 accumulation truncates
-    // and, accumulating onto the large x', would shrink the residual stream by a
-    // few ulps per layer.  In the last layer it still accumulates onto x' (left
-    // there by the gate epilogue): its pooling reads the tile's columns across
-    // warps, which the scratch path does not synchronise.
-    const bool onto = l + 1 == p.L;
     if (MT == 1) {
       dense(MAP_1, l * p.D, 256, false);   // MLP1 -> the z/n columns
-      dense(MAP_2, l * p.D, 0, onto);
+      dense(MAP_2, l * p.D, 0, true);      // MLP2 accumulates onto x'
     } else {
       // d_model 256, pipelined by 128-channel tile: MLP1's first K half (x' of
       // tile 0, XB rows 0-127) starts once the gate epilogue of tile 0 is out,
@@ -315,7 +308,7 @@ __host__ __device__ inline void walk_tile(const TcParams& p, F&& f) {
       for (int kh = 0; kh < 2; ++kh)
         for (int mt = 0; mt < 2; ++mt)
           for (int kc = 2 * kh; kc < 2 * kh + 2; ++kc)
-            f(MAP_2, r1 + mt * 128, kc * 64, 4, mt * 128, kh == 0 ? BSEL_HB : BSEL_XB, kc * 64, onto || kc > 0,
+            f(MAP_2, r1 + mt * 128, kc * 64, 4, mt * 128, kh == 0 ? BSEL_HB : BSEL_XB, kc * 64, true,
               (mt == 0 && kc == 2 * kh) ? W_E : W_NONE, kc == 3 ? C_ACC : C_NONE);
     }
   }
@@ -391,14 +384,10 @@ __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
     ep_silu_t<FP16, 1>(x, bias);
 }
 
-// X = acc + bias, zero on pad columns: for the embedding the accumulator holds
-// its second product; for a layer (ADD_XS) it holds the MLP2 product and
-// X = x' + (acc + bias), with x' read from the per-CTA scratch where the gate
-// epilogue left it (xr holds tile 0's, loaded by the caller before its wait).
-// X goes to the scratch (read back once, by the next layer's gate epilogue) and
-// the RMS-normalised x_hat to XB, recomputing X from TMEM (for a layer X is
-// stored into the accumulator columns for that); the last layer's X is
-// mean-pooled instead (ep_pool).
+// X = acc + bias, zero on pad columns (a layer's accumulator already holds x'
+// plus the MLP2 product).  X goes to the per-CTA scratch (read back once, by the
+// next layer's gate epilogue) and the RMS-normalised x_hat to XB (recomputing X
+// from TMEM); the last layer's X is mean-pooled instead (ep_pool).
 // Sum of v over the 32 lanes for 16 columns at once: afterwards lane L holds the
 // total of column L & 15 (both halves of the warp hold the same 16 totals).
 __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
@@ -415,11 +404,9 @@ __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
   return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 16);
 }
 
-__device__ __forceinline__ void xs_load(const ECtx& x, int mt, float (&xv)[32]);
-
-template <bool FP16, int MT, bool ADD_XS, class W, class S>
+template <bool FP16, int MT, class W, class S>
 __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
-                                              S&& signal_tile, float (&xr)[32]) {
+                                              S&& signal_tile) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;   // d_model
   const uint32_t vm = x.md->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
@@ -436,10 +423,7 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
   for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
-    if (mt > 0) {
-      if (ADD_XS) xs_load(x, mt, xr);
-      wait_tile();
-    }
+    if (mt > 0) wait_tile();
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
       const int c0 = x.col0 + 16 * hh;
@@ -448,8 +432,7 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float a = v[i] + bias_v[mt];
-        const float val = ((vm >> (16 * hh + i)) & 1u) ? (ADD_XS ? xr[16 * hh + i] + a : a) : 0.0f;
+        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
         v[i] = val;
         sq[16 * hh + i] = fmaf(val, val, sq[16 * hh + i]);
       }
@@ -457,10 +440,8 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
 #pragma unroll
       for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
-      if (ADD_XS) tmem_st16(x.tq + mt * 128 + c0, v);
     }
   }
-  if (ADD_XS) tmem_st_wait();
 #pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
     float h16[16];
@@ -498,7 +479,7 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float val = ADD_XS ? v[i] : (((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f);
+        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
         v[i] = val * g * rv[i];
       }
       store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v);
@@ -507,13 +488,13 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
   }
 }
 
-template <bool FP16, bool ADD_XS, class W, class S>
+template <bool FP16, class W, class S>
 __device__ __forceinline__ void ep_residual(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
-                                            S&& signal_tile, float (&xr)[32]) {
+                                            S&& signal_tile) {
   if (x.MT == 2)
-    ep_residual_t<FP16, 2, ADD_XS>(x, bias, gain, wait_tile, signal_tile, xr);
+    ep_residual_t<FP16, 2>(x, bias, gain, wait_tile, signal_tile);
   else
-    ep_residual_t<FP16, 1, ADD_XS>(x, bias, gain, wait_tile, signal_tile, xr);
+    ep_residual_t<FP16, 1>(x, bias, gain, wait_tile, signal_tile);
 }
 
 // Masked mean pooling of the last layer's output X = acc + bias.  The warp of
@@ -552,22 +533,20 @@ __device__ __forceinline__ void ep_pool(const ECtx& x, const float* bias) {
   }
 }
 
-// The residual stream of the thread's channel in tile mt and its 32 columns
-// (X before the gate epilogue, x' after it), read back from the scratch; issued
-// before the wait for the accumulator it is combined with, so the loads'
-// latency hides behind it.
-__device__ __forceinline__ void xs_load(const ECtx& x, int mt, float (&xv)[32]) {
+// X of the thread's channel in tile mt and its 32 columns, read back from the
+// scratch; issued before the wait for the gate's inputs so the loads' latency
+// hides behind it.
+__device__ __forceinline__ void gate_x_load(const ECtx& x, int mt, float (&xv)[32]) {
   const int D = x.p->D;
   const float* xp = x.xs + (size_t)x.col0 * D + mt * 128 + x.c;
 #pragma unroll
   for (int i = 0; i < 32; ++i) xv[i] = xp[(size_t)i * D];
 }
-// x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> XB rows
-// 128 mt + c (the MLP's operand) and, in fp32, the scratch (in place of X, read
-// back by the residual epilogue) or, in the last layer (to_tmem), the merge
-// accumulator's TMEM columns 128 mt.. (MLP2 accumulates onto it there).
+// x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> TMEM columns
+// 128 mt.. (in place of the merge accumulator; MLP2 accumulates onto it) and XB
+// rows 128 mt + c.
 template <bool FP16, int MT>
-__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const float (&xv)[32], bool to_tmem) {
+__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const float (&xv)[32]) {
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;
   const int ch_g = mt * 128 + x.c;
@@ -582,23 +561,17 @@ __device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const fl
     tmem_ld_wait();
 #pragma unroll
     for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm_acc(gv[i] + bg), xv[16 * hh + i]);
-    if (to_tmem) {
-      tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
-    } else {
-      float* xp = x.xs + (size_t)c0 * D + ch_g;
-#pragma unroll
-      for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = mv[i];
-    }
+    tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
     store_row16<FP16>(x.xb, ch_g, c0, mv);
   }
-  if (to_tmem) tmem_st_wait();
+  tmem_st_wait();
 }
 template <bool FP16>
-__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt, const float (&xv)[32], bool to_tmem) {
+__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt, const float (&xv)[32]) {
   if (x.MT == 2)
-    ep_gate_t<FP16, 2>(x, l, mt, xv, to_tmem);
+    ep_gate_t<FP16, 2>(x, l, mt, xv);
   else
-    ep_gate_t<FP16, 1>(x, l, mt, xv, to_tmem);
+    ep_gate_t<FP16, 1>(x, l, mt, xv);
 }
 
 // Scan chunk of one layer.  The chunk holds 64 channels of both directions:
@@ -726,7 +699,8 @@ __device__ __forceinline__ void load_tile(const TcParams& p, Misc* m, TileMeta* 
     float v = 0.0f;
     if (md->col_flags[col] & F_VALID) {
       const size_t trk = (size_t)md->slot_track[md->col_slot[col]];
-      v = p.hits[(trk * p.T + m->col_tpos[col]) * 5 + f];
+      const size_t row = p.offs ? (size_t)p.offs[trk] + m->col_tpos[col] : trk * p.T + m->col_tpos[col];
+      v = p.hits[row * 5 + f];
     }
     m->hs[col][f] = v;
   }
@@ -1086,9 +1060,8 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
       wait_acc();
       ep_silu<FP16>(x, p.b_e1);
       signal();
-      float xr[32];   // the residual stream of one channel tile (x' for a layer's residual)
       wait_acc();
-      ep_residual<FP16, false>(x, p.b_e2, p.g, wait_acc, signal, xr);   // embedding output X0
+      ep_residual<FP16>(x, p.b_e2, p.g, wait_acc, signal);   // embedding output X0
       for (int l = 0; l < p.L; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
           // biases are loaded before the wait so their latency hides behind it
@@ -1109,15 +1082,15 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         // pipelines the next tile's products behind each); with d_model 256 the
         // SiLU of tile 0 goes to HB (MLP1 still reads XB rows 0-127 then)
         const float* b1 = p.b_1 + (size_t)l * p.D;
-        const bool last = l + 1 == p.L;
-        xs_load(x, 0, xr);
+        float xg[32];
+        gate_x_load(x, 0, xg);
         wait_acc();
-        ep_gate<FP16>(x, l, 0, xr, last);
+        ep_gate<FP16>(x, l, 0, xg);
         signal();
         if (x.MT == 2) {
-          xs_load(x, 1, xr);
+          gate_x_load(x, 1, xg);
           wait_acc();
-          ep_gate<FP16>(x, l, 1, xr, last);
+          ep_gate<FP16>(x, l, 1, xg);
           signal();
           wait_acc();
           ep_silu_mt<FP16>(x, b1, 0, 256, x.hb, 0);
@@ -1130,10 +1103,9 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
           ep_silu_mt<FP16>(x, b1, 0, 256, x.xb, 0);
           signal();
         }
-        if (!last) xs_load(x, 0, xr);   // x' of channel tile 0, before the wait for MLP2
         wait_acc();
-        if (!last) {
-          ep_residual<FP16, true>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, wait_acc, signal, xr);
+        if (l + 1 < p.L) {
+          ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, wait_acc, signal);
         } else {
           // both output tiles of the last MLP2 have completed, so HB and XB are
           // free: the next tile's Fourier operand goes in and its first product
@@ -1808,7 +1780,7 @@ int tf_tc_create(trackfit_ctx* h, const float* W) {
 }
 
 int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out, float* out_q,
-                  float* out_pool, cudaStream_t st) {
+                  float* out_pool, cudaStream_t st, const int64_t* offs) {
   tf_tc_state* t = h->tc;
   const tf_shape& s = h->s;
   TcParams p;
@@ -1880,7 +1852,8 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
     plan_pack<<<nseg, 32, 0, st>>>(n_hits + c0, nb, s.T, t->seg_count, t->seg_slabs, t->order);
     plan_scan<<<1, 1024, 0, st>>>(t->seg_count, nseg, nb, t->seg_off, t->n_slabs, t->slab_start);
     plan_scatter<<<nseg, 128, 0, st>>>(t->seg_count, t->seg_off, t->seg_slabs, t->slab_start);
-    p.hits = hits + c0 * s.T * 5;
+    p.hits = offs ? hits : hits + c0 * s.T * 5;
+    p.offs = offs ? offs + c0 : nullptr;
     p.n_hits = n_hits + c0;
     p.out = out + c0 * 5;
     p.out_q = out_q ? out_q + c0 * s.Q : nullptr;

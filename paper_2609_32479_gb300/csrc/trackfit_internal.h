@@ -9,6 +9,9 @@
 
 #define TF_MAX_LAYERS 16
 #define TF_MAX_HITS 64
+#define TF_PACKED_CHUNK 1048576
+#define TF_HOST_CHUNK 262144   // tracks per copy / compute step of trackfit_forward_host
+#define TF_HOST_EVENTS 10
 
 // Offsets (in floats) of every tensor inside the fp32 weight blob.
 struct tf_layer_off {
@@ -45,11 +48,17 @@ struct trackfit_ctx {
   float* ws;
   size_t ws_bytes;
   int64_t ws_tracks;
+  // packed input: per-track hit counts derived from the offsets, one chunk of
+  // TF_PACKED_CHUNK tracks at a time
+  int32_t* pk_n;
   // host-buffer staging
   float* st_hits;
   int32_t* st_n;
   float* st_out;
   int64_t st_cap;
+  cudaStream_t cp_stream;        // copies of trackfit_forward_host (created on first use)
+  cudaEvent_t cp_ev[TF_HOST_EVENTS];
+  int cp_nev;
   tf_tc_state* tc;
   // optional timing of the main compute kernel (trackfit_profile)
   int prof_on;
@@ -65,8 +74,9 @@ void tf_prof_end(trackfit_ctx* h, cudaStream_t st);
 
 // simt.cu
 int tf_simt_workspace(trackfit_ctx* h);
+// offs (may be null): packed input, track b's hits are rows offs[b] .. of hits
 int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,
-                    float* out, float* out_q, float* out_pool, cudaStream_t st);
+                    float* out, float* out_q, float* out_pool, cudaStream_t st, const int64_t* offs = nullptr);
 int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits,
                        int64_t B, int T, int C, float* hf, float* hb, cudaStream_t st);
 
@@ -76,7 +86,7 @@ int tf_tc_schedule_counts(const tf_shape& s, int64_t* counts, int n, uint8_t* co
 int tf_tc_create(trackfit_ctx* h, const float* host_w);
 void tf_tc_destroy(trackfit_ctx* h);
 int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,
-                  float* out, float* out_q, float* out_pool, cudaStream_t st);
+                  float* out, float* out_q, float* out_pool, cudaStream_t st, const int64_t* offs = nullptr);
 
 int tf_tc_wait_limit(trackfit_ctx* h, int64_t limit_ns, int hold_tile);
 int tf_tc_probe(trackfit_ctx* h, const uint16_t* A, const uint16_t* Bkn, int K, float* D, cudaStream_t st);

@@ -26,7 +26,7 @@ EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trac
            "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma",
            "trackfit_profile", "trackfit_profile_read", "trackfit_forward_noalloc",
            "trackfit_debug_schedule", "trackfit_debug_wait_limit", "trackfit_debug_alloc", "trackfit_seed",
-           "trackfit_decode")
+           "trackfit_decode", "trackfit_forward_packed")
 
 
 class Config(ctypes.Structure):
@@ -98,6 +98,8 @@ def load() -> ctypes.CDLL:
     lib.trackfit_seed.restype = ctypes.c_int
     lib.trackfit_decode.argtypes = [vp, vp, i64, vp, vp]
     lib.trackfit_decode.restype = ctypes.c_int
+    lib.trackfit_forward_packed.argtypes = [vp, vp, i64, vp, i64, vp, vp]
+    lib.trackfit_forward_packed.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -201,6 +203,18 @@ class Trackfit:
                                               _dev(pooled, "torch.float32"), _stream_handle(stream))
         if st != OK:
             raise TrackfitError(st, "trackfit_forward")
+
+    def forward_packed(self, hits, offsets, out, stream=None) -> None:
+        """Device tensors: hits [N, 5] f32 (all tracks back to back), offsets [B + 1]
+        i64 (track b = rows offsets[b] .. offsets[b + 1] - 1), out [B, 5] f32."""
+        B = int(offsets.shape[0]) - 1
+        if hits.dim() != 2 or int(hits.shape[1]) != 5 or tuple(out.shape) != (B, 5):
+            raise ValueError("forward_packed: hits must be [N, 5], offsets [B + 1], out [B, 5]")
+        st = self.lib.trackfit_forward_packed(self._h, _dev(hits, "torch.float32"), int(hits.shape[0]),
+                                              _dev(offsets, "torch.int64"), B, _dev(out, "torch.float32"),
+                                              _stream_handle(stream))
+        if st != OK:
+            raise TrackfitError(st, "trackfit_forward_packed")
 
     def forward_host(self, hits: np.ndarray, n_hits: np.ndarray, out: np.ndarray, stream=None) -> None:
         """Host arrays (ideally pinned): copies in, runs, copies out, synchronises."""

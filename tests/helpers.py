@@ -34,14 +34,19 @@ def parity_error(got, ref):
 FP32_TOL = 1e-5         # every track, fp32 path
 FP16_TOL = 2e-3         # every track, fp16 operands
 # bf16 operands: the bars come from the fp32 emulation of the oracle on the same
-# tracks (oracle/fp32_emulation.py), in both of its accumulation orders.  Per
-# track error e_b = max over the outputs of the normalised error; the GPU's 90th
-# percentile and maximum of e_b may exceed the worse emulation's by these factors
-# (measured spread between correct fp32 evaluations, see the design notes), and
-# never need to be below BF16_FLOOR.
-BF16_P90_FACTOR = 1.3
-BF16_MAX_FACTOR = 1.5
-BF16_FLOOR = 2e-4
+# tracks (oracle/fp32_emulation.py), in each of its accumulation orders: steps
+# of 16 products rounding to nearest, or toward zero as the tensor core does,
+# the second MLP product accumulating onto x' as on the tensor-core path.  Per
+# track error e_b = max over the outputs of the normalised error.  The gate
+# holds the mean and the 90th percentile of e_b within BF16_BULK_FACTOR of the
+# worse emulation's (the measured spread between correct fp32 evaluations of
+# the same arithmetic, see the design notes) and the maximum within
+# BF16_MAX_FACTOR (the maximum of a few hundred tracks is an extreme value that
+# scatters by tens of percent between two correct evaluations; the bar catches
+# a wrong track, whose error is of order one).  No bar need be below BF16_FLOOR.
+BF16_BULK_FACTOR = 1.3
+BF16_MAX_FACTOR = 2.0
+BF16_FLOOR = 1e-4
 EVERY_TRACK_BAR = 2e-3  # the stated bar for every track, reported beside the gate
 
 
@@ -53,11 +58,14 @@ def emulations(model, blob, hits, n_hits):
 
 
 def bf16_bars(ref, emuls):
-    """(p90 bar, max bar) of the per-track error, from emulation outputs on the same tracks."""
+    """(mean bar, p90 bar, max bar) of the per-track error, from emulation outputs
+    on the same tracks."""
     es = [track_errors(e, ref) for e in emuls]
+    mean = max(float(e.mean()) for e in es)
     p90 = max(float(np.percentile(e, 90)) for e in es)
     mx = max(float(e.max()) for e in es)
-    return max(BF16_P90_FACTOR * p90, BF16_FLOOR), max(BF16_MAX_FACTOR * mx, BF16_FLOOR)
+    return (max(BF16_BULK_FACTOR * mean, BF16_FLOOR), max(BF16_BULK_FACTOR * p90, BF16_FLOOR),
+            max(BF16_MAX_FACTOR * mx, BF16_FLOOR))
 
 
 def parity_ok(got, ref, precision, emul=None):
@@ -73,8 +81,8 @@ def parity_ok(got, ref, precision, emul=None):
     if emul is None:
         raise ValueError("the bf16 gate needs the fp32 emulation's outputs on the same tracks")
     emuls = list(emul) if isinstance(emul, (list, tuple)) else [emul]
-    b90, bmx = bf16_bars(ref, emuls)
-    p90 = float(np.percentile(e, 90))
-    return bool(p90 <= b90 and mx <= bmx), \
-        (f"per-track p90 {p90:.3e} (bar {b90:.3e}), max {mx:.3e} (bar {bmx:.3e}); "
-         f"every track within {EVERY_TRACK_BAR}: {'yes' if mx <= EVERY_TRACK_BAR else 'no'}")
+    bmean, b90, bmx = bf16_bars(ref, emuls)
+    mean, p90 = float(e.mean()), float(np.percentile(e, 90))
+    return bool(mean <= bmean and p90 <= b90 and mx <= bmx), \
+        (f"per-track mean {mean:.3e} (bar {bmean:.3e}), p90 {p90:.3e} (bar {b90:.3e}), "
+         f"max {mx:.3e} (bar {bmx:.3e}); every track within {EVERY_TRACK_BAR}: {'yes' if mx <= EVERY_TRACK_BAR else 'no'}")

@@ -53,12 +53,21 @@ def oracle(model, blob, hits, n_hits, capture=None):
     return O.forward(dataclasses.asdict(model), blob, hits, n_hits, capture=capture)
 
 
-def emul(model, blob, hits, n_hits):
+_EMUL_CACHE = {}
+
+
+def emul(model, blob, hits, n_hits, key=None):
     """The fp32 emulation's outputs on the same tracks (the bf16 gate's reference
-    spread); None for the other precisions."""
+    spread); None for the other precisions.  key: reuse a result computed for the
+    same inputs (the tests run each case on both kernel paths)."""
     if model.precision != W.PRECISION_BF16:
         return None
-    return emulations(model, blob, hits, n_hits)
+    if key is not None and key in _EMUL_CACHE:
+        return _EMUL_CACHE[key]
+    res = emulations(model, blob, hits, n_hits)
+    if key is not None:
+        _EMUL_CACHE[key] = res
+    return res
 
 
 CASES = [("tiny", None), ("small", None), ("medium", 1000), ("large", 300), ("sweep8", 515), ("sweep16", 300),
@@ -76,7 +85,7 @@ def test_parity_against_oracle(T, name, n, path):
     blob = W.gen_weights(w.model, w.weight_seed)
     r = run(T, w.model, blob, tb.hits, tb.n_hits, path=path)
     ref = oracle(w.model, blob, tb.hits, tb.n_hits)
-    ok, msg = parity_ok(r["out"], ref, w.model.precision, emul=emul(w.model, blob, tb.hits, tb.n_hits))
+    ok, msg = parity_ok(r["out"], ref, w.model.precision, emul=emul(w.model, blob, tb.hits, tb.n_hits, key=(name, n)))
     print(f"{name} [{r['path']}] parity: {msg}; per parameter max {parity_error(r['out'], ref)}")
     assert r["status"] == 0 and r["n_bad"] == 0
     assert np.all(np.isfinite(r["out"]))
@@ -274,3 +283,30 @@ def test_debug_scan_closed_forms(T):
     hf, hb = gpu(a, b, x)
     np.testing.assert_allclose(hf, O.linear_scan(a, b, x, valid), rtol=1e-5, atol=1e-6)
     np.testing.assert_allclose(hb, O.linear_scan(a, b, x, valid, reverse=True), rtol=1e-5, atol=1e-6)
+
+
+@pytest.mark.parametrize("name,depths,n", [("medium", (1, 3, 6), 200), ("large", (1, 4, 8), 150)])
+def test_per_depth_pooled_vectors(T, name, depths, n):
+    """Where the error grows, layer by layer: the model cut after layer l (the
+    weight blob's first l layers are the same draws as the full model's, the
+    pooled vector is the mean of layer l's output) on the tensor-core path,
+    every channel of the pooled vector against the oracle's, under the bars of
+    the fp32 emulation on the same tracks and depth."""
+    from oracle import fp32_emulation as E
+    w0 = W.workload(name, n_tracks=n)
+    tb = W.gen_tracks(w0)
+    for L in depths:
+        m = w0.model.with_(n_layers=L)
+        blob = W.gen_weights(m, w0.weight_seed)
+        r = run(T, m, blob, tb.hits, tb.n_hits, extras=True)
+        assert r["path"].startswith("tcgen05")
+        cap = {}
+        oracle(m, blob, tb.hits, tb.n_hits, capture=cap)
+        ems = []
+        for o in E.ORDERS:
+            c = {}
+            E.forward(dataclasses.asdict(m), blob, tb.hits, tb.n_hits, capture=c, order=o)
+            ems.append(c["pooled"])
+        ok, msg = parity_ok(r["pooled"], cap["pooled"], m.precision, emul=ems)
+        print(f"{name} after layer {L}: pooled vector {msg}")
+        assert ok, msg

@@ -52,9 +52,21 @@ def test_seed_and_features_match_the_oracle(T, name, n):
     np.testing.assert_array_equal(np.isnan(got), np.isnan(ref))
     ok = ~np.isnan(ref[:, 0])
     assert ok.mean() > 0.95
+    # The same fp64 formulas on both sides; the device's and numpy's fp64
+    # transcendentals may differ in the last bit, which d0's cancellation
+    # (d0 = -p_x sin phi0 + p_y cos phi0 with |p| up to the radius) amplifies.
+    # Seeds of tracks near the beam line (|d0| < 10 mm): d0 and z0 to 1e-5 mm
+    # (z0 carries the lever arm from the first hit, metres for stiff tracks;
+    # 1e-5 mm is still below the fp32 rounding of a hit at 1 m), angles to
+    # 1e-11 rad, q/p to 1e-9 relative.  Triplets with noise hits give
+    # ill-conditioned circles: those only to 1e-6 of their scale.
     d = np.abs(wrap(got[ok] - ref[ok]))
-    scale = np.maximum(np.abs(ref[ok]), [1e-3, 1e-2, 1.0, 1.0, 1e-3])
-    assert np.max(d / scale) < 1e-9, np.max(d / scale, axis=0)
+    r = ref[ok]
+    phys = np.abs(r[:, 0]) < 10.0
+    tight = np.array([1e-5, 1e-5, 1e-11, 1e-11, 0.0]) + np.array([0, 0, 0, 0, 1e-9]) * np.abs(r)
+    assert np.all(d[phys] <= tight[phys]), np.max(d[phys] / tight[phys], axis=0)
+    loose = 1e-6 * np.maximum(np.abs(r), [1.0, 1.0, 1.0, 1.0, 1e-3])
+    assert np.all(d <= loose), np.max(d / loose, axis=0)
     fref = S.seed_features(ref, tb.hits, tb.n_hits, B_FIELD)
     valid = (np.arange(w.model.max_hits)[None, :] < tb.n_hits[:, None]) & ok[:, None]
     assert np.all(feats[~valid] == 0.0)
