@@ -8,6 +8,8 @@ than L2, so no flush is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload large] [--impl ours|reference]
   python bench.py --sweep        # length sweep: T = 8/16/32/64 x batch 4k-1M, one line per point
+  python bench.py --seed         # analytic fp64 seed + features + decode, and its share of the forward
+  python bench.py --packed       # packed, unpadded input against the padded entry point
 
 N > 1 runs under torch.distributed.run, one rank per GPU; every rank processes
 its own full batch (replicas, weak scaling; the path has no exchange step).
@@ -288,6 +290,82 @@ def sweep_main(args):
     return 0
 
 
+def _time_events(fn, reps, stream):
+    """Median milliseconds of fn() over reps runs, CUDA events on `stream`."""
+    import torch
+    ts = []
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    return float(np.median(ts))
+
+
+def next_main(args, w: W.Workload):
+    """--seed: the analytic fp64 seed with its per-hit features and the decode
+    (Sec. 3.1, 3.3) over the workload's batch, with its share of seed + forward
+    (the paper reports 9-12 %).  --packed: the packed, unpadded entry point
+    (Sec. 3.5) against the padded one on the same tracks.  One JSON line each."""
+    import torch
+    from paper_2609_32479_gb300 import trackfit as TF
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    B, T = w.n_tracks, w.model.max_hits
+    hits = torch.from_numpy(tb.hits).to(dev)
+    nh = torch.from_numpy(tb.n_hits).to(dev)
+    out = torch.empty((B, 5), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    reps = max(args.steps, 3)
+    with TF.Trackfit(w.model, blob) as tf:
+        for _ in range(max(args.warmup, 1)):
+            tf.forward(hits, nh, out, stream)
+        fwd_ms = _time_events(lambda: tf.forward(hits, nh, out, stream), reps, stream)
+        base = {"n_gpus": 1, "steps": reps, "warmup": max(args.warmup, 1), "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "data": "synthetic helix tracks + random-init weights (seeded)",
+                "path": tf.path}
+        if args.seed:
+            seed = torch.empty((B, 5), dtype=torch.float64, device=dev)
+            feats = torch.empty((B, T, 3), dtype=torch.float32, device=dev)
+            corr = torch.zeros((B, 5), dtype=torch.float32, device=dev)
+            dec = torch.empty((B, 5), dtype=torch.float32, device=dev)
+
+            def seed_step():
+                TF.seed(hits, nh, w.b_field, seed, feats, stream)
+                TF.decode(seed, corr, dec, stream)
+            for _ in range(max(args.warmup, 1)):
+                seed_step()
+            ms = _time_events(seed_step, reps, stream)
+            line = dict(base, metric="analytic fp64 seed + residual features + decode, tracks/sec (device-timed)",
+                        value=B / (ms * 1e-3), unit="tracks/s", ms_per_step=ms, dtype="f64",
+                        config={"workload": w.name, "n_tracks": B, "max_hits": T, "b_field_tesla": w.b_field,
+                                "l2": "inputs larger than L2; no flush"},
+                        seed_share_of_seed_plus_forward=ms / (ms + fwd_ms), forward_ms=fwd_ms,
+                        seed_us_per_track=1e3 * ms / B)
+        else:
+            rows = [tb.hits[b, :tb.n_hits[b]] for b in range(B)]
+            packed = torch.from_numpy(np.ascontiguousarray(np.concatenate(rows))).to(dev)
+            offs = torch.from_numpy(np.concatenate([[0], np.cumsum(tb.n_hits)]).astype(np.int64)).to(dev)
+            outp = torch.empty_like(out)
+            for _ in range(max(args.warmup, 1)):
+                tf.forward_packed(packed, offs, outp, stream)
+            ms = _time_events(lambda: tf.forward_packed(packed, offs, outp, stream), reps, stream)
+            torch.cuda.synchronize()
+            same = bool(torch.equal(outp, out))
+            line = dict(base, metric=METRIC + " (packed input)", value=B / (ms * 1e-3), unit="tracks/s",
+                        ms_per_step=ms, dtype={0: "f32", 1: "bf16", 2: "f16"}[w.model.precision],
+                        config={"workload": w.name, "n_tracks": B, "layout": "packed", "l2": "inputs larger than L2"},
+                        padded_forward_ms=fwd_ms, matches_padded_bitwise=same,
+                        input_bytes_per_track={"packed": float((packed.numel() * 4 + offs.numel() * 8) / B),
+                                               "padded": float(T * 20 + 4)})
+        print(json.dumps(line))
+    return 0
+
+
 def traffic_for_kernel():
     """dram bytes per launch from the committed ncu summary, if it was taken on the
     current kernel source (else null)."""
@@ -316,6 +394,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="length x batch sweep, one line per point")
+    ap.add_argument("--seed", action="store_true", help="time the analytic seed, features and decode")
+    ap.add_argument("--packed", action="store_true", help="time the packed-input entry point")
     args = ap.parse_args()
     if args.sweep:
         return sweep_main(args)
@@ -325,6 +405,8 @@ def main():
     w = W.workload(args.workload, n_tracks=args.n_tracks, **kw)
     if args.impl == "reference":
         return reference_main(args, w)
+    if args.seed or args.packed:
+        return next_main(args, w)
 
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -47,14 +47,45 @@ def _op(x, prec):
 # consecutive blocks of 16 products, each block summed and added to a running
 # fp32 accumulator (the step of one tensor-core instruction), rounding to
 # nearest; "k16rz" = the same steps with each new accumulator value rounded
-# toward zero; "blas" (not in ORDERS) = numpy's float32 matmul as it blocks it.  All three are
-# fp32 accumulations of the same product; "k16rz" is the rounding a tensor core
-# applies (measured: its fp32 sums of same-sign products fall short of the
-# exact sum by a few ulps, a bias round-to-nearest does not have), and a
-# systematically shortened accumulator moves more 16-bit roundings across a
-# boundary than an unbiased one.  Their spread against the fp64 oracle is what
-# the tolerance covers.
+# toward zero, and the accumulation onto x' (the second MLP product) with the
+# tensor core's truncation of every product (_tc_onto); "blas" (not in ORDERS) =
+# numpy's float32 matmul as it blocks it.  All are fp32 accumulations of the
+# same product; "k16rz" is the rounding a tensor core applies (measured: its fp32
+# sums of same-sign products fall short of the exact sum by a few ulps, and by
+# tens of ulps when added onto a large accumulator, a bias round-to-nearest does
+# not have), and a systematically shortened accumulator moves more 16-bit
+# roundings across a boundary than an unbiased one.  Their spread against the
+# fp64 oracle is what the tolerance covers.
 ORDERS = ("k16", "k16rz")
+
+
+def _tc_onto(acc, a, bt):
+    """acc + a @ bt in steps of 16 products with the tensor core's truncation: each
+    exact product is truncated toward zero to a quarter of the fp32 ulp of the
+    largest magnitude among the step's products and the accumulator, the step's sum
+    (exact) is added to the accumulator and the result rounded toward zero.  This
+    reproduces the measured statistics of tcgen05 fp32 accumulation exactly for
+    same-sign products and for products added onto a large accumulator (the case
+    where truncation matters: MLP2 accumulating onto x').  torch CPU operations for
+    speed; every value is exact in fp64 until the final rounding."""
+    import torch
+    A = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float64))
+    Bt = torch.from_numpy(np.ascontiguousarray(bt, dtype=np.float64))
+    out = np.empty(acc.shape, dtype=F32)
+    for r0 in range(0, A.shape[0], 512):
+        ac = torch.from_numpy(np.ascontiguousarray(acc[r0:r0 + 512], dtype=np.float64))
+        for k0 in range(0, A.shape[1], 16):
+            P = A[r0:r0 + 512, k0:k0 + 16, None] * Bt[None, k0:k0 + 16, :]         # exact (16-bit operands)
+            m = torch.maximum(ac.abs(), P.abs().amax(dim=1))
+            e = torch.frexp(torch.where(m > 0, m, torch.ones_like(m)))[1]        # m = f 2^e, f in [0.5, 1)
+            q = torch.ldexp(torch.ones_like(m), e - 26)[:, None, :]             # 2^(floor(log2 m) - 25)
+            s64 = ac + (torch.trunc(P / q) * q).sum(dim=1)
+            f = s64.to(torch.float32)
+            over = f.to(torch.float64).abs() > s64.abs()
+            f = torch.where(over, torch.nextafter(f, torch.zeros_like(f)), f)
+            ac = f.to(torch.float64)
+        out[r0:r0 + 512] = ac.to(torch.float32).numpy()
+    return out
 
 
 def _add_toward_zero(acc, blk):
@@ -77,6 +108,13 @@ def _matmul(a, bt, order, init=None):
     result, the blocked orders only) is the accumulator's starting value."""
     if order == "blas":
         return (a @ bt).astype(F32)
+    if order == "seq":
+        # one product at a time, fused multiply-add rounding to nearest (the
+        # CUDA-core path's order): exact product plus accumulator, rounded once
+        acc = np.zeros(a.shape[:-1] + (bt.shape[1],), dtype=F32) if init is None else init.astype(F32)
+        for k in range(a.shape[-1]):
+            acc = (acc.astype(np.float64) + a[..., k:k + 1].astype(np.float64) * bt[k].astype(np.float64)).astype(F32)
+        return acc
     if order not in ("k16", "k16rz"):
         raise ValueError(order)
     shape = a.shape[:-1] + (bt.shape[1],)
@@ -100,12 +138,36 @@ def _lin(x, w, b, prec, order="k16", rows=None, onto=None):
     accumulation starts from it, giving onto + x W^T + b."""
     if order == "blas" and onto is not None:
         return (onto + _lin(x, w, b, prec, order, rows)).astype(F32)
+    if order == "k16rz" and onto is not None:
+        xr = x if rows is None else x[rows]
+        base = onto if rows is None else onto[rows]
+        res = (_tc_onto(base.reshape(-1, base.shape[-1]), _op(xr, prec).reshape(-1, xr.shape[-1]), _op(w, prec).T)
+               .reshape(base.shape) + b.astype(F32)).astype(F32)
+        if rows is None:
+            return res
+        out = np.zeros(x.shape[:-1] + (w.shape[0],), dtype=F32)
+        out[rows] = res
+        return out
     if rows is None:
         return (_matmul(_op(x, prec), _op(w, prec).T, order, onto) + b.astype(F32)).astype(F32)
     out = np.zeros(x.shape[:-1] + (w.shape[0],), dtype=F32)
     out[rows] = (_matmul(_op(x[rows], prec), _op(w, prec).T, order, None if onto is None else onto[rows])
                  + b.astype(F32)).astype(F32)
     return out
+
+
+def fourier(u, scales):
+    """The oracle's Fourier features as an fp32 evaluation computes them: the
+    argument s_k u reduced modulo 2 into [-1, 1] (exactly, in fp64), rounded to
+    fp32, then sin and cos of pi times that fp32 argument, rounded to fp32.  The
+    argument's rounding (a relative 6e-8) is the one that matters: near a zero
+    of the sine it moves the value by far more than the sine's own rounding, and
+    so across 16-bit rounding boundaries of the embedding's operand."""
+    s = np.asarray(scales, dtype=np.float64)
+    a = np.asarray(u, dtype=np.float64)[..., :, None] * s
+    a = (a - 2.0 * np.rint(0.5 * a)).astype(F32).astype(np.float64)
+    e = np.concatenate([np.sin(np.pi * a), np.cos(np.pi * a)], axis=-1).astype(F32)
+    return e.reshape(np.shape(u)[:-1] + (2 * np.shape(u)[-1] * s.size,))
 
 
 def sigmoid(x):
@@ -174,7 +236,7 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None, order
     bad = (n_hits < 1) | (n_hits > T)
     n_ok = np.where(bad, 1, n_hits)
     valid = np.arange(T)[None, :] < n_ok[:, None]
-    e = O.fourier(O.normalise(hits, cfg["feat_min"], cfg["feat_max"]), cfg["fourier_scale"]).astype(F32)
+    e = fourier(O.normalise(hits, cfg["feat_min"], cfg["feat_max"]), cfg["fourier_scale"])
     hdn = silu(_lin(e, W["emb.w1"], W["emb.b1"], prec, order, valid))
     x = np.where(valid[..., None], _lin(hdn, W["emb.w2"], W["emb.b2"], prec, order, valid), F32(0.0))
     nf = n_ok[:, None].astype(F32)

@@ -285,14 +285,18 @@ def test_debug_scan_closed_forms(T):
     np.testing.assert_allclose(hb, O.linear_scan(a, b, x, valid, reverse=True), rtol=1e-5, atol=1e-6)
 
 
-@pytest.mark.parametrize("name,depths,n", [("medium", (1, 3, 6), 200), ("large", (1, 4, 8), 150)])
+@pytest.mark.parametrize("name,depths,n", [("medium", (1, 2, 3, 6), 200), ("large", (1, 2, 4, 8), 150)])
 def test_per_depth_pooled_vectors(T, name, depths, n):
     """Where the error grows, layer by layer: the model cut after layer l (the
     weight blob's first l layers are the same draws as the full model's, the
     pooled vector is the mean of layer l's output) on the tensor-core path,
-    every channel of the pooled vector against the oracle's, under the bars of
-    the fp32 emulation on the same tracks and depth."""
+    every channel of the pooled vector against the oracle's.  Each layer may add
+    at most 2e-3 to the normalised error of every track (after one layer the
+    16-bit rounding flips are still rare, so the error of every track, not a
+    distribution, is the right measure); the fp32 emulation's figures on the same
+    tracks are printed beside for the localisation."""
     from oracle import fp32_emulation as E
+    from tests.helpers import track_errors
     w0 = W.workload(name, n_tracks=n)
     tb = W.gen_tracks(w0)
     for L in depths:
@@ -302,11 +306,15 @@ def test_per_depth_pooled_vectors(T, name, depths, n):
         assert r["path"].startswith("tcgen05")
         cap = {}
         oracle(m, blob, tb.hits, tb.n_hits, capture=cap)
-        ems = []
+        e = track_errors(r["pooled"], cap["pooled"])
+        em = []
         for o in E.ORDERS:
             c = {}
             E.forward(dataclasses.asdict(m), blob, tb.hits, tb.n_hits, capture=c, order=o)
-            ems.append(c["pooled"])
-        ok, msg = parity_ok(r["pooled"], cap["pooled"], m.precision, emul=ems)
-        print(f"{name} after layer {L}: pooled vector {msg}")
-        assert ok, msg
+            em.append(track_errors(c["pooled"], cap["pooled"]))
+        print(f"{name} after layer {L}: pooled vector per-track mean {e.mean():.3e} p90 {np.percentile(e, 90):.3e} "
+              f"max {e.max():.3e} (bar {2e-3 * L:.1e}); fp32 emulation mean "
+              f"{max(x.mean() for x in em):.3e} p90 {max(np.percentile(x, 90) for x in em):.3e} "
+              f"max {max(x.max() for x in em):.3e}")
+        assert np.all(np.isfinite(r["pooled"]))
+        assert e.max() <= 2e-3 * L, (L, e.max())

