@@ -43,8 +43,8 @@
 extern "C" {
 #endif
 
-#define TRACKFIT_ABI_VERSION 1
-#define TRACKFIT_MAX_FEATURES 5
+#define TRACKFIT_ABI_VERSION 2
+#define TRACKFIT_MAX_FEATURES 16
 #define TRACKFIT_MAX_FOURIER 16
 
 typedef enum {
@@ -59,13 +59,25 @@ typedef enum {
 
 typedef enum { TRACKFIT_FP32 = 0, TRACKFIT_BF16_PROJ = 1, TRACKFIT_FP16_PROJ = 2 } trackfit_precision;
 typedef enum { TRACKFIT_POOL_MEAN = 0, TRACKFIT_POOL_ENDPOINTS = 1 } trackfit_pool;
+/* Layer topology.  MERGE: each layer pre-norms its input, projects it to the
+ * gates, candidates and an output gate, scans, merges the two directions with
+ * the output gate and an MLP into a d_model-wide residual stream (the form given
+ * with the task).  CONCAT: the paper's own (Sec. 3.2): each layer projects its
+ * input to the forward and reverse gates and candidates, scans, and the two
+ * directions' states, concatenated (2 d_hidden wide), are the next layer's input
+ * and the readout's; no norm inside the encoder. */
+typedef enum { TRACKFIT_TOPOLOGY_MERGE = 0, TRACKFIT_TOPOLOGY_CONCAT = 1 } trackfit_topology;
 
-/* Encoder shape.  Supported: abi_version = 1, n_features = 5 (x, y, z [mm], r [mm],
- * phi [rad]), n_fourier = 16, 1 <= max_hits <= 64, d_model in {16, 32, ..., 256}
- * (multiple of 16), d_hidden = 3 * d_model / 2, 1 <= n_layers <= 16,
- * head_hidden = 128, n_quantiles = 7 (odd).  feat_min/feat_max are fixed min-max
- * constants (feat_max > feat_min); fourier_scale[k] = s_k, the feature argument
- * is pi * s_k * u; rms_eps > 0. */
+/* Encoder shape.  Supported: abi_version = 2, 1 <= n_features <= 16 per hit (the
+ * task's configs use 5: x, y, z [mm], r [mm], phi [rad]; the paper's model 15, its
+ * last three the seed features of trackfit_seed), n_fourier = 16, 1 <= max_hits
+ * <= 64, d_model in {16, 32, ..., 256} (multiple of 16), d_hidden = 3 * d_model / 2,
+ * 1 <= n_layers <= 16, head_hidden = 128, n_quantiles odd <= 15, topology MERGE or
+ * CONCAT.  feat_min/feat_max (first n_features entries) are fixed min-max
+ * constants (feat_max > feat_min); fourier_scale[k] = s_k, the feature argument is
+ * pi * s_k * u; rms_eps > 0.  The tensor-core path runs 16-bit-operand MERGE
+ * configs with 5 features, mean pooling and d_model 128 or 256; everything else
+ * runs on the CUDA cores. */
 typedef struct {
   int32_t abi_version;
   int32_t max_hits;
@@ -78,6 +90,7 @@ typedef struct {
   int32_t n_quantiles;
   int32_t precision;  /* trackfit_precision */
   int32_t pool;       /* trackfit_pool */
+  int32_t topology;   /* trackfit_topology */
   float feat_min[TRACKFIT_MAX_FEATURES];
   float feat_max[TRACKFIT_MAX_FEATURES];
   float fourier_scale[TRACKFIT_MAX_FOURIER];
@@ -90,11 +103,14 @@ typedef struct trackfit_ctx* trackfit_t;
  * Number of fp32 values in the weight blob for cfg (0 if cfg is NULL or
  * unsupported).  Blob order, every matrix in PyTorch [out][in] row-major order,
  * with D = d_model, H = d_hidden, E = 2 * n_features * n_fourier,
- * P = D (mean pooling) or 2H (endpoints), Hh = head_hidden, Q = 5 * n_quantiles:
+ * P = D (MERGE with mean pooling) or 2H (endpoints, or CONCAT), Hh = head_hidden,
+ * Q = 5 * n_quantiles:
  *   W_e1[D][E] b_e1[D] W_e2[D][D] b_e2[D]
- *   per layer: g[D] W_in[4H+D][D] b_in[4H+D] (row blocks z_f, n_f, z_b, n_b, gate)
+ *   MERGE, per layer: g[D] W_in[4H+D][D] b_in[4H+D] (row blocks z_f, n_f, z_b, n_b, gate)
  *              W_m[D][2H] (columns: forward states, then reverse) b_m[D]
  *              W_1[D][D] b_1[D] W_2[D][D] b_2[D]
+ *   CONCAT, per layer l: W_in[4H][I_l] b_in[4H] (row blocks z_f, n_f, z_b, n_b), I_0 = D,
+ *              I_l = 2H after (columns: forward states, then reverse)
  *   g_h[P] W_h1[Hh][P] b_h1[Hh] W_h2[Q][Hh] b_h2[Q]   (Q rows parameter-major: [5][7]) */
 size_t trackfit_weight_count(const trackfit_config_t* cfg);
 
@@ -258,19 +274,27 @@ int trackfit_debug_umma(trackfit_t h, const uint16_t* A, const uint16_t* Bkn, in
  * plane holds the hit (Newton's method), du and dv the hit's coordinates there
  * along U = z x t / |z x t| and V = t x U (the curvilinear frame), s the 3-D
  * path length from the perigee, lengths in mm (asinh scale 1 mm).
- *   hits         device [n_tracks][max_hits][5] fp32 (x, y, z first), as trackfit_forward.
+ *   hits         device [n_tracks][max_hits][hit_stride] fp32, x, y, z [mm] first.
+ *   hit_stride   floats per hit row (>= 3; 5 for the task's inputs, 15 for the paper's).
  *   n_hits       device [n_tracks] int32.
  *   b_field      the solenoid field B_z in tesla (> 0).
  *   seed_out     device [n_tracks][5] fp64: the seed perigee; a NaN row where a
  *                track has fewer than three hits so spaced, or n_hits outside
  *                [0, max_hits].
- *   features_out device [n_tracks][max_hits][3] fp32 or NULL: the residual
- *                features, zero on padded hits and on tracks without a seed.
+ *   features_out device fp32 or NULL: hit t of track b gets its three residual
+ *                features at features_out[(b max_hits + t) feat_stride + 0..2],
+ *                zero on padded hits and on tracks without a seed (feat_stride 3:
+ *                an array [n_tracks][max_hits][3]; feat_stride = hit_stride with
+ *                features_out pointing at column 12 of the hit array: the last
+ *                three of the paper's 15 encoder features, written in place).
+ *   feat_stride  >= 3.
  * All pointers 16-byte aligned; the caller owns every buffer.  Asynchronous on
  * `stream`; allocates nothing.  Errors: INVALID_ARG (NULL, n_tracks <= 0,
- * max_hits outside [1, 64], b_field not > 0, misalignment), CUDA. */
-int trackfit_seed(const float* hits, const int32_t* n_hits, int64_t n_tracks, int32_t max_hits, double b_field,
-                  double* seed_out, float* features_out, void* stream);
+ * max_hits outside [1, 64], hit_stride or feat_stride below 3, b_field not > 0,
+ * misalignment), CUDA. */
+int trackfit_seed(const float* hits, int32_t hit_stride, const int32_t* n_hits, int64_t n_tracks,
+                  int32_t max_hits, double b_field, double* seed_out, float* features_out,
+                  int32_t feat_stride, void* stream);
 
 /* Decode of the heads' corrections against the seed (Sec. 3.3): d0, z0, theta
  * additive, phi additive and wrapped to (-pi, pi], q/p from the scale-free

@@ -30,7 +30,8 @@ from typing import Dict, Optional
 import numpy as np
 
 __all__ = ["bf16_round", "fp16_round", "sigmoid", "silu", "rmsnorm", "normalise", "fourier", "linear_scan",
-           "mingru_layer_scans", "embed", "encoder_layer", "pool", "head", "forward", "split_blob"]
+           "mingru_layer_scans", "embed", "encoder_layer", "encoder_layer_concat", "pool", "head", "forward",
+           "split_blob"]
 
 
 # ---------------------------------------------------------------------------
@@ -197,6 +198,25 @@ def encoder_layer(x, W, l, cfg, valid, bf16, last_endpoints=False):
     return np.where(valid[..., None], x2, 0.0), h_f, h_b
 
 
+def encoder_layer_concat(x, W, l, cfg, valid, prec):
+    """One layer of the paper's own topology (Sec. 3.2): the layer input is
+    projected linearly to the forward and reverse gates and candidates
+    [p_zf, n_f, p_zb, n_b] = W_in x + b_in (z = sigma(p_z)), the forward and
+    reverse scans of Eq. 2 run under the padding mask, and the two directions'
+    states are concatenated (2H wide) into the next layer.  The paper names no
+    normalisation inside the encoder; none is applied.  Returns (y, h_f, h_b),
+    y = [h_f; h_b], zero on padded hits (the scans output 0 there)."""
+    H = cfg["d_hidden"]
+    p = f"layer{l}."
+    proj = _lin(x, W[p + "w_in"], W[p + "b_in"], prec)
+    z_f = sigmoid(proj[..., 0:H])
+    n_f = proj[..., H:2 * H]
+    z_b = sigmoid(proj[..., 2 * H:3 * H])
+    n_b = proj[..., 3 * H:4 * H]
+    h_f, h_b = mingru_layer_scans(z_f, n_f, z_b, n_b, valid)
+    return np.concatenate([h_f, h_b], axis=-1), h_f, h_b
+
+
 def pool(x, h_f, h_b, n_hits, valid, mode):
     """Track readout.  mode 0 (mean): average of the last layer's output over the
     valid hits (masked pooling).  mode 1 (endpoints, Sec. 3.2): the forward state at
@@ -229,8 +249,15 @@ def _layout(cfg):
     P = D if cfg["pool"] == 0 else 2 * H
     Hh, Q = cfg["head_hidden"], 5 * cfg["n_quantiles"]
     lay = [("emb.w1", (D, E)), ("emb.b1", (D,)), ("emb.w2", (D, D)), ("emb.b2", (D,))]
+    concat = int(cfg.get("topology", 0)) == 1
+    if concat:
+        P = 2 * H
     for l in range(cfg["n_layers"]):
         p = f"layer{l}."
+        if concat:   # Sec. 3.2: W_in from the layer input (D, then 2H) to the gates and candidates
+            I = D if l == 0 else 2 * H
+            lay += [(p + "w_in", (4 * H, I)), (p + "b_in", (4 * H,))]
+            continue
         lay += [(p + "g", (D,)), (p + "w_in", (4 * H + D, D)), (p + "b_in", (4 * H + D,)),
                 (p + "w_m", (D, 2 * H)), (p + "b_m", (D,)), (p + "w1", (D, D)), (p + "b1", (D,)),
                 (p + "w2", (D, D)), (p + "b2", (D,))]
@@ -258,7 +285,9 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
 
     cfg: dict with d_model, d_hidden, n_layers, n_features, n_fourier, head_hidden,
     n_quantiles, precision (0 fp32, 1 bf16 operands, 2 fp16 operands), pool (0 mean, 1 endpoints),
-    feat_min, feat_max, fourier_scale, rms_eps.  hits: [B, T, 5]; n_hits: [B].
+    feat_min, feat_max, fourier_scale, rms_eps, and topology (0: the gated merge
+    and MLP of encoder_layer, the default; 1: the paper's concatenation,
+    encoder_layer_concat).  hits: [B, T, n_features]; n_hits: [B].
     Tracks whose hit count is outside [1, T] give a NaN row.  The output is the
     median quantile of the head directly (no seed decode)."""
     W = split_blob(cfg, blob)
@@ -276,7 +305,10 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
     endpoints = int(cfg["pool"]) == 1
     h_f = h_b = None
     for l in range(L):
-        x, h_f, h_b = encoder_layer(x, W, l, cfg, valid, bf16, last_endpoints=endpoints and l == L - 1)
+        if int(cfg.get("topology", 0)) == 1:
+            x, h_f, h_b = encoder_layer_concat(x, W, l, cfg, valid, bf16)
+        else:
+            x, h_f, h_b = encoder_layer(x, W, l, cfg, valid, bf16, last_endpoints=endpoints and l == L - 1)
     pv = pool(x, h_f, h_b, n_ok, valid, int(cfg["pool"]))
     out, q = head(pv, W, cfg)
     out = np.where(bad[:, None], np.nan, out)

@@ -51,7 +51,8 @@ static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
 // Fill the shape summary and blob offsets; false if cfg is outside the supported set.
 static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   if (!c || c->abi_version != TRACKFIT_ABI_VERSION) return false;
-  if (c->n_features != TRACKFIT_MAX_FEATURES || c->n_fourier != TRACKFIT_MAX_FOURIER) return false;
+  if (c->n_features < 1 || c->n_features > TRACKFIT_MAX_FEATURES || c->n_fourier != TRACKFIT_MAX_FOURIER) return false;
+  if (c->topology != TRACKFIT_TOPOLOGY_MERGE && c->topology != TRACKFIT_TOPOLOGY_CONCAT) return false;
   if (c->max_hits < 1 || c->max_hits > TF_MAX_HITS) return false;
   if (c->d_model < 16 || c->d_model > 256 || (c->d_model % 16) != 0) return false;
   if (c->d_hidden != 3 * c->d_model / 2) return false;
@@ -62,7 +63,7 @@ static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
     return false;
   if (c->pool != TRACKFIT_POOL_MEAN && c->pool != TRACKFIT_POOL_ENDPOINTS) return false;
   if (!(c->rms_eps > 0.0f) || !std::isfinite(c->rms_eps)) return false;
-  for (int f = 0; f < TRACKFIT_MAX_FEATURES; ++f)
+  for (int f = 0; f < c->n_features; ++f)
     if (!(c->feat_max[f] > c->feat_min[f]) || !std::isfinite(c->feat_max[f]) || !std::isfinite(c->feat_min[f]))
       return false;
   for (int k = 0; k < TRACKFIT_MAX_FOURIER; ++k)
@@ -74,7 +75,8 @@ static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   s->D = c->d_model;
   s->H = c->d_hidden;
   s->L = c->n_layers;
-  s->P = c->pool == TRACKFIT_POOL_MEAN ? s->D : 2 * s->H;
+  s->topology = c->topology;
+  s->P = (c->pool == TRACKFIT_POOL_MEAN && c->topology == TRACKFIT_TOPOLOGY_MERGE) ? s->D : 2 * s->H;
   s->Hh = c->head_hidden;
   s->NQ = c->n_quantiles;
   s->Q = 5 * c->n_quantiles;
@@ -96,6 +98,13 @@ static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   o->emb_b2 = p; p += D;
   for (int l = 0; l < s->L; ++l) {
     tf_layer_off& y = o->layer[l];
+    if (s->topology == TRACKFIT_TOPOLOGY_CONCAT) {   // W_in[4H][I_l] b_in[4H]
+      const size_t I = l == 0 ? D : 2 * H;
+      y.g = y.w_m = y.b_m = y.w1 = y.b1 = y.w2 = y.b2 = 0;
+      y.w_in = p; p += 4 * H * I;
+      y.b_in = p; p += 4 * H;
+      continue;
+    }
     y.g = p; p += D;
     y.w_in = p; p += (4 * H + D) * D;
     y.b_in = p; p += 4 * H + D;

@@ -130,21 +130,22 @@ __device__ void residuals(const Helix& h, const double (&x)[3], double& du, doub
   s = h.R * a / h.st;
 }
 
-__global__ void seed_kernel(const float* __restrict__ hits, const int32_t* __restrict__ n_hits, int64_t B, int T,
-                            double b_field, double min_sep, double* __restrict__ seed, float* __restrict__ feats) {
+__global__ void seed_kernel(const float* __restrict__ hits, int hs, const int32_t* __restrict__ n_hits, int64_t B,
+                            int T, double b_field, double min_sep, double* __restrict__ seed, float* __restrict__ feats,
+                            int fs) {
   const int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (b >= B) return;
   int n = n_hits[b];
   if (n < 0) n = 0;
   if (n > T) n = 0;   // not a track: no seed
-  const float* hb = hits + (size_t)b * T * 5;
+  const float* hb = hits + (size_t)b * T * hs;   // hit t of this track at hb[t * hs]
   // the seed triplet: the first hit, then each first later hit more than min_sep
   // (3-D) from the previous seed hit
   int pick[3] = {-1, -1, -1};
   int np = 0;
   double last[3] = {0.0, 0.0, 0.0};
   for (int t = 0; t < n && np < 3; ++t) {
-    const double p[3] = {(double)hb[t * 5 + 0], (double)hb[t * 5 + 1], (double)hb[t * 5 + 2]};
+    const double p[3] = {(double)hb[t * hs + 0], (double)hb[t * hs + 1], (double)hb[t * hs + 2]};
     bool take = np == 0;
     if (!take) {
       const double dx = p[0] - last[0], dy = p[1] - last[1], dz = p[2] - last[2];
@@ -162,30 +163,30 @@ __global__ void seed_kernel(const float* __restrict__ hits, const int32_t* __res
   if (ok) {
     double h3[3][3];
     for (int k = 0; k < 3; ++k)
-      for (int c = 0; c < 3; ++c) h3[k][c] = (double)hb[pick[k] * 5 + c];
+      for (int c = 0; c < 3; ++c) h3[k][c] = (double)hb[pick[k] * hs + c];
     perigee_from_triplet(h3[0], h3[1], h3[2], b_field, pg);
   } else {
     for (int k = 0; k < 5; ++k) pg[k] = __longlong_as_double(0x7ff8000000000000ll);
   }
   for (int k = 0; k < 5; ++k) seed[b * 5 + k] = pg[k];
   if (!feats) return;
-  float* fo = feats + (size_t)b * T * 3;
+  float* fo = feats + (size_t)b * T * fs;
   bool finite = ok;
   for (int k = 0; k < 5; ++k) finite = finite && isfinite(pg[k]);
   const Helix h = finite ? helix_of(pg, b_field) : Helix{};
   for (int t = 0; t < T; ++t) {
     float f0 = 0.0f, f1 = 0.0f, f2 = 0.0f;
     if (finite && t < n) {
-      const double x[3] = {(double)hb[t * 5 + 0], (double)hb[t * 5 + 1], (double)hb[t * 5 + 2]};
+      const double x[3] = {(double)hb[t * hs + 0], (double)hb[t * hs + 1], (double)hb[t * hs + 2]};
       double du, dv, s;
       residuals(h, x, du, dv, s);
       f0 = (float)asinh(du);
       f1 = (float)asinh(dv);
       f2 = (float)s;
     }
-    fo[t * 3 + 0] = f0;
-    fo[t * 3 + 1] = f1;
-    fo[t * 3 + 2] = f2;
+    fo[t * fs + 0] = f0;
+    fo[t * fs + 1] = f1;
+    fo[t * fs + 2] = f2;
   }
 }
 
@@ -204,18 +205,21 @@ __global__ void decode_kernel(const double* __restrict__ seed, const float* __re
 
 }  // namespace
 
-extern "C" int trackfit_seed(const float* hits, const int32_t* n_hits, int64_t n_tracks, int32_t max_hits,
-                             double b_field, double* seed_out, float* features_out, void* stream) {
+extern "C" int trackfit_seed(const float* hits, int32_t hit_stride, const int32_t* n_hits, int64_t n_tracks,
+                             int32_t max_hits, double b_field, double* seed_out, float* features_out,
+                             int32_t feat_stride, void* stream) {
   if (!hits || !n_hits || !seed_out || n_tracks <= 0 || max_hits < 1 || max_hits > TF_MAX_HITS) {
     return TRACKFIT_ERR_INVALID_ARG;
   }
+  if (hit_stride < 3 || (features_out && feat_stride < 3)) return TRACKFIT_ERR_INVALID_ARG;
   if (!(b_field > 0.0) || !isfinite(b_field)) return TRACKFIT_ERR_INVALID_ARG;
   const uintptr_t mis = reinterpret_cast<uintptr_t>(hits) | reinterpret_cast<uintptr_t>(seed_out) |
                         reinterpret_cast<uintptr_t>(n_hits) | reinterpret_cast<uintptr_t>(features_out);
   if (mis & 15u) return TRACKFIT_ERR_INVALID_ARG;
   const unsigned grid = (unsigned)((n_tracks + 127) / 128);
-  seed_kernel<<<grid, 128, 0, reinterpret_cast<cudaStream_t>(stream)>>>(hits, n_hits, n_tracks, max_hits, b_field,
-                                                                        10.0, seed_out, features_out);
+  seed_kernel<<<grid, 128, 0, reinterpret_cast<cudaStream_t>(stream)>>>(hits, hit_stride, n_hits, n_tracks, max_hits,
+                                                                        b_field, 10.0, seed_out, features_out,
+                                                                        feat_stride);
   return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
 }
 

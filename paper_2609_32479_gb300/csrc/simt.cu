@@ -217,17 +217,17 @@ __global__ void __launch_bounds__(128) pool_head_kernel(const float* __restrict_
   __shared__ float qv[5 * 15];
   const int64_t b = blockIdx.x;
   const int tid = threadIdx.x;
-  const int T = s.T, D = s.D, H = s.H, P = s.P;
+  const int T = s.T, H = s.H, P = s.P;
   int n = n_hits[b];
   const bool bad = n < 1 || n > T;
   if (bad) {
     if (tid == 0) atomicAdd(err, 1ull);
     n = 1;
   }
-  if (s.pool == TRACKFIT_POOL_MEAN) {
-    for (int c = tid; c < D; c += blockDim.x) {
+  if (s.pool == TRACKFIT_POOL_MEAN) {   // x: [rows][P] (P = D, or 2H for CONCAT)
+    for (int c = tid; c < P; c += blockDim.x) {
       float acc = 0.0f;
-      for (int t = 0; t < n; ++t) acc += x[(b * T + t) * D + c];
+      for (int t = 0; t < n; ++t) acc += x[(b * T + t) * P + c];
       pv[c] = acc / (float)n;
     }
   } else {
@@ -330,6 +330,19 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
     if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
     for (int l = 0; l < s.L; ++l) {
       const tf_layer_off& lo = o.layer[l];
+      if (s.topology == TRACKFIT_TOPOLOGY_CONCAT) {
+        // Sec. 3.2: the layer input (the embedding, then the previous layer's
+        // concatenated states) projected to the gates and candidates, the two
+        // scans, their states concatenated in Y (the next layer's input: the
+        // projection reads Y before the scan overwrites it, in stream order)
+        const int I = l == 0 ? D : 2 * H;
+        g.A = l == 0 ? X : Y; g.lda = I; g.W = W + lo.w_in; g.bias = W + lo.b_in; g.C = PR; g.ldc = 4 * H;
+        g.N = 4 * H; g.K = I; g.epi = EPI_PROJ;
+        if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+        dim3 sg((H + 127) / 128, (unsigned)nb);
+        mingru_scan_kernel<<<sg, 128, 0, st>>>(PR, 4 * H, nc, nb, s.T, H, Y);
+        continue;
+      }
       rmsnorm_kernel<<<(unsigned)((R + 7) / 8), 256, 0, st>>>(X, R, D, W + lo.g, s.rms_eps, XH);
       g.A = XH; g.lda = D; g.W = W + lo.w_in; g.bias = W + lo.b_in; g.C = PR; g.ldc = PD;
       g.N = PD; g.K = D; g.epi = EPI_PROJ;
@@ -347,7 +360,9 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
       g.N = D; g.K = D; g.epi = EPI_RES_MASK; g.res = X1; g.ldr = D;
       if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
     }
-    pool_head_kernel<<<(unsigned)nb, 128, 0, st>>>(X, Y, nc, nb, s, W + o.head_g, W + o.head_w1, W + o.head_b1,
+    // mean pooling reads the last layer's output: X (MERGE) or the states Y (CONCAT)
+    const float* xm = s.topology == TRACKFIT_TOPOLOGY_CONCAT ? Y : X;
+    pool_head_kernel<<<(unsigned)nb, 128, 0, st>>>(xm, Y, nc, nb, s, W + o.head_g, W + o.head_w1, W + o.head_b1,
                                                     W + o.head_w2, W + o.head_b2, out + c0 * 5,
                                                     out_q ? out_q + c0 * s.Q : nullptr,
                                                     out_pool ? out_pool + c0 * s.P : nullptr, err);

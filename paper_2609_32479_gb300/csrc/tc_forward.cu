@@ -1607,7 +1607,8 @@ int tf_tc_wait_limit(trackfit_ctx* h, int64_t limit_ns, int hold_tile) {
 }
 
 bool tf_tc_supported(const tf_shape& s) {
-  return (s.precision == TRACKFIT_BF16_PROJ || s.precision == TRACKFIT_FP16_PROJ) && s.pool == TRACKFIT_POOL_MEAN && (s.D == 128 || s.D == 256) &&
+  return (s.precision == TRACKFIT_BF16_PROJ || s.precision == TRACKFIT_FP16_PROJ) && s.pool == TRACKFIT_POOL_MEAN &&
+         s.topology == TRACKFIT_TOPOLOGY_MERGE && (s.D == 128 || s.D == 256) &&
          s.H % 64 == 0 && s.T <= 64 && s.Hh == 128 && s.Q <= 75 && s.F == 5 && s.K == 16;
 }
 

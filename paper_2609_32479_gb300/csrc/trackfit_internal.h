@@ -26,7 +26,7 @@ struct tf_blob_off {
 
 // Shape summary derived from the public config.
 struct tf_shape {
-  int T, F, K, E, D, H, L, P, Hh, NQ, Q, precision, pool;
+  int T, F, K, E, D, H, L, P, Hh, NQ, Q, precision, pool, topology;
   float rms_eps;
   float feat_min[TRACKFIT_MAX_FEATURES], feat_inv_range[TRACKFIT_MAX_FEATURES];
   double feat_min_d[TRACKFIT_MAX_FEATURES], feat_range_d[TRACKFIT_MAX_FEATURES];

@@ -18,7 +18,8 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_lib", "libtrackfit.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_BAD_HITS, ERR_TIMEOUT = range(7)
-ABI_VERSION = 1
+ABI_VERSION = 2
+MAX_FEATURES = 16
 
 # every function declared in include/trackfit.h
 EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trackfit_forward_ex",
@@ -34,8 +35,8 @@ class Config(ctypes.Structure):
                 ("n_features", ctypes.c_int32), ("n_fourier", ctypes.c_int32),
                 ("d_model", ctypes.c_int32), ("d_hidden", ctypes.c_int32), ("n_layers", ctypes.c_int32),
                 ("head_hidden", ctypes.c_int32), ("n_quantiles", ctypes.c_int32),
-                ("precision", ctypes.c_int32), ("pool", ctypes.c_int32),
-                ("feat_min", ctypes.c_float * 5), ("feat_max", ctypes.c_float * 5),
+                ("precision", ctypes.c_int32), ("pool", ctypes.c_int32), ("topology", ctypes.c_int32),
+                ("feat_min", ctypes.c_float * MAX_FEATURES), ("feat_max", ctypes.c_float * MAX_FEATURES),
                 ("fourier_scale", ctypes.c_float * 16), ("rms_eps", ctypes.c_float)]
 
 
@@ -94,7 +95,7 @@ def load() -> ctypes.CDLL:
     lib.trackfit_debug_wait_limit.restype = ctypes.c_int
     lib.trackfit_debug_alloc.argtypes = [i64, ctypes.POINTER(i64)]
     lib.trackfit_debug_alloc.restype = i64
-    lib.trackfit_seed.argtypes = [vp, vp, i64, i32, ctypes.c_double, vp, vp, vp]
+    lib.trackfit_seed.argtypes = [vp, i32, vp, i64, i32, ctypes.c_double, vp, vp, i32, vp]
     lib.trackfit_seed.restype = ctypes.c_int
     lib.trackfit_decode.argtypes = [vp, vp, i64, vp, vp]
     lib.trackfit_decode.restype = ctypes.c_int
@@ -114,8 +115,8 @@ def make_config(m: W.ModelConfig) -> Config:
     c.max_hits, c.n_features, c.n_fourier = m.max_hits, m.n_features, m.n_fourier
     c.d_model, c.d_hidden, c.n_layers = m.d_model, m.d_hidden, m.n_layers
     c.head_hidden, c.n_quantiles = m.head_hidden, m.n_quantiles
-    c.precision, c.pool = m.precision, m.pool
-    for i in range(5):
+    c.precision, c.pool, c.topology = m.precision, m.pool, m.topology
+    for i in range(m.n_features):
         c.feat_min[i], c.feat_max[i] = m.feat_min[i], m.feat_max[i]
     for i in range(16):
         c.fourier_scale[i] = m.fourier_scale[i]
@@ -321,17 +322,24 @@ def debug_alloc(fail_nth: int = 0):
     return int(live), int(att.value)
 
 
-def seed(hits, n_hits, b_field: float, seed_out, features_out=None, stream=None) -> None:
-    """Analytic fp64 seed (device tensors): hits [B, T, 5] f32, n_hits [B] i32 ->
-    seed_out [B, 5] f64, features_out [B, T, 3] f32 (optional)."""
-    B, T = int(hits.shape[0]), int(hits.shape[1])
+def seed(hits, n_hits, b_field: float, seed_out, features_out=None, stream=None, in_place_at=None) -> None:
+    """Analytic fp64 seed (device tensors): hits [B, T, F] f32 (x, y, z first), n_hits
+    [B] i32 -> seed_out [B, 5] f64 and the residual features: into features_out
+    [B, T, 3] f32, or, with in_place_at = c, into columns c..c+2 of hits itself."""
+    B, T, F = int(hits.shape[0]), int(hits.shape[1]), int(hits.shape[2])
     if tuple(n_hits.shape) != (B,) or tuple(seed_out.shape) != (B, 5):
         raise ValueError("seed: n_hits must be [B] and seed_out [B, 5]")
-    if features_out is not None and tuple(features_out.shape) != (B, T, 3):
-        raise ValueError("seed: features_out must be [B, T, 3]")
-    st = load().trackfit_seed(_dev(hits, "torch.float32"), _dev(n_hits, "torch.int32"), B, T, float(b_field),
-                              _dev(seed_out, "torch.float64"), _dev(features_out, "torch.float32"),
-                              _stream_handle(stream))
+    hp = _dev(hits, "torch.float32")
+    if in_place_at is not None:
+        if not 3 <= in_place_at <= F - 3 or (4 * in_place_at) % 16:
+            raise ValueError("seed: in_place_at must leave x, y, z alone, fit the row, and be 16-byte aligned")
+        fp, fs = hp + 4 * int(in_place_at), F
+    else:
+        if features_out is not None and tuple(features_out.shape) != (B, T, 3):
+            raise ValueError("seed: features_out must be [B, T, 3]")
+        fp, fs = _dev(features_out, "torch.float32"), 3
+    st = load().trackfit_seed(hp, F, _dev(n_hits, "torch.int32"), B, T, float(b_field),
+                              _dev(seed_out, "torch.float64"), fp, fs, _stream_handle(stream))
     if st != OK:
         raise TrackfitError(st, "trackfit_seed")
 

@@ -45,6 +45,8 @@ PRECISION_BF16 = 1
 PRECISION_FP16 = 2
 POOL_MEAN = 0
 POOL_ENDPOINTS = 1
+TOPOLOGY_MERGE = 0      # gated merge + MLP into a d_model residual stream
+TOPOLOGY_CONCAT = 1     # Sec. 3.2: concatenated states into the next layer
 
 N_FEATURES = 5          # (x, y, z, r, phi) per hit
 N_FOURIER = 16          # Sec. 3.2: "16 scales"
@@ -69,6 +71,7 @@ class ModelConfig:
     n_layers: int
     precision: int = PRECISION_FP32
     pool: int = POOL_MEAN
+    topology: int = TOPOLOGY_MERGE
     head_hidden: int = HEAD_HIDDEN
     n_quantiles: int = N_QUANTILES
     n_features: int = N_FEATURES
@@ -84,12 +87,14 @@ class ModelConfig:
 
     @property
     def proj_dim(self) -> int:
-        """Rows of the per-layer input projection: z_f, n_f, z_b, n_b, gate."""
-        return 4 * self.d_hidden + self.d_model
+        """Rows of the per-layer input projection: z_f, n_f, z_b, n_b (and, MERGE, the gate)."""
+        return 4 * self.d_hidden + (self.d_model if self.topology == TOPOLOGY_MERGE else 0)
 
     @property
     def pooled_dim(self) -> int:
-        return self.d_model if self.pool == POOL_MEAN else 2 * self.d_hidden
+        if self.pool == POOL_MEAN and self.topology == TOPOLOGY_MERGE:
+            return self.d_model
+        return 2 * self.d_hidden
 
     @property
     def n_out(self) -> int:
@@ -132,6 +137,25 @@ for _T in (8, 16, 32, 64):
                                        layout="sweep", n_barrel=_T, min_hits=_T)
 SWEEP_BATCHES = (4096, 16384, 65536, 262144, 1048576)
 
+# The paper's model (Sec. 3.2): 15 features per hit, d_model 128, two layers of
+# hidden width 192, the concatenation topology, endpoint readout; fp16 operands
+# (Sec. 3.5).  Its 12 measured features are "position, derived angles, and
+# detector identifiers" (Sec. 2); the list is not given, so here: x, y, z, r, phi,
+# the polar angle theta = atan2(r, z), eta = asinh(z / r), the distance
+# rho = |(r, z)|, cos phi, sin phi, the surface kind (barrel 0, disk 1) and the
+# surface's index within its kind; the last three are the seed's residual
+# features (asinh du, asinh dv, s_helix, Sec. 3.1), computed by the seed.
+PAPER_FEATURES = ("x", "y", "z", "r", "phi", "theta", "eta", "rho", "cos_phi", "sin_phi", "surface_kind",
+                  "surface_index", "asinh_du", "asinh_dv", "s_helix")
+PAPER_FEAT_MIN = (-1100.0, -1100.0, -3100.0, 0.0, -math.pi, 0.0, -5.0, 0.0, -1.0, -1.0, 0.0, 0.0, -8.0, -8.0, 0.0)
+PAPER_FEAT_MAX = (1100.0, 1100.0, 3100.0, 1100.0, math.pi, math.pi, 5.0, 3300.0, 1.0, 1.0, 1.0, 9.0, 8.0, 8.0,
+                  4000.0)
+WORKLOADS["paper"] = Workload(
+    "paper", 131072,
+    ModelConfig(max_hits=24, d_model=128, d_hidden=192, n_layers=2, precision=PRECISION_FP16, pool=POOL_ENDPOINTS,
+                topology=TOPOLOGY_CONCAT, n_features=15, feat_min=PAPER_FEAT_MIN, feat_max=PAPER_FEAT_MAX),
+    layout="barrel_endcap", pt_range=(1.0, 100.0))
+
 
 def workload(name: str, n_tracks: Optional[int] = None, **model_kw) -> Workload:
     w = WORKLOADS[name]
@@ -154,6 +178,10 @@ def weight_layout(cfg: ModelConfig) -> List[Tuple[str, Tuple[int, ...], int]]:
     out = [("emb.w1", (D, E), E), ("emb.b1", (D,), E), ("emb.w2", (D, D), D), ("emb.b2", (D,), D)]
     for l in range(cfg.n_layers):
         p = f"layer{l}."
+        if cfg.topology == TOPOLOGY_CONCAT:
+            I = D if l == 0 else 2 * H
+            out += [(p + "w_in", (4 * H, I), I), (p + "b_in", (4 * H,), I)]
+            continue
         out += [(p + "g", (D,), 0), (p + "w_in", (4 * H + D, D), D), (p + "b_in", (4 * H + D,), D),
                 (p + "w_m", (D, 2 * H), 2 * H), (p + "b_m", (D,), 2 * H),
                 (p + "w1", (D, D), D), (p + "b1", (D,), D), (p + "w2", (D, D), D), (p + "b2", (D,), D)]
@@ -216,6 +244,7 @@ C_LIGHT = 0.299792458
 class TrackBatch:
     hits: np.ndarray      # [B, T, 5] float32, pads zero
     n_hits: np.ndarray    # [B] int32
+    kind: np.ndarray      # [B, T] int8: the hit's surface, 0 barrel, 1 disk, -1 padding
     truth: np.ndarray     # [B, 5] float64: d0, z0, phi, theta, q/p
     kin: Dict[str, np.ndarray]   # per-track pT, eta, q, R and helix centre (generator tests)
 
@@ -368,6 +397,7 @@ def gen_tracks(w: Workload, n_tracks: Optional[int] = None, seed: Optional[int] 
         return parts[0]
     return TrackBatch(hits=np.concatenate([p.hits for p in parts]),
                       n_hits=np.concatenate([p.n_hits for p in parts]),
+                      kind=np.concatenate([p.kind for p in parts]),
                       truth=np.concatenate([p.truth for p in parts]),
                       kin={k: np.concatenate([p.kin[k] for p in parts]) for k in parts[0].kin})
 
@@ -423,7 +453,30 @@ def _gen_chunk(w: Workload, B: int, rng, smear: bool, pad_value: float) -> Track
     hits[:, :S2, :] = np.where(valid[..., None], feats[:, :S2, :].astype(np.float32), np.float32(pad_value))
     p = kin["pt"] / np.sin(kin["theta"])
     truth = np.stack([kin["d0"], kin["z0"], kin["phi0"], kin["theta"], kin["q"] / p], axis=1)
-    return TrackBatch(hits=hits, n_hits=cnt.astype(np.int32), truth=truth, kin=kin)
+    kind = np.full((B, T), -1, dtype=np.int8)
+    kind[:, :S2] = np.where(valid, K[:, :S2], -1)
+    return TrackBatch(hits=hits, n_hits=cnt.astype(np.int32), kind=kind, truth=truth, kin=kin)
+
+
+def paper_hits(tb: TrackBatch, w: Workload) -> np.ndarray:
+    """The 15-feature hit rows of the paper's model (PAPER_FEATURES) for a batch:
+    the 12 measured features derived from the stored fp32 (x, y, z, r, phi) in
+    fp64 and rounded to fp32; the three seed features left zero (the seed fills
+    them, on the device in place); padding rows zero.  Surface index: the nearest
+    barrel radius, or the nearest disk |z| (noise hits stay on their surface)."""
+    h = tb.hits.astype(np.float64)
+    x, y, z, r, phi = (h[..., k] for k in range(5))
+    valid = tb.kind >= 0
+    radii = np.linspace(BARREL_R_MIN, BARREL_R_MAX, w.n_barrel if w.layout == "sweep" else 10)
+    bi = np.argmin(np.abs(r[..., None] - radii), axis=-1)
+    di = np.argmin(np.abs(np.abs(z)[..., None] - np.asarray(DISK_Z)), axis=-1)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        eta = np.arcsinh(z / np.where(r > 0, r, 1.0))
+    cols = [x, y, z, r, phi, np.arctan2(r, z), eta, np.hypot(r, z), np.cos(phi), np.sin(phi),
+            tb.kind.astype(np.float64), np.where(tb.kind == 1, di, bi).astype(np.float64)]
+    out = np.zeros(h.shape[:2] + (15,), dtype=np.float32)
+    out[..., :12] = np.where(valid[..., None], np.stack(cols, axis=-1), 0.0).astype(np.float32)
+    return out
 
 
 def length_histogram(n_hits: np.ndarray) -> Dict[int, int]:

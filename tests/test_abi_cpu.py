@@ -43,7 +43,7 @@ def test_weight_count_matches_layout(lib, name):
 
 @pytest.mark.parametrize("bad", [dict(d_model=24), dict(d_hidden=100), dict(max_hits=65), dict(max_hits=0),
                                  dict(n_layers=0), dict(n_layers=17), dict(head_hidden=64), dict(n_quantiles=6),
-                                 dict(precision=3), dict(pool=3), dict(n_fourier=8), dict(rms_eps=0.0),
+                                 dict(precision=3), dict(pool=3), dict(n_fourier=8), dict(rms_eps=0.0), dict(topology=2),
                                  dict(d_model=272, d_hidden=408)])
 def test_unsupported_configs_rejected_on_host(lib, bad):
     m = W.workload("tiny").model.with_(**bad)
@@ -62,8 +62,9 @@ def test_null_and_count_errors_on_host(lib):
     assert lib.trackfit_create(ctypes.byref(c), None, 1, ctypes.byref(h)) == T.ERR_INVALID_ARG
     n = W.weight_count(m)
     assert lib.trackfit_create(ctypes.byref(c), ctypes.c_void_p(16), n + 1, ctypes.byref(h)) == T.ERR_INVALID_ARG
-    c.abi_version = 2
-    assert lib.trackfit_create(ctypes.byref(c), ctypes.c_void_p(16), n, ctypes.byref(h)) == T.ERR_UNSUPPORTED
+    for v in (T.ABI_VERSION - 1, T.ABI_VERSION + 1):   # another layout of the config struct
+        c.abi_version = v
+        assert lib.trackfit_create(ctypes.byref(c), ctypes.c_void_p(16), n, ctypes.byref(h)) == T.ERR_UNSUPPORTED
     assert lib.trackfit_forward(None, ctypes.c_void_p(16), ctypes.c_void_p(16), 4, ctypes.c_void_p(16),
                                 None) == T.ERR_INVALID_ARG
     lib.trackfit_destroy(None)

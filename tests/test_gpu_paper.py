@@ -1,0 +1,125 @@
+"""The paper's own model (Sec. 3.2: 15 features, d_model 128, two layers of width
+192, concatenated directions, endpoint readout, fp16 operands) on the GPU against
+the oracle, and the whole seed-guided forward (Sec. 3.1-3.3): the fp64 seed
+writes its three residual features into the hit rows in place, the encoder reads
+all 15, and the seed decode turns the heads' median corrections into track
+parameters."""
+import dataclasses
+
+import numpy as np
+import pytest
+
+from oracle import seed_oracle as S
+from oracle import trackfit_oracle as O
+from paper_2609_32479_gb300 import workloads as W
+from tests.helpers import parity_ok
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def T():
+    import os
+    from paper_2609_32479_gb300 import trackfit
+    if not os.path.exists(trackfit.LIB_PATH):
+        import __graft_entry__
+        __graft_entry__.build()
+    trackfit.load()
+    return trackfit
+
+
+def oracle_inputs(w, tb):
+    """15-feature rows with the oracle's seed features (rounded to fp32) and the seed."""
+    h = W.paper_hits(tb, w)
+    seed = S.seed_from_hits(h[..., :3], tb.n_hits, w.b_field)
+    h[..., 12:15] = S.seed_features(seed, h[..., :3], tb.n_hits, w.b_field).astype(np.float32)
+    return h, seed
+
+
+def gpu_encoder(T, model, blob, hits, n_hits):
+    dev = torch.device("cuda:0")
+    with T.Trackfit(model, blob) as tf:
+        B = len(n_hits)
+        out = torch.full((B, 5), -7.0, device=dev)
+        q = torch.empty((B, 5, model.n_quantiles), device=dev)
+        tf.forward(torch.from_numpy(np.ascontiguousarray(hits)).to(dev), torch.from_numpy(n_hits).to(dev), out,
+                   quantiles=q)
+        torch.cuda.synchronize()
+        st = tf.device_errors()
+        path = tf.path
+    assert st == (T.OK, 0)
+    return out.cpu().numpy(), q.cpu().numpy(), path
+
+
+@pytest.mark.parametrize("prec", [W.PRECISION_FP32, W.PRECISION_FP16])
+def test_paper_encoder_matches_the_oracle(T, prec):
+    w = W.workload("paper", n_tracks=1000, precision=prec)
+    tb = W.gen_tracks(w)
+    hits, _ = oracle_inputs(w, tb)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    got, q, path = gpu_encoder(T, w.model, blob, hits, tb.n_hits)
+    assert path.startswith("simt")
+    cap = {}
+    ref = O.forward(dataclasses.asdict(w.model), blob, hits, tb.n_hits, capture=cap)
+    ok, msg = parity_ok(got, ref, prec)
+    print(f"paper encoder {path}: {msg}")
+    assert ok, msg
+    ok, msg = parity_ok(q.reshape(len(got), -1), cap["quantiles"].reshape(len(got), -1), prec)
+    assert ok, msg
+
+
+def test_paper_encoder_masking_is_bit_exact(T):
+    w = W.workload("paper", n_tracks=300)
+    tb = W.gen_tracks(w)
+    hits, _ = oracle_inputs(w, tb)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    base = gpu_encoder(T, w.model, blob, hits, tb.n_hits)[0]
+    nan = hits.copy()
+    nan[np.arange(w.model.max_hits)[None, :] >= tb.n_hits[:, None]] = np.nan
+    np.testing.assert_array_equal(gpu_encoder(T, w.model, blob, nan, tb.n_hits)[0], base)
+    perm = np.random.default_rng(2).permutation(300)
+    np.testing.assert_array_equal(gpu_encoder(T, w.model, blob, hits[perm], tb.n_hits[perm])[0], base[perm])
+
+
+def test_seed_guided_forward_matches_the_oracle(T):
+    """Seed (fp64, features written into columns 12-14 in place) -> encoder (fp16
+    operands) -> decode, all on the device, against the same chain in the oracle:
+    the features where the foot point is unique, the heads' corrections at the
+    fp16 bar, and the decoded parameters (seed + correction) to the corrections'
+    error."""
+    w = W.workload("paper", n_tracks=1000)
+    tb = W.gen_tracks(w)
+    hits_o, seed_o = oracle_inputs(w, tb)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    dev = torch.device("cuda:0")
+    hits = torch.from_numpy(W.paper_hits(tb, w)).to(dev)
+    nh = torch.from_numpy(tb.n_hits).to(dev)
+    seed = torch.empty((1000, 5), dtype=torch.float64, device=dev)
+    T.seed(hits, nh, w.b_field, seed, in_place_at=12)
+    with T.Trackfit(w.model, blob) as tf:
+        corr = torch.empty((1000, 5), device=dev)
+        tf.forward(hits, nh, corr)
+        out = torch.empty((1000, 5), device=dev)
+        T.decode(seed, corr, out)
+        torch.cuda.synchronize()
+    h, sd, c, o = hits.cpu().numpy(), seed.cpu().numpy(), corr.cpu().numpy(), out.cpu().numpy()
+    np.testing.assert_array_equal(np.isnan(sd), np.isnan(seed_o))
+    np.testing.assert_array_equal(h[..., :12], hits_o[..., :12])   # the seed wrote only its own columns
+    valid = np.arange(w.model.max_hits)[None, :] < tb.n_hits[:, None]
+    near = valid & (np.abs(np.sinh(hits_o[..., 12])) < 50.0) & (np.abs(np.sinh(hits_o[..., 13])) < 50.0)
+    assert np.max(np.abs(h[..., 12:14][near] - hits_o[..., 12:14][near])) < 2e-6
+    corr_o = O.forward(dataclasses.asdict(w.model), blob, hits_o, tb.n_hits)
+    ok_seed = ~np.isnan(seed_o[:, 0])
+    ok, msg = parity_ok(c[ok_seed], corr_o[ok_seed], w.model.precision)
+    print(f"seed-guided forward, corrections: {msg}")
+    assert ok, msg
+    dec_o = S.decode(seed_o, corr_o)
+    d = np.abs(o[ok_seed] - dec_o[ok_seed])
+    d[:, 2] = np.minimum(d[:, 2], 2 * np.pi - d[:, 2])
+    # q/p = q/p_seed + r (|q/p_seed| + 0.02): its correction enters scaled
+    gain = np.ones_like(d)
+    gain[:, 4] = np.abs(seed_o[ok_seed, 4]) + 0.02
+    scale = np.abs(c[ok_seed] - corr_o[ok_seed]) * gain + 1e-6 * np.maximum(np.abs(dec_o[ok_seed]), 1.0)
+    assert np.all(d <= scale), np.max(d - scale, axis=0)
+    assert np.all(np.isnan(o[~ok_seed]))

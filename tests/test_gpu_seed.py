@@ -74,11 +74,12 @@ def test_seed_and_features_match_the_oracle(T, name, n):
     # is unique near the helix; for a hit far off it (the noise hits of the large
     # workload) the normal-plane condition has several roots and the Newton
     # iteration may settle on a different one from a last-bit difference, so
-    # those hits (|du| or |dv| above 1 mm, against the 10 um smearing) are only
-    # required to be finite.
+    # those hits (|du| or |dv| above 50 mm: a three-hit seed extrapolated to the
+    # outer layers misses real hits by millimetres, noise hits lie hundreds of
+    # millimetres off) are only required to be finite.
     fv, rv = feats[valid], fref[valid]
-    near = (np.abs(np.sinh(rv[:, 0])) < 1.0) & (np.abs(np.sinh(rv[:, 1])) < 1.0)
-    assert near.mean() > 0.85
+    near = (np.abs(np.sinh(rv[:, 0])) < 50.0) & (np.abs(np.sinh(rv[:, 1])) < 50.0)
+    assert near.mean() > 0.8
     df = np.abs(fv[near] - rv[near])
     assert np.max(df[:, :2]) < 2e-6, np.max(df[:, :2])
     assert np.max(df[:, 2] / np.maximum(np.abs(rv[near][:, 2]), 1.0)) < 1e-6
@@ -141,8 +142,11 @@ def test_seed_argument_errors(T):
     sd = torch.zeros((4, 5), dtype=torch.float64, device=dev)
     lib = T.load()
     s = torch.cuda.current_stream().cuda_stream
-    assert lib.trackfit_seed(h.data_ptr(), n.data_ptr(), 0, 10, 2.0, sd.data_ptr(), None, s) == T.ERR_INVALID_ARG
-    assert lib.trackfit_seed(h.data_ptr(), n.data_ptr(), 4, 10, 0.0, sd.data_ptr(), None, s) == T.ERR_INVALID_ARG
-    assert lib.trackfit_seed(h.data_ptr(), n.data_ptr(), 4, 65, 2.0, sd.data_ptr(), None, s) == T.ERR_INVALID_ARG
-    assert lib.trackfit_seed(h.data_ptr() + 4, n.data_ptr(), 4, 10, 2.0, sd.data_ptr(), None, s) == T.ERR_INVALID_ARG
+    hp, np_, sp = h.data_ptr(), n.data_ptr(), sd.data_ptr()
+    assert lib.trackfit_seed(hp, 5, np_, 0, 10, 2.0, sp, None, 3, s) == T.ERR_INVALID_ARG
+    assert lib.trackfit_seed(hp, 5, np_, 4, 10, 0.0, sp, None, 3, s) == T.ERR_INVALID_ARG
+    assert lib.trackfit_seed(hp, 5, np_, 4, 65, 2.0, sp, None, 3, s) == T.ERR_INVALID_ARG
+    assert lib.trackfit_seed(hp + 4, 5, np_, 4, 10, 2.0, sp, None, 3, s) == T.ERR_INVALID_ARG
+    assert lib.trackfit_seed(hp, 2, np_, 4, 10, 2.0, sp, None, 3, s) == T.ERR_INVALID_ARG
+    assert lib.trackfit_seed(hp, 5, np_, 4, 10, 2.0, sp, hp, 2, s) == T.ERR_INVALID_ARG
     assert lib.trackfit_decode(None, h.data_ptr(), 4, h.data_ptr(), s) == T.ERR_INVALID_ARG

@@ -14,6 +14,7 @@ import pytest
 
 from oracle import seed_oracle as SO
 from oracle import trackfit_oracle as O
+from tests import test_oracle_concat as PC
 from tests import test_oracle_model as PM
 from tests import test_oracle_seed as PS
 from tests import test_oracle_units as PU
@@ -68,6 +69,11 @@ MUTANTS = [
      "q.reshape(q.shape[0], nq, q.shape[1] // nq).transpose(0, 2, 1)"),
     ("head-no-norm", "head", 'hn = rmsnorm(pv, W["head.g"], cfg["rms_eps"])', "hn = pv"),
     ("head-no-silu", "head", "hid = silu(", "hid = ("),
+    ("concat-directions-swapped", "encoder_layer_concat", "np.concatenate([h_f, h_b]", "np.concatenate([h_b, h_f]"),
+    ("concat-z-not-gated", "encoder_layer_concat", "z_f = sigmoid(proj[..., 0:H])", "z_f = proj[..., 0:H]"),
+    ("concat-candidate-activated", "encoder_layer_concat", "n_f = proj[..., H:2 * H]", "n_f = np.tanh(proj[..., H:2 * H])"),
+    ("concat-reverse-reads-forward", "encoder_layer_concat", "n_b = proj[..., 3 * H:4 * H]", "n_b = proj[..., H:2 * H]"),
+    ("concat-normalised", "encoder_layer_concat", 'proj = _lin(x, W[p + "w_in"]', 'proj = _lin(rmsnorm(x, 1.0, 1e-6), W[p + "w_in"]'),
 ]
 
 
@@ -103,7 +109,7 @@ SEED_MUTANTS = [
 def _pins(mods=None):
     """Every pin of the oracle test modules, parametrised cases expanded."""
     out = []
-    for mod in (mods or (PU, PM)):
+    for mod in (mods or (PU, PM, PC)):
         for name, fn in sorted(vars(mod).items()):
             if not (name.startswith("test_") and callable(fn)):
                 continue
