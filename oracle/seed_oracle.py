@@ -46,6 +46,7 @@ import numpy as np
 
 C_LIGHT = 0.299792458          # GeV / (T m)
 SEED_MIN_SEPARATION_MM = 10.0
+PITCH_MIN_MM = 1.0             # below this pitch z does not choose the helix turn of a hit
 
 __all__ = ["circle_through_three", "seed_perigee", "seed_triplet", "seed_from_hits", "helix_point",
            "helix_tangent", "curvilinear_residuals", "seed_features", "decode", "C_LIGHT",
@@ -189,13 +190,20 @@ def curvilinear_residuals(perigee, hit, b_field, iters=60):
     """(du, dv, s) of one hit [..., 3] against the helix of perigee [..., 5].
 
     The foot point is the helix point whose normal plane holds the hit:
-    (hit - p(a)) . t(a) = 0, solved for the turning angle a by Newton's method from
-    the transverse angle of the hit around the circle's centre (a few steps reach
-    fp64 rounding; the iteration stops when a no longer changes).  In that plane
+    (hit - p(a)) . t(a) = 0, solved for the turning angle a by Newton's method (a
+    few steps reach fp64 rounding; the iteration stops when a no longer changes).
+    The start is the hit's transverse angle around the circle's centre, counted
+    from the perigee into [-pi, pi) so that it is continuous across the perigee
+    (a hit just behind it gets a small negative angle, not nearly a full turn),
+    moved by the whole number of turns that brings it closest to the angle the
+    hit's z gives, (z - z0) tan(theta) / R, where the helix's pitch 2 pi R |cot
+    theta| exceeds PITCH_MIN_MM (turns closer than that are not told apart by z;
+    where they coincide, du and dv are the same on each).  In that plane
     the curvilinear axes are U = z x t / |z x t| and V = t x U (the frame of the
     linearised Kalman filter); du, dv are the hit's coordinates along them and s
     the 3-D path length R a / sin(theta) from the perigee to the foot point.
-    Readings: the foot point as defined here, s measured from the perigee."""
+    Readings: the foot point as defined here, s measured from the perigee (negative
+    behind it)."""
     perigee = np.asarray(perigee, dtype=np.float64)
     hit = np.asarray(hit, dtype=np.float64)
     d0, z0, phi0, theta, qop = (perigee[..., k] for k in range(5))
@@ -205,7 +213,12 @@ def curvilinear_residuals(perigee, hit, b_field, iters=60):
     cx, cy = x0 + q * R * np.sin(phi0), y0 - q * R * np.cos(phi0)
     g0 = np.arctan2(y0 - cy, x0 - cx)
     gh = np.arctan2(hit[..., 1] - cy, hit[..., 0] - cx)
-    a = np.mod(-q * (gh - g0), 2.0 * np.pi)
+    a = np.mod(-q * (gh - g0) + np.pi, 2.0 * np.pi) - np.pi
+    Rcot = R / np.tan(theta)
+    resolved = 2.0 * np.pi * np.abs(Rcot) > PITCH_MIN_MM
+    a_z = (hit[..., 2] - z0) / np.where(resolved, Rcot, 1.0)
+    turns = np.floor((a_z - a) / (2.0 * np.pi) + 0.5)
+    a = np.where(resolved, a + 2.0 * np.pi * turns, a)
     for _ in range(iters):
         p = helix_point(perigee, a, b_field)
         t = helix_tangent(perigee, a)

@@ -21,6 +21,7 @@ constexpr double TWO_PI = 6.283185307179586476925286766559;
 constexpr double PI = 3.1415926535897932384626433832795;
 constexpr double QOP_FLOOR = 0.02;   // 1/GeV: floor of the scale-free q/p residual (Sec. 3.3)
 constexpr int NEWTON_MAX = 60;
+constexpr double PITCH_MIN_MM = 1.0;   // below this pitch z does not choose the helix turn of a hit
 
 // x mod 2 pi in [0, 2 pi)
 __device__ __forceinline__ double mod2pi(double x) {
@@ -94,12 +95,18 @@ __device__ void perigee_from_triplet(const double (&a)[3], const double (&b)[3],
 }
 
 // (du, dv, s) of a hit against the helix: the foot point is the helix point whose
-// normal plane holds the hit, found by Newton's method on g(a) = (hit - p(a)) . t(a)
-// from the hit's transverse angle around the centre; du, dv are the hit's
-// coordinates along U = z x t / |z x t| and V = t x U there, s = R a / sin(theta).
+// normal plane holds the hit, found by Newton's method on g(a) = (hit - p(a)) . t(a).
+// The start is the hit's transverse angle around the centre counted from the
+// perigee into [-pi, pi) (continuous across the perigee), moved by the whole
+// turns that bring it closest to the angle of the hit's z, (z - z0) / (R cot theta),
+// where the pitch 2 pi R |cot theta| exceeds PITCH_MIN_MM.  du, dv are the hit's
+// coordinates along U = z x t / |z x t| and V = t x U at the foot point,
+// s = R a / sin(theta) (negative behind the perigee).
 __device__ void residuals(const Helix& h, const double (&x)[3], double& du, double& dv, double& s) {
   const double cot = h.ct / h.st;
-  double a = mod2pi(-h.q * (atan2(x[1] - h.cy, x[0] - h.cx) - h.g0));
+  double a = mod2pi(-h.q * (atan2(x[1] - h.cy, x[0] - h.cx) - h.g0) + PI) - PI;
+  const double rcot = h.R / tan(h.theta);
+  if (2.0 * PI * fabs(rcot) > PITCH_MIN_MM) a += TWO_PI * floor(((x[2] - h.z0) / rcot - a) / TWO_PI + 0.5);
   double px = 0.0, py = 0.0, pz = 0.0, tx = 0.0, ty = 0.0, tz = h.ct, sphi = 0.0, cphi = 1.0;
   auto at = [&](double aa) {
     sincos(h.phi0 - h.q * aa, &sphi, &cphi);

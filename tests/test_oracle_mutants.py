@@ -98,6 +98,10 @@ SEED_MUTANTS = [
     ("residual-v-sign", "curvilinear_residuals", "V = np.cross(t, U)", "V = np.cross(U, t)"),
     ("residual-no-foot-search", "curvilinear_residuals", "a_new = a - step", "a_new = a"),
     ("residual-transverse-path", "curvilinear_residuals", "R * a / np.sin(theta)", "R * a"),
+    ("residual-no-turn-choice", "curvilinear_residuals", "a = np.where(resolved, a + 2.0 * np.pi * turns, a)",
+     "a = a"),
+    ("residual-start-from-zero", "curvilinear_residuals", "np.mod(-q * (gh - g0) + np.pi, 2.0 * np.pi) - np.pi",
+     "np.mod(-q * (gh - g0), 2.0 * np.pi)"),
     ("features-no-asinh", "seed_features", "np.arcsinh(du / scale_mm)", "du / scale_mm"),
     ("decode-phi-unwrapped", "decode", "out[..., 2] = np.pi - np.mod(np.pi - out[..., 2], 2.0 * np.pi)",
      "out[..., 2] = out[..., 2]"),

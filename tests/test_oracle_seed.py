@@ -182,6 +182,56 @@ def test_displacements_in_the_normal_plane_are_recovered():
         np.testing.assert_allclose(gv, dv, rtol=0, atol=1e-9)
 
 
+def test_looping_and_behind_the_perigee():
+    """Points a turn or two along the helix (low-momentum tracks loop) and just
+    behind the perigee, displaced in their normal plane: z picks the turn, so the
+    foot point is the point itself and s = R a / sin(theta) with the sign and the
+    whole turns; a point behind the perigee gets a small negative s, not almost a
+    full turn.  Helices whose pitch 2 pi R |cot theta| is at least 100 mm (z tells
+    the turns apart by more than the 5 mm displacement)."""
+    g = np.random.default_rng(24)
+    n = 600
+    w = W.Workload("seed", n, W.workload("large").model, pt_range=(0.5, 5.0), b_field=B_FIELD)
+    pt, eta, phi0, q, d0, z0 = W._draw_kinematics(g, n, w)
+    theta = 2.0 * np.arctan(np.exp(-eta))
+    R = 1000.0 * pt / (W.C_LIGHT * B_FIELD)
+    keep = 2.0 * np.pi * R * np.abs(np.sinh(eta)) > 100.0
+    pt, eta, phi0, q, d0, z0, theta, R = (v[keep] for v in (pt, eta, phi0, q, d0, z0, theta, R))
+    truth = np.stack([d0, z0, phi0, theta, q * np.sin(theta) / pt], axis=-1)
+    x0, y0 = -d0 * np.sin(phi0), d0 * np.cos(phi0)
+    cx, cy = x0 + q * R * np.sin(phi0), y0 - q * R * np.cos(phi0)
+    for base in (-0.3, 0.4, 2.0 * np.pi + 1.0, 4.0 * np.pi + 2.5):
+        al = base + g.uniform(-0.2, 0.2, len(R))
+        x, y = W._helix_point(cx, cy, R, q, phi0, al)
+        p = np.stack([x, y, z0 + R * al * np.sinh(eta)], axis=-1)
+        _, U, V = _frame(truth, al)
+        du, dv = g.uniform(-5.0, 5.0, len(al)), g.uniform(-5.0, 5.0, len(al))
+        gu, gv, s = S.curvilinear_residuals(truth, p + du[:, None] * U + dv[:, None] * V, B_FIELD)
+        np.testing.assert_allclose(gu, du, rtol=0, atol=1e-7)
+        np.testing.assert_allclose(gv, dv, rtol=0, atol=1e-7)
+        np.testing.assert_allclose(s, R * al / np.sin(theta), rtol=1e-9)
+
+
+def test_flat_helix_behind_the_perigee():
+    """theta = pi/2 (zero pitch: every turn is the same circle, z tells none apart):
+    a point just behind the perigee has the small negative s of its own turn, and
+    one ahead the small positive s."""
+    g = np.random.default_rng(25)
+    n = 200
+    R = g.uniform(500.0, 5000.0, n)
+    q = np.where(g.random(n) < 0.5, -1.0, 1.0)
+    phi0, d0, z0 = g.uniform(-np.pi, np.pi, n), g.normal(0.0, 0.1, n), g.normal(0.0, 50.0, n)
+    theta = np.full(n, np.pi / 2)
+    truth = np.stack([d0, z0, phi0, theta, q * 1000.0 / (W.C_LIGHT * B_FIELD * R)], axis=-1)
+    x0, y0 = -d0 * np.sin(phi0), d0 * np.cos(phi0)
+    cx, cy = x0 + q * R * np.sin(phi0), y0 - q * R * np.cos(phi0)
+    for al in (g.uniform(-0.5, -0.01, n), g.uniform(0.01, 0.5, n)):
+        x, y = W._helix_point(cx, cy, R, q, phi0, al)
+        du, dv, s = S.curvilinear_residuals(truth, np.stack([x, y, z0], axis=-1), B_FIELD)
+        assert np.all(np.abs(du) < 1e-6) and np.all(np.abs(dv) < 1e-6)
+        np.testing.assert_allclose(s, R * al, rtol=1e-9)
+
+
 def test_seed_features_layout_and_padding():
     pts, truth, alphas = _helices(20, seed=23)
     B = len(truth)
