@@ -30,7 +30,8 @@ from typing import Dict, Optional
 import numpy as np
 
 __all__ = ["bf16_round", "fp16_round", "sigmoid", "silu", "rmsnorm", "normalise", "fourier", "linear_scan",
-           "mingru_layer_scans", "embed", "encoder_layer", "encoder_layer_concat", "pool", "head", "forward",
+           "mingru_layer_scans", "embed", "encoder_layer", "encoder_layer_concat", "attention",
+           "encoder_layer_attention", "pool", "head", "forward",
            "split_blob"]
 
 
@@ -217,6 +218,46 @@ def encoder_layer_concat(x, W, l, cfg, valid, prec):
     return np.concatenate([h_f, h_b], axis=-1), h_f, h_b
 
 
+def attention(q, k, v, valid, n_heads):
+    """Multi-head self-attention within each track (Vaswani et al. 2017), the
+    token mixing of the paper's Transformer encoder (App. A.3, Tab. A.1: full
+    attention over a track's hits).  q, k, v: [B, T, D], split into n_heads heads
+    of D / n_heads channels; per head the weights are the softmax over the track's
+    valid hits of q . k / sqrt(D / n_heads) and the output their weighted sum of v.
+    Padded hits are no keys (their weight is exactly 0); a padded query's output
+    is 0."""
+    B, T, D = q.shape
+    dh = D // n_heads
+    qh, kh, vh = (np.asarray(a, dtype=np.float64).reshape(B, T, n_heads, dh) for a in (q, k, v))
+    sc = np.einsum("bthd,bshd->bhts", qh, kh) / np.sqrt(dh)
+    sc = np.where(valid[:, None, None, :], sc, -np.inf)
+    sc = sc - np.max(sc, axis=-1, keepdims=True)      # the softmax is unchanged by the shift
+    w = np.exp(sc)
+    w = w / np.sum(w, axis=-1, keepdims=True)
+    o = np.einsum("bhts,bshd->bthd", w, vh).reshape(B, T, D)
+    return np.where(valid[..., None], o, 0.0)
+
+
+def encoder_layer_attention(x, W, l, cfg, valid, prec):
+    """One layer of the Transformer encoder (reading; the paper names only a
+    general-purpose Transformer of the same parameter count, App. A.3): pre-norm
+    attention and MLP blocks with residuals (MLP hidden width d_hidden),
+      x' = x + W_o attention(W_qkv RMSNorm(x) g_1 + b_qkv) + b_o
+      x_next = x' + W_2 SiLU(W_1 RMSNorm(x') g_2 + b_1) + b_2,  padded hits set to 0.
+    With 16-bit operands the projections' operands are rounded as in the
+    recurrent encoder; the attention itself (scores, softmax, weighted sum) is
+    full precision.  No positional encoding: the Fourier features of the hit
+    positions carry where a hit is."""
+    D = cfg["d_model"]
+    p = f"layer{l}."
+    qkv = _lin(rmsnorm(x, W[p + "g1"], cfg["rms_eps"]), W[p + "w_qkv"], W[p + "b_qkv"], prec)
+    o = attention(qkv[..., 0:D], qkv[..., D:2 * D], qkv[..., 2 * D:3 * D], valid, cfg["n_heads"])
+    x1 = x + _lin(o, W[p + "w_o"], W[p + "b_o"], prec)
+    u = silu(_lin(rmsnorm(x1, W[p + "g2"], cfg["rms_eps"]), W[p + "w1"], W[p + "b1"], prec))
+    x2 = x1 + _lin(u, W[p + "w2"], W[p + "b2"], prec)
+    return np.where(valid[..., None], x2, 0.0), None, None
+
+
 def pool(x, h_f, h_b, n_hits, valid, mode):
     """Track readout.  mode 0 (mean): average of the last layer's output over the
     valid hits (masked pooling).  mode 1 (endpoints, Sec. 3.2): the forward state at
@@ -250,10 +291,18 @@ def _layout(cfg):
     Hh, Q = cfg["head_hidden"], 5 * cfg["n_quantiles"]
     lay = [("emb.w1", (D, E)), ("emb.b1", (D,)), ("emb.w2", (D, D)), ("emb.b2", (D,))]
     concat = int(cfg.get("topology", 0)) == 1
+    attn = int(cfg.get("topology", 0)) == 2
     if concat:
         P = 2 * H
+    if attn:
+        P = D
     for l in range(cfg["n_layers"]):
         p = f"layer{l}."
+        if attn:
+            lay += [(p + "g1", (D,)), (p + "w_qkv", (3 * D, D)), (p + "b_qkv", (3 * D,)), (p + "w_o", (D, D)),
+                    (p + "b_o", (D,)), (p + "g2", (D,)), (p + "w1", (H, D)), (p + "b1", (H,)),
+                    (p + "w2", (D, H)), (p + "b2", (D,))]
+            continue
         if concat:   # Sec. 3.2: W_in from the layer input (D, then 2H) to the gates and candidates
             I = D if l == 0 else 2 * H
             lay += [(p + "w_in", (4 * H, I)), (p + "b_in", (4 * H,))]
@@ -287,7 +336,8 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
     n_quantiles, precision (0 fp32, 1 bf16 operands, 2 fp16 operands), pool (0 mean, 1 endpoints),
     feat_min, feat_max, fourier_scale, rms_eps, and topology (0: the gated merge
     and MLP of encoder_layer, the default; 1: the paper's concatenation,
-    encoder_layer_concat).  hits: [B, T, n_features]; n_hits: [B].
+    encoder_layer_concat; 2: the Transformer encoder, encoder_layer_attention, with
+    n_heads, mean pooling only).  hits: [B, T, n_features]; n_hits: [B].
     Tracks whose hit count is outside [1, T] give a NaN row.  The output is the
     median quantile of the head directly (no seed decode)."""
     W = split_blob(cfg, blob)
@@ -307,6 +357,8 @@ def forward(cfg: dict, blob, hits, n_hits, capture: Optional[dict] = None):
     for l in range(L):
         if int(cfg.get("topology", 0)) == 1:
             x, h_f, h_b = encoder_layer_concat(x, W, l, cfg, valid, bf16)
+        elif int(cfg.get("topology", 0)) == 2:
+            x, h_f, h_b = encoder_layer_attention(x, W, l, cfg, valid, bf16)
         else:
             x, h_f, h_b = encoder_layer(x, W, l, cfg, valid, bf16, last_endpoints=endpoints and l == L - 1)
     pv = pool(x, h_f, h_b, n_ok, valid, int(cfg["pool"]))

@@ -14,6 +14,7 @@ import pytest
 
 from oracle import seed_oracle as SO
 from oracle import trackfit_oracle as O
+from tests import test_oracle_attention as PA
 from tests import test_oracle_concat as PC
 from tests import test_oracle_model as PM
 from tests import test_oracle_seed as PS
@@ -74,6 +75,22 @@ MUTANTS = [
     ("concat-candidate-activated", "encoder_layer_concat", "n_f = proj[..., H:2 * H]", "n_f = np.tanh(proj[..., H:2 * H])"),
     ("concat-reverse-reads-forward", "encoder_layer_concat", "n_b = proj[..., 3 * H:4 * H]", "n_b = proj[..., H:2 * H]"),
     ("concat-normalised", "encoder_layer_concat", 'proj = _lin(x, W[p + "w_in"]', 'proj = _lin(rmsnorm(x, 1.0, 1e-6), W[p + "w_in"]'),
+    ("attention-scaled-by-width", "attention", "/ np.sqrt(dh)", "/ np.sqrt(D)"),
+    ("attention-no-key-mask", "attention", "sc = np.where(valid[:, None, None, :], sc, -np.inf)", "sc = sc"),
+    ("attention-scores-transposed", "attention", '"bthd,bshd->bhts"', '"bthd,bshd->bhst"'),
+    ("attention-not-normalised", "attention", "w = w / np.sum(w, axis=-1, keepdims=True)", "w = w"),
+    ("attention-heads-interleaved", "attention", ".reshape(B, T, n_heads, dh) for a in (q, k, v)",
+     ".reshape(B, T, dh, n_heads).swapaxes(2, 3) for a in (q, k, v)"),
+    ("attention-pads-not-zeroed", "attention", "return np.where(valid[..., None], o, 0.0)", "return o"),
+    ("attnlayer-no-prenorm", "encoder_layer_attention", 'qkv = _lin(rmsnorm(x, W[p + "g1"], cfg["rms_eps"])',
+     "qkv = _lin(x"),
+    ("attnlayer-k-v-swapped", "encoder_layer_attention", "qkv[..., D:2 * D], qkv[..., 2 * D:3 * D]",
+     "qkv[..., 2 * D:3 * D], qkv[..., D:2 * D]"),
+    ("attnlayer-no-attention-residual", "encoder_layer_attention", "x1 = x + _lin(o", "x1 = _lin(o"),
+    ("attnlayer-mlp-reads-x", "encoder_layer_attention", 'rmsnorm(x1, W[p + "g2"]', 'rmsnorm(x, W[p + "g2"]'),
+    ("attnlayer-no-mlp-residual", "encoder_layer_attention", "x2 = x1 + _lin(u", "x2 = _lin(u"),
+    ("attnlayer-pads-not-zeroed", "encoder_layer_attention", "return np.where(valid[..., None], x2, 0.0), None, None",
+     "return x2, None, None"),
 ]
 
 
@@ -113,7 +130,7 @@ SEED_MUTANTS = [
 def _pins(mods=None):
     """Every pin of the oracle test modules, parametrised cases expanded."""
     out = []
-    for mod in (mods or (PU, PM, PC)):
+    for mod in (mods or (PU, PM, PC, PA)):
         for name, fn in sorted(vars(mod).items()):
             if not (name.startswith("test_") and callable(fn)):
                 continue
