@@ -11,6 +11,7 @@ than L2, so no flush is needed between steps.
   python bench.py --seed         # analytic fp64 seed + features + decode, and its share of the forward
   python bench.py --packed       # packed, unpadded input against the padded entry point
   python bench.py --paper        # the paper's model: seed, 15-feature encoder, decode per step
+  python bench.py --transformer  # the same with the Transformer encoder of the encoder comparison
 
 N > 1 runs under torch.distributed.run, one rank per GPU; every rank processes
 its own full batch (replicas, weak scaling; the path has no exchange step).
@@ -372,18 +373,40 @@ def next_main(args, w: W.Workload):
 FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 
 
-def paper_main(args):
+def encoder_flops(m, n_hits):
+    """Algorithmic flops of the encoder over tracks with these hit counts: the
+    per-hit products (embedding, then per layer the projections; for the
+    Transformer also q.k and p.v over each track's hits) and the head."""
+    D, H, E = m.d_model, m.d_hidden, m.embed_dim
+    n = np.asarray(n_hits, dtype=np.int64)
+    per_hit = 2 * (E * D + D * D)
+    if m.topology == W.TOPOLOGY_ATTENTION:
+        per_hit += m.n_layers * 2 * (3 * D * D + D * D + 2 * H * D)
+        attn = m.n_layers * 4 * D * int((n * n).sum())
+    else:
+        per_hit += sum(2 * (D if l == 0 else 2 * H) * 4 * H for l in range(m.n_layers))
+        attn = 0
+    return int(n.sum()) * per_hit + attn + len(n) * flops_per_track_head(m)
+
+
+PAPER_CONTEXT = {"paper": "the paper reports 5.41 M tracks/s on one H100 NVL for its trained minGRU model on its data",
+                 "transformer": "the paper reports 3.18 M tracks/s on one H100 NVL for its Transformer of the same "
+                                "parameter count (Tab. A.1)"}
+
+
+def paper_main(args, name="paper"):
     """The paper's model and its whole forward as deployed (Sec. 3.1-3.3, 4.2): per
     step the fp64 seed writes its three features into the 15-feature hit rows in
-    place, the encoder (concatenation topology, endpoint readout, fp16 operands,
-    CUDA-core path) runs, and the decode turns the median corrections into track
-    parameters.  The paper's 5.41 M tracks/s (H100 NVL, its own kernels and data)
-    is context, not a baseline for this workload."""
+    place, the encoder (the paper's concatenation topology with endpoint readout,
+    or the Transformer of its encoder comparison, fp16 operands) runs, and the
+    decode turns the median corrections into track parameters.  The paper's
+    figures (H100 NVL, its own kernels and data) are context, not a baseline for
+    this workload."""
     import torch
     from paper_2609_32479_gb300 import trackfit as TF
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    w = W.workload("paper", n_tracks=args.n_tracks)
+    w = W.workload(name, n_tracks=args.n_tracks)
     m = w.model
     tb = W.gen_tracks(w)
     blob = W.gen_weights(m, w.weight_seed)
@@ -406,24 +429,24 @@ def paper_main(args):
         enc_ms = _time_events(lambda: tf.forward(hits, nh, corr, stream), reps, stream)
         st, nbad = tf.device_errors(stream)
         path = tf.path
-    D, H, E = m.d_model, m.d_hidden, m.embed_dim
-    per_hit = 2 * (E * D + D * D) + sum(2 * (D if l == 0 else 2 * H) * 4 * H for l in range(m.n_layers))
-    flops = int(tb.n_hits.sum()) * per_hit + B * flops_per_track_head(m)
-    achieved = flops / (enc_ms * 1e-3) / 1e12
-    line = {"metric": "tracks/sec at 1 GB300, the paper's model and seed-guided forward (device-timed)",
+    D, H = m.d_model, m.d_hidden
+    achieved = encoder_flops(m, tb.n_hits) / (enc_ms * 1e-3) / 1e12
+    topo = {W.TOPOLOGY_CONCAT: "concat", W.TOPOLOGY_ATTENTION: "attention"}.get(m.topology, "merge")
+    what = "the paper's model" if name == "paper" else "the paper's Transformer encoder"
+    line = {"metric": f"tracks/sec at 1 GB300, {what} and seed-guided forward (device-timed)",
             "value": B / (ms * 1e-3), "unit": "tracks/s", "n_gpus": 1, "steps": reps, "warmup": max(args.warmup, 1),
             "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f16",
             "data": "synthetic helix tracks + random-init weights (seeded)", "path": path,
-            "config": {"workload": "paper", "n_tracks": B, "max_hits": m.max_hits, "n_features": m.n_features,
-                       "d_model": D, "d_hidden": H, "n_layers": m.n_layers, "topology": "concat",
-                       "pool": "endpoints", "l2": "inputs larger than L2; no flush",
-                       "parameters": W.weight_count(m)},
+            "config": {"workload": name, "n_tracks": B, "max_hits": m.max_hits, "n_features": m.n_features,
+                       "d_model": D, "d_hidden": H, "n_layers": m.n_layers, "topology": topo,
+                       "pool": "endpoints" if m.pool == W.POOL_ENDPOINTS else "mean",
+                       "l2": "inputs larger than L2; no flush", "parameters": W.weight_count(m)},
             "encoder_ms": enc_ms, "seed_and_decode_ms": ms - enc_ms,
             "roofline": {"bound": "alu", "kernel": "CUDA-core encoder (fp32 FMA, 16-bit operands)",
                          "achieved": achieved, "peak": FP32_ALU_TFLOPS, "unit": "TFLOP/s",
                          "frac": achieved / FP32_ALU_TFLOPS,
                          "peak_kind": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz"},
-            "context": "the paper reports 5.41 M tracks/s on one H100 NVL for its trained model on its data",
+            "context": PAPER_CONTEXT[name],
             "device_errors": {"status": st, "bad_tracks": nbad}}
     print(json.dumps(line))
     return 0
@@ -460,11 +483,14 @@ def main():
     ap.add_argument("--seed", action="store_true", help="time the analytic seed, features and decode")
     ap.add_argument("--packed", action="store_true", help="time the packed-input entry point")
     ap.add_argument("--paper", action="store_true", help="the paper's model, seed-guided forward")
+    ap.add_argument("--transformer", action="store_true", help="the paper's Transformer encoder, seed-guided")
     args = ap.parse_args()
     if args.sweep:
         return sweep_main(args)
     if args.paper:
         return paper_main(args)
+    if args.transformer:
+        return paper_main(args, "transformer")
     kw = {}
     if args.precision != "config":
         kw["precision"] = W.PRECISION_BF16 if args.precision == "bf16" else W.PRECISION_FP16

@@ -43,7 +43,7 @@
 extern "C" {
 #endif
 
-#define TRACKFIT_ABI_VERSION 2
+#define TRACKFIT_ABI_VERSION 3
 #define TRACKFIT_MAX_FEATURES 16
 #define TRACKFIT_MAX_FOURIER 16
 
@@ -65,15 +65,25 @@ typedef enum { TRACKFIT_POOL_MEAN = 0, TRACKFIT_POOL_ENDPOINTS = 1 } trackfit_po
  * with the task).  CONCAT: the paper's own (Sec. 3.2): each layer projects its
  * input to the forward and reverse gates and candidates, scans, and the two
  * directions' states, concatenated (2 d_hidden wide), are the next layer's input
- * and the readout's; no norm inside the encoder. */
-typedef enum { TRACKFIT_TOPOLOGY_MERGE = 0, TRACKFIT_TOPOLOGY_CONCAT = 1 } trackfit_topology;
+ * and the readout's; no norm inside the encoder.  ATTENTION: the Transformer of
+ * the paper's encoder comparison (App. A.3, Tab. A.1): per layer, pre-norm
+ * multi-head self-attention over the track's own hits and a pre-norm SiLU MLP of
+ * hidden width d_hidden, each added to a d_model-wide residual stream; no
+ * positional encoding; mean pooling. */
+typedef enum {
+  TRACKFIT_TOPOLOGY_MERGE = 0,
+  TRACKFIT_TOPOLOGY_CONCAT = 1,
+  TRACKFIT_TOPOLOGY_ATTENTION = 2
+} trackfit_topology;
 
-/* Encoder shape.  Supported: abi_version = 2, 1 <= n_features <= 16 per hit (the
+/* Encoder shape.  Supported: abi_version = 3, 1 <= n_features <= 16 per hit (the
  * task's configs use 5: x, y, z [mm], r [mm], phi [rad]; the paper's model 15, its
  * last three the seed features of trackfit_seed), n_fourier = 16, 1 <= max_hits
- * <= 64, d_model in {16, 32, ..., 256} (multiple of 16), d_hidden = 3 * d_model / 2,
- * 1 <= n_layers <= 16, head_hidden = 128, n_quantiles odd <= 15, topology MERGE or
- * CONCAT.  feat_min/feat_max (first n_features entries) are fixed min-max
+ * <= 64, d_model in {16, 32, ..., 256} (multiple of 16), d_hidden = 3 * d_model / 2
+ * (MERGE, CONCAT) or, ATTENTION, the MLP width, a multiple of 16 in [16, 1024],
+ * 1 <= n_layers <= 16, head_hidden = 128, n_quantiles odd <= 15.  n_heads is read
+ * for ATTENTION only: d_model / n_heads a multiple of 8, at most 64 (ATTENTION
+ * pools by the mean).  feat_min/feat_max (first n_features entries) are fixed min-max
  * constants (feat_max > feat_min); fourier_scale[k] = s_k, the feature argument is
  * pi * s_k * u; rms_eps > 0.  The tensor-core path runs 16-bit-operand MERGE
  * configs with 5 features, mean pooling and d_model 128 or 256; everything else
@@ -91,6 +101,7 @@ typedef struct {
   int32_t precision;  /* trackfit_precision */
   int32_t pool;       /* trackfit_pool */
   int32_t topology;   /* trackfit_topology */
+  int32_t n_heads;    /* attention heads (ATTENTION) */
   float feat_min[TRACKFIT_MAX_FEATURES];
   float feat_max[TRACKFIT_MAX_FEATURES];
   float fourier_scale[TRACKFIT_MAX_FOURIER];
@@ -103,7 +114,7 @@ typedef struct trackfit_ctx* trackfit_t;
  * Number of fp32 values in the weight blob for cfg (0 if cfg is NULL or
  * unsupported).  Blob order, every matrix in PyTorch [out][in] row-major order,
  * with D = d_model, H = d_hidden, E = 2 * n_features * n_fourier,
- * P = D (MERGE with mean pooling) or 2H (endpoints, or CONCAT), Hh = head_hidden,
+ * P = D (MERGE with mean pooling, ATTENTION) or 2H (endpoints, or CONCAT), Hh = head_hidden,
  * Q = 5 * n_quantiles:
  *   W_e1[D][E] b_e1[D] W_e2[D][D] b_e2[D]
  *   MERGE, per layer: g[D] W_in[4H+D][D] b_in[4H+D] (row blocks z_f, n_f, z_b, n_b, gate)
@@ -111,6 +122,9 @@ typedef struct trackfit_ctx* trackfit_t;
  *              W_1[D][D] b_1[D] W_2[D][D] b_2[D]
  *   CONCAT, per layer l: W_in[4H][I_l] b_in[4H] (row blocks z_f, n_f, z_b, n_b), I_0 = D,
  *              I_l = 2H after (columns: forward states, then reverse)
+ *   ATTENTION, per layer: g_1[D] W_qkv[3D][D] b_qkv[3D] (row blocks q, k, v; head h
+ *              owns rows h D/n_heads .. of each block) W_o[D][D] b_o[D] g_2[D]
+ *              W_1[H][D] b_1[H] W_2[D][H] b_2[D]
  *   g_h[P] W_h1[Hh][P] b_h1[Hh] W_h2[Q][Hh] b_h2[Q]   (Q rows parameter-major: [5][7]) */
 size_t trackfit_weight_count(const trackfit_config_t* cfg);
 

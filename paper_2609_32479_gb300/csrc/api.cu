@@ -52,10 +52,19 @@ static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
 static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   if (!c || c->abi_version != TRACKFIT_ABI_VERSION) return false;
   if (c->n_features < 1 || c->n_features > TRACKFIT_MAX_FEATURES || c->n_fourier != TRACKFIT_MAX_FOURIER) return false;
-  if (c->topology != TRACKFIT_TOPOLOGY_MERGE && c->topology != TRACKFIT_TOPOLOGY_CONCAT) return false;
+  const bool attn = c->topology == TRACKFIT_TOPOLOGY_ATTENTION;
+  if (c->topology != TRACKFIT_TOPOLOGY_MERGE && c->topology != TRACKFIT_TOPOLOGY_CONCAT && !attn) return false;
   if (c->max_hits < 1 || c->max_hits > TF_MAX_HITS) return false;
   if (c->d_model < 16 || c->d_model > 256 || (c->d_model % 16) != 0) return false;
-  if (c->d_hidden != 3 * c->d_model / 2) return false;
+  if (attn) {
+    if (c->d_hidden < 16 || c->d_hidden > 1024 || (c->d_hidden % 16) != 0) return false;
+    if (c->n_heads < 1 || (c->d_model % c->n_heads) != 0) return false;
+    const int dh = c->d_model / c->n_heads;
+    if ((dh % 8) != 0 || dh > 64) return false;
+    if (c->pool != TRACKFIT_POOL_MEAN) return false;
+  } else if (c->d_hidden != 3 * c->d_model / 2) {
+    return false;
+  }
   if (c->n_layers < 1 || c->n_layers > TF_MAX_LAYERS) return false;
   if (c->head_hidden != 128) return false;
   if (c->n_quantiles < 1 || c->n_quantiles > 15 || (c->n_quantiles % 2) == 0) return false;
@@ -76,7 +85,8 @@ static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   s->H = c->d_hidden;
   s->L = c->n_layers;
   s->topology = c->topology;
-  s->P = (c->pool == TRACKFIT_POOL_MEAN && c->topology == TRACKFIT_TOPOLOGY_MERGE) ? s->D : 2 * s->H;
+  s->NH = attn ? c->n_heads : 0;
+  s->P = (c->pool == TRACKFIT_POOL_MEAN && c->topology != TRACKFIT_TOPOLOGY_CONCAT) ? s->D : 2 * s->H;
   s->Hh = c->head_hidden;
   s->NQ = c->n_quantiles;
   s->Q = 5 * c->n_quantiles;
@@ -98,6 +108,20 @@ static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   o->emb_b2 = p; p += D;
   for (int l = 0; l < s->L; ++l) {
     tf_layer_off& y = o->layer[l];
+    y.g2 = 0;
+    if (attn) {   // g_1 W_qkv b_qkv W_o b_o g_2 W_1 b_1 W_2 b_2
+      y.g = p; p += D;
+      y.w_in = p; p += 3 * D * D;
+      y.b_in = p; p += 3 * D;
+      y.w_m = p; p += D * D;
+      y.b_m = p; p += D;
+      y.g2 = p; p += D;
+      y.w1 = p; p += H * D;
+      y.b1 = p; p += H;
+      y.w2 = p; p += D * H;
+      y.b2 = p; p += D;
+      continue;
+    }
     if (s->topology == TRACKFIT_TOPOLOGY_CONCAT) {   // W_in[4H][I_l] b_in[4H]
       const size_t I = l == 0 ? D : 2 * H;
       y.g = y.w_m = y.b_m = y.w1 = y.b1 = y.w2 = y.b2 = 0;

@@ -9,6 +9,7 @@
 #include <cuda_fp16.h>
 #include <math.h>
 
+#include "attention.cuh"
 #include "trackfit_internal.h"
 
 namespace {
@@ -269,7 +270,14 @@ __global__ void __launch_bounds__(128) pool_head_kernel(const float* __restrict_
   if (tid < 5) out[b * 5 + tid] = qv[tid * s.NQ + s.NQ / 2];
 }
 
-size_t ws_floats_per_track(const tf_shape& s) { return (size_t)s.T * (s.E + 14 * (size_t)s.D); }
+// Per hit row: E (Fourier) + U + X + XH + PR + Y + X1, with U = D and PR = 4H + D,
+// Y = 2H (recurrent topologies) or U = H (the MLP), PR = 3D (q, k, v) and Y = D
+// (the attention output) for ATTENTION.
+size_t ws_floats_per_track(const tf_shape& s) {
+  const size_t D = s.D, H = s.H;
+  const size_t row = s.topology == TRACKFIT_TOPOLOGY_ATTENTION ? H + 7 * D : 5 * D + 6 * H;
+  return (size_t)s.T * (s.E + row);
+}
 
 int launch_gemm(const GemmArgs& g, cudaStream_t st) {
   dim3 grid((g.N + BN - 1) / BN, (g.R + BM - 1) / BM);
@@ -298,17 +306,24 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
                 unsigned long long* err, const float* hits, const int32_t* n_hits, int64_t B, float* out,
                 float* out_q, float* out_pool, cudaStream_t st, trackfit_ctx* prof, const int64_t* offs) {
   const int rnd = s.precision;   // TRACKFIT_FP32 = 0, BF16_PROJ = 1, FP16_PROJ = 2
-  const int D = s.D, H = s.H, PD = 4 * s.H + s.D;
+  const bool attn = s.topology == TRACKFIT_TOPOLOGY_ATTENTION;
+  const int D = s.D, H = s.H, PD = attn ? 3 * s.D : 4 * s.H + s.D;
+  const int UW = attn ? s.H : s.D, YW = attn ? s.D : 2 * s.H;
+  // the attention CTA's dynamic shared memory, when above the default 48 KB
+  if (attn && tf_attn::smem_bytes(s.T, s.D) > 48 * 1024 &&
+      cudaFuncSetAttribute(tf_attn::track_attention_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)tf_attn::smem_bytes(s.T, s.D)) != cudaSuccess)
+    return TRACKFIT_ERR_CUDA;
   for (int64_t c0 = 0; c0 < B; c0 += ws_tracks) {
     const int64_t nb = (B - c0 < ws_tracks) ? B - c0 : ws_tracks;
     const int64_t R = nb * s.T;
     float* EB = ws;
     float* U = EB + R * s.E;
-    float* X = U + R * D;
+    float* X = U + R * UW;
     float* XH = X + R * D;
     float* PR = XH + R * D;
     float* Y = PR + R * PD;
-    float* X1 = Y + R * 2 * H;
+    float* X1 = Y + R * YW;
     const float* hc = offs ? hits : hits + c0 * s.T * 5;
     const int64_t* oc = offs ? offs + c0 : nullptr;
     const int32_t* nc = n_hits + c0;
@@ -341,6 +356,27 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
         if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
         dim3 sg((H + 127) / 128, (unsigned)nb);
         mingru_scan_kernel<<<sg, 128, 0, st>>>(PR, 4 * H, nc, nb, s.T, H, Y);
+        continue;
+      }
+      if (attn) {
+        // App. A.3: x' = x + W_o attention(RMSNorm(x) g_1 W_qkv^T + b_qkv) + b_o,
+        // x <- x' + W_2 SiLU(RMSNorm(x') g_2 W_1^T + b_1) + b_2, padded rows 0
+        rmsnorm_kernel<<<(unsigned)((R + 7) / 8), 256, 0, st>>>(X, R, D, W + lo.g, s.rms_eps, XH);
+        g.A = XH; g.lda = D; g.W = W + lo.w_in; g.bias = W + lo.b_in; g.C = PR; g.ldc = 3 * D;
+        g.N = 3 * D; g.K = D; g.epi = EPI_STORE;
+        if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+        tf_attn::track_attention_kernel<float><<<(unsigned)nb, tf_attn::THREADS, tf_attn::smem_bytes(s.T, D), st>>>(
+            PR, 3 * D, nullptr, nc, nb, s.T, D, s.NH, Y, D);
+        g.A = Y; g.lda = D; g.W = W + lo.w_m; g.bias = W + lo.b_m; g.C = X1; g.ldc = D;
+        g.N = D; g.K = D; g.epi = EPI_RES_MASK; g.res = X; g.ldr = D;
+        if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+        rmsnorm_kernel<<<(unsigned)((R + 7) / 8), 256, 0, st>>>(X1, R, D, W + lo.g2, s.rms_eps, XH);
+        g.A = XH; g.lda = D; g.W = W + lo.w1; g.bias = W + lo.b1; g.C = U; g.ldc = H;
+        g.N = H; g.K = D; g.epi = EPI_SILU;
+        if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+        g.A = U; g.lda = H; g.W = W + lo.w2; g.bias = W + lo.b2; g.C = X; g.ldc = D;
+        g.N = D; g.K = H; g.epi = EPI_RES_MASK; g.res = X1; g.ldr = D;
+        if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
         continue;
       }
       rmsnorm_kernel<<<(unsigned)((R + 7) / 8), 256, 0, st>>>(X, R, D, W + lo.g, s.rms_eps, XH);

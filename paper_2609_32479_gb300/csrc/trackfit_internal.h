@@ -14,8 +14,10 @@
 #define TF_HOST_EVENTS 10
 
 // Offsets (in floats) of every tensor inside the fp32 weight blob.
+// ATTENTION layers reuse the names: g = g_1, w_in/b_in = W_qkv/b_qkv, w_m/b_m =
+// W_o/b_o, g2 = g_2, w1/b1 and w2/b2 the MLP.
 struct tf_layer_off {
-  size_t g, w_in, b_in, w_m, b_m, w1, b1, w2, b2;
+  size_t g, w_in, b_in, w_m, b_m, w1, b1, w2, b2, g2;
 };
 struct tf_blob_off {
   size_t emb_w1, emb_b1, emb_w2, emb_b2;
@@ -26,7 +28,7 @@ struct tf_blob_off {
 
 // Shape summary derived from the public config.
 struct tf_shape {
-  int T, F, K, E, D, H, L, P, Hh, NQ, Q, precision, pool, topology;
+  int T, F, K, E, D, H, L, P, Hh, NQ, Q, precision, pool, topology, NH;
   float rms_eps;
   float feat_min[TRACKFIT_MAX_FEATURES], feat_inv_range[TRACKFIT_MAX_FEATURES];
   double feat_min_d[TRACKFIT_MAX_FEATURES], feat_range_d[TRACKFIT_MAX_FEATURES];

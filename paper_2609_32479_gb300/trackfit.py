@@ -18,7 +18,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_lib", "libtrackfit.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_BAD_HITS, ERR_TIMEOUT = range(7)
-ABI_VERSION = 2
+ABI_VERSION = 3
 MAX_FEATURES = 16
 
 # every function declared in include/trackfit.h
@@ -36,6 +36,7 @@ class Config(ctypes.Structure):
                 ("d_model", ctypes.c_int32), ("d_hidden", ctypes.c_int32), ("n_layers", ctypes.c_int32),
                 ("head_hidden", ctypes.c_int32), ("n_quantiles", ctypes.c_int32),
                 ("precision", ctypes.c_int32), ("pool", ctypes.c_int32), ("topology", ctypes.c_int32),
+                ("n_heads", ctypes.c_int32),
                 ("feat_min", ctypes.c_float * MAX_FEATURES), ("feat_max", ctypes.c_float * MAX_FEATURES),
                 ("fourier_scale", ctypes.c_float * 16), ("rms_eps", ctypes.c_float)]
 
@@ -116,6 +117,7 @@ def make_config(m: W.ModelConfig) -> Config:
     c.d_model, c.d_hidden, c.n_layers = m.d_model, m.d_hidden, m.n_layers
     c.head_hidden, c.n_quantiles = m.head_hidden, m.n_quantiles
     c.precision, c.pool, c.topology = m.precision, m.pool, m.topology
+    c.n_heads = m.n_heads
     for i in range(m.n_features):
         c.feat_min[i], c.feat_max[i] = m.feat_min[i], m.feat_max[i]
     for i in range(16):
@@ -194,8 +196,16 @@ class Trackfit:
             raise TrackfitError(st, "trackfit_set_path")
 
     def forward(self, hits, n_hits, out, stream=None, quantiles=None, pooled=None) -> None:
-        """Device tensors: hits [B, T, 5] f32, n_hits [B] i32, out [B, 5] f32."""
+        """Device tensors: hits [B, T, F] f32 (F = n_features), n_hits [B] i32, out
+        [B, 5] f32; optional quantiles [B, 5, n_quantiles] and pooled [B, P] f32."""
         B = int(n_hits.shape[0])
+        m = self.model
+        if tuple(hits.shape) != (B, m.max_hits, m.n_features) or tuple(out.shape) != (B, 5):
+            raise ValueError(f"forward: hits must be [{B}, {m.max_hits}, {m.n_features}] and out [{B}, 5]")
+        if quantiles is not None and tuple(quantiles.shape) != (B, 5, m.n_quantiles):
+            raise ValueError(f"forward: quantiles must be [{B}, 5, {m.n_quantiles}]")
+        if pooled is not None and tuple(pooled.shape) != (B, m.pooled_dim):
+            raise ValueError(f"forward: pooled must be [{B}, {m.pooled_dim}]")
         args = (self._h, _dev(hits, "torch.float32"), _dev(n_hits, "torch.int32"), B, _dev(out, "torch.float32"))
         if quantiles is None and pooled is None:
             st = self.lib.trackfit_forward(*args, _stream_handle(stream))
@@ -206,11 +216,13 @@ class Trackfit:
             raise TrackfitError(st, "trackfit_forward")
 
     def forward_packed(self, hits, offsets, out, stream=None) -> None:
-        """Device tensors: hits [N, 5] f32 (all tracks back to back), offsets [B + 1]
-        i64 (track b = rows offsets[b] .. offsets[b + 1] - 1), out [B, 5] f32."""
+        """Device tensors: hits [N, F] f32 (all tracks back to back, F = n_features),
+        offsets [B + 1] i64 (track b = rows offsets[b] .. offsets[b + 1] - 1), out
+        [B, 5] f32."""
         B = int(offsets.shape[0]) - 1
-        if hits.dim() != 2 or int(hits.shape[1]) != 5 or tuple(out.shape) != (B, 5):
-            raise ValueError("forward_packed: hits must be [N, 5], offsets [B + 1], out [B, 5]")
+        F = self.model.n_features
+        if hits.dim() != 2 or int(hits.shape[1]) != F or tuple(out.shape) != (B, 5):
+            raise ValueError(f"forward_packed: hits must be [N, {F}], offsets [B + 1], out [B, 5]")
         st = self.lib.trackfit_forward_packed(self._h, _dev(hits, "torch.float32"), int(hits.shape[0]),
                                               _dev(offsets, "torch.int64"), B, _dev(out, "torch.float32"),
                                               _stream_handle(stream))

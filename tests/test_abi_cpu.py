@@ -41,10 +41,23 @@ def test_weight_count_matches_layout(lib, name):
     assert T.weight_count(e) == W.weight_count(e)
 
 
+@pytest.mark.parametrize("name", ["paper", "transformer"])
+def test_weight_count_of_the_paper_models(lib, name):
+    m = W.workload(name).model
+    assert T.weight_count(m) == W.weight_count(m) > 0
+    if m.topology == W.TOPOLOGY_ATTENTION:
+        for kw in (dict(n_heads=2), dict(n_heads=16), dict(d_hidden=16), dict(n_layers=1)):
+            assert T.weight_count(m.with_(**kw)) == W.weight_count(m.with_(**kw))
+        assert T.weight_count(m.with_(n_heads=1)) == 0     # head width 128 > 64
+
+
 @pytest.mark.parametrize("bad", [dict(d_model=24), dict(d_hidden=100), dict(max_hits=65), dict(max_hits=0),
                                  dict(n_layers=0), dict(n_layers=17), dict(head_hidden=64), dict(n_quantiles=6),
-                                 dict(precision=3), dict(pool=3), dict(n_fourier=8), dict(rms_eps=0.0), dict(topology=2),
-                                 dict(d_model=272, d_hidden=408)])
+                                 dict(precision=3), dict(pool=3), dict(n_fourier=8), dict(rms_eps=0.0), dict(topology=3),
+                                 dict(d_model=272, d_hidden=408), dict(topology=2, pool=1),
+                                 dict(topology=2, n_heads=3), dict(topology=2, n_heads=8),
+                                 dict(topology=2, n_heads=0), dict(topology=2, d_hidden=40),
+                                 dict(topology=2, d_hidden=1040)])
 def test_unsupported_configs_rejected_on_host(lib, bad):
     m = W.workload("tiny").model.with_(**bad)
     c = T.make_config(m)
