@@ -85,9 +85,11 @@ typedef enum {
  * for ATTENTION only: d_model / n_heads a multiple of 8, at most 64 (ATTENTION
  * pools by the mean).  feat_min/feat_max (first n_features entries) are fixed min-max
  * constants (feat_max > feat_min); fourier_scale[k] = s_k, the feature argument is
- * pi * s_k * u; rms_eps > 0.  The tensor-core path runs 16-bit-operand MERGE
- * configs with 5 features, mean pooling and d_model 128 or 256; everything else
- * runs on the CUDA cores. */
+ * pi * s_k * u; rms_eps > 0.  The fused tensor-core path runs 16-bit-operand
+ * MERGE configs with 5 features, mean pooling and d_model 128 or 256; the
+ * packed-row tensor-core path runs 16-bit-operand CONCAT and ATTENTION configs
+ * (valid hits only, one tensor-core product per matrix of Sec. 3.2 / App. A.3);
+ * everything else runs on the CUDA cores. */
 typedef struct {
   int32_t abi_version;
   int32_t max_hits;
@@ -332,8 +334,11 @@ int trackfit_decode(const double* seed, const float* corrections, int64_t n_trac
  * expires; -1 holds nothing.  The outputs of a forward that timed out are not
  * valid; trackfit_device_errors reports TRACKFIT_ERR_TIMEOUT and resets the
  * counters, after which the handle is usable again.  Host side only; launches
- * nothing.  Errors: INVALID_ARG (NULL handle, limit_ns < 0, hold_tile < -1),
- * UNSUPPORTED (the handle runs the CUDA-core path, which has no waits). */
+ * nothing.  On a handle of the packed-row tensor-core path (16-bit CONCAT and
+ * ATTENTION configs) only the limit applies: hold_tile must be -1 there.
+ * Errors: INVALID_ARG (NULL handle, limit_ns < 0, hold_tile < -1), UNSUPPORTED
+ * (the handle runs the CUDA-core path, which has no waits, or hold_tile >= 0 on
+ * the packed-row path). */
 int trackfit_debug_wait_limit(trackfit_t h, int64_t limit_ns, int32_t hold_tile);
 
 /* Test hook for allocation failures (host side, not thread-safe): every device

@@ -43,6 +43,11 @@ extern "C" int64_t trackfit_debug_alloc(int64_t fail_nth, int64_t* attempted) {
 
 extern "C" int trackfit_debug_wait_limit(trackfit_t h, int64_t limit_ns, int32_t hold_tile) {
   if (!h) return TRACKFIT_ERR_INVALID_ARG;
+  if (h->rows) {   // the packed-row path: the limit only (it has no loader hand-over to hold)
+    if (limit_ns < 0 || hold_tile != -1) return limit_ns < 0 || hold_tile < -1 ? TRACKFIT_ERR_INVALID_ARG
+                                                                               : TRACKFIT_ERR_UNSUPPORTED;
+    return tf_rows_wait_limit(h, limit_ns);
+  }
   return tf_tc_wait_limit(h, limit_ns, hold_tile);
 }
 
@@ -221,6 +226,7 @@ extern "C" void trackfit_destroy(trackfit_t h) {
   if (!h) return;
   if (h->prof_on) trackfit_profile(h, 0);
   tf_tc_destroy(h);
+  tf_rows_destroy(h);
   tf_free(h->d_w);
   tf_free(h->d_err);
   tf_free(h->ws);
@@ -256,6 +262,9 @@ extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weight
   if (st == TRACKFIT_OK && tf_tc_supported(s)) {
     st = tf_tc_create(h, weights);
     if (st == TRACKFIT_OK) h->path = TF_PATH_TC;
+  } else if (st == TRACKFIT_OK && tf_rows_supported(s)) {
+    st = tf_rows_create(h, weights);
+    if (st == TRACKFIT_OK) h->path = TF_PATH_ROWS;
   }
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaDeviceSynchronize());
   if (st != TRACKFIT_OK) {
@@ -268,9 +277,9 @@ extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weight
 
 extern "C" const char* trackfit_path_name(trackfit_t h) {
   if (!h) return "none";
-  const bool tc = h->path == TF_PATH_TC;
-  if (h->s.precision == TRACKFIT_FP16_PROJ) return tc ? "tcgen05-fp16" : "simt-fp16";
-  if (h->s.precision == TRACKFIT_BF16_PROJ) return tc ? "tcgen05-bf16" : "simt-bf16";
+  const bool tc = h->path == TF_PATH_TC, rows = h->path == TF_PATH_ROWS;
+  if (h->s.precision == TRACKFIT_FP16_PROJ) return tc ? "tcgen05-fp16" : rows ? "tcgen05-rows-fp16" : "simt-fp16";
+  if (h->s.precision == TRACKFIT_BF16_PROJ) return tc ? "tcgen05-bf16" : rows ? "tcgen05-rows-bf16" : "simt-bf16";
   return "simt-fp32";
 }
 
@@ -281,7 +290,7 @@ extern "C" int trackfit_set_path(trackfit_t h, int path) {
     return TRACKFIT_OK;
   }
   if (path != 0) return TRACKFIT_ERR_INVALID_ARG;
-  h->path = (h->tc != nullptr) ? TF_PATH_TC : TF_PATH_SIMT;
+  h->path = (h->tc != nullptr) ? TF_PATH_TC : (h->rows != nullptr) ? TF_PATH_ROWS : TF_PATH_SIMT;
   return TRACKFIT_OK;
 }
 
@@ -293,6 +302,7 @@ extern "C" int trackfit_forward_ex(trackfit_t h, const float* hits, const int32_
   if ((out_q && !aligned16(out_q)) || (out_pool && !aligned16(out_pool))) return TRACKFIT_ERR_INVALID_ARG;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (h->path == TF_PATH_TC) return tf_tc_forward(h, hits, n_hits, n_tracks, out_params, out_q, out_pool, st);
+  if (h->path == TF_PATH_ROWS) return tf_rows_forward(h, hits, n_hits, n_tracks, out_params, out_q, out_pool, st);
   return tf_simt_forward(h, hits, n_hits, n_tracks, out_params, out_q, out_pool, st);
 }
 
@@ -316,9 +326,12 @@ extern "C" int trackfit_forward_packed(trackfit_t h, const float* hits, int64_t 
     const int64_t nb = (n_tracks - c0 < TF_PACKED_CHUNK) ? n_tracks - c0 : TF_PACKED_CHUNK;
     counts_from_offsets<<<(unsigned)((nb + 255) / 256), 256, 0, st>>>(offsets + c0, nb, n_hit_rows, h->s.T, h->pk_n);
     if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
-    const int r = h->path == TF_PATH_TC
-                      ? tf_tc_forward(h, hits, h->pk_n, nb, out_params + c0 * 5, nullptr, nullptr, st, offsets + c0)
-                      : tf_simt_forward(h, hits, h->pk_n, nb, out_params + c0 * 5, nullptr, nullptr, st, offsets + c0);
+    const int r =
+        h->path == TF_PATH_TC
+            ? tf_tc_forward(h, hits, h->pk_n, nb, out_params + c0 * 5, nullptr, nullptr, st, offsets + c0)
+        : h->path == TF_PATH_ROWS
+            ? tf_rows_forward(h, hits, h->pk_n, nb, out_params + c0 * 5, nullptr, nullptr, st, offsets + c0)
+            : tf_simt_forward(h, hits, h->pk_n, nb, out_params + c0 * 5, nullptr, nullptr, st, offsets + c0);
     if (r != TRACKFIT_OK) return r;
   }
   return TRACKFIT_OK;

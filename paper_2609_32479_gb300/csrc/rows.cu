@@ -1,0 +1,833 @@
+// Packed-row tensor-core path for the paper's own topology (Sec. 3.2: concatenated
+// directions, endpoint or mean readout) and for the Transformer encoder of its
+// encoder comparison (App. A.3), with 16-bit operands (Sec. 3.5: fp16 projections,
+// fp32 accumulation and recurrence).
+//
+// Layout: only valid hits are stored (Sec. 3.5, packed and unpadded).  Track b's
+// hit t is row row0[b] + t of every per-hit matrix; row0 is the exclusive prefix
+// sum of the valid hit counts (a track whose count is outside [1, max_hits] has
+// no rows and a NaN output).  Every per-hit matrix product is one launch of
+// row_gemm_kernel over all rows of a chunk:
+//   C[row][n] = epilogue(sum_k A[row][k] W[n][k])
+// A (16-bit activations, [rows][K]) and W (16-bit weights, PyTorch [N][K]) are
+// both K-major, TMA-staged with 128-byte swizzle; the fp32 accumulator lives in
+// tensor memory with lane = row, column = output channel, so one epilogue thread
+// owns one hit row: bias, SiLU, the sigmoid of the update gates, the residual
+// addition and the RMSNorm of the next pre-norm block (a reduction over the row)
+// are applied in registers and the results leave in the precision their consumer
+// reads (16-bit operands for the next product, fp32 for the residual stream and
+// the scans).  Between products run the CUDA-core kernels that are not
+// contractions: the Fourier featurisation, the gated scans along each track (the
+// concatenation topology) and the attention within each track (the Transformer),
+// the pooling and the head.
+//
+// Kernel roles (192 threads, one CTA per SM, persistent over 128-row x Nt tiles):
+//   warp 0     TMA producer (one elected lane): A and W chunks of 64 k into a ring of stages
+//   warp 1     MMA issuer (one elected lane) and TMEM owner: two accumulator buffers
+//   warps 2-5  epilogue, TMEM lane quadrant = warp % 4
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include <cstring>
+#include <vector>
+
+#include "attention.cuh"
+#include "sm100_ptx.cuh"
+#include "trackfit_internal.h"
+
+using namespace sm100;
+
+namespace {
+
+constexpr int RG_THREADS = 192;
+constexpr int RG_ROWS = 128;                      // rows per tile (MMA M)
+constexpr int RG_KC = 64;                         // k per stage (one 128-byte swizzle row of 16-bit values)
+constexpr int RG_A_BYTES = RG_ROWS * RG_KC * 2;   // 16 KB
+constexpr int RG_MAX_NT = 256;                    // MMA N per tile (two buffers fill the 512 TMEM columns)
+constexpr int RG_SMEM_BUDGET = 200 * 1024;
+constexpr int RG_MAX_STAGES = 8;
+constexpr uint64_t RG_WAIT_NS = 2000000000ull;
+constexpr uint64_t RG_DRAIN_NS = 200000000ull;
+constexpr size_t RG_WS_BUDGET = (size_t)4 << 30;  // workspace bytes of one handle
+
+// epilogues
+enum {
+  EP_F32 = 0,        // out32 = v
+  EP_PROJ = 1,       // out32 = v, sigmoid on the update-gate blocks z_f, z_b (columns [0, H) and [2H, 3H))
+  EP_16 = 2,         // out16 = v
+  EP_SILU16 = 3,     // out16 = SiLU(v)
+  EP_NORM = 4,       // x = v (+ res): out32 = x, out16 = RMSNorm(x) g
+  EP_RES = 5         // out32 = res + v
+};
+
+struct RowGemm {
+  CUtensorMap ta;             // A [cap][K] 16-bit, box 64 x 128, 128-byte swizzle
+  CUtensorMap tw;             // W [N][K] 16-bit, box 64 x Nt, 128-byte swizzle
+  const int64_t* n_rows;      // device: rows of this chunk
+  int K, N, Nt, n_ntiles, kchunks, stages;
+  int epi;
+  int H;                      // EP_PROJ: gate block width
+  uint32_t idesc;
+  const float* bias;          // [N]
+  const float* res;           // EP_NORM (optional), EP_RES: fp32 [rows][N]
+  const float* gain;          // EP_NORM: [N]
+  float rms_eps;
+  float* out32;               // fp32 [rows][N]
+  void* out16;                // 16-bit [rows][N]
+  int fp16;                   // 16-bit format of A, W and out16: 1 fp16, 0 bf16
+  unsigned long long* err;    // [1]: expired bounded waits
+  uint64_t wait_ns;
+};
+
+struct RgBars {
+  uint64_t full[RG_MAX_STAGES], empty[RG_MAX_STAGES];
+  uint64_t acc_full[2], acc_empty[2], drain;
+  uint32_t tmem_base;
+  int abort;
+  int never;                  // a flag nothing sets: for the waits at exit that must not give up on abort
+};
+
+__device__ __forceinline__ float sigm(float x) { return 1.0f / (1.0f + expf(-x)); }
+
+__device__ __forceinline__ uint32_t pack16(float a, float b, int fp16) {   // a -> low half
+  if (fp16) {
+    const __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&h);
+  }
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+}  // namespace
+
+namespace {
+
+// ------------------------------------------------------------------ the GEMM
+// One 16-column chunk of an epilogue: v[i] is column n = nbase + i of this row.
+__device__ __forceinline__ void store16(const RowGemm& g, int64_t row, int nbase, const float (&v)[16]) {
+  if (g.out32) {
+    float4* o = reinterpret_cast<float4*>(g.out32 + row * g.N + nbase);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+  }
+}
+__device__ __forceinline__ void store16_h(const RowGemm& g, int64_t row, int nbase, const float (&v)[16]) {
+  uint4* o = reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(g.out16) + row * g.N + nbase);
+  o[0] = make_uint4(pack16(v[0], v[1], g.fp16), pack16(v[2], v[3], g.fp16), pack16(v[4], v[5], g.fp16),
+                    pack16(v[6], v[7], g.fp16));
+  o[1] = make_uint4(pack16(v[8], v[9], g.fp16), pack16(v[10], v[11], g.fp16), pack16(v[12], v[13], g.fp16),
+                    pack16(v[14], v[15], g.fp16));
+}
+
+// acc + bias (+ res) of 16 columns; the same arithmetic in both passes of EP_NORM
+__device__ __forceinline__ void biased(const RowGemm& g, int64_t row, bool live, int nbase, float (&v)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] += g.bias[nbase + i];
+  if (g.res && live) {
+    const float4* r = reinterpret_cast<const float4*>(g.res + row * g.N + nbase);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float4 a = r[i];
+      v[4 * i] = a.x + v[4 * i];
+      v[4 * i + 1] = a.y + v[4 * i + 1];
+      v[4 * i + 2] = a.z + v[4 * i + 2];
+      v[4 * i + 3] = a.w + v[4 * i + 3];
+    }
+  }
+}
+
+__device__ void rg_fail(const RowGemm& g, RgBars* b) {
+  if (atomicExch(&b->abort, 1) == 0) atomicAdd(g.err + 1, 1ull);
+}
+
+__global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_constant__ RowGemm g) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const int stage_bytes = RG_A_BYTES + g.Nt * 128;
+  RgBars* bars = reinterpret_cast<RgBars*>(smem_raw + (base - raw) + (size_t)g.stages * stage_bytes);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < g.stages; ++s) {
+      mbar_init(smem_u32(&bars->full[s]), 1);
+      mbar_init(smem_u32(&bars->empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&bars->acc_full[b]), 1);
+      mbar_init(smem_u32(&bars->acc_empty[b]), 4);   // one arrival per epilogue warp
+    }
+    mbar_init(smem_u32(&bars->drain), 1);
+    bars->abort = 0;
+    bars->never = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&bars->tmem_base), 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  const int64_t rows = *g.n_rows;
+  const int64_t total = ((rows + RG_ROWS - 1) / RG_ROWS) * g.n_ntiles;
+  volatile int* abort = &bars->abort;
+  volatile int* never = &bars->never;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer
+    uint32_t armed[RG_MAX_STAGES];
+    for (int s = 0; s < RG_MAX_STAGES; ++s) armed[s] = 0;
+    int s = 0;
+    uint32_t ph = 0;
+    for (int64_t t = blockIdx.x; t < total && !*abort; t += gridDim.x) {
+      const int m0 = (int)(t / g.n_ntiles) * RG_ROWS, n0 = (int)(t % g.n_ntiles) * g.Nt;
+      for (int kc = 0; kc < g.kchunks; ++kc) {
+        if (!mbar_wait(smem_u32(&bars->empty[s]), ph ^ 1u, abort, g.wait_ns)) {
+          rg_fail(g, bars);
+          break;
+        }
+        const uint32_t a_s = base + (uint32_t)(s * stage_bytes), fb = smem_u32(&bars->full[s]);
+        mbar_arrive_expect_tx(fb, (uint32_t)stage_bytes);
+        tma_load_2d(a_s, &g.ta, fb, kc * RG_KC, m0);
+        tma_load_2d(a_s + RG_A_BYTES, &g.tw, fb, kc * RG_KC, n0);
+        ++armed[s];
+        if (++s == g.stages) {
+          s = 0;
+          ph ^= 1u;
+        }
+      }
+    }
+    // no copy may land after the CTA has gone: wait for the last phase armed on
+    // every stage (already complete on the normal path)
+    for (int i = 0; i < g.stages; ++i)
+      if (armed[i] && !mbar_wait(smem_u32(&bars->full[i]), (armed[i] - 1) & 1u, never, RG_DRAIN_NS))
+        rg_fail(g, bars);
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer
+    int s = 0;
+    uint32_t ph = 0;
+    int acc_k = 0;
+    bool issued = false;
+    for (int64_t t = blockIdx.x; t < total && !*abort; t += gridDim.x) {
+      const int buf = acc_k & 1;
+      const uint32_t aph = (uint32_t)(acc_k >> 1) & 1u;
+      if (!mbar_wait(smem_u32(&bars->acc_empty[buf]), aph ^ 1u, abort, g.wait_ns)) {
+        rg_fail(g, bars);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d = tmem + (uint32_t)(buf * RG_MAX_NT);
+      bool ok = true;
+      for (int kc = 0; kc < g.kchunks; ++kc) {
+        if (!mbar_wait(smem_u32(&bars->full[s]), ph, abort, g.wait_ns)) {
+          rg_fail(g, bars);
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_s = base + (uint32_t)(s * stage_bytes), w_s = a_s + RG_A_BYTES;
+#pragma unroll
+        for (int k = 0; k < RG_KC / 16; ++k)
+          umma_f16(d, sdesc_sw128(a_s + 32 * k, 16, 1024), sdesc_sw128(w_s + 32 * k, 16, 1024), g.idesc,
+                   (kc | k) ? 1u : 0u);
+        issued = true;
+        umma_commit(smem_u32(&bars->empty[s]));
+        if (++s == g.stages) {
+          s = 0;
+          ph ^= 1u;
+        }
+      }
+      if (!ok) break;
+      umma_commit(smem_u32(&bars->acc_full[buf]));
+      ++acc_k;
+    }
+    // every MMA complete before TMEM is freed
+    if (issued) {
+      umma_commit(smem_u32(&bars->drain));
+      if (!mbar_wait(smem_u32(&bars->drain), 0, never, RG_DRAIN_NS)) rg_fail(g, bars);
+    }
+  } else if (warp >= 2) {
+    // ---------------- epilogue: this warp's 32 rows of each tile
+    const int q = warp & 3;
+    int acc_k = 0;
+    for (int64_t t = blockIdx.x; t < total; t += gridDim.x) {
+      const int buf = acc_k & 1;
+      const uint32_t aph = (uint32_t)(acc_k >> 1) & 1u;
+      if (!mbar_wait(smem_u32(&bars->acc_full[buf]), aph, abort, g.wait_ns)) {
+        if (lane == 0) rg_fail(g, bars);
+        break;
+      }
+      tc_fence_after();
+      const int64_t row = (t / g.n_ntiles) * RG_ROWS + 32 * q + lane;
+      const int n0 = (int)(t % g.n_ntiles) * g.Nt;
+      const bool live = row < rows;
+      const uint32_t tq = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * RG_MAX_NT);
+      if (g.epi == EP_NORM) {
+        float ss = 0.0f;
+        for (int c = 0; c < g.Nt; c += 16) {
+          float v[16];
+          tmem_ld16(tq + c, v);
+          tmem_ld_wait();
+          biased(g, row, live, n0 + c, v);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) ss = fmaf(v[i], v[i], ss);
+          if (live) store16(g, row, n0 + c, v);
+        }
+        const float inv = 1.0f / sqrtf(ss / (float)g.N + g.rms_eps);
+        for (int c = 0; c < g.Nt; c += 16) {
+          float v[16];
+          tmem_ld16(tq + c, v);
+          tmem_ld_wait();
+          biased(g, row, live, n0 + c, v);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) v[i] = v[i] * inv * g.gain[n0 + c + i];
+          if (live) store16_h(g, row, n0 + c, v);
+        }
+      } else {
+        for (int c = 0; c < g.Nt; c += 16) {
+          float v[16];
+          tmem_ld16(tq + c, v);
+          tmem_ld_wait();
+          const int nb = n0 + c;
+          biased(g, row, live, nb, v);
+          if (g.epi == EP_PROJ) {
+            // the update-gate blocks of the projection rows (z_f, n_f, z_b, n_b)
+            const bool z = nb < g.H || (nb >= 2 * g.H && nb < 3 * g.H);
+            if (z) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) v[i] = sigm(v[i]);
+            }
+          } else if (g.epi == EP_SILU16) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = v[i] * sigm(v[i]);
+          }
+          if (live) {
+            if (g.epi == EP_16 || g.epi == EP_SILU16)
+              store16_h(g, row, nb, v);
+            else
+              store16(g, row, nb, v);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty[buf]));
+      ++acc_k;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+}  // namespace
+
+namespace {
+
+// ------------------------------------------------------------------ row plan
+// row0[b] = sum of the valid hit counts of tracks < b (a count outside [1, T]
+// counts 0); row0[B] = the chunk's rows.  Three launches: block totals, one CTA
+// scanning the totals, each block's scan.
+constexpr int PLAN_NT = 1024;
+
+__device__ __forceinline__ int64_t valid_count(const int32_t* n_hits, int64_t b, int64_t B, int T) {
+  if (b >= B) return 0;
+  const int n = n_hits[b];
+  return (n >= 1 && n <= T) ? n : 0;
+}
+
+// inclusive scan of one value per thread over the CTA (PLAN_NT threads)
+__device__ int64_t cta_inclusive_scan(int64_t v, int64_t* warp_tot) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int64_t u = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += u;
+  }
+  if (lane == 31) warp_tot[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    int64_t w = warp_tot[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int64_t u = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += u;
+    }
+    warp_tot[lane] = w;
+  }
+  __syncthreads();
+  const int64_t r = v + (warp ? warp_tot[warp - 1] : 0);
+  __syncthreads();
+  return r;
+}
+
+__global__ void __launch_bounds__(PLAN_NT) plan_totals(const int32_t* __restrict__ n_hits, int64_t B, int T,
+                                                       int64_t* __restrict__ tot) {
+  __shared__ int64_t wt[32];
+  const int64_t b = blockIdx.x * (int64_t)PLAN_NT + threadIdx.x;
+  const int64_t s = cta_inclusive_scan(valid_count(n_hits, b, B, T), wt);
+  if (threadIdx.x == PLAN_NT - 1) tot[blockIdx.x] = s;
+}
+
+__global__ void __launch_bounds__(PLAN_NT) plan_scan_totals(int64_t* __restrict__ tot, int nblk) {
+  __shared__ int64_t wt[32];
+  __shared__ int64_t last;
+  int64_t carry = 0;
+  for (int i0 = 0; i0 < nblk; i0 += PLAN_NT) {   // exclusive scan in place
+    const int i = i0 + threadIdx.x;
+    const int64_t v = i < nblk ? tot[i] : 0;
+    const int64_t s = cta_inclusive_scan(v, wt);
+    if (i < nblk) tot[i] = carry + s - v;
+    if (threadIdx.x == PLAN_NT - 1) last = s;
+    __syncthreads();
+    carry += last;
+    __syncthreads();
+  }
+}
+
+__global__ void __launch_bounds__(PLAN_NT) plan_rows(const int32_t* __restrict__ n_hits, int64_t B, int T,
+                                                     const int64_t* __restrict__ tot, int64_t* __restrict__ row0) {
+  __shared__ int64_t wt[32];
+  const int64_t b = blockIdx.x * (int64_t)PLAN_NT + threadIdx.x;
+  const int64_t v = valid_count(n_hits, b, B, T);
+  const int64_t s = cta_inclusive_scan(v, wt) + tot[blockIdx.x];
+  if (b < B) row0[b] = s - v;
+  if (b == B - 1) row0[B] = s;
+}
+
+// ------------------------------------------------------------------ Fourier rows
+// Sec. 3.2: u = (v - min) / (max - min) per feature, then sin(pi s_k u) and
+// cos(pi s_k u) for the 16 scales, feature-major ([f][sin k, cos k]); the argument
+// s_k u is formed in fp64 and reduced modulo 2 before the fp32 sinpi / cospi.  One
+// thread per (track, hit, feature); the 2 n_fourier values leave as 16-bit
+// operands of the embedding product.  Hit rows: padded hits[b][t] or packed
+// hits[offs[b] + t].
+template <typename T16>
+__global__ void fourier_rows_kernel(const float* __restrict__ hits, const int64_t* __restrict__ offs,
+                                    const int32_t* __restrict__ n_hits, int64_t B, tf_shape s,
+                                    const int64_t* __restrict__ row0, T16* __restrict__ e) {
+  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= B * s.T * s.F) return;
+  const int64_t b = i / (s.T * s.F);
+  const int r = (int)(i - b * s.T * s.F), t = r / s.F, f = r - t * s.F;
+  const int n = n_hits[b];
+  if (n < 1 || n > s.T || t >= n) return;
+  const float v = offs ? hits[(offs[b] + t) * s.F + f] : hits[(b * s.T + t) * s.F + f];
+  const double u = ((double)v - s.feat_min_d[f]) / s.feat_range_d[f];
+  float sv[TRACKFIT_MAX_FOURIER], cv[TRACKFIT_MAX_FOURIER];
+#pragma unroll
+  for (int k = 0; k < TRACKFIT_MAX_FOURIER; ++k) {
+    double a = u * (double)s.scale[k];
+    a -= 2.0 * rint(0.5 * a);
+    const float af = (float)a;
+    sv[k] = sinpif(af);
+    cv[k] = cospif(af);
+  }
+  T16* o = e + (row0[b] + t) * s.E + f * 2 * TRACKFIT_MAX_FOURIER;
+#pragma unroll
+  for (int k = 0; k < TRACKFIT_MAX_FOURIER; ++k) {
+    tf_attn::put(o + k, sv[k]);
+    tf_attn::put(o + TRACKFIT_MAX_FOURIER + k, cv[k]);
+  }
+}
+
+// ------------------------------------------------------------------ scans
+// The two gated scans of one concatenation layer (Sec. 3.2, Eq. 2) over each
+// track's rows: h_t = (1 - z_t) h_{t-1} + z_t n_t forward, the same backward with
+// the reverse gates; z already through the sigmoid.  One thread per (track,
+// channel).  y16 (optional): the concatenated states [h_f | h_b] per row as the
+// next layer's 16-bit operand.  pooled (optional, the last layer): endpoints, the
+// forward state at the last hit and the reverse state at the first, or the mean
+// of [h_f | h_b] over the hits.
+template <typename T16>
+__global__ void concat_scan_rows_kernel(const float* __restrict__ pr, const int64_t* __restrict__ row0,
+                                        const int32_t* __restrict__ n_hits, int64_t B, int T, int H,
+                                        T16* __restrict__ y16, float* __restrict__ pooled, int pool) {
+  const int64_t b = blockIdx.x;
+  const int c = blockIdx.y * blockDim.x + threadIdx.x;
+  if (b >= B || c >= H) return;
+  const int n = n_hits[b];
+  if (n < 1 || n > T) return;
+  const int64_t r0 = row0[b];
+  const int ldp = 4 * H;
+  float h = 0.0f, sum = 0.0f;
+  for (int t = 0; t < n; ++t) {
+    const float* p = pr + (r0 + t) * ldp;
+    h = fmaf(p[c], p[H + c] - h, h);
+    if (y16) tf_attn::put(y16 + (r0 + t) * 2 * H + c, h);
+    sum += h;
+  }
+  if (pooled) pooled[b * 2 * H + c] = pool == TRACKFIT_POOL_ENDPOINTS ? h : sum / (float)n;
+  h = 0.0f;
+  sum = 0.0f;
+  for (int t = n - 1; t >= 0; --t) {
+    const float* p = pr + (r0 + t) * ldp;
+    h = fmaf(p[2 * H + c], p[3 * H + c] - h, h);
+    if (y16) tf_attn::put(y16 + (r0 + t) * 2 * H + H + c, h);
+    sum += h;
+  }
+  if (pooled) pooled[b * 2 * H + H + c] = pool == TRACKFIT_POOL_ENDPOINTS ? h : sum / (float)n;
+}
+
+// Mean over each track's rows of the last layer's output x [rows][D] (the
+// Transformer's readout); one thread per (track, channel), hits in order.
+__global__ void pool_mean_rows_kernel(const float* __restrict__ x, const int64_t* __restrict__ row0,
+                                      const int32_t* __restrict__ n_hits, int64_t B, int T, int D,
+                                      float* __restrict__ pooled) {
+  const int64_t b = blockIdx.x;
+  const int c = blockIdx.y * blockDim.x + threadIdx.x;
+  if (b >= B || c >= D) return;
+  const int n = n_hits[b];
+  if (n < 1 || n > T) return;
+  const int64_t r0 = row0[b];
+  float acc = 0.0f;
+  for (int t = 0; t < n; ++t) acc += x[(r0 + t) * D + c];
+  pooled[b * D + c] = acc / (float)n;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ host side
+struct tf_rows_state {
+  int fp16;
+  int nsm;
+  uint16_t* w16;            // every product's weights, 16-bit, back to back
+  int64_t chunk, cap;       // tracks per chunk; rows of the workspace (chunk * max_hits)
+  int64_t* row0;            // [chunk + 1]
+  int64_t* tot;             // [chunk / 1024 + 1]
+  uint16_t *a0, *hs16, *xy16, *o16;
+  float *p32, *x32, *x1, *pooled;
+  RowGemm e1, e2;
+  RowGemm lay[TF_MAX_LAYERS][4];
+  size_t smem;
+  uint64_t wait_ns;
+};
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 rows_encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 16-bit matrix [rows][cols] row-major -> tensor map of 64-column x box_rows boxes
+// with 128-byte swizzle (out-of-range elements read as zero).
+bool rows_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows, int fp16) {
+  auto fn = rows_encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, fp16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr),
+            dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The MMA N of one tile: N itself up to 256, else the smallest equal split into
+// multiples of 16 (0 if there is none).
+int tile_n(int N) {
+  for (int parts = (N + RG_MAX_NT - 1) / RG_MAX_NT; parts <= N / 16; ++parts)
+    if (N % parts == 0 && (N / parts) % 16 == 0) return N / parts;
+  return 0;
+}
+
+size_t gemm_smem(const RowGemm& g) {
+  return 1024 + (size_t)g.stages * (RG_A_BYTES + g.Nt * 128) + sizeof(RgBars);
+}
+
+// A [cap][K] (16-bit, row stride K) times W [N][K]; the epilogue's pointers are set by the caller.
+bool make_gemm(RowGemm& g, const tf_rows_state* r, const void* A, int K, const uint16_t* W, int N, int epi) {
+  std::memset(&g, 0, sizeof(g));
+  g.K = K;
+  g.N = N;
+  g.Nt = tile_n(N);
+  if (!g.Nt || (K % 8) != 0) return false;
+  g.n_ntiles = N / g.Nt;
+  g.kchunks = (K + RG_KC - 1) / RG_KC;
+  const int stage = RG_A_BYTES + g.Nt * 128;
+  g.stages = (int)((RG_SMEM_BUDGET - 1024 - (int)sizeof(RgBars)) / stage);
+  if (g.stages > RG_MAX_STAGES) g.stages = RG_MAX_STAGES;
+  if (g.stages < 2) return false;
+  g.epi = epi;
+  g.idesc = idesc_f16(RG_ROWS, g.Nt, r->fp16 ? 0u : 1u, false, false);
+  g.fp16 = r->fp16;
+  g.wait_ns = RG_WAIT_NS;
+  return rows_map(&g.ta, A, (uint64_t)r->cap, (uint64_t)K, RG_ROWS, r->fp16) &&
+         rows_map(&g.tw, W, (uint64_t)N, (uint64_t)K, (uint32_t)g.Nt, r->fp16);
+}
+
+int launch_gemm(const tf_rows_state* r, RowGemm& g, const int64_t* n_rows, unsigned long long* err,
+                cudaStream_t st) {
+  g.n_rows = n_rows;
+  g.err = err;
+  g.wait_ns = r->wait_ns;
+  row_gemm_kernel<<<r->nsm, RG_THREADS, gemm_smem(g), st>>>(g);
+  return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
+}
+
+uint16_t to16(float f, int fp16) {
+  if (fp16) {
+    const __half v = __float2half_rn(f);
+    return *reinterpret_cast<const uint16_t*>(&v);
+  }
+  const __nv_bfloat16 v = __float2bfloat16_rn(f);
+  return *reinterpret_cast<const uint16_t*>(&v);
+}
+
+}  // namespace
+
+bool tf_rows_supported(const tf_shape& s) {
+  if (s.precision != TRACKFIT_BF16_PROJ && s.precision != TRACKFIT_FP16_PROJ) return false;
+  if (s.topology != TRACKFIT_TOPOLOGY_CONCAT && s.topology != TRACKFIT_TOPOLOGY_ATTENTION) return false;
+  if (tile_n(s.D) != s.D) return false;   // the row-wide epilogues need a whole row in one tile
+  // CONCAT: the sigmoid of the update-gate blocks is chosen per 16 columns
+  if (s.topology == TRACKFIT_TOPOLOGY_CONCAT) return (s.H % 16) == 0 && tile_n(4 * s.H) != 0;
+  return tile_n(3 * s.D) != 0 && tile_n(s.H) != 0;
+}
+
+void tf_rows_destroy(trackfit_ctx* h) {
+  tf_rows_state* r = h->rows;
+  if (!r) return;
+  tf_free(r->w16);
+  tf_free(r->row0);
+  tf_free(r->tot);
+  tf_free(r->a0);
+  tf_free(r->hs16);
+  tf_free(r->xy16);
+  tf_free(r->o16);
+  tf_free(r->p32);
+  tf_free(r->x32);
+  tf_free(r->x1);
+  tf_free(r->pooled);
+  delete r;
+  h->rows = nullptr;
+}
+
+int tf_rows_wait_limit(trackfit_ctx* h, int64_t limit_ns) {
+  if (!h->rows) return TRACKFIT_ERR_UNSUPPORTED;
+  h->rows->wait_ns = limit_ns > 0 ? (uint64_t)limit_ns : RG_WAIT_NS;
+  return TRACKFIT_OK;
+}
+
+int tf_rows_create(trackfit_ctx* h, const float* host_w) {
+  const tf_shape& s = h->s;
+  const tf_blob_off& o = h->off;
+  tf_rows_state* r = new (std::nothrow) tf_rows_state();
+  if (!r) return TRACKFIT_ERR_OOM;
+  h->rows = r;   // freed by tf_rows_destroy on any failure below
+  r->fp16 = s.precision == TRACKFIT_FP16_PROJ;
+  r->wait_ns = RG_WAIT_NS;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&r->nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return TRACKFIT_ERR_CUDA;
+  const bool attn = s.topology == TRACKFIT_TOPOLOGY_ATTENTION;
+  const size_t D = s.D, H = s.H, E = s.E;
+  // the 16-bit weights of every product: (blob offset, N, K)
+  struct Mat { size_t off, n, k, at; };
+  std::vector<Mat> mats;
+  mats.push_back({o.emb_w1, D, E, 0});
+  mats.push_back({o.emb_w2, D, D, 0});
+  for (int l = 0; l < s.L; ++l) {
+    const tf_layer_off& lo = o.layer[l];
+    if (attn) {
+      mats.push_back({lo.w_in, 3 * D, D, 0});
+      mats.push_back({lo.w_m, D, D, 0});
+      mats.push_back({lo.w1, H, D, 0});
+      mats.push_back({lo.w2, D, H, 0});
+    } else {
+      mats.push_back({lo.w_in, 4 * H, l == 0 ? D : 2 * H, 0});
+    }
+  }
+  size_t n16 = 0;
+  for (Mat& m : mats) {
+    m.at = n16;
+    n16 += (m.n * m.k + 63) / 64 * 64;   // 128-byte aligned starts
+  }
+  std::vector<uint16_t> w(n16, 0);
+  for (const Mat& m : mats)
+    for (size_t i = 0; i < m.n * m.k; ++i) w[m.at + i] = to16(host_w[m.off + i], r->fp16);
+  int st = tf_status_from_cuda(tf_malloc((void**)&r->w16, n16 * 2));
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(r->w16, w.data(), n16 * 2, cudaMemcpyHostToDevice));
+  if (st != TRACKFIT_OK) return st;
+  // workspace, sized for whole chunks of full-length tracks
+  const size_t hsw = attn ? (H > D ? H : D) : D;
+  const size_t xyw = attn ? D : (2 * H > D ? 2 * H : D);
+  const size_t pw = attn ? 3 * D : 4 * H;
+  const size_t row_bytes = 2 * (E + hsw + xyw + (attn ? D : 0)) + 4 * (pw + (attn ? 2 * D : 0));
+  const size_t track_bytes = (size_t)s.T * row_bytes + 4 * (size_t)s.P + 16;
+  int64_t chunk = (int64_t)(RG_WS_BUDGET / track_bytes);
+  if (chunk > 4194304) chunk = 4194304;
+  chunk = chunk / PLAN_NT * PLAN_NT;
+  if (chunk < PLAN_NT) return TRACKFIT_ERR_UNSUPPORTED;
+  r->chunk = chunk;
+  r->cap = chunk * s.T;
+  const size_t cap = (size_t)r->cap;
+  auto alloc = [&](void** p, size_t bytes) {
+    if (st == TRACKFIT_OK) st = tf_status_from_cuda(tf_malloc(p, bytes));
+  };
+  alloc((void**)&r->row0, (chunk + 1) * sizeof(int64_t));
+  alloc((void**)&r->tot, (chunk / PLAN_NT + 1) * sizeof(int64_t));
+  alloc((void**)&r->a0, cap * E * 2);
+  alloc((void**)&r->hs16, cap * hsw * 2);
+  alloc((void**)&r->xy16, cap * xyw * 2);
+  alloc((void**)&r->p32, cap * pw * 4);
+  alloc((void**)&r->pooled, (size_t)chunk * s.P * 4);
+  if (attn) {
+    alloc((void**)&r->o16, cap * D * 2);
+    alloc((void**)&r->x32, cap * D * 4);
+    alloc((void**)&r->x1, cap * D * 4);
+  }
+  if (st != TRACKFIT_OK) return st;
+  // the products of one chunk
+  const float* Wd = h->d_w;
+  const uint16_t* w16 = r->w16;
+  size_t mi = 0;
+  bool ok = make_gemm(r->e1, r, r->a0, (int)E, w16 + mats[mi++].at, (int)D, EP_SILU16);
+  r->e1.bias = Wd + o.emb_b1;
+  r->e1.out16 = r->hs16;
+  ok = ok && make_gemm(r->e2, r, r->hs16, (int)D, w16 + mats[mi++].at, (int)D, attn ? EP_NORM : EP_16);
+  r->e2.bias = Wd + o.emb_b2;
+  r->e2.out16 = r->xy16;
+  if (attn) {   // x = embedding; the first layer's pre-norm operand
+    r->e2.out32 = r->x32;
+    r->e2.gain = Wd + o.layer[0].g;
+    r->e2.rms_eps = s.rms_eps;
+  }
+  for (int l = 0; l < s.L && ok; ++l) {
+    const tf_layer_off& lo = o.layer[l];
+    RowGemm* g = r->lay[l];
+    if (!attn) {   // Sec. 3.2: the layer input (D, then 2H wide) to z_f, n_f, z_b, n_b
+      ok = make_gemm(g[0], r, r->xy16, l == 0 ? (int)D : (int)(2 * H), w16 + mats[mi++].at, (int)(4 * H), EP_PROJ);
+      g[0].H = (int)H;
+      g[0].bias = Wd + lo.b_in;
+      g[0].out32 = r->p32;
+      continue;
+    }
+    // App. A.3: qkv of the normed stream; x' = x + W_o o + b_o and its pre-norm;
+    // SiLU(W_1 .. + b_1); x = x' + W_2 u + b_2 and the next layer's pre-norm
+    ok = make_gemm(g[0], r, r->xy16, (int)D, w16 + mats[mi++].at, (int)(3 * D), EP_F32) &&
+         make_gemm(g[1], r, r->o16, (int)D, w16 + mats[mi++].at, (int)D, EP_NORM) &&
+         make_gemm(g[2], r, r->xy16, (int)D, w16 + mats[mi++].at, (int)H, EP_SILU16) &&
+         make_gemm(g[3], r, r->hs16, (int)H, w16 + mats[mi++].at, (int)D, l + 1 < s.L ? EP_NORM : EP_RES);
+    g[0].bias = Wd + lo.b_in;
+    g[0].out32 = r->p32;
+    g[1].bias = Wd + lo.b_m;
+    g[1].res = r->x32;
+    g[1].gain = Wd + lo.g2;
+    g[1].rms_eps = s.rms_eps;
+    g[1].out32 = r->x1;
+    g[1].out16 = r->xy16;
+    g[2].bias = Wd + lo.b1;
+    g[2].out16 = r->hs16;
+    g[3].bias = Wd + lo.b2;
+    g[3].res = r->x1;
+    g[3].out32 = r->x32;
+    if (l + 1 < s.L) {
+      g[3].gain = Wd + o.layer[l + 1].g;
+      g[3].rms_eps = s.rms_eps;
+      g[3].out16 = r->xy16;
+    }
+  }
+  if (!ok) return TRACKFIT_ERR_CUDA;
+  r->smem = gemm_smem(r->e1);
+  auto upd = [&](const RowGemm& g) { r->smem = gemm_smem(g) > r->smem ? gemm_smem(g) : r->smem; };
+  upd(r->e2);
+  for (int l = 0; l < s.L; ++l)
+    for (int k = 0; k < (attn ? 4 : 1); ++k) upd(r->lay[l][k]);
+  if (cudaFuncSetAttribute(row_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r->smem) != cudaSuccess)
+    return TRACKFIT_ERR_CUDA;
+  if (attn) {
+    const int ab = (int)tf_attn::smem_bytes(s.T, s.D);
+    if (cudaFuncSetAttribute(tf_attn::track_attention_kernel<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ab) != cudaSuccess ||
+        cudaFuncSetAttribute(tf_attn::track_attention_kernel<__nv_bfloat16>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, ab) != cudaSuccess)
+      return TRACKFIT_ERR_CUDA;
+  }
+  return TRACKFIT_OK;
+}
+
+namespace {
+
+template <typename T16>
+int rows_chunk(trackfit_ctx* h, const float* hits, const int64_t* offs, const int32_t* nc, int64_t nb, float* out,
+               float* out_q, float* out_pool, cudaStream_t st) {
+  tf_rows_state* r = h->rows;
+  const tf_shape& s = h->s;
+  unsigned long long* err = h->d_err;
+  const bool attn = s.topology == TRACKFIT_TOPOLOGY_ATTENTION;
+  const int nblk = (int)((nb + PLAN_NT - 1) / PLAN_NT);
+  plan_totals<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot);
+  plan_scan_totals<<<1, PLAN_NT, 0, st>>>(r->tot, nblk);
+  plan_rows<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot, r->row0);
+  const int64_t* nrows = r->row0 + nb;
+  const int64_t nf = nb * s.T * s.F;
+  fourier_rows_kernel<T16><<<(unsigned)((nf + 255) / 256), 256, 0, st>>>(hits, offs, nc, nb, s, r->row0,
+                                                                         reinterpret_cast<T16*>(r->a0));
+  if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  if (launch_gemm(r, r->e1, nrows, err, st) || launch_gemm(r, r->e2, nrows, err, st)) return TRACKFIT_ERR_CUDA;
+  for (int l = 0; l < s.L; ++l) {
+    RowGemm* g = r->lay[l];
+    if (!attn) {
+      if (launch_gemm(r, g[0], nrows, err, st)) return TRACKFIT_ERR_CUDA;
+      const bool last = l + 1 == s.L;
+      dim3 grid((unsigned)nb, (unsigned)((s.H + 127) / 128));
+      concat_scan_rows_kernel<T16><<<grid, 128, 0, st>>>(r->p32, r->row0, nc, nb, s.T, s.H,
+                                                         last ? nullptr : reinterpret_cast<T16*>(r->xy16),
+                                                         last ? r->pooled : nullptr, s.pool);
+      continue;
+    }
+    if (launch_gemm(r, g[0], nrows, err, st)) return TRACKFIT_ERR_CUDA;
+    tf_attn::track_attention_kernel<T16><<<(unsigned)nb, tf_attn::THREADS, tf_attn::smem_bytes(s.T, s.D), st>>>(
+        r->p32, 3 * s.D, r->row0, nc, nb, s.T, s.D, s.NH, reinterpret_cast<T16*>(r->o16), s.D);
+    if (launch_gemm(r, g[1], nrows, err, st) || launch_gemm(r, g[2], nrows, err, st) ||
+        launch_gemm(r, g[3], nrows, err, st))
+      return TRACKFIT_ERR_CUDA;
+  }
+  if (attn) {
+    dim3 grid((unsigned)nb, (unsigned)((s.D + 127) / 128));
+    pool_mean_rows_kernel<<<grid, 128, 0, st>>>(r->x32, r->row0, nc, nb, s.T, s.D, r->pooled);
+  }
+  if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
+  return tf_simt_head(s, h->off, h->d_w, r->pooled, nc, nb, out, out_q, out_pool, err, st);
+}
+
+}  // namespace
+
+int tf_rows_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out,
+                    float* out_q, float* out_pool, cudaStream_t st, const int64_t* offs) {
+  tf_rows_state* r = h->rows;
+  const tf_shape& s = h->s;
+  for (int64_t c0 = 0; c0 < B; c0 += r->chunk) {
+    const int64_t nb = B - c0 < r->chunk ? B - c0 : r->chunk;
+    const float* hc = offs ? hits : hits + c0 * s.T * s.F;
+    const int64_t* oc = offs ? offs + c0 : nullptr;
+    if (h->prof_on) tf_prof_begin(h, st);
+    const int e = r->fp16 ? rows_chunk<__half>(h, hc, oc, n_hits + c0, nb, out + c0 * 5,
+                                               out_q ? out_q + c0 * s.Q : nullptr,
+                                               out_pool ? out_pool + c0 * s.P : nullptr, st)
+                          : rows_chunk<__nv_bfloat16>(h, hc, oc, n_hits + c0, nb, out + c0 * 5,
+                                                      out_q ? out_q + c0 * s.Q : nullptr,
+                                                      out_pool ? out_pool + c0 * s.P : nullptr, st);
+    if (h->prof_on) tf_prof_end(h, st);
+    if (e != TRACKFIT_OK) return e;
+  }
+  return TRACKFIT_OK;
+}

@@ -204,8 +204,11 @@ __global__ void linear_scan_kernel(const float* __restrict__ a, const float* __r
   }
 }
 
-// Pooling and head (Sec. 3.2-3.3): one 128-thread block per track.
-__global__ void __launch_bounds__(128) pool_head_kernel(const float* __restrict__ x, const float* __restrict__ y,
+// Pooling and head (Sec. 3.2-3.3): one 128-thread block per track.  With
+// pooled_in the pooled vectors [B][P] are given (the packed-row path pools in its
+// scan or pooling kernel) and x, y are not read.
+__global__ void __launch_bounds__(128) pool_head_kernel(const float* __restrict__ pooled_in,
+                                                        const float* __restrict__ x, const float* __restrict__ y,
                                                         const int32_t* __restrict__ n_hits, int64_t B, tf_shape s,
                                                         const float* __restrict__ gh, const float* __restrict__ w1,
                                                         const float* __restrict__ b1, const float* __restrict__ w2,
@@ -225,7 +228,9 @@ __global__ void __launch_bounds__(128) pool_head_kernel(const float* __restrict_
     if (tid == 0) atomicAdd(err, 1ull);
     n = 1;
   }
-  if (s.pool == TRACKFIT_POOL_MEAN) {   // x: [rows][P] (P = D, or 2H for CONCAT)
+  if (pooled_in) {
+    for (int c = tid; c < P; c += blockDim.x) pv[c] = bad ? 0.0f : pooled_in[b * P + c];
+  } else if (s.pool == TRACKFIT_POOL_MEAN) {   // x: [rows][P] (P = D, or 2H for CONCAT)
     for (int c = tid; c < P; c += blockDim.x) {
       float acc = 0.0f;
       for (int t = 0; t < n; ++t) acc += x[(b * T + t) * P + c];
@@ -398,7 +403,7 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
     }
     // mean pooling reads the last layer's output: X (MERGE) or the states Y (CONCAT)
     const float* xm = s.topology == TRACKFIT_TOPOLOGY_CONCAT ? Y : X;
-    pool_head_kernel<<<(unsigned)nb, 128, 0, st>>>(xm, Y, nc, nb, s, W + o.head_g, W + o.head_w1, W + o.head_b1,
+    pool_head_kernel<<<(unsigned)nb, 128, 0, st>>>(nullptr, xm, Y, nc, nb, s, W + o.head_g, W + o.head_w1, W + o.head_b1,
                                                     W + o.head_w2, W + o.head_b2, out + c0 * 5,
                                                     out_q ? out_q + c0 * s.Q : nullptr,
                                                     out_pool ? out_pool + c0 * s.P : nullptr, err);
@@ -430,3 +435,14 @@ int tf_simt_forward_explicit(const tf_shape& s, const tf_blob_off& o, const floa
 }
 
 size_t tf_simt_bytes_per_track(const tf_shape& s) { return ws_floats_per_track(s) * sizeof(float); }
+
+// The head of Sec. 3.2-3.3 on given pooled vectors [B][P]: out [B][5], optional
+// quantiles [B][Q] and the pooled export (NaN rows for invalid tracks).
+int tf_simt_head(const tf_shape& s, const tf_blob_off& o, const float* W, const float* pooled,
+                 const int32_t* n_hits, int64_t B, float* out, float* out_q, float* out_pool,
+                 unsigned long long* err, cudaStream_t st) {
+  pool_head_kernel<<<(unsigned)B, 128, 0, st>>>(pooled, nullptr, nullptr, n_hits, B, s, W + o.head_g, W + o.head_w1,
+                                                 W + o.head_b1, W + o.head_w2, W + o.head_b2, out, out_q, out_pool,
+                                                 err);
+  return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
+}

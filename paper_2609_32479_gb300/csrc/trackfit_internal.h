@@ -35,9 +35,10 @@ struct tf_shape {
   float scale[TRACKFIT_MAX_FOURIER];
 };
 
-struct tf_tc_state;  // tcgen05 path (tc_forward.cu)
+struct tf_tc_state;    // tcgen05 fused path (tc_forward.cu)
+struct tf_rows_state;  // tcgen05 packed-row path (rows.cu)
 
-enum { TF_PATH_SIMT = 0, TF_PATH_TC = 1 };
+enum { TF_PATH_SIMT = 0, TF_PATH_TC = 1, TF_PATH_ROWS = 2 };
 
 struct trackfit_ctx {
   trackfit_config_t cfg;
@@ -62,6 +63,7 @@ struct trackfit_ctx {
   cudaEvent_t cp_ev[TF_HOST_EVENTS];
   int cp_nev;
   tf_tc_state* tc;
+  tf_rows_state* rows;
   // optional timing of the main compute kernel (trackfit_profile)
   int prof_on;
   int prof_n;
@@ -79,6 +81,9 @@ int tf_simt_workspace(trackfit_ctx* h);
 // offs (may be null): packed input, track b's hits are rows offs[b] .. of hits
 int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B,
                     float* out, float* out_q, float* out_pool, cudaStream_t st, const int64_t* offs = nullptr);
+int tf_simt_head(const tf_shape& s, const tf_blob_off& o, const float* W, const float* pooled,
+                 const int32_t* n_hits, int64_t B, float* out, float* out_q, float* out_pool,
+                 unsigned long long* err, cudaStream_t st);
 int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits,
                        int64_t B, int T, int C, float* hf, float* hb, cudaStream_t st);
 
@@ -92,6 +97,14 @@ int tf_tc_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int
 
 int tf_tc_wait_limit(trackfit_ctx* h, int64_t limit_ns, int hold_tile);
 int tf_tc_probe(trackfit_ctx* h, const uint16_t* A, const uint16_t* Bkn, int K, float* D, cudaStream_t st);
+
+// rows.cu
+bool tf_rows_supported(const tf_shape& s);
+int tf_rows_create(trackfit_ctx* h, const float* host_w);
+void tf_rows_destroy(trackfit_ctx* h);
+int tf_rows_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, int64_t B, float* out,
+                    float* out_q, float* out_pool, cudaStream_t st, const int64_t* offs = nullptr);
+int tf_rows_wait_limit(trackfit_ctx* h, int64_t limit_ns);
 
 // api.cu
 int tf_status_from_cuda(cudaError_t e);

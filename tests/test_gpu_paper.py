@@ -37,9 +37,11 @@ def oracle_inputs(w, tb):
     return h, seed
 
 
-def gpu_encoder(T, model, blob, hits, n_hits):
+def gpu_encoder(T, model, blob, hits, n_hits, path=None):
     dev = torch.device("cuda:0")
     with T.Trackfit(model, blob) as tf:
+        if path is not None:
+            tf.set_path(path)
         B = len(n_hits)
         out = torch.full((B, 5), -7.0, device=dev)
         q = torch.empty((B, 5, model.n_quantiles), device=dev)
@@ -52,14 +54,18 @@ def gpu_encoder(T, model, blob, hits, n_hits):
     return out.cpu().numpy(), q.cpu().numpy(), path
 
 
-@pytest.mark.parametrize("prec", [W.PRECISION_FP32, W.PRECISION_FP16])
-def test_paper_encoder_matches_the_oracle(T, prec):
+# (operand precision, path): fp32 runs on the CUDA cores; fp16 on the packed-row
+# tensor-core path by default and on the CUDA cores when asked (set_path 1)
+@pytest.mark.parametrize("prec,path,want", [(W.PRECISION_FP32, None, "simt"), (W.PRECISION_FP16, None, "tcgen05-rows"),
+                                            (W.PRECISION_FP16, 1, "simt")])
+def test_paper_encoder_matches_the_oracle(T, prec, path, want):
     w = W.workload("paper", n_tracks=1000, precision=prec)
     tb = W.gen_tracks(w)
     hits, _ = oracle_inputs(w, tb)
     blob = W.gen_weights(w.model, w.weight_seed)
-    got, q, path = gpu_encoder(T, w.model, blob, hits, tb.n_hits)
-    assert path.startswith("simt")
+    got, q, used = gpu_encoder(T, w.model, blob, hits, tb.n_hits, path)
+    assert used.startswith(want), used
+    path = used
     cap = {}
     ref = O.forward(dataclasses.asdict(w.model), blob, hits, tb.n_hits, capture=cap)
     ok, msg = parity_ok(got, ref, prec)

@@ -59,14 +59,18 @@ def run(T, model, blob, hits, n_hits, path=None, packed=False):
     return out.cpu().numpy(), q.cpu().numpy(), pooled.cpu().numpy(), st, used
 
 
-@pytest.mark.parametrize("prec", [W.PRECISION_FP32, W.PRECISION_FP16])
-def test_transformer_matches_the_oracle(T, prec):
+# fp32 runs on the CUDA cores; fp16 on the packed-row tensor-core path by
+# default and on the CUDA cores when asked (set_path 1)
+@pytest.mark.parametrize("prec,force,want", [(W.PRECISION_FP32, None, "simt"), (W.PRECISION_FP16, None, "tcgen05-rows"),
+                                             (W.PRECISION_FP16, 1, "simt")])
+def test_transformer_matches_the_oracle(T, prec, force, want):
     w = W.workload("transformer", n_tracks=600, precision=prec)
     tb = W.gen_tracks(w)
     hits = inputs(w, tb)
     blob = W.gen_weights(w.model, w.weight_seed)
-    got, q, pooled, st, path = run(T, w.model, blob, hits, tb.n_hits)
+    got, q, pooled, st, path = run(T, w.model, blob, hits, tb.n_hits, path=force)
     assert st == (T.OK, 0)
+    assert path.startswith(want), path
     cap = {}
     ref = O.forward(dataclasses.asdict(w.model), blob, hits, tb.n_hits, capture=cap)
     ok, msg = parity_ok(got, ref, prec)
@@ -78,11 +82,14 @@ def test_transformer_matches_the_oracle(T, prec):
     assert ok, msg
 
 
-def test_long_tracks_and_wide_heads(T):
+@pytest.mark.parametrize("prec", [W.PRECISION_FP32, W.PRECISION_FP16])
+def test_long_tracks_and_wide_heads(T, prec):
     """64 hits per track at d_model 128 (the attention CTA stages 64 x 257 floats,
-    66 KB of shared memory), 2 heads of width 64, and a one-hit track."""
+    66 KB of shared memory), 2 heads of width 64, and a one-hit track; fp32 on the
+    CUDA cores, fp16 on the packed-row tensor-core path (MLP width 256: one
+    256-column tile; q, k, v: two tiles of 192)."""
     m = W.ModelConfig(max_hits=64, d_model=128, d_hidden=256, n_layers=2, topology=W.TOPOLOGY_ATTENTION,
-                      n_heads=2)
+                      n_heads=2, precision=prec)
     w = W.Workload("long", 120, m, layout="sweep", n_barrel=64, min_hits=64)
     tb = W.gen_tracks(w)
     n = tb.n_hits.copy()
@@ -92,8 +99,8 @@ def test_long_tracks_and_wide_heads(T):
     got, _, _, st, _ = run(T, m, blob, tb.hits, n)
     assert st == (T.OK, 0)
     ref = O.forward(dataclasses.asdict(m), blob, tb.hits, n)
-    ok, msg = parity_ok(got, ref, 0)
-    print(f"long tracks: {msg}")
+    ok, msg = parity_ok(got, ref, prec)
+    print(f"long tracks, precision {prec}: {msg}")
     assert ok, msg
 
 
