@@ -218,18 +218,21 @@ int trackfit_forward_host(trackfit_t h, const float* hits_host, const int32_t* n
 int trackfit_device_errors(trackfit_t h, void* stream, int64_t* n_bad);
 
 /* Name of the kernel path the handle runs: "simt-fp32", "simt-bf16",
- * "simt-fp16", "tcgen05-bf16" or "tcgen05-fp16".  Static string, owned by the
- * library. */
+ * "simt-fp16", "tcgen05-bf16", "tcgen05-fp16", "tcgen05-rows-bf16" or
+ * "tcgen05-rows-fp16".  Static string, owned by the library. */
 const char* trackfit_path_name(trackfit_t h);
 
-/* Select the kernel path: 0 = automatic (tcgen05 for the BF16_PROJ / FP16_PROJ
- * configs it supports: mean pooling, d_model 128 or 256; SIMT otherwise), 1 = force the SIMT path.  Returns UNSUPPORTED if the
- * requested path cannot run this configuration. */
+/* Select the kernel path: 0 = automatic (the fused tcgen05 path for the
+ * BF16_PROJ / FP16_PROJ MERGE configs it supports: mean pooling, d_model 128 or
+ * 256; the packed-row tcgen05 path for 16-bit CONCAT and ATTENTION configs; SIMT
+ * otherwise), 1 = force the SIMT path.  Returns UNSUPPORTED if the requested path
+ * cannot run this configuration. */
 int trackfit_set_path(trackfit_t h, int path);
 
 /* Timing hook: with enable = 1 every forward records CUDA events on its stream
- * around the main compute kernel (the fused tcgen05 kernel, or the SIMT layer
- * sequence); trackfit_profile_read synchronises on them, returns the summed
+ * around the main compute kernel (the fused tcgen05 kernel, every product
+ * launch of the packed-row tcgen05 path, or the SIMT layer sequence);
+ * trackfit_profile_read synchronises on them, returns the summed
  * kernel time in milliseconds and the number of timed launches since the last
  * read, and resets both.  enable = 0 releases the events. */
 int trackfit_profile(trackfit_t h, int enable);

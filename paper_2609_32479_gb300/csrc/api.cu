@@ -100,7 +100,9 @@ static bool derive(const trackfit_config_t* c, tf_shape* s, tf_blob_off* o) {
   s->rms_eps = c->rms_eps;
   for (int f = 0; f < s->F; ++f) {
     s->feat_min[f] = c->feat_min[f];
-    s->feat_inv_range[f] = (float)(1.0 / ((double)c->feat_max[f] - (double)c->feat_min[f]));
+    const double inv = 1.0 / ((double)c->feat_max[f] - (double)c->feat_min[f]);
+    s->feat_inv_range[f] = (float)inv;
+    s->feat_inv_lo[f] = (float)(inv - (double)s->feat_inv_range[f]);
     s->feat_min_d[f] = c->feat_min[f];
     s->feat_range_d[f] = (double)c->feat_max[f] - (double)c->feat_min[f];
   }

@@ -5,6 +5,12 @@
 //   o_t = sum_j softmax_j(q_t . k_j / sqrt(dh)) v_j.
 // q, k, v are the fp32 outputs of the qkv projection; scores, softmax and the
 // weighted sum run in fp32.
+//
+// One CTA per track stages the track's q, k, v rows in shared memory; warp w
+// takes heads w, w + 4, ...; lane i takes queries i and i + 32 and keeps its
+// query and its output (dh values each) in registers, so every key and value is
+// a broadcast read of shared memory.  The softmax takes two passes over the keys:
+// the maximum score, then the exponentials, their sum and the weighted values.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -17,33 +23,46 @@ __device__ __forceinline__ void put(float* p, float v) { *p = v; }
 __device__ __forceinline__ void put(__half* p, float v) { *p = __float2half_rn(v); }
 __device__ __forceinline__ void put(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
 
-constexpr int THREADS = 128;   // 4 warps; warp w takes heads w, w + 4, ...
+constexpr int THREADS = 128;
 
-// Dynamic shared memory of one CTA: the track's keys and values, T rows of 2 D + 1
-// floats (the odd row stride puts key j's channel c in bank (j + c) mod 32).
-__host__ __device__ inline size_t smem_bytes(int T, int D) { return (size_t)T * (2 * D + 1) * sizeof(float); }
+// Shared memory of one CTA: T rows of 3 D + 4 floats (q, k, v; rows 16-byte aligned).
+__host__ __device__ inline size_t smem_bytes(int T, int D) { return (size_t)T * (3 * D + 4) * sizeof(float); }
 
-// One CTA per track.  qkv: rows [q | k | v] of width 3 D at stride ldq; track b's
-// hit t is row row0[b] + t (packed rows) or b T + t (padded rows, row0 null).
-// o: the attention output, row-aligned with qkv at stride ldo.  With padded rows
-// the rows t >= n of a track (all of them for a track whose count is outside
-// [1, T]) are written 0; packed rows have no padding.
-template <typename OutT>
+template <int DH>
+__device__ __forceinline__ float dot(const float (&q)[DH], const float* k) {
+  float s = 0.0f;
+#pragma unroll
+  for (int i = 0; i < DH; i += 4) {
+    const float4 a = *reinterpret_cast<const float4*>(k + i);
+    s = fmaf(q[i], a.x, s);
+    s = fmaf(q[i + 1], a.y, s);
+    s = fmaf(q[i + 2], a.z, s);
+    s = fmaf(q[i + 3], a.w, s);
+  }
+  return s;
+}
+
+// qkv: rows [q | k | v] of width 3 D at stride ldq; track b's hit t is row
+// row0[b] + t (packed rows) or b T + t (padded rows, row0 null).  o: the attention
+// output at stride ldo, row-aligned with qkv.  With padded rows the rows t >= n of
+// a track (all of them for a track whose count is outside [1, T]) are written 0.
+template <int DH, typename OutT>
 __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* __restrict__ qkv, int ldq,
                                                                   const int64_t* __restrict__ row0,
                                                                   const int32_t* __restrict__ n_hits, int64_t B,
                                                                   int T, int D, int NH, OutT* __restrict__ o,
                                                                   int ldo) {
-  extern __shared__ float kv[];
+  extern __shared__ float4 sm4[];
+  float* sm = reinterpret_cast<float*>(sm4);
   const int64_t b = blockIdx.x;
   if (b >= B) return;
   int n = n_hits[b];
   if (n < 1 || n > T) n = 0;
   const int64_t r0 = row0 ? row0[b] : b * (int64_t)T;
-  const int ks = 2 * D + 1;
-  for (int i = threadIdx.x; i < n * 2 * D; i += THREADS) {
-    const int j = i / (2 * D), c = i - j * (2 * D);
-    kv[j * ks + c] = qkv[(r0 + j) * ldq + D + c];
+  const int ls = 3 * D + 4, w4 = (3 * D) / 4;
+  for (int i = threadIdx.x; i < n * w4; i += THREADS) {
+    const int j = i / w4, c = i - j * w4;
+    *reinterpret_cast<float4*>(sm + j * ls + 4 * c) = *reinterpret_cast<const float4*>(qkv + (r0 + j) * ldq + 4 * c);
   }
   if (!row0) {   // padded layout: zero the padding rows
     for (int i = threadIdx.x; i < (T - n) * D; i += THREADS) {
@@ -53,46 +72,89 @@ __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* _
   }
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int dh = D / NH;
-  const float scale = rsqrtf((float)dh);
+  const float scale = rsqrtf((float)DH);
   for (int h = warp; h < NH; h += THREADS / 32) {
-    const int c0 = h * dh;
-    for (int t = 0; t < n; ++t) {
-      const float* q = qkv + (r0 + t) * ldq + c0;
-      const float qa = lane < dh ? q[lane] : 0.0f;
-      const float qb = lane + 32 < dh ? q[lane + 32] : 0.0f;
-      // lane j scores keys j and j + 32
-      float s0 = 0.0f, s1 = 0.0f;
-      const float* k0 = kv + lane * ks + c0;
-      const float* k1 = kv + (lane + 32) * ks + c0;
-      for (int c = 0; c < dh; ++c) {
-        const float qc = __shfl_sync(0xffffffffu, c < 32 ? qa : qb, c & 31);
-        if (lane < n) s0 = fmaf(qc, k0[c], s0);
-        if (lane + 32 < n) s1 = fmaf(qc, k1[c], s1);
+    const int c0 = h * DH;
+    for (int t0 = 0; t0 < n; t0 += 32) {
+      const int t = t0 + lane;
+      const float* qr = sm + (t < n ? t : 0) * ls + c0;
+      float q[DH], acc[DH];
+#pragma unroll
+      for (int i = 0; i < DH; ++i) {
+        q[i] = qr[i];
+        acc[i] = 0.0f;
       }
-      s0 = lane < n ? s0 * scale : -INFINITY;
-      s1 = lane + 32 < n ? s1 * scale : -INFINITY;
-      float m = fmaxf(s0, s1);
-#pragma unroll
-      for (int w = 16; w > 0; w >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, w));
-      const float p0 = lane < n ? expf(s0 - m) : 0.0f;
-      const float p1 = lane + 32 < n ? expf(s1 - m) : 0.0f;
-      float z = p0 + p1;
-#pragma unroll
-      for (int w = 16; w > 0; w >>= 1) z += __shfl_xor_sync(0xffffffffu, z, w);
-      const float inv = 1.0f / z;
-      float oa = 0.0f, ob = 0.0f;   // channels c0 + lane and c0 + lane + 32
+      float m = -INFINITY;
+      for (int j = 0; j < n; ++j) m = fmaxf(m, dot<DH>(q, sm + j * ls + D + c0) * scale);
+      float l = 0.0f;
       for (int j = 0; j < n; ++j) {
-        const float pj = __shfl_sync(0xffffffffu, j < 32 ? p0 : p1, j & 31);
-        const float* v = kv + j * ks + D + c0;
-        if (lane < dh) oa = fmaf(pj, v[lane], oa);
-        if (lane + 32 < dh) ob = fmaf(pj, v[lane + 32], ob);
+        const float p = expf(dot<DH>(q, sm + j * ls + D + c0) * scale - m);
+        l += p;
+        const float* vr = sm + j * ls + 2 * D + c0;
+#pragma unroll
+        for (int i = 0; i < DH; i += 4) {
+          const float4 v = *reinterpret_cast<const float4*>(vr + i);
+          acc[i] = fmaf(p, v.x, acc[i]);
+          acc[i + 1] = fmaf(p, v.y, acc[i + 1]);
+          acc[i + 2] = fmaf(p, v.z, acc[i + 2]);
+          acc[i + 3] = fmaf(p, v.w, acc[i + 3]);
+        }
       }
-      OutT* orow = o + (r0 + t) * ldo + c0;
-      if (lane < dh) put(orow + lane, oa * inv);
-      if (lane + 32 < dh) put(orow + lane + 32, ob * inv);
+      if (t < n) {
+        const float inv = 1.0f / l;
+        OutT* orow = o + (r0 + t) * ldo + c0;
+#pragma unroll
+        for (int i = 0; i < DH; ++i) put(orow + i, acc[i] * inv);
+      }
     }
   }
+}
+
+// Launch for the head width D / NH (a multiple of 8 up to 64; anything else is
+// rejected when the handle is created).
+template <typename OutT>
+inline cudaError_t launch(const float* qkv, int ldq, const int64_t* row0, const int32_t* n_hits, int64_t B, int T,
+                          int D, int NH, OutT* o, int ldo, cudaStream_t st) {
+  const size_t sm = smem_bytes(T, D);
+  const unsigned g = (unsigned)B;
+#define TF_ATTN_CASE(DHV) \
+  case DHV:               \
+    track_attention_kernel<DHV, OutT><<<g, THREADS, sm, st>>>(qkv, ldq, row0, n_hits, B, T, D, NH, o, ldo); break;
+  switch (D / NH) {
+    TF_ATTN_CASE(8)
+    TF_ATTN_CASE(16)
+    TF_ATTN_CASE(24)
+    TF_ATTN_CASE(32)
+    TF_ATTN_CASE(40)
+    TF_ATTN_CASE(48)
+    TF_ATTN_CASE(56)
+    TF_ATTN_CASE(64)
+    default: return cudaErrorInvalidValue;
+  }
+#undef TF_ATTN_CASE
+  return cudaPeekAtLastError();
+}
+
+// The dynamic shared memory of the launches above for tracks of T hits at width D.
+template <typename OutT>
+inline cudaError_t allow_smem(int T, int D, int NH) {
+  const int sm = (int)smem_bytes(T, D);
+  if (sm <= 48 * 1024) return cudaSuccess;
+#define TF_ATTN_ATTR(DHV) \
+  case DHV:               \
+    return cudaFuncSetAttribute(track_attention_kernel<DHV, OutT>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  switch (D / NH) {
+    TF_ATTN_ATTR(8)
+    TF_ATTN_ATTR(16)
+    TF_ATTN_ATTR(24)
+    TF_ATTN_ATTR(32)
+    TF_ATTN_ATTR(40)
+    TF_ATTN_ATTR(48)
+    TF_ATTN_ATTR(56)
+    TF_ATTN_ATTR(64)
+    default: return cudaErrorInvalidValue;
+  }
+#undef TF_ATTN_ATTR
 }
 
 }  // namespace tf_attn

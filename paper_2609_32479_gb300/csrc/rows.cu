@@ -32,6 +32,7 @@
 #include <math.h>
 
 #include <cstring>
+#include <type_traits>
 #include <vector>
 
 #include "attention.cuh"
@@ -47,7 +48,8 @@ constexpr int RG_ROWS = 128;                      // rows per tile (MMA M)
 constexpr int RG_KC = 64;                         // k per stage (one 128-byte swizzle row of 16-bit values)
 constexpr int RG_A_BYTES = RG_ROWS * RG_KC * 2;   // 16 KB
 constexpr int RG_MAX_NT = 256;                    // MMA N per tile (two buffers fill the 512 TMEM columns)
-constexpr int RG_SMEM_BUDGET = 200 * 1024;
+constexpr int RG_SMEM_BUDGET = 196 * 1024;        // the ring of stages and the barriers
+constexpr int RG_STG_WARP = 6144;                 // per epilogue warp: 2 x (32 rows x 16 fp32) + 2 x (32 x 16 16-bit)
 constexpr int RG_MAX_STAGES = 8;
 constexpr uint64_t RG_WAIT_NS = 2000000000ull;
 constexpr uint64_t RG_DRAIN_NS = 200000000ull;
@@ -66,6 +68,8 @@ enum {
 struct RowGemm {
   CUtensorMap ta;             // A [cap][K] 16-bit, box 64 x 128, 128-byte swizzle
   CUtensorMap tw;             // W [N][K] 16-bit, box 64 x Nt, 128-byte swizzle
+  CUtensorMap to32;           // out32 [cap][N] fp32, box 16 x 32 (stores)
+  CUtensorMap to16;           // out16 [cap][N] 16-bit, box 16 x 32 (stores)
   const int64_t* n_rows;      // device: rows of this chunk
   int K, N, Nt, n_ntiles, kchunks, stages;
   int epi;
@@ -106,21 +110,51 @@ __device__ __forceinline__ uint32_t pack16(float a, float b, int fp16) {   // a 
 namespace {
 
 // ------------------------------------------------------------------ the GEMM
-// One 16-column chunk of an epilogue: v[i] is column n = nbase + i of this row.
-__device__ __forceinline__ void store16(const RowGemm& g, int64_t row, int nbase, const float (&v)[16]) {
-  if (g.out32) {
-    float4* o = reinterpret_cast<float4*>(g.out32 + row * g.N + nbase);
+__device__ __forceinline__ void sts4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+
+// Output of one 16-column chunk of a warp's 32 rows: every lane writes its row's
+// 16 values into the warp's staging buffer, then one lane stores the [32][16] box
+// with TMA.  The buffers use the tensor maps' swizzled layouts (fp32 rows of 64
+// bytes: 16-byte piece c of row r at c ^ ((r >> 1) & 3); 16-bit rows of 32 bytes:
+// piece c at c ^ ((r >> 2) & 1)), so the 8 lanes of a quarter warp write 8
+// different bank groups.  Two buffers per output alternate; a buffer is rewritten
+// only after the store that read it two chunks earlier has finished reading.
+struct Emit {
+  uint32_t stg;     // this warp's staging area
+  int chunk;        // chunks emitted so far (buffer parity)
+  __device__ __forceinline__ void operator()(const RowGemm& g, int lane, int nb, int row, const float (&v)[16],
+                                             bool to32, bool to16) {
+    const int p = chunk & 1;
+    if (lane == 0) bulk_wait_read1();
+    __syncwarp();
+    if (to32) {
+      const uint32_t a = stg + p * 2048 + lane * 64;
+      const int sw = (lane >> 1) & 3;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      for (int j = 0; j < 4; ++j)
+        sts4(a + 16 * (j ^ sw), __float_as_uint(v[4 * j]), __float_as_uint(v[4 * j + 1]),
+             __float_as_uint(v[4 * j + 2]), __float_as_uint(v[4 * j + 3]));
+    }
+    if (to16) {
+      const uint32_t a = stg + 4096 + p * 1024 + lane * 32;
+      const int sw = (lane >> 2) & 1;
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        sts4(a + 16 * (j ^ sw), pack16(v[8 * j], v[8 * j + 1], g.fp16), pack16(v[8 * j + 2], v[8 * j + 3], g.fp16),
+             pack16(v[8 * j + 4], v[8 * j + 5], g.fp16), pack16(v[8 * j + 6], v[8 * j + 7], g.fp16));
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      if (to32) tma_store_2d(&g.to32, stg + p * 2048, nb, row);
+      if (to16) tma_store_2d(&g.to16, stg + 4096 + p * 1024, nb, row);
+      bulk_commit();
+    }
+    ++chunk;
   }
-}
-__device__ __forceinline__ void store16_h(const RowGemm& g, int64_t row, int nbase, const float (&v)[16]) {
-  uint4* o = reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(g.out16) + row * g.N + nbase);
-  o[0] = make_uint4(pack16(v[0], v[1], g.fp16), pack16(v[2], v[3], g.fp16), pack16(v[4], v[5], g.fp16),
-                    pack16(v[6], v[7], g.fp16));
-  o[1] = make_uint4(pack16(v[8], v[9], g.fp16), pack16(v[10], v[11], g.fp16), pack16(v[12], v[13], g.fp16),
-                    pack16(v[14], v[15], g.fp16));
-}
+};
 
 // acc + bias (+ res) of 16 columns; the same arithmetic in both passes of EP_NORM
 __device__ __forceinline__ void biased(const RowGemm& g, int64_t row, bool live, int nbase, float (&v)[16]) {
@@ -254,6 +288,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
     // ---------------- epilogue: this warp's 32 rows of each tile
     const int q = warp & 3;
     int acc_k = 0;
+    Emit emit{base + (uint32_t)(g.stages * stage_bytes) + 1024u + (uint32_t)((warp - 2) * RG_STG_WARP), 0};
     for (int64_t t = blockIdx.x; t < total; t += gridDim.x) {
       const int buf = acc_k & 1;
       const uint32_t aph = (uint32_t)(acc_k >> 1) & 1u;
@@ -263,6 +298,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       }
       tc_fence_after();
       const int64_t row = (t / g.n_ntiles) * RG_ROWS + 32 * q + lane;
+      const int rbox = (int)((t / g.n_ntiles) * RG_ROWS + 32 * q);   // first row of this warp's boxes
       const int n0 = (int)(t % g.n_ntiles) * g.Nt;
       const bool live = row < rows;
       const uint32_t tq = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * RG_MAX_NT);
@@ -275,7 +311,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
           biased(g, row, live, n0 + c, v);
 #pragma unroll
           for (int i = 0; i < 16; ++i) ss = fmaf(v[i], v[i], ss);
-          if (live) store16(g, row, n0 + c, v);
+          emit(g, lane, n0 + c, rbox, v, true, false);
         }
         const float inv = 1.0f / sqrtf(ss / (float)g.N + g.rms_eps);
         for (int c = 0; c < g.Nt; c += 16) {
@@ -285,7 +321,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
           biased(g, row, live, n0 + c, v);
 #pragma unroll
           for (int i = 0; i < 16; ++i) v[i] = v[i] * inv * g.gain[n0 + c + i];
-          if (live) store16_h(g, row, n0 + c, v);
+          emit(g, lane, n0 + c, rbox, v, false, true);
         }
       } else {
         for (int c = 0; c < g.Nt; c += 16) {
@@ -305,12 +341,8 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[i] = v[i] * sigm(v[i]);
           }
-          if (live) {
-            if (g.epi == EP_16 || g.epi == EP_SILU16)
-              store16_h(g, row, nb, v);
-            else
-              store16(g, row, nb, v);
-          }
+          const bool h = g.epi == EP_16 || g.epi == EP_SILU16;
+          emit(g, lane, nb, rbox, v, !h, h);
         }
       }
       tc_fence_before();
@@ -318,6 +350,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty[buf]));
       ++acc_k;
     }
+    if (lane == 0) bulk_wait_all();   // every store done before the CTA leaves
   }
   tc_fence_before();
   __syncthreads();
@@ -404,15 +437,19 @@ __global__ void __launch_bounds__(PLAN_NT) plan_rows(const int32_t* __restrict__
 
 // ------------------------------------------------------------------ Fourier rows
 // Sec. 3.2: u = (v - min) / (max - min) per feature, then sin(pi s_k u) and
-// cos(pi s_k u) for the 16 scales, feature-major ([f][sin k, cos k]); the argument
-// s_k u is formed in fp64 and reduced modulo 2 before the fp32 sinpi / cospi.  One
-// thread per (track, hit, feature); the 2 n_fourier values leave as 16-bit
-// operands of the embedding product.  Hit rows: padded hits[b][t] or packed
-// hits[offs[b] + t].
+// cos(pi s_k u) for the 16 scales, feature-major ([f][sin k, cos k]).  One thread
+// per (track, hit, feature); the 2 n_fourier values leave as 16-bit operands of
+// the embedding product.  Hit rows: padded hits[b][t] or packed hits[offs[b] + t].
+// fp32 only (fp64 is slow on this part): v - min (TwoSum) times the two-float
+// 1 / (max - min) and s_k (TwoProduct) give the argument as an unevaluated sum
+// of two floats, reduced modulo 2 exactly, so the sine and cosine carry only the
+// final fp32 rounding of the argument.  When s_{k+3} = 2 s_k for every k (the
+// scales 2^(k/3)), the scales k = 0-2, 6-8, 12-14 are evaluated and the others
+// follow by one double-angle step (2 s c, (c - s)(c + s)).
 template <typename T16>
 __global__ void fourier_rows_kernel(const float* __restrict__ hits, const int64_t* __restrict__ offs,
                                     const int32_t* __restrict__ n_hits, int64_t B, tf_shape s,
-                                    const int64_t* __restrict__ row0, T16* __restrict__ e) {
+                                    const int64_t* __restrict__ row0, int doubling, T16* __restrict__ e) {
   const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (i >= B * s.T * s.F) return;
   const int64_t b = i / (s.T * s.F);
@@ -420,21 +457,36 @@ __global__ void fourier_rows_kernel(const float* __restrict__ hits, const int64_
   const int n = n_hits[b];
   if (n < 1 || n > s.T || t >= n) return;
   const float v = offs ? hits[(offs[b] + t) * s.F + f] : hits[(b * s.T + t) * s.F + f];
-  const double u = ((double)v - s.feat_min_d[f]) / s.feat_range_d[f];
+  const float mn = -s.feat_min[f], ih = s.feat_inv_range[f];
+  const float dh = v + mn;
+  const float bv = dh - v;
+  const float dl = (v - (dh - bv)) + (mn - bv);
+  const float uh = dh * ih;
+  const float ul = fmaf(dh, ih, -uh) + fmaf(dh, s.feat_inv_lo[f], dl * ih);
   float sv[TRACKFIT_MAX_FOURIER], cv[TRACKFIT_MAX_FOURIER];
 #pragma unroll
   for (int k = 0; k < TRACKFIT_MAX_FOURIER; ++k) {
-    double a = u * (double)s.scale[k];
-    a -= 2.0 * rint(0.5 * a);
-    const float af = (float)a;
-    sv[k] = sinpif(af);
-    cv[k] = cospif(af);
+    if (doubling && (k % 6) >= 3) {   // s_k = 2 s_{k-3}
+      sv[k] = 2.0f * sv[k - 3] * cv[k - 3];
+      cv[k] = (cv[k - 3] - sv[k - 3]) * (cv[k - 3] + sv[k - 3]);
+      continue;
+    }
+    const float sk = s.scale[k];
+    const float xh = uh * sk;
+    const float xl = fmaf(uh, sk, -xh) + ul * sk;
+    const float r = (xh - 2.0f * rintf(0.5f * xh)) + xl;
+    sv[k] = sinpif(r);
+    cv[k] = cospif(r);
   }
-  T16* o = e + (row0[b] + t) * s.E + f * 2 * TRACKFIT_MAX_FOURIER;
+  // the feature's 32 values (64 bytes, 16-byte aligned) in four vector stores
+  uint4* o = reinterpret_cast<uint4*>(e + (row0[b] + t) * s.E + f * 2 * TRACKFIT_MAX_FOURIER);
+  const int h16 = sizeof(T16) == 2 && std::is_same<T16, __half>::value;
 #pragma unroll
-  for (int k = 0; k < TRACKFIT_MAX_FOURIER; ++k) {
-    tf_attn::put(o + k, sv[k]);
-    tf_attn::put(o + TRACKFIT_MAX_FOURIER + k, cv[k]);
+  for (int q = 0; q < 2; ++q) {
+    o[q] = make_uint4(pack16(sv[8 * q], sv[8 * q + 1], h16), pack16(sv[8 * q + 2], sv[8 * q + 3], h16),
+                      pack16(sv[8 * q + 4], sv[8 * q + 5], h16), pack16(sv[8 * q + 6], sv[8 * q + 7], h16));
+    o[2 + q] = make_uint4(pack16(cv[8 * q], cv[8 * q + 1], h16), pack16(cv[8 * q + 2], cv[8 * q + 3], h16),
+                          pack16(cv[8 * q + 4], cv[8 * q + 5], h16), pack16(cv[8 * q + 6], cv[8 * q + 7], h16));
   }
 }
 
@@ -492,6 +544,87 @@ __global__ void pool_mean_rows_kernel(const float* __restrict__ x, const int64_t
   pooled[b * D + c] = acc / (float)n;
 }
 
+// ------------------------------------------------------------------ head
+// The head of Sec. 3.2-3.3 on the pooled vectors, in fp32 on the CUDA cores:
+// RMSNorm (gain g_h), W_h1 (P -> 128) + SiLU, W_h2 (128 -> 5 x n_quantiles), the
+// median quantile per parameter.  One CTA per HR_TRK tracks: thread j owns hidden
+// unit j and reads column j of W_h1 transposed ([P][128], coalesced across the
+// CTA) once for all the CTA's tracks.
+constexpr int HR_TRK = 16, HR_NT = 128;
+
+__host__ __device__ inline size_t head_rows_smem(int P, int Q) {
+  return (size_t)HR_TRK * ((size_t)P + 128 + (size_t)Q + 1) * sizeof(float);
+}
+
+__global__ void __launch_bounds__(HR_NT) head_rows_kernel(const float* __restrict__ pooled,
+                                                          const int32_t* __restrict__ n_hits, int64_t B, int T,
+                                                          int P, int Q, int NQ, float eps, const float* __restrict__ g,
+                                                          const float* __restrict__ w1t, const float* __restrict__ b1,
+                                                          const float* __restrict__ w2, const float* __restrict__ b2,
+                                                          float* __restrict__ out, float* __restrict__ out_q,
+                                                          float* __restrict__ out_pool,
+                                                          unsigned long long* __restrict__ err) {
+  extern __shared__ float hsm[];
+  float* pv = hsm;                    // [HR_TRK][P]
+  float* hid = pv + HR_TRK * P;       // [HR_TRK][128]
+  float* qv = hid + HR_TRK * 128;     // [HR_TRK][Q]
+  float* inv = qv + HR_TRK * Q;       // [HR_TRK]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t b0 = blockIdx.x * (int64_t)HR_TRK;
+  const int nt = B - b0 < HR_TRK ? (int)(B - b0) : HR_TRK;
+  for (int i = tid; i < HR_TRK * P; i += HR_NT) pv[i] = i < nt * P ? pooled[b0 * P + i] : 0.0f;
+  if (tid < nt) {
+    const int n = n_hits[b0 + tid];
+    if (n < 1 || n > T) atomicAdd(err, 1ull);
+  }
+  __syncthreads();
+  for (int t = warp; t < HR_TRK; t += HR_NT / 32) {
+    float ss = 0.0f;
+    for (int c = lane; c < P; c += 32) ss = fmaf(pv[t * P + c], pv[t * P + c], ss);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if (lane == 0) inv[t] = 1.0f / sqrtf(ss / (float)P + eps);
+  }
+  __syncthreads();
+  for (int i = tid; i < nt * P; i += HR_NT) {
+    const int t = i / P, c = i - t * P;
+    if (out_pool) {
+      const int n = n_hits[b0 + t];
+      out_pool[b0 * P + i] = (n < 1 || n > T) ? NAN : pv[i];
+    }
+    pv[i] = pv[i] * inv[t] * g[c];
+  }
+  __syncthreads();
+  {
+    float acc[HR_TRK];
+#pragma unroll
+    for (int t = 0; t < HR_TRK; ++t) acc[t] = b1[tid];
+#pragma unroll 8
+    for (int c = 0; c < P; ++c) {
+      const float w = __ldg(w1t + c * 128 + tid);
+#pragma unroll
+      for (int t = 0; t < HR_TRK; ++t) acc[t] = fmaf(w, pv[t * P + c], acc[t]);
+    }
+#pragma unroll
+    for (int t = 0; t < HR_TRK; ++t) hid[t * 128 + tid] = acc[t] * sigm(acc[t]);
+  }
+  __syncthreads();
+  for (int o = tid; o < nt * Q; o += HR_NT) {
+    const int t = o / Q, q = o - t * Q;
+    float acc = b2[q];
+    const float* wr = w2 + (size_t)q * 128;
+    for (int j = 0; j < 128; ++j) acc = fmaf(wr[j], hid[t * 128 + j], acc);
+    const int n = n_hits[b0 + t];
+    qv[o] = (n < 1 || n > T) ? NAN : acc;
+    if (out_q) out_q[b0 * Q + o] = qv[o];
+  }
+  __syncthreads();
+  for (int o = tid; o < nt * 5; o += HR_NT) {
+    const int t = o / 5, p = o - t * 5;
+    out[(b0 + t) * 5 + p] = qv[t * Q + p * NQ + NQ / 2];
+  }
+}
+
 }  // namespace
 
 // ------------------------------------------------------------------ host side
@@ -499,6 +632,8 @@ struct tf_rows_state {
   int fp16;
   int nsm;
   uint16_t* w16;            // every product's weights, 16-bit, back to back
+  float* w1t;               // the head's W_h1 transposed, [P][128] fp32
+  int doubling;             // fourier_scale[k + 3] == 2 fourier_scale[k] for every k
   int64_t chunk, cap;       // tracks per chunk; rows of the workspace (chunk * max_hits)
   int64_t* row0;            // [chunk + 1]
   int64_t* tot;             // [chunk / 1024 + 1]
@@ -539,6 +674,33 @@ bool rows_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uin
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Output matrix [rows][cols] row-major (fp32, or 16-bit) -> tensor map of
+// 16-column x 32-row boxes for the epilogue's TMA stores, swizzled over the box
+// row (64 bytes for fp32, 32 bytes for 16-bit).
+bool out_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, int bytes, int fp16) {
+  auto fn = rows_encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * (uint64_t)bytes};
+  cuuint32_t box[2] = {16, 32};
+  cuuint32_t es[2] = {1, 1};
+  const CUtensorMapDataType t = bytes == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+                                : fp16     ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                           : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  return fn(m, t, 2, const_cast<void*>(ptr), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            bytes == 4 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The store maps of a product whose output pointers are set.
+bool finish_gemm(RowGemm& g, const tf_rows_state* r) {
+  const bool need32 = g.epi == EP_F32 || g.epi == EP_PROJ || g.epi == EP_RES || g.epi == EP_NORM;
+  const bool need16 = g.epi == EP_16 || g.epi == EP_SILU16 || g.epi == EP_NORM;
+  if (need32 != (g.out32 != nullptr) || need16 != (g.out16 != nullptr)) return false;
+  return (!g.out32 || out_map(&g.to32, g.out32, (uint64_t)r->cap, (uint64_t)g.N, 4, r->fp16)) &&
+         (!g.out16 || out_map(&g.to16, g.out16, (uint64_t)r->cap, (uint64_t)g.N, 2, r->fp16));
+}
+
 // The MMA N of one tile: N itself up to 256, else the smallest equal split into
 // multiples of 16 (0 if there is none).
 int tile_n(int N) {
@@ -547,8 +709,10 @@ int tile_n(int N) {
   return 0;
 }
 
+// alignment slack, the ring of stages, the barriers (one 1 KB block), the
+// epilogue warps' staging buffers
 size_t gemm_smem(const RowGemm& g) {
-  return 1024 + (size_t)g.stages * (RG_A_BYTES + g.Nt * 128) + sizeof(RgBars);
+  return 1024 + (size_t)g.stages * (RG_A_BYTES + g.Nt * 128) + 1024 + 4 * RG_STG_WARP;
 }
 
 // A [cap][K] (16-bit, row stride K) times W [N][K]; the epilogue's pointers are set by the caller.
@@ -561,7 +725,7 @@ bool make_gemm(RowGemm& g, const tf_rows_state* r, const void* A, int K, const u
   g.n_ntiles = N / g.Nt;
   g.kchunks = (K + RG_KC - 1) / RG_KC;
   const int stage = RG_A_BYTES + g.Nt * 128;
-  g.stages = (int)((RG_SMEM_BUDGET - 1024 - (int)sizeof(RgBars)) / stage);
+  g.stages = (int)((RG_SMEM_BUDGET - 1024) / stage);
   if (g.stages > RG_MAX_STAGES) g.stages = RG_MAX_STAGES;
   if (g.stages < 2) return false;
   g.epi = epi;
@@ -572,12 +736,16 @@ bool make_gemm(RowGemm& g, const tf_rows_state* r, const void* A, int K, const u
          rows_map(&g.tw, W, (uint64_t)N, (uint64_t)K, (uint32_t)g.Nt, r->fp16);
 }
 
-int launch_gemm(const tf_rows_state* r, RowGemm& g, const int64_t* n_rows, unsigned long long* err,
-                cudaStream_t st) {
+// One product over the chunk's rows; the handle's timing hook (trackfit_profile)
+// brackets every product launch of this path.
+int launch_gemm(trackfit_ctx* h, RowGemm& g, const int64_t* n_rows, cudaStream_t st) {
+  const tf_rows_state* r = h->rows;
   g.n_rows = n_rows;
-  g.err = err;
+  g.err = h->d_err;
   g.wait_ns = r->wait_ns;
+  tf_prof_begin(h, st);
   row_gemm_kernel<<<r->nsm, RG_THREADS, gemm_smem(g), st>>>(g);
+  tf_prof_end(h, st);
   return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
 }
 
@@ -605,6 +773,7 @@ void tf_rows_destroy(trackfit_ctx* h) {
   tf_rows_state* r = h->rows;
   if (!r) return;
   tf_free(r->w16);
+  tf_free(r->w1t);
   tf_free(r->row0);
   tf_free(r->tot);
   tf_free(r->a0);
@@ -633,6 +802,9 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
   h->rows = r;   // freed by tf_rows_destroy on any failure below
   r->fp16 = s.precision == TRACKFIT_FP16_PROJ;
   r->wait_ns = RG_WAIT_NS;
+  r->doubling = 1;
+  for (int k = 0; k + 3 < TRACKFIT_MAX_FOURIER; ++k)
+    if (s.scale[k + 3] != 2.0f * s.scale[k]) r->doubling = 0;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&r->nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
@@ -665,6 +837,13 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
     for (size_t i = 0; i < m.n * m.k; ++i) w[m.at + i] = to16(host_w[m.off + i], r->fp16);
   int st = tf_status_from_cuda(tf_malloc((void**)&r->w16, n16 * 2));
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(r->w16, w.data(), n16 * 2, cudaMemcpyHostToDevice));
+  {
+    std::vector<float> t((size_t)s.P * 128);
+    for (int j = 0; j < 128; ++j)
+      for (int c = 0; c < s.P; ++c) t[(size_t)c * 128 + j] = host_w[o.head_w1 + (size_t)j * s.P + c];
+    if (st == TRACKFIT_OK) st = tf_status_from_cuda(tf_malloc((void**)&r->w1t, t.size() * 4));
+    if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(r->w1t, t.data(), t.size() * 4, cudaMemcpyHostToDevice));
+  }
   if (st != TRACKFIT_OK) return st;
   // workspace, sized for whole chunks of full-length tracks
   const size_t hsw = attn ? (H > D ? H : D) : D;
@@ -745,22 +924,22 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
       g[3].out16 = r->xy16;
     }
   }
+  ok = ok && finish_gemm(r->e1, r) && finish_gemm(r->e2, r);
+  for (int l = 0; l < s.L && ok; ++l)
+    for (int k = 0; k < (attn ? 4 : 1) && ok; ++k) ok = finish_gemm(r->lay[l][k], r);
   if (!ok) return TRACKFIT_ERR_CUDA;
   r->smem = gemm_smem(r->e1);
   auto upd = [&](const RowGemm& g) { r->smem = gemm_smem(g) > r->smem ? gemm_smem(g) : r->smem; };
   upd(r->e2);
   for (int l = 0; l < s.L; ++l)
     for (int k = 0; k < (attn ? 4 : 1); ++k) upd(r->lay[l][k]);
-  if (cudaFuncSetAttribute(row_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r->smem) != cudaSuccess)
+  if (cudaFuncSetAttribute(row_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r->smem) != cudaSuccess ||
+      cudaFuncSetAttribute(head_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)head_rows_smem(s.P, s.Q)) != cudaSuccess)
     return TRACKFIT_ERR_CUDA;
-  if (attn) {
-    const int ab = (int)tf_attn::smem_bytes(s.T, s.D);
-    if (cudaFuncSetAttribute(tf_attn::track_attention_kernel<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             ab) != cudaSuccess ||
-        cudaFuncSetAttribute(tf_attn::track_attention_kernel<__nv_bfloat16>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, ab) != cudaSuccess)
-      return TRACKFIT_ERR_CUDA;
-  }
+  if (attn && (tf_attn::allow_smem<__half>(s.T, s.D, s.NH) != cudaSuccess ||
+               tf_attn::allow_smem<__nv_bfloat16>(s.T, s.D, s.NH) != cudaSuccess))
+    return TRACKFIT_ERR_CUDA;
   return TRACKFIT_OK;
 }
 
@@ -771,7 +950,7 @@ int rows_chunk(trackfit_ctx* h, const float* hits, const int64_t* offs, const in
                float* out_q, float* out_pool, cudaStream_t st) {
   tf_rows_state* r = h->rows;
   const tf_shape& s = h->s;
-  unsigned long long* err = h->d_err;
+  unsigned long long* err = h->d_err;   // bad-track counter of the head
   const bool attn = s.topology == TRACKFIT_TOPOLOGY_ATTENTION;
   const int nblk = (int)((nb + PLAN_NT - 1) / PLAN_NT);
   plan_totals<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot);
@@ -779,14 +958,14 @@ int rows_chunk(trackfit_ctx* h, const float* hits, const int64_t* offs, const in
   plan_rows<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot, r->row0);
   const int64_t* nrows = r->row0 + nb;
   const int64_t nf = nb * s.T * s.F;
-  fourier_rows_kernel<T16><<<(unsigned)((nf + 255) / 256), 256, 0, st>>>(hits, offs, nc, nb, s, r->row0,
+  fourier_rows_kernel<T16><<<(unsigned)((nf + 255) / 256), 256, 0, st>>>(hits, offs, nc, nb, s, r->row0, r->doubling,
                                                                          reinterpret_cast<T16*>(r->a0));
   if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
-  if (launch_gemm(r, r->e1, nrows, err, st) || launch_gemm(r, r->e2, nrows, err, st)) return TRACKFIT_ERR_CUDA;
+  if (launch_gemm(h, r->e1, nrows, st) || launch_gemm(h, r->e2, nrows, st)) return TRACKFIT_ERR_CUDA;
   for (int l = 0; l < s.L; ++l) {
     RowGemm* g = r->lay[l];
     if (!attn) {
-      if (launch_gemm(r, g[0], nrows, err, st)) return TRACKFIT_ERR_CUDA;
+      if (launch_gemm(h, g[0], nrows, st)) return TRACKFIT_ERR_CUDA;
       const bool last = l + 1 == s.L;
       dim3 grid((unsigned)nb, (unsigned)((s.H + 127) / 128));
       concat_scan_rows_kernel<T16><<<grid, 128, 0, st>>>(r->p32, r->row0, nc, nb, s.T, s.H,
@@ -794,19 +973,24 @@ int rows_chunk(trackfit_ctx* h, const float* hits, const int64_t* offs, const in
                                                          last ? r->pooled : nullptr, s.pool);
       continue;
     }
-    if (launch_gemm(r, g[0], nrows, err, st)) return TRACKFIT_ERR_CUDA;
-    tf_attn::track_attention_kernel<T16><<<(unsigned)nb, tf_attn::THREADS, tf_attn::smem_bytes(s.T, s.D), st>>>(
-        r->p32, 3 * s.D, r->row0, nc, nb, s.T, s.D, s.NH, reinterpret_cast<T16*>(r->o16), s.D);
-    if (launch_gemm(r, g[1], nrows, err, st) || launch_gemm(r, g[2], nrows, err, st) ||
-        launch_gemm(r, g[3], nrows, err, st))
+    if (launch_gemm(h, g[0], nrows, st)) return TRACKFIT_ERR_CUDA;
+    if (tf_attn::launch<T16>(r->p32, 3 * s.D, r->row0, nc, nb, s.T, s.D, s.NH, reinterpret_cast<T16*>(r->o16), s.D,
+                             st) != cudaSuccess)
+      return TRACKFIT_ERR_CUDA;
+    if (launch_gemm(h, g[1], nrows, st) || launch_gemm(h, g[2], nrows, st) ||
+        launch_gemm(h, g[3], nrows, st))
       return TRACKFIT_ERR_CUDA;
   }
   if (attn) {
     dim3 grid((unsigned)nb, (unsigned)((s.D + 127) / 128));
     pool_mean_rows_kernel<<<grid, 128, 0, st>>>(r->x32, r->row0, nc, nb, s.T, s.D, r->pooled);
   }
-  if (cudaPeekAtLastError() != cudaSuccess) return TRACKFIT_ERR_CUDA;
-  return tf_simt_head(s, h->off, h->d_w, r->pooled, nc, nb, out, out_q, out_pool, err, st);
+  const tf_blob_off& o = h->off;
+  const float* W = h->d_w;
+  head_rows_kernel<<<(unsigned)((nb + HR_TRK - 1) / HR_TRK), HR_NT, head_rows_smem(s.P, s.Q), st>>>(
+      r->pooled, nc, nb, s.T, s.P, s.Q, s.NQ, s.rms_eps, W + o.head_g, r->w1t, W + o.head_b1, W + o.head_w2,
+      W + o.head_b2, out, out_q, out_pool, err);
+  return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
 }
 
 }  // namespace
@@ -819,14 +1003,12 @@ int tf_rows_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, i
     const int64_t nb = B - c0 < r->chunk ? B - c0 : r->chunk;
     const float* hc = offs ? hits : hits + c0 * s.T * s.F;
     const int64_t* oc = offs ? offs + c0 : nullptr;
-    if (h->prof_on) tf_prof_begin(h, st);
     const int e = r->fp16 ? rows_chunk<__half>(h, hc, oc, n_hits + c0, nb, out + c0 * 5,
                                                out_q ? out_q + c0 * s.Q : nullptr,
                                                out_pool ? out_pool + c0 * s.P : nullptr, st)
                           : rows_chunk<__nv_bfloat16>(h, hc, oc, n_hits + c0, nb, out + c0 * 5,
                                                       out_q ? out_q + c0 * s.Q : nullptr,
                                                       out_pool ? out_pool + c0 * s.P : nullptr, st);
-    if (h->prof_on) tf_prof_end(h, st);
     if (e != TRACKFIT_OK) return e;
   }
   return TRACKFIT_OK;

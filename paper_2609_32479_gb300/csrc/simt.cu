@@ -315,10 +315,7 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
   const int D = s.D, H = s.H, PD = attn ? 3 * s.D : 4 * s.H + s.D;
   const int UW = attn ? s.H : s.D, YW = attn ? s.D : 2 * s.H;
   // the attention CTA's dynamic shared memory, when above the default 48 KB
-  if (attn && tf_attn::smem_bytes(s.T, s.D) > 48 * 1024 &&
-      cudaFuncSetAttribute(tf_attn::track_attention_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)tf_attn::smem_bytes(s.T, s.D)) != cudaSuccess)
-    return TRACKFIT_ERR_CUDA;
+  if (attn && tf_attn::allow_smem<float>(s.T, s.D, s.NH) != cudaSuccess) return TRACKFIT_ERR_CUDA;
   for (int64_t c0 = 0; c0 < B; c0 += ws_tracks) {
     const int64_t nb = (B - c0 < ws_tracks) ? B - c0 : ws_tracks;
     const int64_t R = nb * s.T;
@@ -370,8 +367,8 @@ int tf_simt_run(const tf_shape& s, const tf_blob_off& o, const float* W, float* 
         g.A = XH; g.lda = D; g.W = W + lo.w_in; g.bias = W + lo.b_in; g.C = PR; g.ldc = 3 * D;
         g.N = 3 * D; g.K = D; g.epi = EPI_STORE;
         if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
-        tf_attn::track_attention_kernel<float><<<(unsigned)nb, tf_attn::THREADS, tf_attn::smem_bytes(s.T, D), st>>>(
-            PR, 3 * D, nullptr, nc, nb, s.T, D, s.NH, Y, D);
+        if (tf_attn::launch<float>(PR, 3 * D, nullptr, nc, nb, s.T, D, s.NH, Y, D, st) != cudaSuccess)
+          return TRACKFIT_ERR_CUDA;
         g.A = Y; g.lda = D; g.W = W + lo.w_m; g.bias = W + lo.b_m; g.C = X1; g.ldc = D;
         g.N = D; g.K = D; g.epi = EPI_RES_MASK; g.res = X; g.ldr = D;
         if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;

@@ -30,7 +30,8 @@ struct tf_blob_off {
 struct tf_shape {
   int T, F, K, E, D, H, L, P, Hh, NQ, Q, precision, pool, topology, NH;
   float rms_eps;
-  float feat_min[TRACKFIT_MAX_FEATURES], feat_inv_range[TRACKFIT_MAX_FEATURES];
+  // 1 / (max - min) as the unevaluated sum feat_inv_range + feat_inv_lo of two floats
+  float feat_min[TRACKFIT_MAX_FEATURES], feat_inv_range[TRACKFIT_MAX_FEATURES], feat_inv_lo[TRACKFIT_MAX_FEATURES];
   double feat_min_d[TRACKFIT_MAX_FEATURES], feat_range_d[TRACKFIT_MAX_FEATURES];
   float scale[TRACKFIT_MAX_FOURIER];
 };
