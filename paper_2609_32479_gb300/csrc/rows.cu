@@ -24,7 +24,7 @@
 // Kernel roles (192 threads, one CTA per SM, persistent over 128-row x Nt tiles):
 //   warp 0     TMA producer (one elected lane): A and W chunks of 64 k into a ring of stages
 //   warp 1     MMA issuer (one elected lane) and TMEM owner: two accumulator buffers
-//   warps 2-5  epilogue, TMEM lane quadrant = warp % 4
+//   warps 2-9  epilogue, TMEM lane quadrant = warp % 4, column half = (warp - 2) / 4
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -32,6 +32,7 @@
 #include <math.h>
 
 #include <cstring>
+#include <map>
 #include <type_traits>
 #include <vector>
 
@@ -43,12 +44,13 @@ using namespace sm100;
 
 namespace {
 
-constexpr int RG_THREADS = 192;
+constexpr int RG_THREADS = 320;
+constexpr int RG_EPI_WARPS = 8;                   // two per TMEM lane quadrant, each half of a tile's columns
 constexpr int RG_ROWS = 128;                      // rows per tile (MMA M)
 constexpr int RG_KC = 64;                         // k per stage (one 128-byte swizzle row of 16-bit values)
 constexpr int RG_A_BYTES = RG_ROWS * RG_KC * 2;   // 16 KB
 constexpr int RG_MAX_NT = 256;                    // MMA N per tile (two buffers fill the 512 TMEM columns)
-constexpr int RG_SMEM_BUDGET = 196 * 1024;        // the ring of stages and the barriers
+constexpr int RG_SMEM_BUDGET = 176 * 1024;        // the ring of stages
 constexpr int RG_STG_WARP = 6144;                 // per epilogue warp: 2 x (32 rows x 16 fp32) + 2 x (32 x 16 16-bit)
 constexpr int RG_MAX_STAGES = 8;
 constexpr uint64_t RG_WAIT_NS = 2000000000ull;
@@ -89,12 +91,16 @@ struct RowGemm {
 struct RgBars {
   uint64_t full[RG_MAX_STAGES], empty[RG_MAX_STAGES];
   uint64_t acc_full[2], acc_empty[2], drain;
+  uint64_t ssb[4];            // RMSNorm: the two warps of a lane quadrant exchange their partial sums
   uint32_t tmem_base;
   int abort;
   int never;                  // a flag nothing sets: for the waits at exit that must not give up on abort
 };
 
-__device__ __forceinline__ float sigm(float x) { return 1.0f / (1.0f + expf(-x)); }
+// sigma(x) = 1 / (1 + e^-x) with the hardware exponential (ex2 of -x log2 e) and a
+// correctly rounded reciprocal: a few ulp of fp32, far below the 16-bit rounding
+// of the operands it feeds (e^-x = inf for x < -88 gives 1 / inf = 0).
+__device__ __forceinline__ float sigm(float x) { return __frcp_rn(1.0f + __expf(-x)); }
 
 __device__ __forceinline__ uint32_t pack16(float a, float b, int fp16) {   // a -> low half
   if (fp16) {
@@ -156,10 +162,18 @@ struct Emit {
   }
 };
 
-// acc + bias (+ res) of 16 columns; the same arithmetic in both passes of EP_NORM
+// acc + bias (+ res) of 16 columns; the same arithmetic in both passes of EP_NORM.
+// bias (and gain) vectors are 16-byte aligned copies made at create.
 __device__ __forceinline__ void biased(const RowGemm& g, int64_t row, bool live, int nbase, float (&v)[16]) {
+  const float4* bb = reinterpret_cast<const float4*>(g.bias + nbase);
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] += g.bias[nbase + i];
+  for (int i = 0; i < 4; ++i) {
+    const float4 w = __ldg(bb + i);
+    v[4 * i] += w.x;
+    v[4 * i + 1] += w.y;
+    v[4 * i + 2] += w.z;
+    v[4 * i + 3] += w.w;
+  }
   if (g.res && live) {
     const float4* r = reinterpret_cast<const float4*>(g.res + row * g.N + nbase);
 #pragma unroll
@@ -191,8 +205,9 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&bars->acc_full[b]), 1);
-      mbar_init(smem_u32(&bars->acc_empty[b]), 4);   // one arrival per epilogue warp
+      mbar_init(smem_u32(&bars->acc_empty[b]), RG_EPI_WARPS);   // one arrival per epilogue warp
     }
+    for (int q = 0; q < 4; ++q) mbar_init(smem_u32(&bars->ssb[q]), 2);
     mbar_init(smem_u32(&bars->drain), 1);
     bars->abort = 0;
     bars->never = 0;
@@ -285,10 +300,13 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       if (!mbar_wait(smem_u32(&bars->drain), 0, never, RG_DRAIN_NS)) rg_fail(g, bars);
     }
   } else if (warp >= 2) {
-    // ---------------- epilogue: this warp's 32 rows of each tile
-    const int q = warp & 3;
-    int acc_k = 0;
-    Emit emit{base + (uint32_t)(g.stages * stage_bytes) + 1024u + (uint32_t)((warp - 2) * RG_STG_WARP), 0};
+    // ---------------- epilogue: this warp's 32 rows and half of the columns of each tile
+    const int q = warp & 3, hs = (warp - 2) >> 2;
+    const uint32_t misc = base + (uint32_t)(g.stages * stage_bytes) + 1024u;   // partial sums [2][2][128]
+    float* ssx = reinterpret_cast<float*>(smem_raw + (misc - raw));
+    Emit emit{misc + 2048u + (uint32_t)((warp - 2) * RG_STG_WARP), 0};
+    const int U = g.Nt / 16, ub = hs ? (U + 1) / 2 : 0, ue = hs ? U : (U + 1) / 2;
+    int acc_k = 0, norms = 0;
     for (int64_t t = blockIdx.x; t < total; t += gridDim.x) {
       const int buf = acc_k & 1;
       const uint32_t aph = (uint32_t)(acc_k >> 1) & 1u;
@@ -302,53 +320,80 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       const int n0 = (int)(t % g.n_ntiles) * g.Nt;
       const bool live = row < rows;
       const uint32_t tq = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * RG_MAX_NT);
-      if (g.epi == EP_NORM) {
-        float ss = 0.0f;
-        for (int c = 0; c < g.Nt; c += 16) {
-          float v[16];
-          tmem_ld16(tq + c, v);
+      // one pass over this warp's 16-column units, the next unit's TMEM load in
+      // flight while the current one is processed.  mode 0: the epilogue; 1: the
+      // residual stream of EP_NORM and its sum of squares; 2: its normed operand.
+      auto pass = [&](int mode, float inv) -> float {
+        float ss = 0.0f, cur[16], nxt[16];
+        if (ub < ue) {
+          tmem_ld16(tq + 16 * ub, cur);
           tmem_ld_wait();
-          biased(g, row, live, n0 + c, v);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) ss = fmaf(v[i], v[i], ss);
-          emit(g, lane, n0 + c, rbox, v, true, false);
         }
-        const float inv = 1.0f / sqrtf(ss / (float)g.N + g.rms_eps);
-        for (int c = 0; c < g.Nt; c += 16) {
-          float v[16];
-          tmem_ld16(tq + c, v);
-          tmem_ld_wait();
-          biased(g, row, live, n0 + c, v);
+        for (int u = ub; u < ue; ++u) {
+          if (u + 1 < ue) tmem_ld16(tq + 16 * (u + 1), nxt);
+          const int nb = n0 + 16 * u;
+          biased(g, row, live, nb, cur);
+          if (mode == 1) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] = v[i] * inv * g.gain[n0 + c + i];
-          emit(g, lane, n0 + c, rbox, v, false, true);
-        }
-      } else {
-        for (int c = 0; c < g.Nt; c += 16) {
-          float v[16];
-          tmem_ld16(tq + c, v);
-          tmem_ld_wait();
-          const int nb = n0 + c;
-          biased(g, row, live, nb, v);
-          if (g.epi == EP_PROJ) {
-            // the update-gate blocks of the projection rows (z_f, n_f, z_b, n_b)
-            const bool z = nb < g.H || (nb >= 2 * g.H && nb < 3 * g.H);
-            if (z) {
+            for (int i = 0; i < 16; ++i) ss = fmaf(cur[i], cur[i], ss);
+            emit(g, lane, nb, rbox, cur, true, false);
+          } else if (mode == 2) {
+            const float4* gn = reinterpret_cast<const float4*>(g.gain + nb);
 #pragma unroll
-              for (int i = 0; i < 16; ++i) v[i] = sigm(v[i]);
+            for (int i = 0; i < 4; ++i) {
+              const float4 w = __ldg(gn + i);
+              cur[4 * i] = cur[4 * i] * inv * w.x;
+              cur[4 * i + 1] = cur[4 * i + 1] * inv * w.y;
+              cur[4 * i + 2] = cur[4 * i + 2] * inv * w.z;
+              cur[4 * i + 3] = cur[4 * i + 3] * inv * w.w;
             }
-          } else if (g.epi == EP_SILU16) {
+            emit(g, lane, nb, rbox, cur, false, true);
+          } else {
+            if (g.epi == EP_PROJ) {
+              // the update-gate blocks of the projection rows (z_f, n_f, z_b, n_b)
+              if (nb < g.H || (nb >= 2 * g.H && nb < 3 * g.H)) {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) v[i] = v[i] * sigm(v[i]);
+                for (int i = 0; i < 16; ++i) cur[i] = sigm(cur[i]);
+              }
+            } else if (g.epi == EP_SILU16) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) cur[i] = cur[i] * sigm(cur[i]);
+            }
+            const bool h = g.epi == EP_16 || g.epi == EP_SILU16;
+            emit(g, lane, nb, rbox, cur, !h, h);
           }
-          const bool h = g.epi == EP_16 || g.epi == EP_SILU16;
-          emit(g, lane, nb, rbox, v, !h, h);
+          if (u + 1 < ue) {
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) cur[i] = nxt[i];
+          }
         }
+        return ss;
+      };
+      bool ok = true;
+      if (g.epi == EP_NORM) {
+        // the row's sum of squares: this warp's half, then the partner's through
+        // shared memory (double-buffered by tile) and a two-arrival barrier
+        const int par = norms & 1;
+        ssx[(par * 2 + hs) * 128 + 32 * q + lane] = pass(1, 0.0f);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bars->ssb[q]));
+        ok = mbar_wait(smem_u32(&bars->ssb[q]), (uint32_t)par, abort, g.wait_ns);
+        if (ok) {
+          const float tot = ssx[(par * 2) * 128 + 32 * q + lane] + ssx[(par * 2 + 1) * 128 + 32 * q + lane];
+          pass(2, 1.0f / sqrtf(tot / (float)g.N + g.rms_eps));
+        } else if (lane == 0) {
+          rg_fail(g, bars);
+        }
+        ++norms;
+      } else {
+        pass(0, 0.0f);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&bars->acc_empty[buf]));
       ++acc_k;
+      if (!ok) break;
     }
     if (lane == 0) bulk_wait_all();   // every store done before the CTA leaves
   }
@@ -544,87 +589,6 @@ __global__ void pool_mean_rows_kernel(const float* __restrict__ x, const int64_t
   pooled[b * D + c] = acc / (float)n;
 }
 
-// ------------------------------------------------------------------ head
-// The head of Sec. 3.2-3.3 on the pooled vectors, in fp32 on the CUDA cores:
-// RMSNorm (gain g_h), W_h1 (P -> 128) + SiLU, W_h2 (128 -> 5 x n_quantiles), the
-// median quantile per parameter.  One CTA per HR_TRK tracks: thread j owns hidden
-// unit j and reads column j of W_h1 transposed ([P][128], coalesced across the
-// CTA) once for all the CTA's tracks.
-constexpr int HR_TRK = 16, HR_NT = 128;
-
-__host__ __device__ inline size_t head_rows_smem(int P, int Q) {
-  return (size_t)HR_TRK * ((size_t)P + 128 + (size_t)Q + 1) * sizeof(float);
-}
-
-__global__ void __launch_bounds__(HR_NT) head_rows_kernel(const float* __restrict__ pooled,
-                                                          const int32_t* __restrict__ n_hits, int64_t B, int T,
-                                                          int P, int Q, int NQ, float eps, const float* __restrict__ g,
-                                                          const float* __restrict__ w1t, const float* __restrict__ b1,
-                                                          const float* __restrict__ w2, const float* __restrict__ b2,
-                                                          float* __restrict__ out, float* __restrict__ out_q,
-                                                          float* __restrict__ out_pool,
-                                                          unsigned long long* __restrict__ err) {
-  extern __shared__ float hsm[];
-  float* pv = hsm;                    // [HR_TRK][P]
-  float* hid = pv + HR_TRK * P;       // [HR_TRK][128]
-  float* qv = hid + HR_TRK * 128;     // [HR_TRK][Q]
-  float* inv = qv + HR_TRK * Q;       // [HR_TRK]
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int64_t b0 = blockIdx.x * (int64_t)HR_TRK;
-  const int nt = B - b0 < HR_TRK ? (int)(B - b0) : HR_TRK;
-  for (int i = tid; i < HR_TRK * P; i += HR_NT) pv[i] = i < nt * P ? pooled[b0 * P + i] : 0.0f;
-  if (tid < nt) {
-    const int n = n_hits[b0 + tid];
-    if (n < 1 || n > T) atomicAdd(err, 1ull);
-  }
-  __syncthreads();
-  for (int t = warp; t < HR_TRK; t += HR_NT / 32) {
-    float ss = 0.0f;
-    for (int c = lane; c < P; c += 32) ss = fmaf(pv[t * P + c], pv[t * P + c], ss);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-    if (lane == 0) inv[t] = 1.0f / sqrtf(ss / (float)P + eps);
-  }
-  __syncthreads();
-  for (int i = tid; i < nt * P; i += HR_NT) {
-    const int t = i / P, c = i - t * P;
-    if (out_pool) {
-      const int n = n_hits[b0 + t];
-      out_pool[b0 * P + i] = (n < 1 || n > T) ? NAN : pv[i];
-    }
-    pv[i] = pv[i] * inv[t] * g[c];
-  }
-  __syncthreads();
-  {
-    float acc[HR_TRK];
-#pragma unroll
-    for (int t = 0; t < HR_TRK; ++t) acc[t] = b1[tid];
-#pragma unroll 8
-    for (int c = 0; c < P; ++c) {
-      const float w = __ldg(w1t + c * 128 + tid);
-#pragma unroll
-      for (int t = 0; t < HR_TRK; ++t) acc[t] = fmaf(w, pv[t * P + c], acc[t]);
-    }
-#pragma unroll
-    for (int t = 0; t < HR_TRK; ++t) hid[t * 128 + tid] = acc[t] * sigm(acc[t]);
-  }
-  __syncthreads();
-  for (int o = tid; o < nt * Q; o += HR_NT) {
-    const int t = o / Q, q = o - t * Q;
-    float acc = b2[q];
-    const float* wr = w2 + (size_t)q * 128;
-    for (int j = 0; j < 128; ++j) acc = fmaf(wr[j], hid[t * 128 + j], acc);
-    const int n = n_hits[b0 + t];
-    qv[o] = (n < 1 || n > T) ? NAN : acc;
-    if (out_q) out_q[b0 * Q + o] = qv[o];
-  }
-  __syncthreads();
-  for (int o = tid; o < nt * 5; o += HR_NT) {
-    const int t = o / 5, p = o - t * 5;
-    out[(b0 + t) * 5 + p] = qv[t * Q + p * NQ + NQ / 2];
-  }
-}
-
 }  // namespace
 
 // ------------------------------------------------------------------ host side
@@ -632,7 +596,8 @@ struct tf_rows_state {
   int fp16;
   int nsm;
   uint16_t* w16;            // every product's weights, 16-bit, back to back
-  float* w1t;               // the head's W_h1 transposed, [P][128] fp32
+  float* hws;               // the head's workspace, chunk x (P + 128 + Q) floats
+  float* vec;               // the products' bias and gain vectors, each 16-byte aligned
   int doubling;             // fourier_scale[k + 3] == 2 fourier_scale[k] for every k
   int64_t chunk, cap;       // tracks per chunk; rows of the workspace (chunk * max_hits)
   int64_t* row0;            // [chunk + 1]
@@ -710,9 +675,9 @@ int tile_n(int N) {
 }
 
 // alignment slack, the ring of stages, the barriers (one 1 KB block), the
-// epilogue warps' staging buffers
+// RMSNorm partial sums (2 KB), the epilogue warps' staging buffers
 size_t gemm_smem(const RowGemm& g) {
-  return 1024 + (size_t)g.stages * (RG_A_BYTES + g.Nt * 128) + 1024 + 4 * RG_STG_WARP;
+  return 1024 + (size_t)g.stages * (RG_A_BYTES + g.Nt * 128) + 1024 + 2048 + RG_EPI_WARPS * RG_STG_WARP;
 }
 
 // A [cap][K] (16-bit, row stride K) times W [N][K]; the epilogue's pointers are set by the caller.
@@ -773,7 +738,8 @@ void tf_rows_destroy(trackfit_ctx* h) {
   tf_rows_state* r = h->rows;
   if (!r) return;
   tf_free(r->w16);
-  tf_free(r->w1t);
+  tf_free(r->hws);
+  tf_free(r->vec);
   tf_free(r->row0);
   tf_free(r->tot);
   tf_free(r->a0);
@@ -837,20 +803,13 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
     for (size_t i = 0; i < m.n * m.k; ++i) w[m.at + i] = to16(host_w[m.off + i], r->fp16);
   int st = tf_status_from_cuda(tf_malloc((void**)&r->w16, n16 * 2));
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(r->w16, w.data(), n16 * 2, cudaMemcpyHostToDevice));
-  {
-    std::vector<float> t((size_t)s.P * 128);
-    for (int j = 0; j < 128; ++j)
-      for (int c = 0; c < s.P; ++c) t[(size_t)c * 128 + j] = host_w[o.head_w1 + (size_t)j * s.P + c];
-    if (st == TRACKFIT_OK) st = tf_status_from_cuda(tf_malloc((void**)&r->w1t, t.size() * 4));
-    if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(r->w1t, t.data(), t.size() * 4, cudaMemcpyHostToDevice));
-  }
   if (st != TRACKFIT_OK) return st;
   // workspace, sized for whole chunks of full-length tracks
   const size_t hsw = attn ? (H > D ? H : D) : D;
   const size_t xyw = attn ? D : (2 * H > D ? 2 * H : D);
   const size_t pw = attn ? 3 * D : 4 * H;
   const size_t row_bytes = 2 * (E + hsw + xyw + (attn ? D : 0)) + 4 * (pw + (attn ? 2 * D : 0));
-  const size_t track_bytes = (size_t)s.T * row_bytes + 4 * (size_t)s.P + 16;
+  const size_t track_bytes = (size_t)s.T * row_bytes + 4 * (2 * (size_t)s.P + s.Hh + s.Q) + 16;
   int64_t chunk = (int64_t)(RG_WS_BUDGET / track_bytes);
   if (chunk > 4194304) chunk = 4194304;
   chunk = chunk / PLAN_NT * PLAN_NT;
@@ -868,25 +827,53 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
   alloc((void**)&r->xy16, cap * xyw * 2);
   alloc((void**)&r->p32, cap * pw * 4);
   alloc((void**)&r->pooled, (size_t)chunk * s.P * 4);
+  alloc((void**)&r->hws, (size_t)chunk * (s.P + s.Hh + s.Q) * 4);
   if (attn) {
     alloc((void**)&r->o16, cap * D * 2);
     alloc((void**)&r->x32, cap * D * 4);
     alloc((void**)&r->x1, cap * D * 4);
   }
   if (st != TRACKFIT_OK) return st;
+  // 16-byte aligned copies of the bias and gain vectors the epilogues read
+  std::map<size_t, size_t> at;
+  std::vector<float> hv;
+  auto want = [&](size_t off, size_t n) {
+    if (at.count(off)) return;
+    at[off] = hv.size();
+    hv.insert(hv.end(), host_w + off, host_w + off + n);
+    hv.resize((hv.size() + 3) / 4 * 4, 0.0f);
+  };
+  want(o.emb_b1, D);
+  want(o.emb_b2, D);
+  for (int l = 0; l < s.L; ++l) {
+    const tf_layer_off& lo = o.layer[l];
+    if (!attn) {
+      want(lo.b_in, 4 * H);
+      continue;
+    }
+    want(lo.g, D);
+    want(lo.b_in, 3 * D);
+    want(lo.b_m, D);
+    want(lo.g2, D);
+    want(lo.b1, H);
+    want(lo.b2, D);
+  }
+  st = tf_status_from_cuda(tf_malloc((void**)&r->vec, hv.size() * 4));
+  if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(r->vec, hv.data(), hv.size() * 4, cudaMemcpyHostToDevice));
+  if (st != TRACKFIT_OK) return st;
+  auto V = [&](size_t off) -> const float* { return r->vec + at[off]; };
   // the products of one chunk
-  const float* Wd = h->d_w;
   const uint16_t* w16 = r->w16;
   size_t mi = 0;
   bool ok = make_gemm(r->e1, r, r->a0, (int)E, w16 + mats[mi++].at, (int)D, EP_SILU16);
-  r->e1.bias = Wd + o.emb_b1;
+  r->e1.bias = V(o.emb_b1);
   r->e1.out16 = r->hs16;
   ok = ok && make_gemm(r->e2, r, r->hs16, (int)D, w16 + mats[mi++].at, (int)D, attn ? EP_NORM : EP_16);
-  r->e2.bias = Wd + o.emb_b2;
+  r->e2.bias = V(o.emb_b2);
   r->e2.out16 = r->xy16;
   if (attn) {   // x = embedding; the first layer's pre-norm operand
     r->e2.out32 = r->x32;
-    r->e2.gain = Wd + o.layer[0].g;
+    r->e2.gain = V(o.layer[0].g);
     r->e2.rms_eps = s.rms_eps;
   }
   for (int l = 0; l < s.L && ok; ++l) {
@@ -895,7 +882,7 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
     if (!attn) {   // Sec. 3.2: the layer input (D, then 2H wide) to z_f, n_f, z_b, n_b
       ok = make_gemm(g[0], r, r->xy16, l == 0 ? (int)D : (int)(2 * H), w16 + mats[mi++].at, (int)(4 * H), EP_PROJ);
       g[0].H = (int)H;
-      g[0].bias = Wd + lo.b_in;
+      g[0].bias = V(lo.b_in);
       g[0].out32 = r->p32;
       continue;
     }
@@ -905,21 +892,21 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
          make_gemm(g[1], r, r->o16, (int)D, w16 + mats[mi++].at, (int)D, EP_NORM) &&
          make_gemm(g[2], r, r->xy16, (int)D, w16 + mats[mi++].at, (int)H, EP_SILU16) &&
          make_gemm(g[3], r, r->hs16, (int)H, w16 + mats[mi++].at, (int)D, l + 1 < s.L ? EP_NORM : EP_RES);
-    g[0].bias = Wd + lo.b_in;
+    g[0].bias = V(lo.b_in);
     g[0].out32 = r->p32;
-    g[1].bias = Wd + lo.b_m;
+    g[1].bias = V(lo.b_m);
     g[1].res = r->x32;
-    g[1].gain = Wd + lo.g2;
+    g[1].gain = V(lo.g2);
     g[1].rms_eps = s.rms_eps;
     g[1].out32 = r->x1;
     g[1].out16 = r->xy16;
-    g[2].bias = Wd + lo.b1;
+    g[2].bias = V(lo.b1);
     g[2].out16 = r->hs16;
-    g[3].bias = Wd + lo.b2;
+    g[3].bias = V(lo.b2);
     g[3].res = r->x1;
     g[3].out32 = r->x32;
     if (l + 1 < s.L) {
-      g[3].gain = Wd + o.layer[l + 1].g;
+      g[3].gain = V(o.layer[l + 1].g);
       g[3].rms_eps = s.rms_eps;
       g[3].out16 = r->xy16;
     }
@@ -933,9 +920,7 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
   upd(r->e2);
   for (int l = 0; l < s.L; ++l)
     for (int k = 0; k < (attn ? 4 : 1); ++k) upd(r->lay[l][k]);
-  if (cudaFuncSetAttribute(row_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r->smem) != cudaSuccess ||
-      cudaFuncSetAttribute(head_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)head_rows_smem(s.P, s.Q)) != cudaSuccess)
+  if (cudaFuncSetAttribute(row_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)r->smem) != cudaSuccess)
     return TRACKFIT_ERR_CUDA;
   if (attn && (tf_attn::allow_smem<__half>(s.T, s.D, s.NH) != cudaSuccess ||
                tf_attn::allow_smem<__nv_bfloat16>(s.T, s.D, s.NH) != cudaSuccess))
@@ -985,12 +970,7 @@ int rows_chunk(trackfit_ctx* h, const float* hits, const int64_t* offs, const in
     dim3 grid((unsigned)nb, (unsigned)((s.D + 127) / 128));
     pool_mean_rows_kernel<<<grid, 128, 0, st>>>(r->x32, r->row0, nc, nb, s.T, s.D, r->pooled);
   }
-  const tf_blob_off& o = h->off;
-  const float* W = h->d_w;
-  head_rows_kernel<<<(unsigned)((nb + HR_TRK - 1) / HR_TRK), HR_NT, head_rows_smem(s.P, s.Q), st>>>(
-      r->pooled, nc, nb, s.T, s.P, s.Q, s.NQ, s.rms_eps, W + o.head_g, r->w1t, W + o.head_b1, W + o.head_w2,
-      W + o.head_b2, out, out_q, out_pool, err);
-  return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
+  return tf_simt_head_batched(s, h->off, h->d_w, r->pooled, nc, nb, r->hws, out, out_q, out_pool, err, st);
 }
 
 }  // namespace

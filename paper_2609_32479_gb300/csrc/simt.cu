@@ -278,6 +278,24 @@ __global__ void __launch_bounds__(128) pool_head_kernel(const float* __restrict_
 // Per hit row: E (Fourier) + U + X + XH + PR + Y + X1, with U = D and PR = 4H + D,
 // Y = 2H (recurrent topologies) or U = H (the MLP), PR = 3D (q, k, v) and Y = D
 // (the attention output) for ATTENTION.
+// The head's last step on given quantiles qv [B][Q]: invalid tracks (count
+// outside [1, T]) get NaN rows and are counted; the medians go to out, the
+// quantiles and the pooled vectors to the optional exports.
+__global__ void head_finish_kernel(const float* __restrict__ qv, const float* __restrict__ pooled,
+                                   const int32_t* __restrict__ n_hits, int64_t B, tf_shape s, float* __restrict__ out,
+                                   float* __restrict__ out_q, float* __restrict__ out_pool, unsigned long long* err) {
+  const int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const int n = n_hits[b];
+  const bool bad = n < 1 || n > s.T;
+  if (bad) atomicAdd(err, 1ull);
+  for (int p = 0; p < 5; ++p) out[b * 5 + p] = bad ? NAN : qv[b * s.Q + p * s.NQ + s.NQ / 2];
+  if (out_q)
+    for (int o = 0; o < s.Q; ++o) out_q[b * s.Q + o] = bad ? NAN : qv[b * s.Q + o];
+  if (out_pool)
+    for (int c = 0; c < s.P; ++c) out_pool[b * s.P + c] = bad ? NAN : pooled[b * s.P + c];
+}
+
 size_t ws_floats_per_track(const tf_shape& s) {
   const size_t D = s.D, H = s.H;
   const size_t row = s.topology == TRACKFIT_TOPOLOGY_ATTENTION ? H + 7 * D : 5 * D + 6 * H;
@@ -432,6 +450,29 @@ int tf_simt_forward_explicit(const tf_shape& s, const tf_blob_off& o, const floa
 }
 
 size_t tf_simt_bytes_per_track(const tf_shape& s) { return ws_floats_per_track(s) * sizeof(float); }
+
+// The head of Sec. 3.2-3.3 on given pooled vectors [B][P] as three batched
+// steps over all tracks: RMSNorm, the tiled product with W_h1 (SiLU), the tiled
+// product with W_h2, then the medians.  ws: B (P + 128 + Q) floats.
+int tf_simt_head_batched(const tf_shape& s, const tf_blob_off& o, const float* W, const float* pooled,
+                         const int32_t* n_hits, int64_t B, float* ws, float* out, float* out_q, float* out_pool,
+                         unsigned long long* err, cudaStream_t st) {
+  float* pn = ws;
+  float* hid = pn + B * s.P;
+  float* qv = hid + B * s.Hh;
+  rmsnorm_kernel<<<(unsigned)((B + 7) / 8), 256, 0, st>>>(pooled, B, s.P, W + o.head_g, s.rms_eps, pn);
+  GemmArgs g{};
+  g.R = (int)B;
+  g.rnd = 0;
+  g.A = pn; g.lda = s.P; g.W = W + o.head_w1; g.bias = W + o.head_b1; g.C = hid; g.ldc = s.Hh;
+  g.N = s.Hh; g.K = s.P; g.epi = EPI_SILU;
+  if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+  g.A = hid; g.lda = s.Hh; g.W = W + o.head_w2; g.bias = W + o.head_b2; g.C = qv; g.ldc = s.Q;
+  g.N = s.Q; g.K = s.Hh; g.epi = EPI_STORE;
+  if (launch_gemm(g, st)) return TRACKFIT_ERR_CUDA;
+  head_finish_kernel<<<(unsigned)((B + 255) / 256), 256, 0, st>>>(qv, pooled, n_hits, B, s, out, out_q, out_pool, err);
+  return cudaPeekAtLastError() == cudaSuccess ? TRACKFIT_OK : TRACKFIT_ERR_CUDA;
+}
 
 // The head of Sec. 3.2-3.3 on given pooled vectors [B][P]: out [B][5], optional
 // quantiles [B][Q] and the pooled export (NaN rows for invalid tracks).

@@ -85,6 +85,9 @@ int tf_simt_forward(trackfit_ctx* h, const float* hits, const int32_t* n_hits, i
 int tf_simt_head(const tf_shape& s, const tf_blob_off& o, const float* W, const float* pooled,
                  const int32_t* n_hits, int64_t B, float* out, float* out_q, float* out_pool,
                  unsigned long long* err, cudaStream_t st);
+int tf_simt_head_batched(const tf_shape& s, const tf_blob_off& o, const float* W, const float* pooled,
+                         const int32_t* n_hits, int64_t B, float* ws, float* out, float* out_q, float* out_pool,
+                         unsigned long long* err, cudaStream_t st);
 int tf_simt_debug_scan(const float* a, const float* b, const float* x, const int32_t* n_hits,
                        int64_t B, int T, int C, float* hf, float* hb, cudaStream_t st);
 
