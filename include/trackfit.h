@@ -247,6 +247,11 @@ void trackfit_destroy(trackfit_t h);
 /* Static description of a status code. */
 const char* trackfit_strerror(int status);
 
+/* The CUDA error behind the calling thread's last TRACKFIT_ERR_CUDA or
+ * TRACKFIT_ERR_OOM, with the step it came from ("" if none yet).  The string is
+ * owned by the library and valid until the thread's next failing call. */
+const char* trackfit_last_error(void);
+
 /* Test hook: masked bidirectional linear recurrence h_t = a_t h_{t-1} + b_t x_t
  * (Eq. 2 written as a linear recurrence, with a = 1 - z, b = z, x = n) on the device.
  * a, b, x, h_fwd, h_bwd: device [n_tracks][T][C] fp32; n_hits device [n_tracks].

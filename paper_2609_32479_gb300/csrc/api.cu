@@ -8,11 +8,21 @@
 
 #include "trackfit_internal.h"
 
+// The CUDA error behind this thread's last TRACKFIT_ERR_CUDA / ERR_OOM.
+static thread_local char g_last_error[160] = "";
+
+void tf_note_cuda(cudaError_t e, const char* where) {
+  std::snprintf(g_last_error, sizeof(g_last_error), "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
 int tf_status_from_cuda(cudaError_t e) {
   if (e == cudaSuccess) return TRACKFIT_OK;
+  tf_note_cuda(e, "CUDA call");
   if (e == cudaErrorMemoryAllocation) return TRACKFIT_ERR_OOM;
   return TRACKFIT_ERR_CUDA;
 }
+
+extern "C" const char* trackfit_last_error(void) { return g_last_error; }
 
 // Allocation bookkeeping for the test hook trackfit_debug_alloc (host side; the
 // counters are not meant for concurrent use).

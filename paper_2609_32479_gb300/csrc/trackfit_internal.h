@@ -112,6 +112,9 @@ int tf_rows_wait_limit(trackfit_ctx* h, int64_t limit_ns);
 
 // api.cu
 int tf_status_from_cuda(cudaError_t e);
+// Record e as the calling thread's last CUDA error (trackfit_last_error), with
+// where it happened.
+void tf_note_cuda(cudaError_t e, const char* where);
 // Every device allocation of a handle goes through these two (counted; a test
 // hook can make one fail as if the device were out of memory).  tf_free
 // accepts null.

@@ -27,7 +27,7 @@ EXPORTS = ("trackfit_weight_count", "trackfit_create", "trackfit_forward", "trac
            "trackfit_destroy", "trackfit_strerror", "trackfit_debug_scan", "trackfit_debug_umma",
            "trackfit_profile", "trackfit_profile_read", "trackfit_forward_noalloc",
            "trackfit_debug_schedule", "trackfit_debug_wait_limit", "trackfit_debug_alloc", "trackfit_seed",
-           "trackfit_decode", "trackfit_forward_packed")
+           "trackfit_decode", "trackfit_forward_packed", "trackfit_last_error")
 
 
 class Config(ctypes.Structure):
@@ -44,7 +44,10 @@ class Config(ctypes.Structure):
 class TrackfitError(RuntimeError):
     def __init__(self, status: int, what: str):
         self.status = status
-        super().__init__(f"{what}: {strerror(status)} (status {status})")
+        detail = ""
+        if status in (ERR_CUDA, ERR_OOM):
+            detail = load().trackfit_last_error().decode()
+        super().__init__(f"{what}: {strerror(status)} (status {status})" + (f" [{detail}]" if detail else ""))
 
 
 _lib: Optional[ctypes.CDLL] = None
@@ -80,6 +83,8 @@ def load() -> ctypes.CDLL:
     lib.trackfit_destroy.restype = None
     lib.trackfit_strerror.argtypes = [ctypes.c_int]
     lib.trackfit_strerror.restype = ctypes.c_char_p
+    lib.trackfit_last_error.argtypes = []
+    lib.trackfit_last_error.restype = ctypes.c_char_p
     lib.trackfit_debug_scan.argtypes = [vp, vp, vp, vp, i64, i32, i32, vp, vp, vp]
     lib.trackfit_debug_scan.restype = ctypes.c_int
     lib.trackfit_debug_umma.argtypes = [vp, vp, vp, i32, vp, vp]

@@ -75,17 +75,32 @@ def test_paper_encoder_matches_the_oracle(T, prec, path, want):
     assert ok, msg
 
 
-def test_paper_encoder_masking_is_bit_exact(T):
+@pytest.mark.parametrize("path", [None, 1])
+def test_paper_encoder_masking_and_order(T, path):
+    """NaN in the padded entries changes nothing, bit for bit, on both paths.  A
+    permuted batch: bit-exact on the CUDA cores (each track's arithmetic is fixed);
+    on the tensor-core path the fused scans compose a track's per-hit maps in an
+    order that depends on where the track crosses a 32-row lane quadrant of its
+    tile, so a track moved to another position may round differently in fp32,
+    and a 16-bit operand rounding downstream can then differ: there the permuted
+    results must agree within the fp16 bar."""
     w = W.workload("paper", n_tracks=300)
     tb = W.gen_tracks(w)
     hits, _ = oracle_inputs(w, tb)
     blob = W.gen_weights(w.model, w.weight_seed)
-    base = gpu_encoder(T, w.model, blob, hits, tb.n_hits)[0]
+    base = gpu_encoder(T, w.model, blob, hits, tb.n_hits, path)[0]
     nan = hits.copy()
     nan[np.arange(w.model.max_hits)[None, :] >= tb.n_hits[:, None]] = np.nan
-    np.testing.assert_array_equal(gpu_encoder(T, w.model, blob, nan, tb.n_hits)[0], base)
+    np.testing.assert_array_equal(gpu_encoder(T, w.model, blob, nan, tb.n_hits, path)[0], base)
     perm = np.random.default_rng(2).permutation(300)
-    np.testing.assert_array_equal(gpu_encoder(T, w.model, blob, hits[perm], tb.n_hits[perm])[0], base[perm])
+    got = gpu_encoder(T, w.model, blob, hits[perm], tb.n_hits[perm], path)[0]
+    if path == 1:
+        np.testing.assert_array_equal(got, base[perm])
+    else:
+        ok, msg = parity_ok(got, base[perm], W.PRECISION_FP16)
+        print(f"paper encoder, permuted batch on the tensor cores: {msg}")
+        assert ok, msg
+        np.testing.assert_array_equal(gpu_encoder(T, w.model, blob, hits, tb.n_hits, path)[0], base)  # repeatable
 
 
 def test_seed_guided_forward_matches_the_oracle(T):
@@ -129,3 +144,39 @@ def test_seed_guided_forward_matches_the_oracle(T):
     scale = np.abs(c[ok_seed] - corr_o[ok_seed]) * gain + 1e-6 * np.maximum(np.abs(dec_o[ok_seed]), 1.0)
     assert np.all(d <= scale), np.max(d - scale, axis=0)
     assert np.all(np.isnan(o[~ok_seed]))
+
+
+@pytest.mark.parametrize("T_,L,pool,n_tracks", [(64, 3, W.POOL_ENDPOINTS, 700), (24, 2, W.POOL_MEAN, 500),
+                                                (8, 1, W.POOL_ENDPOINTS, 600)])
+def test_concatenation_shapes_on_the_tensor_cores(T, T_, L, pool, n_tracks):
+    """The concatenation topology with fp16 operands on the packed-row tensor-core
+    path beyond the paper's shape: tracks of 1-64 hits (whole tracks per 128-row
+    tile, so a 64-hit track fills half a tile and segments of 256 tracks close
+    partial tiles), three layers (a layer's operand and its output alternate
+    between two buffers), mean pooling (the scans then run as their own kernel),
+    invalid counts; against the oracle at the fp16 bar, invalid tracks NaN."""
+    m = W.ModelConfig(max_hits=T_, d_model=128, d_hidden=192, n_layers=L, precision=W.PRECISION_FP16, pool=pool,
+                      topology=W.TOPOLOGY_CONCAT)
+    w = W.Workload("c", n_tracks, m, layout="sweep", n_barrel=T_, min_hits=T_)
+    tb = W.gen_tracks(w)
+    n = np.random.default_rng(T_ + L).integers(1, T_ + 1, n_tracks).astype(np.int32)
+    n[:40] = T_
+    n[40:60] = 1
+    n[77], n[300] = 0, T_ + 1
+    blob = W.gen_weights(m, 5)
+    dev = torch.device("cuda:0")
+    with T.Trackfit(m, blob) as tf:
+        out = torch.full((n_tracks, 5), -7.0, device=dev)
+        tf.forward(torch.from_numpy(tb.hits).to(dev), torch.from_numpy(n).to(dev), out)
+        torch.cuda.synchronize()
+        st = tf.device_errors()
+        path = tf.path
+    got = out.cpu().numpy()
+    assert path.startswith("tcgen05-rows"), path
+    assert st == (T.ERR_BAD_HITS, 2)
+    assert np.all(np.isnan(got[[77, 300]]))
+    good = np.setdiff1d(np.arange(n_tracks), [77, 300])
+    ref = O.forward(dataclasses.asdict(m), blob, tb.hits[good], n[good])
+    ok, msg = parity_ok(got[good], ref, W.PRECISION_FP16)
+    print(f"concatenation T={T_} L={L} pool={pool}: {msg}")
+    assert ok, msg
