@@ -6,11 +6,15 @@
 // q, k, v are the fp32 outputs of the qkv projection; scores, softmax and the
 // weighted sum run in fp32.
 //
-// One CTA per track stages the track's q, k, v rows in shared memory; warp w
-// takes heads w, w + 4, ...; lane i takes queries i and i + 32 and keeps its
-// query and its output (dh values each) in registers, so every key and value is
-// a broadcast read of shared memory.  The softmax takes two passes over the keys:
-// the maximum score, then the exponentials, their sum and the weighted values.
+// One CTA per track stages the track's keys and values in shared memory, each
+// head's slice of a row padded by 4 floats so that the heads fall in different
+// banks; thread i takes the (head, query) items i, i + 128, ... (head = item / n,
+// query = item % n), keeps its query and its output (dh values each) in
+// registers and reads every key and value of its head as a broadcast within the
+// threads of that head.  With n hits a track keeps n x heads threads busy (52 at
+// 13 hits and 4 heads); the other warps only stage.  The softmax takes two passes
+// over the keys: the maximum score, then the exponentials, their sum and the
+// weighted values.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -25,8 +29,10 @@ __device__ __forceinline__ void put(__nv_bfloat16* p, float v) { *p = __float2bf
 
 constexpr int THREADS = 128;
 
-// Shared memory of one CTA: T rows of 3 D + 4 floats (q, k, v; rows 16-byte aligned).
-__host__ __device__ inline size_t smem_bytes(int T, int D) { return (size_t)T * (3 * D + 4) * sizeof(float); }
+// Shared memory of one CTA: keys and values, T rows x NH heads x (dh + 4) floats each.
+__host__ __device__ inline size_t smem_bytes(int T, int D, int NH) {
+  return (size_t)2 * T * (D + 4 * NH) * sizeof(float);
+}
 
 template <int DH>
 __device__ __forceinline__ float dot(const float (&q)[DH], const float* k) {
@@ -59,10 +65,15 @@ __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* _
   int n = n_hits[b];
   if (n < 1 || n > T) n = 0;
   const int64_t r0 = row0 ? row0[b] : b * (int64_t)T;
-  const int ls = 3 * D + 4, w4 = (3 * D) / 4;
+  const int hs = DH + 4, rs = NH * hs;   // padded head slice, row of one matrix
+  float* ks = sm;
+  float* vs = sm + (size_t)T * rs;
+  const int w4 = (2 * D) / 4;            // float4s of k and v per row
   for (int i = threadIdx.x; i < n * w4; i += THREADS) {
-    const int j = i / w4, c = i - j * w4;
-    *reinterpret_cast<float4*>(sm + j * ls + 4 * c) = *reinterpret_cast<const float4*>(qkv + (r0 + j) * ldq + 4 * c);
+    const int j = i / w4, c = 4 * (i - j * w4);
+    const int m = c >= D, cc = c - m * D, h = cc / DH, e = cc - h * DH;
+    *reinterpret_cast<float4*>((m ? vs : ks) + j * rs + h * hs + e) =
+        *reinterpret_cast<const float4*>(qkv + (r0 + j) * ldq + D + c);
   }
   if (!row0) {   // padded layout: zero the padding rows
     for (int i = threadIdx.x; i < (T - n) * D; i += THREADS) {
@@ -71,42 +82,42 @@ __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* _
     }
   }
   __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float scale = rsqrtf((float)DH);
-  for (int h = warp; h < NH; h += THREADS / 32) {
-    const int c0 = h * DH;
-    for (int t0 = 0; t0 < n; t0 += 32) {
-      const int t = t0 + lane;
-      const float* qr = sm + (t < n ? t : 0) * ls + c0;
-      float q[DH], acc[DH];
+  for (int it = threadIdx.x; it < NH * n; it += THREADS) {
+    const int h = it / n, t = it - h * n;
+    const float* qr = qkv + (r0 + t) * ldq + h * DH;
+    float q[DH], acc[DH];
 #pragma unroll
-      for (int i = 0; i < DH; ++i) {
-        q[i] = qr[i];
-        acc[i] = 0.0f;
-      }
-      float m = -INFINITY;
-      for (int j = 0; j < n; ++j) m = fmaxf(m, dot<DH>(q, sm + j * ls + D + c0) * scale);
-      float l = 0.0f;
-      for (int j = 0; j < n; ++j) {
-        const float p = expf(dot<DH>(q, sm + j * ls + D + c0) * scale - m);
-        l += p;
-        const float* vr = sm + j * ls + 2 * D + c0;
+    for (int i = 0; i < DH; i += 4) {
+      const float4 a = *reinterpret_cast<const float4*>(qr + i);
+      q[i] = a.x;
+      q[i + 1] = a.y;
+      q[i + 2] = a.z;
+      q[i + 3] = a.w;
+      acc[i] = acc[i + 1] = acc[i + 2] = acc[i + 3] = 0.0f;
+    }
+    const float* kh = ks + h * hs;
+    const float* vh = vs + h * hs;
+    float m = -INFINITY;
+    for (int j = 0; j < n; ++j) m = fmaxf(m, dot<DH>(q, kh + j * rs) * scale);
+    float l = 0.0f;
+    for (int j = 0; j < n; ++j) {
+      const float p = expf(dot<DH>(q, kh + j * rs) * scale - m);
+      l += p;
+      const float* vr = vh + j * rs;
 #pragma unroll
-        for (int i = 0; i < DH; i += 4) {
-          const float4 v = *reinterpret_cast<const float4*>(vr + i);
-          acc[i] = fmaf(p, v.x, acc[i]);
-          acc[i + 1] = fmaf(p, v.y, acc[i + 1]);
-          acc[i + 2] = fmaf(p, v.z, acc[i + 2]);
-          acc[i + 3] = fmaf(p, v.w, acc[i + 3]);
-        }
-      }
-      if (t < n) {
-        const float inv = 1.0f / l;
-        OutT* orow = o + (r0 + t) * ldo + c0;
-#pragma unroll
-        for (int i = 0; i < DH; ++i) put(orow + i, acc[i] * inv);
+      for (int i = 0; i < DH; i += 4) {
+        const float4 v = *reinterpret_cast<const float4*>(vr + i);
+        acc[i] = fmaf(p, v.x, acc[i]);
+        acc[i + 1] = fmaf(p, v.y, acc[i + 1]);
+        acc[i + 2] = fmaf(p, v.z, acc[i + 2]);
+        acc[i + 3] = fmaf(p, v.w, acc[i + 3]);
       }
     }
+    const float inv = 1.0f / l;
+    OutT* orow = o + (r0 + t) * ldo + h * DH;
+#pragma unroll
+    for (int i = 0; i < DH; ++i) put(orow + i, acc[i] * inv);
   }
 }
 
@@ -115,7 +126,7 @@ __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* _
 template <typename OutT>
 inline cudaError_t launch(const float* qkv, int ldq, const int64_t* row0, const int32_t* n_hits, int64_t B, int T,
                           int D, int NH, OutT* o, int ldo, cudaStream_t st) {
-  const size_t sm = smem_bytes(T, D);
+  const size_t sm = smem_bytes(T, D, NH);
   const unsigned g = (unsigned)B;
 #define TF_ATTN_CASE(DHV) \
   case DHV:               \
@@ -138,7 +149,7 @@ inline cudaError_t launch(const float* qkv, int ldq, const int64_t* row0, const 
 // The dynamic shared memory of the launches above for tracks of T hits at width D.
 template <typename OutT>
 inline cudaError_t allow_smem(int T, int D, int NH) {
-  const int sm = (int)smem_bytes(T, D);
+  const int sm = (int)smem_bytes(T, D, NH);
   if (sm <= 48 * 1024) return cudaSuccess;
 #define TF_ATTN_ATTR(DHV) \
   case DHV:               \

@@ -51,8 +51,7 @@ constexpr int RG_KC = 64;                         // k per stage (one 128-byte s
 constexpr int RG_A_BYTES = RG_ROWS * RG_KC * 2;   // 16 KB
 constexpr int RG_MAX_NT = 256;                    // MMA N per tile (two buffers fill the 512 TMEM columns)
 constexpr int RG_SMEM_BUDGET = 170 * 1024;        // the ring of stages
-constexpr int SCB = 8;                            // channels per batch of the fused scans
-constexpr int RG_MISC = 7168;                     // RMSNorm partial sums, scan carries and flags
+constexpr int RG_MISC = 2048;                     // RMSNorm partial sums
 constexpr int RG_STG_WARP = 6144;                 // per epilogue warp: 2 x (32 rows x 16 fp32) + 2 x (32 x 16 16-bit)
 constexpr int RG_MAX_STAGES = 8;
 constexpr uint64_t RG_WAIT_NS = 2000000000ull;
@@ -66,8 +65,7 @@ enum {
   EP_16 = 2,         // out16 = v
   EP_SILU16 = 3,     // out16 = SiLU(v)
   EP_NORM = 4,       // x = v (+ res): out32 = x, out16 = RMSNorm(x) g
-  EP_RES = 5,        // out32 = res + v
-  EP_SCAN = 6        // the concatenation layer's projection and both scans (rows: whole tracks per tile)
+  EP_RES = 5         // out32 = res + v
 };
 
 struct RowGemm {
@@ -75,7 +73,6 @@ struct RowGemm {
   CUtensorMap tw;             // W [N][K] 16-bit, box 64 x Nt, 128-byte swizzle
   CUtensorMap to32;           // out32 [cap][N] fp32, box 16 x 32 (stores)
   CUtensorMap to16;           // out16 [cap][N] 16-bit, box 16 x 32 (stores)
-  CUtensorMap to16h;          // the same, box 8 x 32 (EP_SCAN)
   const int64_t* n_rows;      // device: rows of this chunk
   int K, N, Nt, n_ntiles, kchunks, stages;
   int epi;
@@ -88,16 +85,7 @@ struct RowGemm {
   float* out32;               // fp32 [rows][N]
   void* out16;                // 16-bit [rows][N]
   int fp16;                   // 16-bit format of A, W and out16: 1 fp16, 0 bf16
-  int N16;                    // columns of out16 (N, or 2H for EP_SCAN)
-  // EP_SCAN: the W_in rows come in groups of 64 channels [z_f | n_f | z_b | n_b], one
-  // group per 256-column tile; out16 = the states [h_f | h_b] (the next layer's
-  // operand) or, on the last layer, pooled = the endpoint states
-  const int32_t* rtrk;        // the row's track (-1: padding)
-  int64_t ntrk;               // tracks of the chunk (a larger index is treated as padding)
   int64_t cap;                // rows of the workspace (the row count is clamped to it)
-  const int64_t* row0;        // first row of each track
-  const int32_t* nh;          // hit count of each track
-  float* pooled;              // [B][2H] fp32
   unsigned long long* err;    // [1]: expired bounded waits
   uint64_t wait_ns;
 };
@@ -106,7 +94,6 @@ struct RgBars {
   uint64_t full[RG_MAX_STAGES], empty[RG_MAX_STAGES];
   uint64_t acc_full[2], acc_empty[2], drain;
   uint64_t ssb[4];            // RMSNorm: the two warps of a lane quadrant exchange their partial sums
-  uint64_t xb[2];             // EP_SCAN: the four lane-quadrant warps of a column half exchange scan carries
   uint32_t tmem_base;
   int abort;
   int never;                  // a flag nothing sets: for the waits at exit that must not give up on abort
@@ -175,22 +162,6 @@ struct Emit {
     }
     ++chunk;
   }
-  // an 8-column 16-bit box (16 bytes a row, no swizzle), in the 16-bit buffers
-  __device__ __forceinline__ void half(const RowGemm& g, int lane, int nb, int row, const float (&v)[SCB]) {
-    const int p = chunk & 1;
-    if (lane == 0) bulk_wait_read1();
-    __syncwarp();
-    const uint32_t a = stg + 4096 + p * 1024 + lane * 16;
-    sts4(a, pack16(v[0], v[1], g.fp16), pack16(v[2], v[3], g.fp16), pack16(v[4], v[5], g.fp16),
-         pack16(v[6], v[7], g.fp16));
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) {
-      tma_store_2d(&g.to16h, stg + 4096 + p * 1024, nb, row);
-      bulk_commit();
-    }
-    ++chunk;
-  }
 };
 
 // acc + bias (+ res) of 16 columns; the same arithmetic in both passes of EP_NORM.
@@ -218,155 +189,8 @@ __device__ __forceinline__ void biased(const RowGemm& g, int64_t row, bool live,
   }
 }
 
-// acc + bias of 8 columns
-__device__ __forceinline__ void biased8(const RowGemm& g, int nbase, float (&v)[8]) {
-  const float4* bb = reinterpret_cast<const float4*>(g.bias + nbase);
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {
-    const float4 w = __ldg(bb + i);
-    v[4 * i] += w.x;
-    v[4 * i + 1] += w.y;
-    v[4 * i + 2] += w.z;
-    v[4 * i + 3] += w.w;
-  }
-}
-
 __device__ void rg_fail(const RowGemm& g, RgBars* b) {
   if (atomicExch(&b->abort, 1) == 0) atomicAdd(g.err + 1, 1ull);
-}
-
-// ------------------------------------------------------------------ fused scans
-// EP_SCAN epilogue of one tile (Sec. 3.2, Eq. 2): the tile holds whole tracks, its
-// 256 columns are z_f, n_f, z_b, n_b of 64 channels; this warp takes 32 rows (lanes)
-// and 32 channels (batches of SCB).  Per channel the recurrence
-// h_t = (1 - z_t) h_{t-1} + z_t n_t is an affine map of h_{t-1}; the maps of a
-// warp's rows are composed by a segmented scan over the lanes (a track's first row
-// starts a segment forward, its last row backward; a padding row is a segment of
-// its own), then the carries enter from the other lane-quadrant warps of the tile
-// (tracks span quadrants, never tiles) through shared memory.  Out: the states
-// [h_f | h_b] as the next layer's 16-bit operand, or, on the last layer, the
-// forward state at each track's last hit and the reverse state at its first.
-// Returns false when the exchange's bounded wait gave up.
-__device__ __forceinline__ bool scan_tile(const RowGemm& g, RgBars* bars, volatile int* abort, Emit& emit,
-                                          float* xch, int* xfl, uint32_t tq, int64_t row, int rbox, int n0, int q,
-                                          int hs, int lane, int& uses) {
-  constexpr unsigned FULL = 0xffffffffu;
-  int trk = g.rtrk[row];
-  if (trk >= g.ntrk) trk = -1;
-  bool f0 = true, e0 = true;
-  if (trk >= 0) {
-    const int64_t r0 = g.row0[trk];
-    f0 = row == r0;
-    e0 = row == r0 + g.nh[trk] - 1;
-  }
-  const int H = g.H, cbase = n0 / 4;
-  for (int k = 0; k < 32 / SCB; ++k) {
-    const int co = 32 * hs + SCB * k;
-    float af[SCB], bf[SCB], ab[SCB], bb[SCB];
-    tmem_ld8(tq + co, af);
-    tmem_ld8(tq + 64 + co, bf);
-    tmem_ld8(tq + 128 + co, ab);
-    tmem_ld8(tq + 192 + co, bb);
-    tmem_ld_wait();
-    biased8(g, n0 + co, af);
-    biased8(g, n0 + 64 + co, bf);
-    biased8(g, n0 + 128 + co, ab);
-    biased8(g, n0 + 192 + co, bb);
-#pragma unroll
-    for (int i = 0; i < SCB; ++i) {
-      const float z = sigm(af[i]), y = sigm(ab[i]);
-      af[i] = 1.0f - z;
-      bf[i] = z * bf[i];
-      ab[i] = 1.0f - y;
-      bb[i] = y * bb[i];
-    }
-    bool f = f0, e = e0;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {   // forward: compose with lane - d
-      const bool fp = __shfl_up_sync(FULL, f, d);
-#pragma unroll
-      for (int i = 0; i < SCB; ++i) {
-        const float ap = __shfl_up_sync(FULL, af[i], d), bp = __shfl_up_sync(FULL, bf[i], d);
-        if (lane >= d && !f) {
-          bf[i] = fmaf(af[i], bp, bf[i]);
-          af[i] *= ap;
-        }
-      }
-      if (lane >= d) f = f || fp;
-    }
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {   // reverse: compose with lane + d
-      const bool ep = __shfl_down_sync(FULL, e, d);
-#pragma unroll
-      for (int i = 0; i < SCB; ++i) {
-        const float an = __shfl_down_sync(FULL, ab[i], d), bn = __shfl_down_sync(FULL, bb[i], d);
-        if (lane + d < 32 && !e) {
-          bb[i] = fmaf(ab[i], bn, bb[i]);
-          ab[i] *= an;
-        }
-      }
-      if (lane + d < 32) e = e || ep;
-    }
-    // this warp's carries out: the forward map at its last row, the reverse at its first
-    const int par = uses & 1;
-    float* X = xch + (par * 2 + hs) * 4 * 4 * SCB;
-    int* XF = xfl + (par * 2 + hs) * 4 * 2;
-    if (lane == 31) {
-#pragma unroll
-      for (int i = 0; i < SCB; ++i) {
-        X[q * 2 * SCB * 2 + 2 * i] = af[i];
-        X[q * 2 * SCB * 2 + 2 * i + 1] = bf[i];
-      }
-      XF[q * 2] = f;
-    }
-    if (lane == 0) {
-#pragma unroll
-      for (int i = 0; i < SCB; ++i) {
-        X[q * 2 * SCB * 2 + 2 * SCB + 2 * i] = ab[i];
-        X[q * 2 * SCB * 2 + 2 * SCB + 2 * i + 1] = bb[i];
-      }
-      XF[q * 2 + 1] = e;
-    }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(smem_u32(&bars->xb[hs]));
-    if (!mbar_wait(smem_u32(&bars->xb[hs]), (uint32_t)par, abort, g.wait_ns)) return false;
-    ++uses;
-    float hi[SCB], hr[SCB];
-#pragma unroll
-    for (int i = 0; i < SCB; ++i) hi[i] = hr[i] = 0.0f;
-    for (int w = 0; w < q; ++w) {   // the state entering this warp, forward
-      const bool fw = XF[w * 2] != 0;
-#pragma unroll
-      for (int i = 0; i < SCB; ++i) hi[i] = fw ? X[w * 4 * SCB + 2 * i + 1] : fmaf(X[w * 4 * SCB + 2 * i], hi[i], X[w * 4 * SCB + 2 * i + 1]);
-    }
-    for (int w = 3; w > q; --w) {   // and backward
-      const bool ew = XF[w * 2 + 1] != 0;
-#pragma unroll
-      for (int i = 0; i < SCB; ++i)
-        hr[i] = ew ? X[w * 4 * SCB + 2 * SCB + 2 * i + 1] : fmaf(X[w * 4 * SCB + 2 * SCB + 2 * i], hr[i], X[w * 4 * SCB + 2 * SCB + 2 * i + 1]);
-    }
-#pragma unroll
-    for (int i = 0; i < SCB; ++i) {
-      bf[i] = f ? bf[i] : fmaf(af[i], hi[i], bf[i]);
-      bb[i] = e ? bb[i] : fmaf(ab[i], hr[i], bb[i]);
-    }
-    if (g.pooled) {
-      if (trk >= 0 && e0) {
-        float4* o = reinterpret_cast<float4*>(g.pooled + (int64_t)trk * 2 * H + cbase + co);
-#pragma unroll
-        for (int i = 0; i < SCB / 4; ++i) o[i] = make_float4(bf[4 * i], bf[4 * i + 1], bf[4 * i + 2], bf[4 * i + 3]);
-      }
-      if (trk >= 0 && f0) {
-        float4* o = reinterpret_cast<float4*>(g.pooled + (int64_t)trk * 2 * H + H + cbase + co);
-#pragma unroll
-        for (int i = 0; i < SCB / 4; ++i) o[i] = make_float4(bb[4 * i], bb[4 * i + 1], bb[4 * i + 2], bb[4 * i + 3]);
-      }
-    } else {
-      emit.half(g, lane, cbase + co, rbox, bf);
-      emit.half(g, lane, H + cbase + co, rbox, bb);
-    }
-  }
-  return true;
 }
 
 __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_constant__ RowGemm g) {
@@ -386,7 +210,6 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       mbar_init(smem_u32(&bars->acc_empty[b]), RG_EPI_WARPS);   // one arrival per epilogue warp
     }
     for (int q = 0; q < 4; ++q) mbar_init(smem_u32(&bars->ssb[q]), 2);
-    for (int h = 0; h < 2; ++h) mbar_init(smem_u32(&bars->xb[h]), 4);
     mbar_init(smem_u32(&bars->drain), 1);
     bars->abort = 0;
     bars->never = 0;
@@ -481,13 +304,10 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
   } else if (warp >= 2) {
     // ---------------- epilogue: this warp's 32 rows and half of the columns of each tile
     const int q = warp & 3, hs = (warp - 2) >> 2;
-    // misc: RMSNorm partial sums [2][2][128], scan carries [2][2][4][64], their flags [2][2][4][2]
+    // misc: RMSNorm partial sums [2][2][128]
     const uint32_t misc = base + (uint32_t)(g.stages * stage_bytes) + 1024u;
     float* ssx = reinterpret_cast<float*>(smem_raw + (misc - raw));
-    float* xch = ssx + 512;
-    int* xfl = reinterpret_cast<int*>(xch + 1024);
     Emit emit{misc + (uint32_t)RG_MISC + (uint32_t)((warp - 2) * RG_STG_WARP), 0};
-    int scans = 0;
     const int U = g.Nt / 16, ub = hs ? (U + 1) / 2 : 0, ue = hs ? U : (U + 1) / 2;
     int acc_k = 0, norms = 0;
     for (int64_t t = blockIdx.x; t < total; t += gridDim.x) {
@@ -554,10 +374,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
         return ss;
       };
       bool ok = true;
-      if (g.epi == EP_SCAN) {
-        ok = scan_tile(g, bars, abort, emit, xch, xfl, tq, row, rbox, n0, q, hs, lane, scans);
-        if (!ok && lane == 0) rg_fail(g, bars);
-      } else if (g.epi == EP_NORM) {
+      if (g.epi == EP_NORM) {
         // the row's sum of squares: this warp's half, then the partner's through
         // shared memory (double-buffered by tile) and a two-arrival barrier
         const int par = norms & 1;
@@ -665,58 +482,6 @@ __global__ void __launch_bounds__(PLAN_NT) plan_rows(const int32_t* __restrict__
   const int64_t s = cta_inclusive_scan(v, wt) + tot[blockIdx.x];
   if (b < B) row0[b] = s - v;
   if (b == B - 1) row0[B] = s;
-}
-
-// Tile-aligned plan (the fused scan): no track crosses a 128-row tile.  Tracks
-// are packed next-fit, in order, into whole tiles, independently per segment of
-// SEG_TRK tracks (one warp per segment; the sequential fit runs on values every
-// lane holds).  mode 0 writes each segment's tile count; mode 1, after the
-// exclusive scan of those counts into seg, writes row0[b] for every track,
-// row0[B] = all rows (tiles x 128), and rtrk[row] = the row's track (-1 for the
-// padding rows that close a tile).
-constexpr int SEG_TRK = 256;
-
-__global__ void __launch_bounds__(128) plan_aligned(const int32_t* __restrict__ n_hits, int64_t B, int T, int mode,
-                                                    int64_t* __restrict__ seg, int64_t* __restrict__ row0,
-                                                    int32_t* __restrict__ rtrk, int64_t cap) {
-  const int64_t sg = blockIdx.x * 4 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  const int64_t nseg = (B + SEG_TRK - 1) / SEG_TRK;
-  if (sg >= nseg) return;
-  const int64_t b0 = sg * SEG_TRK;
-  int nv[SEG_TRK / 32];
-#pragma unroll
-  for (int k = 0; k < SEG_TRK / 32; ++k) nv[k] = (int)valid_count(n_hits, b0 + 32 * k + lane, B, T);
-  int64_t tile = mode ? seg[sg] : 0;
-  int cur = 0;
-#pragma unroll
-  for (int k = 0; k < SEG_TRK / 32; ++k) {
-    for (int i = 0; i < 32; ++i) {
-      const int n = __shfl_sync(0xffffffffu, nv[k], i);
-      const int64_t b = b0 + 32 * k + i;
-      if (n && cur + n > RG_ROWS) {   // close the tile
-        if (mode && (tile + 1) * RG_ROWS <= cap)
-          for (int r = cur + lane; r < RG_ROWS; r += 32) rtrk[tile * RG_ROWS + r] = -1;
-        ++tile;
-        cur = 0;
-      }
-      if (mode && b < B) {
-        if (lane == 0) row0[b] = tile * RG_ROWS + cur;
-        if ((tile + 1) * RG_ROWS <= cap)   // (the workspace is sized so that this always holds)
-          for (int t = lane; t < n; t += 32) rtrk[tile * RG_ROWS + cur + t] = (int32_t)b;
-      }
-      cur += n;
-    }
-  }
-  if (cur) {
-    if (mode && (tile + 1) * RG_ROWS <= cap)
-      for (int r = cur + lane; r < RG_ROWS; r += 32) rtrk[tile * RG_ROWS + r] = -1;
-    ++tile;
-  }
-  if (lane == 0) {
-    if (!mode) seg[sg] = tile;
-    if (mode && sg == nseg - 1) row0[B] = seg[nseg] * RG_ROWS;
-  }
 }
 
 // ------------------------------------------------------------------ Fourier rows
@@ -838,13 +603,10 @@ struct tf_rows_state {
   float* hws;               // the head's workspace, chunk x (P + 128 + Q) floats
   float* vec;               // the products' bias and gain vectors, each 16-byte aligned
   int doubling;             // fourier_scale[k + 3] == 2 fourier_scale[k] for every k
-  int fused;                // concatenation layers with the scans in the product's epilogue (EP_SCAN)
-  int32_t* rtrk;            // fused: each row's track, -1 for padding [cap]
   int64_t chunk, cap;       // tracks per chunk; rows of the workspace (chunk * max_hits)
   int64_t* row0;            // [chunk + 1]
   int64_t* tot;             // [chunk / 1024 + 1]
   uint16_t *a0, *hs16, *xy16, *o16;
-  uint16_t* xy16b;          // fused: the other layer-operand buffer (a layer never writes its own input)
   float *p32, *x32, *x1, *pooled;
   RowGemm e1, e2;
   RowGemm lay[TF_MAX_LAYERS][4];
@@ -884,20 +646,18 @@ bool rows_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uin
 // Output matrix [rows][cols] row-major (fp32, or 16-bit) -> tensor map of
 // 16-column x 32-row boxes for the epilogue's TMA stores, swizzled over the box
 // row (64 bytes for fp32, 32 bytes for 16-bit).
-bool out_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, int bytes, int fp16, uint32_t bw = 16) {
+bool out_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, int bytes, int fp16) {
   auto fn = rows_encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * (uint64_t)bytes};
-  cuuint32_t box[2] = {bw, 32};
+  cuuint32_t box[2] = {16, 32};
   cuuint32_t es[2] = {1, 1};
   const CUtensorMapDataType t = bytes == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
                                 : fp16     ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
                                            : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   return fn(m, t, 2, const_cast<void*>(ptr), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-            bw * bytes == 16 ? CU_TENSOR_MAP_SWIZZLE_NONE
-            : bytes == 4     ? CU_TENSOR_MAP_SWIZZLE_64B
-                             : CU_TENSOR_MAP_SWIZZLE_32B,
+            bytes == 4 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B,
             CU_TENSOR_MAP_L2_PROMOTION_NONE,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -905,13 +665,10 @@ bool out_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, int 
 // The store maps of a product whose output pointers are set.
 bool finish_gemm(RowGemm& g, const tf_rows_state* r) {
   const bool need32 = g.epi == EP_F32 || g.epi == EP_PROJ || g.epi == EP_RES || g.epi == EP_NORM;
-  const bool need16 =
-      g.epi == EP_16 || g.epi == EP_SILU16 || g.epi == EP_NORM || (g.epi == EP_SCAN && g.pooled == nullptr);
+  const bool need16 = g.epi == EP_16 || g.epi == EP_SILU16 || g.epi == EP_NORM;
   if (need32 != (g.out32 != nullptr) || need16 != (g.out16 != nullptr)) return false;
-  if (!g.N16) g.N16 = g.N;
   return (!g.out32 || out_map(&g.to32, g.out32, (uint64_t)r->cap, (uint64_t)g.N, 4, r->fp16)) &&
-         (!g.out16 || out_map(&g.to16, g.out16, (uint64_t)r->cap, (uint64_t)g.N16, 2, r->fp16)) &&
-         (!g.out16 || out_map(&g.to16h, g.out16, (uint64_t)r->cap, (uint64_t)g.N16, 2, r->fp16, 8));
+         (!g.out16 || out_map(&g.to16, g.out16, (uint64_t)r->cap, (uint64_t)g.N, 2, r->fp16));
 }
 
 // The MMA N of one tile: N itself up to 256, else the smallest equal split into
@@ -992,13 +749,11 @@ void tf_rows_destroy(trackfit_ctx* h) {
   tf_free(r->w16);
   tf_free(r->hws);
   tf_free(r->vec);
-  tf_free(r->rtrk);
   tf_free(r->row0);
   tf_free(r->tot);
   tf_free(r->a0);
   tf_free(r->hs16);
   tf_free(r->xy16);
-  tf_free(r->xy16b);
   tf_free(r->o16);
   tf_free(r->p32);
   tf_free(r->x32);
@@ -1031,28 +786,20 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
     return TRACKFIT_ERR_CUDA;
   const bool attn = s.topology == TRACKFIT_TOPOLOGY_ATTENTION;
   const size_t D = s.D, H = s.H, E = s.E;
-  // the scans run inside the projection's epilogue when a 256-column tile holds
-  // z_f, n_f, z_b, n_b of 64 whole channels and the readout takes the endpoints
-  r->fused = !attn && (H % 64) == 0 && s.pool == TRACKFIT_POOL_ENDPOINTS;
-  // fused: projection row (and bias) j of group gi = j / 256 is row
-  // (j % 256 / 64) H + 64 gi + j % 64 of W_in's [z_f; n_f; z_b; n_b]
-  auto src_row = [&](size_t j) -> size_t {
-    return r->fused ? (j % 256 / 64) * H + 64 * (j / 256) + j % 64 : j;
-  };
-  // the 16-bit weights of every product: (blob offset, N, K, permuted rows)
-  struct Mat { size_t off, n, k, at; bool perm; };
+  // the 16-bit weights of every product: (blob offset, N, K)
+  struct Mat { size_t off, n, k, at; };
   std::vector<Mat> mats;
-  mats.push_back({o.emb_w1, D, E, 0, false});
-  mats.push_back({o.emb_w2, D, D, 0, false});
+  mats.push_back({o.emb_w1, D, E, 0});
+  mats.push_back({o.emb_w2, D, D, 0});
   for (int l = 0; l < s.L; ++l) {
     const tf_layer_off& lo = o.layer[l];
     if (attn) {
-      mats.push_back({lo.w_in, 3 * D, D, 0, false});
-      mats.push_back({lo.w_m, D, D, 0, false});
-      mats.push_back({lo.w1, H, D, 0, false});
-      mats.push_back({lo.w2, D, H, 0, false});
+      mats.push_back({lo.w_in, 3 * D, D, 0});
+      mats.push_back({lo.w_m, D, D, 0});
+      mats.push_back({lo.w1, H, D, 0});
+      mats.push_back({lo.w2, D, H, 0});
     } else {
-      mats.push_back({lo.w_in, 4 * H, l == 0 ? D : 2 * H, 0, true});
+      mats.push_back({lo.w_in, 4 * H, l == 0 ? D : 2 * H, 0});
     }
   }
   size_t n16 = 0;
@@ -1062,10 +809,7 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
   }
   std::vector<uint16_t> w(n16, 0);
   for (const Mat& m : mats)
-    for (size_t j = 0; j < m.n; ++j) {
-      const size_t sj = m.perm ? src_row(j) : j;
-      for (size_t c = 0; c < m.k; ++c) w[m.at + j * m.k + c] = to16(host_w[m.off + sj * m.k + c], r->fp16);
-    }
+    for (size_t i = 0; i < m.n * m.k; ++i) w[m.at + i] = to16(host_w[m.off + i], r->fp16);
   int st = tf_status_from_cuda(tf_malloc((void**)&r->w16, n16 * 2));
   if (st == TRACKFIT_OK) st = tf_status_from_cuda(cudaMemcpy(r->w16, w.data(), n16 * 2, cudaMemcpyHostToDevice));
   if (st != TRACKFIT_OK) return st;
@@ -1073,34 +817,24 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
   const size_t hsw = attn ? (H > D ? H : D) : D;
   const size_t xyw = attn ? D : (2 * H > D ? 2 * H : D);
   const size_t pw = attn ? 3 * D : 4 * H;
-  const size_t row_bytes =
-      2 * (E + hsw + xyw + (attn ? D : 0) + (r->fused ? 2 * H : 0)) + 4 * (pw + (attn ? 2 * D : 0));
+  const size_t row_bytes = 2 * (E + hsw + xyw + (attn ? D : 0)) + 4 * (pw + (attn ? 2 * D : 0));
   const size_t track_bytes = (size_t)s.T * row_bytes + 4 * (2 * (size_t)s.P + s.Hh + s.Q) + 16;
-  // fused: whole tracks per tile; a closed tile holds more than 128 - T rows, and
-  // each segment's last tile may be partly empty
-  const double rows_per_track =
-      r->fused ? (double)RG_ROWS * s.T / (RG_ROWS + 1 - s.T) + (double)RG_ROWS / SEG_TRK + 4.0 / SEG_TRK : s.T;
-  int64_t chunk = (int64_t)(RG_WS_BUDGET / (track_bytes / s.T * rows_per_track + 4 * rows_per_track));
+  int64_t chunk = (int64_t)(RG_WS_BUDGET / track_bytes);
   if (chunk > 4194304) chunk = 4194304;
   chunk = chunk / PLAN_NT * PLAN_NT;
   if (chunk < PLAN_NT) return TRACKFIT_ERR_UNSUPPORTED;
   r->chunk = chunk;
-  r->cap = r->fused ? RG_ROWS * ((chunk * s.T + RG_ROWS - s.T) / (RG_ROWS + 1 - s.T) + chunk / SEG_TRK + 1)
-                    : chunk * s.T;
+  r->cap = chunk * s.T;
   const size_t cap = (size_t)r->cap;
   auto alloc = [&](void** p, size_t bytes) {
     if (st == TRACKFIT_OK) st = tf_status_from_cuda(tf_malloc(p, bytes));
   };
   alloc((void**)&r->row0, (chunk + 1) * sizeof(int64_t));
-  alloc((void**)&r->tot, (chunk / SEG_TRK + 2) * sizeof(int64_t));
-  if (r->fused) alloc((void**)&r->rtrk, cap * sizeof(int32_t));
+  alloc((void**)&r->tot, (chunk / PLAN_NT + 2) * sizeof(int64_t));
   alloc((void**)&r->a0, cap * E * 2);
   alloc((void**)&r->hs16, cap * hsw * 2);
   alloc((void**)&r->xy16, cap * xyw * 2);
-  if (r->fused)
-    alloc((void**)&r->xy16b, cap * 2 * H * 2);
-  else
-    alloc((void**)&r->p32, cap * pw * 4);
+  alloc((void**)&r->p32, cap * pw * 4);
   alloc((void**)&r->pooled, (size_t)chunk * s.P * 4);
   alloc((void**)&r->hws, (size_t)chunk * (s.P + s.Hh + s.Q) * 4);
   if (attn) {
@@ -1112,10 +846,10 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
   // 16-byte aligned copies of the bias and gain vectors the epilogues read
   std::map<size_t, size_t> at;
   std::vector<float> hv;
-  auto want = [&](size_t off, size_t n, bool perm = false) {
+  auto want = [&](size_t off, size_t n) {
     if (at.count(off)) return;
     at[off] = hv.size();
-    for (size_t j = 0; j < n; ++j) hv.push_back(host_w[off + (perm ? src_row(j) : j)]);
+    hv.insert(hv.end(), host_w + off, host_w + off + n);
     hv.resize((hv.size() + 3) / 4 * 4, 0.0f);
   };
   want(o.emb_b1, D);
@@ -1123,7 +857,7 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
   for (int l = 0; l < s.L; ++l) {
     const tf_layer_off& lo = o.layer[l];
     if (!attn) {
-      want(lo.b_in, 4 * H, true);
+      want(lo.b_in, 4 * H);
       continue;
     }
     want(lo.g, D);
@@ -1155,24 +889,10 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
     const tf_layer_off& lo = o.layer[l];
     RowGemm* g = r->lay[l];
     if (!attn) {   // Sec. 3.2: the layer input (D, then 2H wide) to z_f, n_f, z_b, n_b
-      // fused: layer l reads xy16 (l even) or xy16b (l odd) and writes the other
-      uint16_t* in = (r->fused && (l & 1)) ? r->xy16b : r->xy16;
-      ok = make_gemm(g[0], r, in, l == 0 ? (int)D : (int)(2 * H), w16 + mats[mi++].at, (int)(4 * H),
-                     r->fused ? EP_SCAN : EP_PROJ);
+      ok = make_gemm(g[0], r, r->xy16, l == 0 ? (int)D : (int)(2 * H), w16 + mats[mi++].at, (int)(4 * H), EP_PROJ);
       g[0].H = (int)H;
       g[0].bias = V(lo.b_in);
-      if (!r->fused) {
-        g[0].out32 = r->p32;
-        continue;
-      }
-      // the scans in the epilogue: the next layer's operand [h_f | h_b], or the endpoints
-      g[0].rtrk = r->rtrk;
-      g[0].row0 = r->row0;
-      g[0].N16 = (int)(2 * H);
-      if (l + 1 < s.L)
-        g[0].out16 = in == r->xy16 ? r->xy16b : r->xy16;
-      else
-        g[0].pooled = r->pooled;
+      g[0].out32 = r->p32;
       continue;
     }
     // App. A.3: qkv of the normed stream; x' = x + W_o o + b_o and its pre-norm;
@@ -1235,17 +955,10 @@ int rows_chunk(trackfit_ctx* h, const float* hits, const int64_t* offs, const in
   const tf_shape& s = h->s;
   unsigned long long* err = h->d_err;   // bad-track counter of the head
   const bool attn = s.topology == TRACKFIT_TOPOLOGY_ATTENTION;
-  if (r->fused) {   // whole tracks per 128-row tile
-    const int nseg = (int)((nb + SEG_TRK - 1) / SEG_TRK);
-    plan_aligned<<<(nseg + 3) / 4, 128, 0, st>>>(nc, nb, s.T, 0, r->tot, r->row0, r->rtrk, r->cap);
-    plan_scan_totals<<<1, PLAN_NT, 0, st>>>(r->tot, nseg);
-    plan_aligned<<<(nseg + 3) / 4, 128, 0, st>>>(nc, nb, s.T, 1, r->tot, r->row0, r->rtrk, r->cap);
-  } else {
-    const int nblk = (int)((nb + PLAN_NT - 1) / PLAN_NT);
-    plan_totals<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot);
-    plan_scan_totals<<<1, PLAN_NT, 0, st>>>(r->tot, nblk);
-    plan_rows<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot, r->row0);
-  }
+  const int nblk = (int)((nb + PLAN_NT - 1) / PLAN_NT);
+  plan_totals<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot);
+  plan_scan_totals<<<1, PLAN_NT, 0, st>>>(r->tot, nblk);
+  plan_rows<<<nblk, PLAN_NT, 0, st>>>(nc, nb, s.T, r->tot, r->row0);
   const int64_t* nrows = r->row0 + nb;
   const int64_t nf = nb * s.T * s.F;
   fourier_rows_kernel<T16><<<(unsigned)((nf + 255) / 256), 256, 0, st>>>(hits, offs, nc, nb, s, r->row0, r->doubling,
@@ -1261,10 +974,7 @@ int rows_chunk(trackfit_ctx* h, const float* hits, const int64_t* offs, const in
   for (int l = 0; l < s.L; ++l) {
     RowGemm* g = r->lay[l];
     if (!attn) {
-      g[0].nh = nc;
-      g[0].ntrk = nb;
       if (launch_gemm(h, g[0], nrows, st)) return TRACKFIT_ERR_CUDA;
-      if (r->fused) continue;   // the scans ran in the product's epilogue
       const bool last = l + 1 == s.L;
       dim3 grid((unsigned)nb, (unsigned)((s.H + 127) / 128));
       concat_scan_rows_kernel<T16><<<grid, 128, 0, st>>>(r->p32, r->row0, nc, nb, s.T, s.H,
