@@ -13,8 +13,8 @@
 // registers and reads every key and value of its head as a broadcast within the
 // threads of that head.  With n hits a track keeps n x heads threads busy (52 at
 // 13 hits and 4 heads); the other warps only stage.  The softmax takes two passes
-// over the keys: the maximum score, then the exponentials, their sum and the
-// weighted values.
+// over the keys: the scores (kept in registers, up to KMAX = 32 or 64 keys) and
+// their maximum, then the exponentials, their sum and the weighted values.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -52,7 +52,7 @@ __device__ __forceinline__ float dot(const float (&q)[DH], const float* k) {
 // row0[b] + t (packed rows) or b T + t (padded rows, row0 null).  o: the attention
 // output at stride ldo, row-aligned with qkv.  With padded rows the rows t >= n of
 // a track (all of them for a track whose count is outside [1, T]) are written 0.
-template <int DH, typename OutT>
+template <int DH, int KMAX, typename OutT>
 __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* __restrict__ qkv, int ldq,
                                                                   const int64_t* __restrict__ row0,
                                                                   const int32_t* __restrict__ n_hits, int64_t B,
@@ -98,11 +98,19 @@ __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* _
     }
     const float* kh = ks + h * hs;
     const float* vh = vs + h * hs;
+    float sc[KMAX];
     float m = -INFINITY;
-    for (int j = 0; j < n; ++j) m = fmaxf(m, dot<DH>(q, kh + j * rs) * scale);
+#pragma unroll
+    for (int j = 0; j < KMAX; ++j) {
+      if (j >= n) break;
+      sc[j] = dot<DH>(q, kh + j * rs) * scale;
+      m = fmaxf(m, sc[j]);
+    }
     float l = 0.0f;
-    for (int j = 0; j < n; ++j) {
-      const float p = expf(dot<DH>(q, kh + j * rs) * scale - m);
+#pragma unroll
+    for (int j = 0; j < KMAX; ++j) {
+      if (j >= n) break;
+      const float p = expf(sc[j] - m);
       l += p;
       const float* vr = vh + j * rs;
 #pragma unroll
@@ -128,9 +136,13 @@ inline cudaError_t launch(const float* qkv, int ldq, const int64_t* row0, const 
                           int D, int NH, OutT* o, int ldo, cudaStream_t st) {
   const size_t sm = smem_bytes(T, D, NH);
   const unsigned g = (unsigned)B;
-#define TF_ATTN_CASE(DHV) \
-  case DHV:               \
-    track_attention_kernel<DHV, OutT><<<g, THREADS, sm, st>>>(qkv, ldq, row0, n_hits, B, T, D, NH, o, ldo); break;
+#define TF_ATTN_CASE(DHV)                                                                                  \
+  case DHV:                                                                                                \
+    if (T <= 32)                                                                                           \
+      track_attention_kernel<DHV, 32, OutT><<<g, THREADS, sm, st>>>(qkv, ldq, row0, n_hits, B, T, D, NH, o, ldo); \
+    else                                                                                                   \
+      track_attention_kernel<DHV, 64, OutT><<<g, THREADS, sm, st>>>(qkv, ldq, row0, n_hits, B, T, D, NH, o, ldo); \
+    break;
   switch (D / NH) {
     TF_ATTN_CASE(8)
     TF_ATTN_CASE(16)
@@ -151,9 +163,12 @@ template <typename OutT>
 inline cudaError_t allow_smem(int T, int D, int NH) {
   const int sm = (int)smem_bytes(T, D, NH);
   if (sm <= 48 * 1024) return cudaSuccess;
-#define TF_ATTN_ATTR(DHV) \
-  case DHV:               \
-    return cudaFuncSetAttribute(track_attention_kernel<DHV, OutT>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+#define TF_ATTN_ATTR(DHV)                                                                                    \
+  case DHV:                                                                                                  \
+    return T <= 32 ? cudaFuncSetAttribute(track_attention_kernel<DHV, 32, OutT>,                             \
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, sm)                   \
+                   : cudaFuncSetAttribute(track_attention_kernel<DHV, 64, OutT>,                             \
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
   switch (D / NH) {
     TF_ATTN_ATTR(8)
     TF_ATTN_ATTR(16)

@@ -50,9 +50,10 @@ constexpr int RG_ROWS = 128;                      // rows per tile (MMA M)
 constexpr int RG_KC = 64;                         // k per stage (one 128-byte swizzle row of 16-bit values)
 constexpr int RG_A_BYTES = RG_ROWS * RG_KC * 2;   // 16 KB
 constexpr int RG_MAX_NT = 256;                    // MMA N per tile (two buffers fill the 512 TMEM columns)
-constexpr int RG_SMEM_BUDGET = 170 * 1024;        // the ring of stages
+constexpr int RG_SMEM_BUDGET = 158 * 1024;        // the ring of stages
 constexpr int RG_MISC = 2048;                     // RMSNorm partial sums
-constexpr int RG_STG_WARP = 6144;                 // per epilogue warp: 2 x (32 rows x 16 fp32) + 2 x (32 x 16 16-bit)
+constexpr int RG_STG_BUFS = 4;                    // staging buffers per epilogue warp (stores in flight)
+constexpr int RG_STG_WARP = RG_STG_BUFS * 2048;   // each a 32 x 16 fp32 (or 16-bit) box
 constexpr int RG_MAX_STAGES = 8;
 constexpr uint64_t RG_WAIT_NS = 2000000000ull;
 constexpr uint64_t RG_DRAIN_NS = 200000000ull;
@@ -61,7 +62,7 @@ constexpr size_t RG_WS_BUDGET = (size_t)4 << 30;  // workspace bytes of one hand
 // epilogues
 enum {
   EP_F32 = 0,        // out32 = v
-  EP_PROJ = 1,       // out32 = v, sigmoid on the update-gate blocks z_f, z_b (columns [0, H) and [2H, 3H))
+  EP_PROJ = 1,       // out32 = v: the pre-activations of z_f, n_f, z_b, n_b (the scan applies the sigmoid)
   EP_16 = 2,         // out16 = v
   EP_SILU16 = 3,     // out16 = SiLU(v)
   EP_NORM = 4,       // x = v (+ res): out32 = x, out16 = RMSNorm(x) g
@@ -76,7 +77,6 @@ struct RowGemm {
   const int64_t* n_rows;      // device: rows of this chunk
   int K, N, Nt, n_ntiles, kchunks, stages;
   int epi;
-  int H;                      // EP_PROJ: gate block width
   uint32_t idesc;
   const float* bias;          // [N]
   const float* res;           // EP_NORM (optional), EP_RES: fp32 [rows][N]
@@ -99,10 +99,11 @@ struct RgBars {
   int never;                  // a flag nothing sets: for the waits at exit that must not give up on abort
 };
 
-// sigma(x) = 1 / (1 + e^-x) with the hardware exponential (ex2 of -x log2 e) and a
-// correctly rounded reciprocal: a few ulp of fp32, far below the 16-bit rounding
-// of the operands it feeds (e^-x = inf for x < -88 gives 1 / inf = 0).
-__device__ __forceinline__ float sigm(float x) { return __frcp_rn(1.0f + __expf(-x)); }
+// sigma(x) = 1 / (1 + e^-x) with the hardware exponential (ex2 of -x log2 e) and
+// the hardware reciprocal (two MUFU operations, no branch): a few ulp of fp32, far
+// below the 16-bit rounding of the operands it feeds (e^-x = inf for x < -88
+// gives 1 / inf = 0).
+__device__ __forceinline__ float sigm(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
 
 __device__ __forceinline__ uint32_t pack16(float a, float b, int fp16) {   // a -> low half
   if (fp16) {
@@ -122,72 +123,55 @@ __device__ __forceinline__ void sts4(uint32_t addr, uint32_t a, uint32_t b, uint
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
-// Output of one 16-column chunk of a warp's 32 rows: every lane writes its row's
-// 16 values into the warp's staging buffer, then one lane stores the [32][16] box
-// with TMA.  The buffers use the tensor maps' swizzled layouts (fp32 rows of 64
-// bytes: 16-byte piece c of row r at c ^ ((r >> 1) & 3); 16-bit rows of 32 bytes:
-// piece c at c ^ ((r >> 2) & 1)), so the 8 lanes of a quarter warp write 8
-// different bank groups.  Two buffers per output alternate; a buffer is rewritten
-// only after the store that read it two chunks earlier has finished reading.
+// Output of a warp's 32 rows, 16 columns (one box) at a time, fp32 or 16-bit:
+// every lane writes its row's 16 values into one of the warp's staging buffers,
+// then one lane stores the [32][16] boxes of a group of two with TMA.  The
+// buffers use the tensor maps' swizzled layouts (fp32 rows of 64 bytes: 16-byte
+// piece c of row r at c ^ ((r >> 1) & 3); 16-bit rows of 32 bytes: piece c at
+// c ^ ((r >> 2) & 1)), so the 8 lanes of a quarter warp write 8 different bank
+// groups.  Two groups of two buffers alternate; a group's buffers are rewritten
+// only after the stores that read them two groups earlier have finished reading.
 struct Emit {
-  uint32_t stg;     // this warp's staging area
-  int chunk;        // chunks emitted so far (buffer parity)
-  __device__ __forceinline__ void operator()(const RowGemm& g, int lane, int nb, int row, const float (&v)[16],
-                                             bool to32, bool to16) {
-    const int p = chunk & 1;
-    if (lane == 0) bulk_wait_read1();
+  uint32_t stg;     // this warp's staging area (RG_STG_BUFS = 4 buffers of 2 KB)
+  int group;        // groups flushed so far
+  __device__ __forceinline__ uint32_t buf(int slot) const {
+    return stg + (uint32_t)((((group & 1) << 1) + slot) * 2048);
+  }
+  __device__ __forceinline__ void begin(int lane) {
+    if (lane == 0) bulk_wait_read_keep(1);
     __syncwarp();
-    if (to32) {
-      const uint32_t a = stg + p * 2048 + lane * 64;
+  }
+  __device__ __forceinline__ void put(const RowGemm& g, int lane, int slot, const float (&v)[16], bool is32) {
+    if (is32) {
+      const uint32_t a = buf(slot) + lane * 64;
       const int sw = (lane >> 1) & 3;
 #pragma unroll
       for (int j = 0; j < 4; ++j)
         sts4(a + 16 * (j ^ sw), __float_as_uint(v[4 * j]), __float_as_uint(v[4 * j + 1]),
              __float_as_uint(v[4 * j + 2]), __float_as_uint(v[4 * j + 3]));
-    }
-    if (to16) {
-      const uint32_t a = stg + 4096 + p * 1024 + lane * 32;
+    } else {
+      const uint32_t a = buf(slot) + lane * 32;
       const int sw = (lane >> 2) & 1;
 #pragma unroll
       for (int j = 0; j < 2; ++j)
         sts4(a + 16 * (j ^ sw), pack16(v[8 * j], v[8 * j + 1], g.fp16), pack16(v[8 * j + 2], v[8 * j + 3], g.fp16),
              pack16(v[8 * j + 4], v[8 * j + 5], g.fp16), pack16(v[8 * j + 6], v[8 * j + 7], g.fp16));
     }
+  }
+  // count (1 or 2) boxes at columns nb0, nb0 + 16 of rows row .. row + 31
+  __device__ __forceinline__ void flush(const RowGemm& g, int lane, bool is32, int nb0, int count, int row) {
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) {
-      if (to32) tma_store_2d(&g.to32, stg + p * 2048, nb, row);
-      if (to16) tma_store_2d(&g.to16, stg + 4096 + p * 1024, nb, row);
+      const CUtensorMap* m = is32 ? &g.to32 : &g.to16;
+      tma_store_2d(m, buf(0), nb0, row);
+      if (count > 1) tma_store_2d(m, buf(1), nb0 + 16, row);
       bulk_commit();
     }
-    ++chunk;
+    ++group;
   }
 };
 
-// acc + bias (+ res) of 16 columns; the same arithmetic in both passes of EP_NORM.
-// bias (and gain) vectors are 16-byte aligned copies made at create.
-__device__ __forceinline__ void biased(const RowGemm& g, int64_t row, bool live, int nbase, float (&v)[16]) {
-  const float4* bb = reinterpret_cast<const float4*>(g.bias + nbase);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float4 w = __ldg(bb + i);
-    v[4 * i] += w.x;
-    v[4 * i + 1] += w.y;
-    v[4 * i + 2] += w.z;
-    v[4 * i + 3] += w.w;
-  }
-  if (g.res && live) {
-    const float4* r = reinterpret_cast<const float4*>(g.res + row * g.N + nbase);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float4 a = r[i];
-      v[4 * i] = a.x + v[4 * i];
-      v[4 * i + 1] = a.y + v[4 * i + 1];
-      v[4 * i + 2] = a.z + v[4 * i + 2];
-      v[4 * i + 3] = a.w + v[4 * i + 3];
-    }
-  }
-}
 
 __device__ void rg_fail(const RowGemm& g, RgBars* b) {
   if (atomicExch(&b->abort, 1) == 0) atomicAdd(g.err + 1, 1ull);
@@ -308,6 +292,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
     const uint32_t misc = base + (uint32_t)(g.stages * stage_bytes) + 1024u;
     float* ssx = reinterpret_cast<float*>(smem_raw + (misc - raw));
     Emit emit{misc + (uint32_t)RG_MISC + (uint32_t)((warp - 2) * RG_STG_WARP), 0};
+    static_assert(RG_STG_BUFS == 4, "the epilogue's staging rotates two groups of two buffers");
     const int U = g.Nt / 16, ub = hs ? (U + 1) / 2 : 0, ue = hs ? U : (U + 1) / 2;
     int acc_k = 0, norms = 0;
     for (int64_t t = blockIdx.x; t < total; t += gridDim.x) {
@@ -327,19 +312,40 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       // flight while the current one is processed.  mode 0: the epilogue; 1: the
       // residual stream of EP_NORM and its sum of squares; 2: its normed operand.
       auto pass = [&](int mode, float inv) -> float {
+        const bool is32 = mode == 1 || (mode == 0 && g.epi != EP_16 && g.epi != EP_SILU16);
         float ss = 0.0f, cur[16], nxt[16];
         if (ub < ue) {
           tmem_ld16(tq + 16 * ub, cur);
           tmem_ld_wait();
         }
         for (int u = ub; u < ue; ++u) {
+          const int slot = (u - ub) & 1;
+          if (slot == 0) emit.begin(lane);
           if (u + 1 < ue) tmem_ld16(tq + 16 * (u + 1), nxt);
           const int nb = n0 + 16 * u;
-          biased(g, row, live, nb, cur);
+          const float4* bb = reinterpret_cast<const float4*>(g.bias + nb);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float4 w = __ldg(bb + i);
+            cur[4 * i] += w.x;
+            cur[4 * i + 1] += w.y;
+            cur[4 * i + 2] += w.z;
+            cur[4 * i + 3] += w.w;
+          }
+          if (g.res && live) {   // x + (acc + b), the same arithmetic in both passes of EP_NORM
+            const float4* rr = reinterpret_cast<const float4*>(g.res + row * g.N + nb);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const float4 a = rr[i];
+              cur[4 * i] = a.x + cur[4 * i];
+              cur[4 * i + 1] = a.y + cur[4 * i + 1];
+              cur[4 * i + 2] = a.z + cur[4 * i + 2];
+              cur[4 * i + 3] = a.w + cur[4 * i + 3];
+            }
+          }
           if (mode == 1) {
 #pragma unroll
             for (int i = 0; i < 16; ++i) ss = fmaf(cur[i], cur[i], ss);
-            emit(g, lane, nb, rbox, cur, true, false);
           } else if (mode == 2) {
             const float4* gn = reinterpret_cast<const float4*>(g.gain + nb);
 #pragma unroll
@@ -350,21 +356,12 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
               cur[4 * i + 2] = cur[4 * i + 2] * inv * w.z;
               cur[4 * i + 3] = cur[4 * i + 3] * inv * w.w;
             }
-            emit(g, lane, nb, rbox, cur, false, true);
-          } else {
-            if (g.epi == EP_PROJ) {
-              // the update-gate blocks of the projection rows (z_f, n_f, z_b, n_b)
-              if (nb < g.H || (nb >= 2 * g.H && nb < 3 * g.H)) {
+          } else if (g.epi == EP_SILU16) {
 #pragma unroll
-                for (int i = 0; i < 16; ++i) cur[i] = sigm(cur[i]);
-              }
-            } else if (g.epi == EP_SILU16) {
-#pragma unroll
-              for (int i = 0; i < 16; ++i) cur[i] = cur[i] * sigm(cur[i]);
-            }
-            const bool h = g.epi == EP_16 || g.epi == EP_SILU16;
-            emit(g, lane, nb, rbox, cur, !h, h);
+            for (int i = 0; i < 16; ++i) cur[i] = cur[i] * sigm(cur[i]);
           }
+          emit.put(g, lane, slot, cur, is32);
+          if (slot == 1 || u + 1 == ue) emit.flush(g, lane, is32, nb - 16 * slot, slot + 1, rbox);
           if (u + 1 < ue) {
             tmem_ld_wait();
 #pragma unroll
@@ -541,8 +538,9 @@ __global__ void fourier_rows_kernel(const float* __restrict__ hits, const int64_
 
 // ------------------------------------------------------------------ scans
 // The two gated scans of one concatenation layer (Sec. 3.2, Eq. 2) over each
-// track's rows: h_t = (1 - z_t) h_{t-1} + z_t n_t forward, the same backward with
-// the reverse gates; z already through the sigmoid.  One thread per (track,
+// track's rows: z_t = sigma(p_z), h_t = (1 - z_t) h_{t-1} + z_t n_t forward, the
+// same backward with the reverse gates (the projection stores the
+// pre-activations; the sigmoid runs here, in a kernel bound by HBM).  One thread per (track,
 // channel).  y16 (optional): the concatenated states [h_f | h_b] per row as the
 // next layer's 16-bit operand.  pooled (optional, the last layer): endpoints, the
 // forward state at the last hit and the reverse state at the first, or the mean
@@ -558,23 +556,26 @@ __global__ void concat_scan_rows_kernel(const float* __restrict__ pr, const int6
   if (n < 1 || n > T) return;
   const int64_t r0 = row0[b];
   const int ldp = 4 * H;
-  float h = 0.0f, sum = 0.0f;
+  // the two directions are independent chains: step t forward and step n - 1 - t
+  // backward run together, each in hit order for its own direction
+  float hf = 0.0f, hb = 0.0f, sf = 0.0f, sb = 0.0f;
   for (int t = 0; t < n; ++t) {
-    const float* p = pr + (r0 + t) * ldp;
-    h = fmaf(p[c], p[H + c] - h, h);
-    if (y16) tf_attn::put(y16 + (r0 + t) * 2 * H + c, h);
-    sum += h;
+    const float* pf = pr + (r0 + t) * ldp;
+    const float* pb = pr + (r0 + n - 1 - t) * ldp;
+    const float zf = pf[c], nf = pf[H + c], zb = pb[2 * H + c], nb = pb[3 * H + c];
+    hf = fmaf(sigm(zf), nf - hf, hf);
+    hb = fmaf(sigm(zb), nb - hb, hb);
+    if (y16) {
+      tf_attn::put(y16 + (r0 + t) * 2 * H + c, hf);
+      tf_attn::put(y16 + (r0 + n - 1 - t) * 2 * H + H + c, hb);
+    }
+    sf += hf;
+    sb += hb;
   }
-  if (pooled) pooled[b * 2 * H + c] = pool == TRACKFIT_POOL_ENDPOINTS ? h : sum / (float)n;
-  h = 0.0f;
-  sum = 0.0f;
-  for (int t = n - 1; t >= 0; --t) {
-    const float* p = pr + (r0 + t) * ldp;
-    h = fmaf(p[2 * H + c], p[3 * H + c] - h, h);
-    if (y16) tf_attn::put(y16 + (r0 + t) * 2 * H + H + c, h);
-    sum += h;
+  if (pooled) {
+    pooled[b * 2 * H + c] = pool == TRACKFIT_POOL_ENDPOINTS ? hf : sf / (float)n;
+    pooled[b * 2 * H + H + c] = pool == TRACKFIT_POOL_ENDPOINTS ? hb : sb / (float)n;
   }
-  if (pooled) pooled[b * 2 * H + H + c] = pool == TRACKFIT_POOL_ENDPOINTS ? h : sum / (float)n;
 }
 
 // Mean over each track's rows of the last layer's output x [rows][D] (the
@@ -890,7 +891,6 @@ int tf_rows_create(trackfit_ctx* h, const float* host_w) {
     RowGemm* g = r->lay[l];
     if (!attn) {   // Sec. 3.2: the layer input (D, then 2H wide) to z_f, n_f, z_b, n_b
       ok = make_gemm(g[0], r, r->xy16, l == 0 ? (int)D : (int)(2 * H), w16 + mats[mi++].at, (int)(4 * H), EP_PROJ);
-      g[0].H = (int)H;
       g[0].bias = V(lo.b_in);
       g[0].out32 = r->p32;
       continue;
