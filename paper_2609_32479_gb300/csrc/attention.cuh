@@ -8,11 +8,11 @@
 //
 // One CTA per track stages the track's keys and values in shared memory, each
 // head's slice of a row padded by 4 floats so that the heads fall in different
-// banks; thread i takes the (head, query) items i, i + 128, ... (head = item / n,
+// banks; thread i takes the (head, query) items i, i + 64, ... (head = item / n,
 // query = item % n), keeps its query and its output (dh values each) in
 // registers and reads every key and value of its head as a broadcast within the
 // threads of that head.  With n hits a track keeps n x heads threads busy (52 at
-// 13 hits and 4 heads); the other warps only stage.  The softmax takes two passes
+// 13 hits and 4 heads, of 64).  The softmax takes two passes
 // over the keys: the scores (kept in registers, up to KMAX = 32 or 64 keys) and
 // their maximum, then the exponentials, their sum and the weighted values.
 #pragma once
@@ -27,7 +27,7 @@ __device__ __forceinline__ void put(float* p, float v) { *p = v; }
 __device__ __forceinline__ void put(__half* p, float v) { *p = __float2half_rn(v); }
 __device__ __forceinline__ void put(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
 
-constexpr int THREADS = 128;
+constexpr int THREADS = 64;   // a track: heads x hits items (52 at 13 hits and 4 heads)
 
 // Shared memory of one CTA: keys and values, T rows x NH heads x (dh + 4) floats each.
 __host__ __device__ inline size_t smem_bytes(int T, int D, int NH) {
