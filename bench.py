@@ -655,12 +655,24 @@ def main():
     peak = float(peaks.get(dtype_tf, FALLBACK_PEAKS["bf16_tflops"]))
     peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
     achieved = flops_launch / kern_avg_s / 1e12 if kern_n else None
-    traffic = traffic_for_kernel()
+    bound, peak_kind = "tensor", f"{peak_kind} bf16 dense burst (fp16 runs at the bf16 rate)"
+    if m.precision == 0:
+        # fp32 configs run on the CUDA cores: the denominator is the FP32 FFMA
+        # rate derived from unit counts and clock (SMs x 128 lanes x 2 flop x
+        # maximum SM clock), not a tensor-core peak
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        mhz = float(peaks.get("sm_max_mhz", 2070.0))
+        peak = sms * 128 * 2 * mhz * 1e6 / 1e12
+        peak_sus = peak
+        bound = "alu"
+        peak_kind = f"FP32 FFMA peak derived: {sms} SMs x 128 lanes x 2 flop x {mhz:.0f} MHz"
+    # the committed capture is of the fused kernel on the large workload's model
+    traffic = traffic_for_kernel() if (tf.path.startswith("tcgen05") and w.name == "large") else None
     if traffic is not None:   # the summary scales its capture to 1,048,576 tracks
         traffic *= (B / launches_per_step) / 1048576
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+    roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": (achieved / peak) if achieved else None, "traffic": traffic,
-                "peak_kind": f"{peak_kind} bf16 dense burst (fp16 runs at the bf16 rate)",
+                "peak_kind": peak_kind,
                 "frac_of_sustained": (achieved / peak_sus) if achieved else None,
                 "kernel": "tc_forward_kernel" if tf.path.startswith("tcgen05") else "simt layer sequence",
                 "kernel_ms_avg": kern_avg_s * 1e3, "launches_per_step": launches_per_step,

@@ -129,7 +129,7 @@ struct Misc {
   uint8_t col_tpos[TILE];   // the loader's own
   alignas(16) float part[4][TILE];
   float carry[2][128];   // [slab][channel]: scan states between a slab's column segments
-  alignas(16) float rinv[TILE];
+  alignas(16) float rinv[NE / 32][32];   // per epilogue warp: 1 / RMS of its 32 columns
   float hs[TILE][5];   // the loader's own
 };
 static_assert(sizeof(Misc) <= MISC_BYTES, "misc region too small");
@@ -154,15 +154,20 @@ __device__ __forceinline__ float silu(float x) { return x * sigm(x); }
 // oracle).  The output gate does not: its value scales the merge into the fp32
 // residual stream, where that error showed up on every track, so it takes the
 // two-operation sigmoid, as do the scan gates (a = 1 - sigma there also needs
-// relative accuracy as sigma -> 1).
-__device__ __forceinline__ float sigm_acc(float x) { return rcp_approx(1.0f + ex2_approx(-x * LOG2E_F)); }
+// relative accuracy as sigma -> 1).  (A reciprocal by Newton steps on the FMA
+// pipe instead of rcp was measured slower: these epilogues are bound by issued
+// instructions more than by the MUFU unit.)  sigm_pre takes its argument
+// already scaled by -log2 e, with the bias folded in by one FMA.
+__device__ __forceinline__ float sigm_pre(float t) { return rcp_approx(1.0f + ex2_approx(t)); }
 __device__ __forceinline__ float tanh_approx(float x) {
   float y;
   asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-__device__ __forceinline__ float silu_t(float x) {
-  const float h = 0.5f * x;
+// SiLU(v + b) in that form, with hb = b / 2: the half argument (v + b) / 2 comes
+// from one FMA, bit for bit the value of halving the rounded sum (halving is exact)
+__device__ __forceinline__ float silu_tb(float v, float hb) {
+  const float h = fmaf(v, 0.5f, hb);
   return fmaf(h, tanh_approx(h), h);
 }
 
@@ -348,40 +353,44 @@ __device__ __forceinline__ void carry_wait(const ECtx& x) {
   asm volatile("bar.sync %0, 64;" ::"r"(2 + 2 * x.q + x.half) : "memory");
 }
 
-// silu(acc + bias) of the 128-channel tile mt -> k-rows row0 + c of buf
+// silu(acc + b) of the 128-channel tile mt -> k-rows row0 + c of buf (b: the
+// thread's channel's bias, loaded before the wait for the product)
 template <bool FP16>
-__device__ __forceinline__ void ep_silu_mt(const ECtx& x, const float* bias, int mt, uint32_t tcol, uint32_t buf,
-                                           int row0) {
+__device__ __forceinline__ void ep_silu_mt(const ECtx& x, float b, int mt, uint32_t tcol, uint32_t buf, int row0) {
   float v[32];
   tmem_ld32(x.tq + tcol + mt * 128 + x.col0, v);
-  const float b = bias[mt * 128 + x.c];
   tmem_ld_wait();
 #pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = silu_t(v[i] + b);
+  for (int i = 0; i < 32; ++i) v[i] = silu_tb(v[i], 0.5f * b);
   store_row32<FP16>(buf, row0 + x.c, x.col0, v);
 }
 // silu(acc + bias) of the embedding's first product (accumulator columns
-// 256 + mt*128) -> XB rows [mt*128 + c], all tiles read under one TMEM wait
-template <bool FP16, int MT>
-__device__ __forceinline__ void ep_silu_t(const ECtx& x, const float* bias) {
+// 256 + mt*128) -> XB rows [mt*128 + c], all tiles read under one TMEM wait;
+// the biases are loaded before the wait for the product (wait_first)
+template <bool FP16, int MT, class W>
+__device__ __forceinline__ void ep_silu_t(const ECtx& x, const float* bias, W&& wait_first) {
+  float bv[MT];
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) bv[mt] = bias[mt * 128 + x.c];
+  wait_first();
   float v[MT][32];
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) tmem_ld32(x.tq + 256 + mt * 128 + x.col0, v[mt]);
   tmem_ld_wait();
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
-    const float b = bias[mt * 128 + x.c];
+    const float b = bv[mt];
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[mt][i] = silu(v[mt][i] + b);
     store_row32<FP16>(x.xb, mt * 128 + x.c, x.col0, v[mt]);
   }
 }
-template <bool FP16>
-__device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias) {
+template <bool FP16, class W>
+__device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias, W&& wait_first) {
   if (x.MT == 2)
-    ep_silu_t<FP16, 2>(x, bias);
+    ep_silu_t<FP16, 2>(x, bias, wait_first);
   else
-    ep_silu_t<FP16, 1>(x, bias);
+    ep_silu_t<FP16, 1>(x, bias, wait_first);
 }
 
 // X = acc + bias, zero on pad columns (a layer's accumulator already holds x'
@@ -407,39 +416,47 @@ __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
 template <bool FP16, int MT, class W, class S>
 __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, const float* gain, W&& wait_tile,
                                               S&& signal_tile) {
+  // bias and gain of the thread's channels, loaded before the wait for the
+  // first tile's product so that their latency hides behind it
   const TcParams& p = *x.p;
   constexpr int D = 128 * MT;   // d_model
   const uint32_t vm = x.md->m_valid[x.half][x.sub];   // bit i: column col0 + i holds a hit
   // X = acc + bias (the accumulator already holds x' + MLP for a layer, the
-  // embedding product for the embedding), zero on pad columns.  The products
-  // complete one 128-channel tile at a time: tile 0 is processed while tile 1 is
-  // still being computed (wait_tile), and x_hat is handed over per tile
-  // (signal_tile) so the next products can start on its K rows.
-  float bias_v[MT];
+  // embedding product for the embedding).  Pad columns are not cleared in X:
+  // their x_hat is 0 (their inverse RMS is set to 0), so every product gives
+  // them its bias, and their values stay finite and in their own columns (the
+  // products and norms are per column, the scans restart at each track's ends,
+  // pooling skips them).  The products
+  // complete one 128-channel tile at a time, each waited for in turn
+  // (wait_tile): tile 0 is summed while tile 1 is still being computed, and
+  // x_hat is handed over per tile
+  // (signal_tile) so the next products can start on its K rows.  Only the sums
+  // of squares stand between the last product and the first hand-over: X goes
+  // to the scratch after both hand-overs (each thread later reads back only its
+  // own values, and the accumulator columns still hold X until the next layer's
+  // first merge, which waits for this thread's scan hand-over).
+  float bias_v[MT], gain_v[MT];
 #pragma unroll
-  for (int mt = 0; mt < MT; ++mt) bias_v[mt] = bias[mt * 128 + x.c];
+  for (int mt = 0; mt < MT; ++mt) {
+    bias_v[mt] = bias[mt * 128 + x.c];
+    gain_v[mt] = gain[mt * 128 + x.c];
+  }
   float sq[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) sq[i] = 0.0f;
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
-    if (mt > 0) wait_tile();
+    wait_tile();
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
-      const int c0 = x.col0 + 16 * hh;
       float v[16];
-      tmem_ld16(x.tq + mt * 128 + c0, v);
+      tmem_ld16(x.tq + mt * 128 + x.col0 + 16 * hh, v);
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
-        v[i] = val;
+        const float val = v[i] + bias_v[mt];
         sq[16 * hh + i] = fmaf(val, val, sq[16 * hh + i]);
       }
-      // the residual stream to the scratch (a warp's store: one 128-byte line)
-      float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
-#pragma unroll
-      for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i];
     }
   }
 #pragma unroll
@@ -451,23 +468,26 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
     if (x.lane < 16) x.m->part[x.q][x.col0 + 16 * hh + x.lane] = t;
   }
   // the column sums over all channels: the four quadrants' partial sums of this
-  // segment's columns
+  // segment's columns; every warp then forms the 32 inverse RMS values itself
+  // (the same sum in the same order, so the four copies are identical) in a
+  // slice of its own
   seg_sync(x.seg);
-  if (x.q == 0) {
+  float* rw = x.m->rinv[x.e];
+  {
     const int c = x.col0 + x.lane;
     const float t = x.m->part[0][c] + x.m->part[1][c] + x.m->part[2][c] + x.m->part[3][c];
-    x.m->rinv[c] = 1.0f / sqrtf(t / (float)D + p.rms_eps);
+    rw[x.lane] = ((vm >> x.lane) & 1u) ? 1.0f / sqrtf(t / (float)D + p.rms_eps) : 0.0f;
   }
-  seg_sync(x.seg);
+  __syncwarp();
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
-    const float g = gain[mt * 128 + x.c];
+    const float g = gain_v[mt];
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
       const int c0 = x.col0 + 16 * hh;
       float v[16], rv[16];
       tmem_ld16(x.tq + mt * 128 + c0, v);
-      const float4* rp = reinterpret_cast<const float4*>(x.m->rinv + c0);
+      const float4* rp = reinterpret_cast<const float4*>(rw + 16 * hh);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         const float4 r4 = rp[i];
@@ -478,13 +498,24 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
       }
       tmem_ld_wait();
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const float val = ((vm >> (16 * hh + i)) & 1u) ? v[i] + bias_v[mt] : 0.0f;
-        v[i] = val * g * rv[i];
-      }
+      for (int i = 0; i < 16; ++i) v[i] = (v[i] + bias_v[mt]) * g * rv[i];
       store_row16<FP16>(x.xb, mt * 128 + x.c, c0, v);
     }
     signal_tile();   // x_hat of this tile is in XB
+  }
+  // the residual stream to the scratch (a warp's store: one 128-byte line)
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      const int c0 = x.col0 + 16 * hh;
+      float v[16];
+      tmem_ld16(x.tq + mt * 128 + c0, v);
+      tmem_ld_wait();
+      float* xp = x.xs + (size_t)c0 * D + mt * 128 + x.c;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) xp[(size_t)i * D] = v[i] + bias_v[mt];
+    }
   }
 }
 
@@ -545,13 +576,10 @@ __device__ __forceinline__ void gate_x_load(const ECtx& x, int mt, float (&xv)[3
 // x' = X + (M + b_m) * sigma(p_g + b_g) for the 128-channel tile mt -> TMEM columns
 // 128 mt.. (in place of the merge accumulator; MLP2 accumulates onto it) and XB
 // rows 128 mt + c.
-template <bool FP16, int MT>
-__device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const float (&xv)[32]) {
-  const TcParams& p = *x.p;
-  constexpr int D = 128 * MT;
+template <bool FP16>
+__device__ __forceinline__ void ep_gate(const ECtx& x, int mt, const float (&xv)[32], float bm, float bg) {
   const int ch_g = mt * 128 + x.c;
-  const float bm = p.b_m[l * D + ch_g];
-  const float bg = p.b_in[(size_t)l * p.ROWS_IN + p.NDC * 256 + ch_g];
+  const float cg = -bg * LOG2E_F;
 #pragma unroll
   for (int hh = 0; hh < 2; ++hh) {
     const int c0 = x.col0 + 16 * hh;
@@ -560,18 +588,11 @@ __device__ __forceinline__ void ep_gate_t(const ECtx& x, int l, int mt, const fl
     tmem_ld16(x.tq + 256 + mt * 128 + c0, gv);
     tmem_ld_wait();
 #pragma unroll
-    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm_acc(gv[i] + bg), xv[16 * hh + i]);
+    for (int i = 0; i < 16; ++i) mv[i] = fmaf(mv[i] + bm, sigm_pre(fmaf(gv[i], -LOG2E_F, cg)), xv[16 * hh + i]);
     tmem_st16(x.tq + mt * 128 + c0, mv);   // x' where MLP2 will accumulate
     store_row16<FP16>(x.xb, ch_g, c0, mv);
   }
   tmem_st_wait();
-}
-template <bool FP16>
-__device__ __forceinline__ void ep_gate(const ECtx& x, int l, int mt, const float (&xv)[32]) {
-  if (x.MT == 2)
-    ep_gate_t<FP16, 2>(x, l, mt, xv);
-  else
-    ep_gate_t<FP16, 1>(x, l, mt, xv);
 }
 
 // Scan chunk of one layer.  The chunk holds 64 channels of both directions:
@@ -606,9 +627,10 @@ __device__ __forceinline__ void scan_gates(const ECtx& x, float (&z)[32], float 
 // Eq. 2 per channel over this thread's 32 columns (one FMA per hit on the serial
 // path), the states replacing z.  Tracks fill a slab from its first column, so
 // padding only trails the last track: the forward state is never read after it,
-// and in reverse the last track's end restarts the state.  Values left in
+// and in reverse the last track's end restarts the state (a = 0 there: the
+// finite state coming from the padding is multiplied away).  Values left in
 // padding columns stay in padding columns (every product and norm is per
-// column, every residual masks them), so they need no clearing here.
+// column) and stay finite (their x_hat is 0), so they need no clearing here.
 template <bool FP16>
 __device__ __forceinline__ void scan_chain_store(const ECtx& x, float (&a)[32], const float (&b)[32]) {
   const bool fwd = x.q < 2;
@@ -763,12 +785,14 @@ __device__ __forceinline__ void load_tile(const TcParams& p, Misc* m, TileMeta* 
 // buffer into HB (five 16-byte chunks per thread, all loads in flight at once).
 // The loads bypass L1 (ld.global.cg): the buffer is rewritten by the loader warp
 // every other tile, and a line of an earlier tile's operand must not be served
-// from L1.
-__device__ __forceinline__ void ep_fourier_in(const ECtx& x, const uint8_t* fb) {
-  static_assert(EB_BYTES == 5 * 16 * NE, "one chunk per thread per round");
-  uint4 v[5];
+// from L1.  The loads (fourier_fetch) can be issued before HB is free; the
+// stores (fourier_put) only after.
+static_assert(EB_BYTES == 5 * 16 * NE, "one chunk per thread per round");
+__device__ __forceinline__ void fourier_fetch(const ECtx& x, const uint8_t* fb, uint4 (&v)[5]) {
 #pragma unroll
   for (int r = 0; r < 5; ++r) v[r] = __ldcg(reinterpret_cast<const uint4*>(fb) + r * NE + x.te);
+}
+__device__ __forceinline__ void fourier_put(const ECtx& x, const uint4 (&v)[5]) {
 #pragma unroll
   for (int r = 0; r < 5; ++r) st_shared_v4(x.hb + 16 * (r * NE + x.te), v[r].x, v[r].y, v[r].z, v[r].w);
 }
@@ -1047,20 +1071,28 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
     const uint8_t* fbuf = p.fbuf + (size_t)blockIdx.x * 2 * EB_BYTES;
     uint32_t meta_ph[2] = {0u, 0u};
     // tile start: the loader's metadata and Fourier operand of the CTA's i-th tile
-    auto tile_in = [&](int i) {
+    // the loads wait for the loader's hand-over of tile i; the stores, after
+    // which the operand is handed to the issuer, need HB free
+    auto tile_fetch = [&](int i, uint4 (&v)[5]) {
       const int b = i & 1;
       wait_on(smem_u32(&m->meta_full[b]), meta_ph[b]);
-      ep_fourier_in(x, fbuf + b * EB_BYTES);
+      fourier_fetch(x, fbuf + b * EB_BYTES, v);
+    };
+    auto tile_put = [&](const uint4 (&v)[5]) {
+      fourier_put(x, v);
       signal();
+    };
+    auto tile_in = [&](int i) {
+      uint4 v[5];
+      tile_fetch(i, v);
+      tile_put(v);
     };
     if ((int)blockIdx.x < n_tiles) tile_in(0);
     int i = 0;
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
       x.md = &m->meta[i & 1];
-      wait_acc();
-      ep_silu<FP16>(x, p.b_e1);
+      ep_silu<FP16>(x, p.b_e1, wait_acc);
       signal();
-      wait_acc();
       ep_residual<FP16>(x, p.b_e2, p.g, wait_acc, signal);   // embedding output X0
       for (int l = 0; l < p.L; ++l) {
         for (int dc = 0; dc < p.NDC; ++dc) {
@@ -1081,37 +1113,46 @@ __global__ void __launch_bounds__(NT, 1) tc_forward_kernel(const __grid_constant
         // gate and MLP1 epilogues one 128-channel tile at a time (the issuer
         // pipelines the next tile's products behind each); with d_model 256 the
         // SiLU of tile 0 goes to HB (MLP1 still reads XB rows 0-127 then)
+        // the biases of the thread's channels are loaded ahead of the waits
         const float* b1 = p.b_1 + (size_t)l * p.D;
+        const float* bmp = p.b_m + (size_t)l * p.D;
+        const float* bgp = p.b_in + (size_t)l * p.ROWS_IN + p.NDC * 256;
+        const float bm0 = bmp[x.c], bg0 = bgp[x.c], b10 = b1[x.c];
         float xg[32];
         gate_x_load(x, 0, xg);
         wait_acc();
-        ep_gate<FP16>(x, l, 0, xg);
+        ep_gate<FP16>(x, 0, xg, bm0, bg0);
         signal();
         if (x.MT == 2) {
+          const float bm1 = bmp[128 + x.c], bg1 = bgp[128 + x.c], b11 = b1[128 + x.c];
           gate_x_load(x, 1, xg);
           wait_acc();
-          ep_gate<FP16>(x, l, 1, xg);
+          ep_gate<FP16>(x, 1, xg, bm1, bg1);
           signal();
           wait_acc();
-          ep_silu_mt<FP16>(x, b1, 0, 256, x.hb, 0);
+          ep_silu_mt<FP16>(x, b10, 0, 256, x.hb, 0);
           signal();
           wait_acc();
-          ep_silu_mt<FP16>(x, b1, 1, 256, x.xb, 128);
+          ep_silu_mt<FP16>(x, b11, 1, 256, x.xb, 128);
           signal();
         } else {
           wait_acc();
-          ep_silu_mt<FP16>(x, b1, 0, 256, x.xb, 0);
+          ep_silu_mt<FP16>(x, b10, 0, 256, x.xb, 0);
           signal();
         }
-        wait_acc();
         if (l + 1 < p.L) {
           ep_residual<FP16>(x, p.b_2 + (size_t)l * p.D, p.g + (size_t)(l + 1) * p.D, wait_acc, signal);
         } else {
-          // both output tiles of the last MLP2 have completed, so HB and XB are
-          // free: the next tile's Fourier operand goes in and its first product
-          // (into the z/n columns) runs while this tile is pooled
+          // once both output tiles of the last MLP2 have completed, HB and XB
+          // are free: the next tile's Fourier operand (fetched before the
+          // waits) goes in and its first product (into the z/n columns) runs
+          // while this tile is pooled
+          const bool more = t + (int)gridDim.x < n_tiles;
+          uint4 fv[5];
+          if (more) tile_fetch(i + 1, fv);
+          wait_acc();
           if (x.MT == 2) wait_acc();
-          if (t + (int)gridDim.x < n_tiles) tile_in(i + 1);
+          if (more) tile_put(fv);
           ep_pool(x, p.b_2 + (size_t)l * p.D);
           signal_to(smem_u32(&m->meta_free[i & 1]), false);   // this tile's metadata is no longer read
         }
