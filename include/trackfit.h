@@ -194,9 +194,10 @@ int trackfit_forward_packed(trackfit_t h, const float* hits, int64_t n_hit_rows,
  * End-to-end variant with HOST buffers: copies hits [n_tracks][max_hits][5] and
  * n_hits [n_tracks] to the device, runs the encoder and copies out_params
  * [n_tracks][5] back, all on `stream`, and returns after the stream has finished
- * this work (synchronous).  The batch moves in steps of 1,048,576 tracks: a
+ * this work (synchronous).  The batch moves in steps of 262,144 tracks: a
  * step's inputs are copied on a stream of the handle's own while the previous
- * step computes on `stream`, and its outputs are copied back behind it.  Pinned
+ * step computes on `stream` (only the first step's copy is not hidden), and
+ * its outputs are copied back behind it.  Pinned
  * (page-locked) host memory makes the copies asynchronous and lets them
  * overlap; pageable memory works too.  The device staging
  * buffers are owned by the handle and grow on demand (this call may allocate).

@@ -404,26 +404,38 @@ extern "C" int trackfit_forward_host(trackfit_t h, const float* hits_host, const
   cudaStream_t cs = h->cp_stream;
   cudaEvent_t* ev = h->cp_ev;
   const int64_t chunk = TF_HOST_CHUNK;
+  const int64_t n_chunks = (n_tracks + chunk - 1) / chunk;
+  // chunk k's events: in(k) (its inputs have landed), done(k) (its outputs are
+  // computed), from a ring (each is waited for before it is recorded again)
+  auto ev_in = [&](int64_t k) { return ev[1 + (2 * k) % (TF_HOST_EVENTS - 2)]; };
+  auto ev_done = [&](int64_t k) { return ev[2 + (2 * k) % (TF_HOST_EVENTS - 2)]; };
+  auto send = [&](int64_t k) -> cudaError_t {   // chunk k's inputs, on the copy stream
+    const int64_t c0 = k * chunk, nb = (n_tracks - c0 < chunk) ? n_tracks - c0 : chunk;
+    cudaError_t r = cudaMemcpyAsync(h->st_hits + c0 * row, hits_host + c0 * row, nb * row * sizeof(float),
+                                    cudaMemcpyHostToDevice, cs);
+    if (r == cudaSuccess)
+      r = cudaMemcpyAsync(h->st_n + c0, n_hits_host + c0, nb * sizeof(int32_t), cudaMemcpyHostToDevice, cs);
+    if (r == cudaSuccess) r = cudaEventRecord(ev_in(k), cs);
+    return r;
+  };
   // the staging buffers may still be read by earlier work on the caller's stream
   cudaError_t e = cudaEventRecord(ev[0], st);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev[0], 0);
-  int k = 0;
-  for (int64_t c0 = 0; c0 < n_tracks && e == cudaSuccess; c0 += chunk, ++k) {
-    const int64_t nb = (n_tracks - c0 < chunk) ? n_tracks - c0 : chunk;
-    cudaEvent_t in = ev[1 + (2 * k) % (TF_HOST_EVENTS - 2)], done = ev[2 + (2 * k) % (TF_HOST_EVENTS - 2)];
-    e = cudaMemcpyAsync(h->st_hits + c0 * row, hits_host + c0 * row, nb * row * sizeof(float), cudaMemcpyHostToDevice, cs);
-    if (e == cudaSuccess)
-      e = cudaMemcpyAsync(h->st_n + c0, n_hits_host + c0, nb * sizeof(int32_t), cudaMemcpyHostToDevice, cs);
-    if (e == cudaSuccess) e = cudaEventRecord(in, cs);
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, in, 0);
+  if (e == cudaSuccess) e = send(0);
+  for (int64_t k = 0; k < n_chunks && e == cudaSuccess; ++k) {
+    // chunk k + 1's inputs are queued on the copy stream before that stream waits
+    // for chunk k's outputs, so they travel while chunk k computes
+    if (k + 1 < n_chunks) e = send(k + 1);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, ev_in(k), 0);
     if (e != cudaSuccess) break;
+    const int64_t c0 = k * chunk, nb = (n_tracks - c0 < chunk) ? n_tracks - c0 : chunk;
     const int r = trackfit_forward(h, h->st_hits + c0 * row, h->st_n + c0, nb, h->st_out + c0 * 5, stream);
     if (r != TRACKFIT_OK) {
       cudaStreamSynchronize(cs);
       return r;
     }
-    e = cudaEventRecord(done, st);
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, done, 0);
+    e = cudaEventRecord(ev_done(k), st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev_done(k), 0);
     if (e == cudaSuccess)
       e = cudaMemcpyAsync(out_host + c0 * 5, h->st_out + c0 * 5, nb * 5 * sizeof(float), cudaMemcpyDeviceToHost, cs);
   }

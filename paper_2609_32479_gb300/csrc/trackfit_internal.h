@@ -10,7 +10,7 @@
 #define TF_MAX_LAYERS 16
 #define TF_MAX_HITS 64
 #define TF_PACKED_CHUNK 1048576
-#define TF_HOST_CHUNK 1048576  // tracks per copy / compute step of trackfit_forward_host
+#define TF_HOST_CHUNK 262144  // tracks per copy / compute step of trackfit_forward_host
 #define TF_HOST_EVENTS 10
 
 // Offsets (in floats) of every tensor inside the fp32 weight blob.

@@ -239,6 +239,24 @@ def test_host_buffer_entry_point_matches_device(T):
         np.testing.assert_array_equal(o2, base)
 
 
+def test_host_buffer_entry_point_in_several_steps(T):
+    """A batch of three copy/compute steps (262,144 + 262,144 + 75,712 tracks) through
+    the host-buffer entry point equals one device forward bit for bit."""
+    B = 600000
+    w = W.workload("sweep8", n_tracks=B)
+    tb = W.gen_tracks(w)
+    blob = W.gen_weights(w.model, w.weight_seed)
+    base = run(T, w.model, blob, tb.hits, tb.n_hits)["out"]
+    with T.Trackfit(w.model, blob) as tf:
+        hits = torch.from_numpy(tb.hits).pin_memory()
+        n = torch.from_numpy(tb.n_hits).pin_memory()
+        out = torch.empty((B, 5), dtype=torch.float32).pin_memory()
+        for _ in range(2):                           # the second call reuses the staging buffers
+            out.fill_(float("nan"))
+            tf.forward_host_ptr(hits.data_ptr(), n.data_ptr(), B, out.data_ptr())
+            np.testing.assert_array_equal(out.numpy(), base)
+
+
 def test_abi_argument_errors_launch_nothing(T):
     w = W.workload("tiny", n_tracks=8)
     blob = W.gen_weights(w.model, 1)
