@@ -27,25 +27,67 @@ __device__ __forceinline__ void put(float* p, float v) { *p = v; }
 __device__ __forceinline__ void put(__half* p, float v) { *p = __float2half_rn(v); }
 __device__ __forceinline__ void put(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
 
+// One head's output row o[0 .. DH) = acc * inv in 16-byte stores (DH is a
+// multiple of 8; a row that does not start on a 16-byte boundary, which a
+// workspace carved at an odd offset could give, is written value by value);
+// each value is rounded as put() rounds it.
+template <int DH>
+__device__ __forceinline__ void put_row(float* o, const float (&acc)[DH], float inv) {
+  if (reinterpret_cast<uintptr_t>(o) & 15u) {
+#pragma unroll
+    for (int i = 0; i < DH; ++i) put(o + i, acc[i] * inv);
+    return;
+  }
+#pragma unroll
+  for (int i = 0; i < DH; i += 4)
+    *reinterpret_cast<float4*>(o + i) = make_float4(acc[i] * inv, acc[i + 1] * inv, acc[i + 2] * inv, acc[i + 3] * inv);
+}
+template <int DH>
+__device__ __forceinline__ void put_row(__half* o, const float (&acc)[DH], float inv) {
+  if (reinterpret_cast<uintptr_t>(o) & 15u) {
+#pragma unroll
+    for (int i = 0; i < DH; ++i) put(o + i, acc[i] * inv);
+    return;
+  }
+#pragma unroll
+  for (int i = 0; i < DH; i += 8) {
+    uint4 w;
+    __half2 h0 = __floats2half2_rn(acc[i] * inv, acc[i + 1] * inv), h1 = __floats2half2_rn(acc[i + 2] * inv, acc[i + 3] * inv);
+    __half2 h2 = __floats2half2_rn(acc[i + 4] * inv, acc[i + 5] * inv), h3 = __floats2half2_rn(acc[i + 6] * inv, acc[i + 7] * inv);
+    w.x = *reinterpret_cast<uint32_t*>(&h0);
+    w.y = *reinterpret_cast<uint32_t*>(&h1);
+    w.z = *reinterpret_cast<uint32_t*>(&h2);
+    w.w = *reinterpret_cast<uint32_t*>(&h3);
+    *reinterpret_cast<uint4*>(o + i) = w;
+  }
+}
+template <int DH>
+__device__ __forceinline__ void put_row(__nv_bfloat16* o, const float (&acc)[DH], float inv) {
+  if (reinterpret_cast<uintptr_t>(o) & 15u) {
+#pragma unroll
+    for (int i = 0; i < DH; ++i) put(o + i, acc[i] * inv);
+    return;
+  }
+#pragma unroll
+  for (int i = 0; i < DH; i += 8) {
+    uint4 w;
+    __nv_bfloat162 h0 = __floats2bfloat162_rn(acc[i] * inv, acc[i + 1] * inv);
+    __nv_bfloat162 h1 = __floats2bfloat162_rn(acc[i + 2] * inv, acc[i + 3] * inv);
+    __nv_bfloat162 h2 = __floats2bfloat162_rn(acc[i + 4] * inv, acc[i + 5] * inv);
+    __nv_bfloat162 h3 = __floats2bfloat162_rn(acc[i + 6] * inv, acc[i + 7] * inv);
+    w.x = *reinterpret_cast<uint32_t*>(&h0);
+    w.y = *reinterpret_cast<uint32_t*>(&h1);
+    w.z = *reinterpret_cast<uint32_t*>(&h2);
+    w.w = *reinterpret_cast<uint32_t*>(&h3);
+    *reinterpret_cast<uint4*>(o + i) = w;
+  }
+}
+
 constexpr int THREADS = 64;   // a track: heads x hits items (52 at 13 hits and 4 heads)
 
 // Shared memory of one CTA: keys and values, T rows x NH heads x (dh + 4) floats each.
 __host__ __device__ inline size_t smem_bytes(int T, int D, int NH) {
   return (size_t)2 * T * (D + 4 * NH) * sizeof(float);
-}
-
-template <int DH>
-__device__ __forceinline__ float dot(const float (&q)[DH], const float* k) {
-  float s = 0.0f;
-#pragma unroll
-  for (int i = 0; i < DH; i += 4) {
-    const float4 a = *reinterpret_cast<const float4*>(k + i);
-    s = fmaf(q[i], a.x, s);
-    s = fmaf(q[i + 1], a.y, s);
-    s = fmaf(q[i + 2], a.z, s);
-    s = fmaf(q[i + 3], a.w, s);
-  }
-  return s;
 }
 
 // qkv: rows [q | k | v] of width 3 D at stride ldq; track b's hit t is row
@@ -98,13 +140,57 @@ __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* _
     }
     const float* kh = ks + h * hs;
     const float* vh = vs + h * hs;
+    // the scores four keys at a time: four independent chains, each summed over
+    // the head's dimensions in order (rows past the last key are read from the
+    // last key's row and their scores dropped, so every read stays within the
+    // track's keys)
     float sc[KMAX];
     float m = -INFINITY;
 #pragma unroll
-    for (int j = 0; j < KMAX; ++j) {
-      if (j >= n) break;
-      sc[j] = dot<DH>(q, kh + j * rs) * scale;
-      m = fmaxf(m, sc[j]);
+    for (int j0 = 0; j0 < KMAX; j0 += 4) {
+      if (j0 >= n) break;
+      const float* k0 = kh + j0 * rs;
+      const float* k1 = kh + min(j0 + 1, n - 1) * rs;
+      const float* k2 = kh + min(j0 + 2, n - 1) * rs;
+      const float* k3 = kh + min(j0 + 3, n - 1) * rs;
+      float s0 = 0.0f, s1 = 0.0f, s2 = 0.0f, s3 = 0.0f;
+#pragma unroll
+      for (int i = 0; i < DH; i += 4) {
+        const float4 a0 = *reinterpret_cast<const float4*>(k0 + i);
+        const float4 a1 = *reinterpret_cast<const float4*>(k1 + i);
+        const float4 a2 = *reinterpret_cast<const float4*>(k2 + i);
+        const float4 a3 = *reinterpret_cast<const float4*>(k3 + i);
+        s0 = fmaf(q[i], a0.x, s0);
+        s1 = fmaf(q[i], a1.x, s1);
+        s2 = fmaf(q[i], a2.x, s2);
+        s3 = fmaf(q[i], a3.x, s3);
+        s0 = fmaf(q[i + 1], a0.y, s0);
+        s1 = fmaf(q[i + 1], a1.y, s1);
+        s2 = fmaf(q[i + 1], a2.y, s2);
+        s3 = fmaf(q[i + 1], a3.y, s3);
+        s0 = fmaf(q[i + 2], a0.z, s0);
+        s1 = fmaf(q[i + 2], a1.z, s1);
+        s2 = fmaf(q[i + 2], a2.z, s2);
+        s3 = fmaf(q[i + 2], a3.z, s3);
+        s0 = fmaf(q[i + 3], a0.w, s0);
+        s1 = fmaf(q[i + 3], a1.w, s1);
+        s2 = fmaf(q[i + 3], a2.w, s2);
+        s3 = fmaf(q[i + 3], a3.w, s3);
+      }
+      sc[j0] = s0 * scale;
+      m = fmaxf(m, sc[j0]);
+      if (j0 + 1 < n) {
+        sc[j0 + 1] = s1 * scale;
+        m = fmaxf(m, sc[j0 + 1]);
+      }
+      if (j0 + 2 < n) {
+        sc[j0 + 2] = s2 * scale;
+        m = fmaxf(m, sc[j0 + 2]);
+      }
+      if (j0 + 3 < n) {
+        sc[j0 + 3] = s3 * scale;
+        m = fmaxf(m, sc[j0 + 3]);
+      }
     }
     float l = 0.0f;
 #pragma unroll
@@ -123,9 +209,7 @@ __global__ void __launch_bounds__(THREADS) track_attention_kernel(const float* _
       }
     }
     const float inv = 1.0f / l;
-    OutT* orow = o + (r0 + t) * ldo + h * DH;
-#pragma unroll
-    for (int i = 0; i < DH; ++i) put(orow + i, acc[i] * inv);
+    put_row<DH>(o + (r0 + t) * ldo + h * DH, acc, inv);
   }
 }
 

@@ -313,15 +313,25 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       // residual stream of EP_NORM and its sum of squares; 2: its normed operand.
       auto pass = [&](int mode, float inv) -> float {
         const bool is32 = mode == 1 || (mode == 0 && g.epi != EP_16 && g.epi != EP_SILU16);
+        const bool use_res = g.res && live;
+        // a unit's residual (64 bytes of the thread's row) is prefetched into L1
+        // together with that unit's TMEM load, one unit ahead
+        auto prefetch_res = [&](int u) {
+          if (use_res) asm volatile("prefetch.global.L1 [%0];" ::"l"(g.res + row * g.N + n0 + 16 * u));
+        };
         float ss = 0.0f, cur[16], nxt[16];
         if (ub < ue) {
           tmem_ld16(tq + 16 * ub, cur);
+          prefetch_res(ub);
           tmem_ld_wait();
         }
         for (int u = ub; u < ue; ++u) {
           const int slot = (u - ub) & 1;
           if (slot == 0) emit.begin(lane);
-          if (u + 1 < ue) tmem_ld16(tq + 16 * (u + 1), nxt);
+          if (u + 1 < ue) {
+            tmem_ld16(tq + 16 * (u + 1), nxt);
+            prefetch_res(u + 1);
+          }
           const int nb = n0 + 16 * u;
           const float4* bb = reinterpret_cast<const float4*>(g.bias + nb);
 #pragma unroll
@@ -332,7 +342,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
             cur[4 * i + 2] += w.z;
             cur[4 * i + 3] += w.w;
           }
-          if (g.res && live) {   // x + (acc + b), the same arithmetic in both passes of EP_NORM
+          if (use_res) {   // x + (acc + b), the same arithmetic in both passes of EP_NORM
             const float4* rr = reinterpret_cast<const float4*>(g.res + row * g.N + nb);
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
