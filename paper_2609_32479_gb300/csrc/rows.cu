@@ -313,7 +313,10 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
       // residual stream of EP_NORM and its sum of squares; 2: its normed operand.
       auto pass = [&](int mode, float inv) -> float {
         const bool is32 = mode == 1 || (mode == 0 && g.epi != EP_16 && g.epi != EP_SILU16);
-        const bool use_res = g.res && live;
+        // EP_NORM's first pass writes x = res + (acc + b) back over the accumulator,
+        // so the second pass reads x from TMEM instead of forming it again
+        const bool x_in_tmem = mode == 2;
+        const bool use_res = g.res && live && !x_in_tmem;
         // a unit's residual (64 bytes of the thread's row) is prefetched into L1
         // together with that unit's TMEM load, one unit ahead
         auto prefetch_res = [&](int u) {
@@ -333,16 +336,18 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
             prefetch_res(u + 1);
           }
           const int nb = n0 + 16 * u;
-          const float4* bb = reinterpret_cast<const float4*>(g.bias + nb);
+          if (!x_in_tmem) {
+            const float4* bb = reinterpret_cast<const float4*>(g.bias + nb);
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float4 w = __ldg(bb + i);
-            cur[4 * i] += w.x;
-            cur[4 * i + 1] += w.y;
-            cur[4 * i + 2] += w.z;
-            cur[4 * i + 3] += w.w;
+            for (int i = 0; i < 4; ++i) {
+              const float4 w = __ldg(bb + i);
+              cur[4 * i] += w.x;
+              cur[4 * i + 1] += w.y;
+              cur[4 * i + 2] += w.z;
+              cur[4 * i + 3] += w.w;
+            }
           }
-          if (use_res) {   // x + (acc + b), the same arithmetic in both passes of EP_NORM
+          if (use_res) {   // x + (acc + b)
             const float4* rr = reinterpret_cast<const float4*>(g.res + row * g.N + nb);
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
@@ -354,6 +359,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
             }
           }
           if (mode == 1) {
+            tmem_st16(tq + 16 * u, cur);   // x for the second pass (not the unit being loaded)
 #pragma unroll
             for (int i = 0; i < 16; ++i) ss = fmaf(cur[i], cur[i], ss);
           } else if (mode == 2) {
@@ -386,6 +392,7 @@ __global__ void __launch_bounds__(RG_THREADS, 1) row_gemm_kernel(const __grid_co
         // shared memory (double-buffered by tile) and a two-arrival barrier
         const int par = norms & 1;
         ssx[(par * 2 + hs) * 128 + 32 * q + lane] = pass(1, 0.0f);
+        tmem_st_wait();   // x is in TMEM before the second pass reads it
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&bars->ssb[q]));
         ok = mbar_wait(smem_u32(&bars->ssb[q]), (uint32_t)par, abort, g.wait_ns);
