@@ -253,6 +253,7 @@ extern "C" void trackfit_destroy(trackfit_t h) {
 
 extern "C" int trackfit_create(const trackfit_config_t* cfg, const float* weights, size_t n_weights,
                                trackfit_t* out) {
+  tf_nvtx_range nvtx_range("trackfit_create");
   if (!cfg || !weights || !out) return TRACKFIT_ERR_INVALID_ARG;
   tf_shape s;
   tf_blob_off o;
@@ -308,6 +309,7 @@ extern "C" int trackfit_set_path(trackfit_t h, int path) {
 
 extern "C" int trackfit_forward_ex(trackfit_t h, const float* hits, const int32_t* n_hits, int64_t n_tracks,
                                    float* out_params, float* out_q, float* out_pool, void* stream) {
+  tf_nvtx_range nvtx_range("trackfit_forward_ex");
   if (!h || !hits || !n_hits || !out_params) return TRACKFIT_ERR_INVALID_ARG;
   if (n_tracks <= 0) return TRACKFIT_ERR_INVALID_ARG;
   if (!aligned16(hits) || !aligned16(out_params) || !aligned16(n_hits)) return TRACKFIT_ERR_INVALID_ARG;
@@ -331,6 +333,7 @@ __global__ void counts_from_offsets(const int64_t* __restrict__ offs, int64_t B,
 
 extern "C" int trackfit_forward_packed(trackfit_t h, const float* hits, int64_t n_hit_rows, const int64_t* offsets,
                                        int64_t n_tracks, float* out_params, void* stream) {
+  tf_nvtx_range nvtx_range("trackfit_forward_packed");
   if (!h || !hits || !offsets || !out_params || n_tracks <= 0 || n_hit_rows < 0) return TRACKFIT_ERR_INVALID_ARG;
   if (!aligned16(hits) || !aligned16(offsets) || !aligned16(out_params)) return TRACKFIT_ERR_INVALID_ARG;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -356,6 +359,7 @@ extern "C" int trackfit_forward(trackfit_t h, const float* hits, const int32_t* 
 
 extern "C" int trackfit_forward_host(trackfit_t h, const float* hits_host, const int32_t* n_hits_host,
                                      int64_t n_tracks, float* out_host, void* stream) {
+  tf_nvtx_range nvtx_range("trackfit_forward_host");
   if (!h || !hits_host || !n_hits_host || !out_host || n_tracks <= 0) return TRACKFIT_ERR_INVALID_ARG;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const size_t row = (size_t)h->s.T * 5;

@@ -45,6 +45,7 @@ int scratch_address(void** out) {
 extern "C" int trackfit_forward_noalloc(const trackfit_config_t* cfg, const float* weights, const float* hits,
                                         const int32_t* n_hits, int64_t n_tracks, float* out_params,
                                         void* stream) {
+  tf_nvtx_range nvtx_range("trackfit_forward_noalloc");
   tf_shape s;
   tf_blob_off o;
   if (!cfg || !weights || !hits || !n_hits || !out_params || n_tracks <= 0) return TRACKFIT_ERR_INVALID_ARG;

@@ -215,6 +215,7 @@ __global__ void decode_kernel(const double* __restrict__ seed, const float* __re
 extern "C" int trackfit_seed(const float* hits, int32_t hit_stride, const int32_t* n_hits, int64_t n_tracks,
                              int32_t max_hits, double b_field, double* seed_out, float* features_out,
                              int32_t feat_stride, void* stream) {
+  tf_nvtx_range nvtx_range("trackfit_seed");
   if (!hits || !n_hits || !seed_out || n_tracks <= 0 || max_hits < 1 || max_hits > TF_MAX_HITS) {
     return TRACKFIT_ERR_INVALID_ARG;
   }
@@ -232,6 +233,7 @@ extern "C" int trackfit_seed(const float* hits, int32_t hit_stride, const int32_
 
 extern "C" int trackfit_decode(const double* seed, const float* corrections, int64_t n_tracks, float* out_params,
                                void* stream) {
+  tf_nvtx_range nvtx_range("trackfit_decode");
   if (!seed || !corrections || !out_params || n_tracks <= 0) return TRACKFIT_ERR_INVALID_ARG;
   const uintptr_t mis = reinterpret_cast<uintptr_t>(seed) | reinterpret_cast<uintptr_t>(corrections) |
                         reinterpret_cast<uintptr_t>(out_params);

@@ -2,10 +2,21 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 #include <stdint.h>
 #include <stddef.h>
 
 #include "trackfit.h"
+
+// An NVTX range over an entry point's host-side work (its launches included), so
+// that timeline tools show each call; with no tool attached a push and a pop cost
+// a few instructions.
+struct tf_nvtx_range {
+  explicit tf_nvtx_range(const char* name) { nvtxRangePushA(name); }
+  ~tf_nvtx_range() { nvtxRangePop(); }
+  tf_nvtx_range(const tf_nvtx_range&) = delete;
+  tf_nvtx_range& operator=(const tf_nvtx_range&) = delete;
+};
 
 #define TF_MAX_LAYERS 16
 #define TF_MAX_HITS 64
