@@ -393,10 +393,10 @@ __device__ __forceinline__ void ep_silu(const ECtx& x, const float* bias, W&& wa
     ep_silu_t<FP16, 1>(x, bias, wait_first);
 }
 
-// X = acc + bias, zero on pad columns (a layer's accumulator already holds x'
-// plus the MLP2 product).  X goes to the per-CTA scratch (read back once, by the
-// next layer's gate epilogue) and the RMS-normalised x_hat to XB (recomputing X
-// from TMEM); the last layer's X is mean-pooled instead (ep_pool).
+// X = acc + bias (a layer's accumulator already holds x' plus the MLP2 product).
+// X goes to the per-CTA scratch (read back once, by the next layer's gate
+// epilogue) and the RMS-normalised x_hat to XB (recomputing X from TMEM); the
+// last layer's X is mean-pooled instead (ep_pool).
 // Sum of v over the 32 lanes for 16 columns at once: afterwards lane L holds the
 // total of column L & 15 (both halves of the warp hold the same 16 totals).
 __device__ __forceinline__ float reduce_scatter16(float (&v)[16], int lane) {
@@ -426,15 +426,14 @@ __device__ __forceinline__ void ep_residual_t(const ECtx& x, const float* bias, 
   // their x_hat is 0 (their inverse RMS is set to 0), so every product gives
   // them its bias, and their values stay finite and in their own columns (the
   // products and norms are per column, the scans restart at each track's ends,
-  // pooling skips them).  The products
-  // complete one 128-channel tile at a time, each waited for in turn
-  // (wait_tile): tile 0 is summed while tile 1 is still being computed, and
-  // x_hat is handed over per tile
-  // (signal_tile) so the next products can start on its K rows.  Only the sums
-  // of squares stand between the last product and the first hand-over: X goes
-  // to the scratch after both hand-overs (each thread later reads back only its
-  // own values, and the accumulator columns still hold X until the next layer's
-  // first merge, which waits for this thread's scan hand-over).
+  // pooling skips them).  The products complete one 128-channel tile at a time,
+  // each waited for in turn (wait_tile): tile 0 is summed while tile 1 is still
+  // being computed, and x_hat is handed over per tile (signal_tile) so the next
+  // products can start on its K rows.  Only the sums of squares stand between
+  // the last product and the first hand-over: X goes to the scratch after both
+  // hand-overs (each thread later reads back only its own values, and the
+  // accumulator columns still hold X until the next layer's first merge, which
+  // waits for this thread's scan hand-over).
   float bias_v[MT], gain_v[MT];
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
